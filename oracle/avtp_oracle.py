@@ -1,0 +1,401 @@
+"""AVTP pruning-stage oracle: a plain, slow, fp64 CPU restatement of the method.
+
+TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``
+(its ``cpu_baseline`` leg and its ``--impl reference`` arm) may import or run this
+module. The product path (``paper_2608_26806_gb300`` and its CUDA library) never
+does, and this module imports nothing from it: the two share no code.
+
+What it computes (paper: "Multi-Image Visual Token Pruning in Large Visual
+Language Models", AVTP):
+
+1A. Token importance from hidden-state variation (§3.3.1):
+    ``I_v = 1 - Sim(h^l_v, h^prior_v)``; ``Sim`` is read as cosine similarity with
+    each norm guarded below by 1e-8.
+1B. Text-to-visual attention importance (the attention quantity of §3.3.2, kept
+    per visual token): for each visual key t of request r,
+    ``s_t = 1/(Hq*|Q_r|) * sum_h sum_{q in Q_r, q >= t} softmax_{h,q}(t)``, where
+    Q_r are the request's text tokens, the softmax runs over the keys causally
+    visible to q inside the request, logits are ``scale * q_h . k_{g(h)}`` and
+    ``g(h) = h // (Hq/Hkv)`` (grouped-query attention).
+2.  Per-image mean importance and adaptive keep ratio (§3.3.3):
+    ``Ibar_i = mean_{v in V_i} I_v``, ``r_i = r_base + alpha*(Ibar_i - Ibar_avg)``,
+    clamped to [5%, 95%] (App. A.2), then integer budgets whose total is the
+    request's global budget.
+3.  Per image, keep the ``k_i`` most important visual tokens; text is kept (§3.1,
+    §3.3.3); the result is an order-preserving subsequence (§3.1).
+4.  Compaction: a row gather of the kept tokens (§3.1, ``E_pruned = p(E_v)``).
+
+Readings of points the paper leaves open (each is also listed with its reason in
+the design notes of the repository):
+
+* Per-image sums are taken in fixed point, ``S_i = sum rint(fx(I_t) * 2^32)`` on the
+  fp32-rounded score, with ``fx`` mapping NaN to 0 and clamping to +-2^10, so that
+  every summation order gives the same integer.
+* ``Ibar_avg`` is the token-weighted mean ``sum_i S_i / 2^32 / N_vis``.
+* The global budget is ``B_r = floor(keep_ratio_r * N_vis_r + 0.5)``.
+* ``relative=1`` replaces the additive rule by ``r_i = r_base*(1 + alpha*(Ibar_i/Ibar_avg - 1))``
+  (``r_base`` when ``Ibar_avg == 0``); criterion 1B's raw values are of order
+  1/N, where the additive rule would leave every ratio at ``r_base``.
+* A shift lambda (water-fill) restores ``sum_i n_i * clamp(r_i + lambda)`` to ``B_r``
+  after clamping: 64 fp64 bisection steps on ``[r_min - max r, r_max - min r]``,
+  midpoint ``lo + (hi - lo) * 0.5``, move ``hi`` iff ``F(mid) >= B_r``, take ``hi``.
+* Integer budgets: ``x_i = n_i * clamp(r_i + lambda)``, ``k_i = min(floor(x_i), n_i)``,
+  then largest remainder (ties to the lower image index) until ``sum k_i = B_r``;
+  a surplus is removed from the smallest remainders (ties to the higher index).
+* Top-k order: score descending, position ascending; NaN ranks below -inf;
+  -0 equals +0.
+
+All floating-point steps of the budget rule are single fp64 operations in a
+fixed order (Python floats: no fused multiply-add), so a correct device
+implementation that rounds each operation to nearest reproduces them exactly.
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, List, Optional, Sequence
+
+import numpy as np
+
+FX_FRAC_BITS = 32
+FX_SCORE_LIMIT = 1024.0  # |score| is clamped to 2^10 before the fixed-point conversion
+NORM_EPS = 1e-8
+BISECTION_STEPS = 64
+
+
+# ----------------------------------------------------------------------------
+# helpers
+# ----------------------------------------------------------------------------
+def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Decode bf16 bit patterns (uint16) to fp64 (exact widening)."""
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return u.view(np.float32).astype(np.float64)
+
+
+def _image_rows(layout, r: int, i: int) -> np.ndarray:
+    base = int(layout.cu_seqlens[r]) + int(layout.img_start[i])
+    return np.arange(base, base + int(layout.img_len[i]), dtype=np.int64)
+
+
+def _request_visual_local(layout, r: int) -> np.ndarray:
+    """Boolean mask over the request's local positions: True inside an image span."""
+    T_r = int(layout.cu_seqlens[r + 1]) - int(layout.cu_seqlens[r])
+    m = np.zeros(T_r, dtype=bool)
+    for i in range(int(layout.img_cu[r]), int(layout.img_cu[r + 1])):
+        s = int(layout.img_start[i])
+        m[s:s + int(layout.img_len[i])] = True
+    return m
+
+
+# ----------------------------------------------------------------------------
+# Step 1A: hidden-state variation (paper §3.3.1)
+# ----------------------------------------------------------------------------
+def score_hidden_variation(layout, h_cur: np.ndarray, h_prior: np.ndarray) -> np.ndarray:
+    """``I_v = 1 - cos(h^l_v, h^prior_v)`` for every visual token (fp64); text entries are 0.
+
+    ``h_cur`` / ``h_prior``: bf16 bits [T, D]. Paper §3.3.1 (importance score).
+    """
+    T = int(layout.cu_seqlens[-1])
+    out = np.zeros(T, dtype=np.float64)
+    for r in range(len(layout.cu_seqlens) - 1):
+        for i in range(int(layout.img_cu[r]), int(layout.img_cu[r + 1])):
+            rows = _image_rows(layout, r, i)
+            a = bf16_to_f64(h_cur[rows])
+            b = bf16_to_f64(h_prior[rows])
+            dot = np.sum(a * b, axis=1)
+            na = np.sqrt(np.sum(a * a, axis=1))
+            nb = np.sqrt(np.sum(b * b, axis=1))
+            cos = dot / (np.maximum(na, NORM_EPS) * np.maximum(nb, NORM_EPS))
+            out[rows] = 1.0 - cos
+    return out
+
+
+# ----------------------------------------------------------------------------
+# Step 1B: text-to-visual attention (attention quantity of paper §3.3.2)
+# ----------------------------------------------------------------------------
+def attention_logits(layout, q, k, r: int, h: int, n_q_heads: int, n_kv_heads: int, scale: float):
+    """Scaled logits of request r, head h: text queries (rows) x all request keys.
+
+    Returns ``(z, text_local)``; ``z`` is fp64 [|Q_r|, T_r] with ``-inf`` where the key
+    lies after the query (causal mask).
+    """
+    a = int(layout.cu_seqlens[r])
+    b = int(layout.cu_seqlens[r + 1])
+    vis = _request_visual_local(layout, r)
+    text_local = np.nonzero(~vis)[0]
+    g = h // (n_q_heads // n_kv_heads)
+    Qh = bf16_to_f64(q[a + text_local, h, :])        # [nq, d]
+    Kg = bf16_to_f64(k[a:b, g, :])                   # [T_r, d]
+    z = float(scale) * (Qh @ Kg.T)                   # [nq, T_r]
+    keys = np.arange(b - a)
+    visible = keys[None, :] <= text_local[:, None]
+    z = np.where(visible, z, -np.inf)
+    return z, text_local
+
+
+def logsumexp_rows(z: np.ndarray) -> np.ndarray:
+    """Natural-log sum of exp over each row, with max subtraction."""
+    m = np.max(z, axis=1)
+    return m + np.log(np.sum(np.exp(z - m[:, None]), axis=1))
+
+
+def text_lse(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float) -> np.ndarray:
+    """Per (head, text query) natural-log LSE of the scaled causal logits: fp64 [Hq, T].
+
+    This is the normaliser a FlashAttention-style forward pass keeps per query row;
+    visual rows are left 0.
+    """
+    T = int(layout.cu_seqlens[-1])
+    out = np.zeros((n_q_heads, T), dtype=np.float64)
+    for r in range(len(layout.cu_seqlens) - 1):
+        a = int(layout.cu_seqlens[r])
+        for h in range(n_q_heads):
+            z, text_local = attention_logits(layout, q, k, r, h, n_q_heads, n_kv_heads, scale)
+            if text_local.size:
+                out[h, a + text_local] = logsumexp_rows(z)
+    return out
+
+
+def score_text_attention(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float,
+                         lse: Optional[np.ndarray] = None) -> np.ndarray:
+    """Mean over heads and text queries of the causal softmax probability of each visual key.
+
+    ``q``: bf16 bits [T, Hq, d]; ``k``: bf16 bits [T, Hkv, d]; ``lse`` (optional) [Hq, T]
+    natural-log normalisers for the text rows; when given they replace the
+    oracle's own. Returns fp64 [T] (text entries 0).
+    """
+    T = int(layout.cu_seqlens[-1])
+    out = np.zeros(T, dtype=np.float64)
+    for r in range(len(layout.cu_seqlens) - 1):
+        a = int(layout.cu_seqlens[r])
+        b = int(layout.cu_seqlens[r + 1])
+        vis = _request_visual_local(layout, r)
+        nq = int((~vis).sum())
+        if nq == 0:
+            continue
+        acc = np.zeros(b - a, dtype=np.float64)
+        for h in range(n_q_heads):
+            z, text_local = attention_logits(layout, q, k, r, h, n_q_heads, n_kv_heads, scale)
+            if lse is None:
+                norm = logsumexp_rows(z)
+            else:
+                norm = np.asarray(lse, dtype=np.float64)[h, a + text_local]
+            P = np.exp(z - norm[:, None])  # exp(-inf) = 0 on masked keys
+            acc += np.sum(P, axis=0)
+        out[a:b][vis] = acc[vis] / (n_q_heads * nq)
+    return out
+
+
+# ----------------------------------------------------------------------------
+# Step 2: per-image sums, adaptive ratios and integer budgets (paper §3.3.3, App. A.2)
+# ----------------------------------------------------------------------------
+def to_fp32(scores: np.ndarray) -> np.ndarray:
+    """The interface type of scores is fp32 (round to nearest)."""
+    return np.asarray(scores, dtype=np.float64).astype(np.float32)
+
+
+def fixed_point(scores_f32: np.ndarray) -> np.ndarray:
+    """``rint(fx(s) * 2^32)`` as int64; fx: NaN -> 0, clamp to [-2^10, 2^10]."""
+    s = np.asarray(scores_f32, dtype=np.float32).astype(np.float64)
+    s = np.where(np.isnan(s), 0.0, s)
+    s = np.clip(s, -FX_SCORE_LIMIT, FX_SCORE_LIMIT)
+    return np.rint(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)
+
+
+def image_sums(layout, scores_f32: np.ndarray) -> np.ndarray:
+    """Fixed-point per-image sums ``S_i`` (int64 [n_img]) of the fp32 scores."""
+    fx = fixed_point(scores_f32)
+    n_img = len(layout.img_len)
+    out = np.zeros(n_img, dtype=np.int64)
+    for r in range(len(layout.cu_seqlens) - 1):
+        for i in range(int(layout.img_cu[r]), int(layout.img_cu[r + 1])):
+            out[i] = int(sum(int(v) for v in fx[_image_rows(layout, r, i)]))
+    return out
+
+
+def global_budget(keep_ratio_f32: float, n_vis: int) -> int:
+    """``B_r = floor(keep_ratio * N_vis + 0.5)`` with the fp32 ratio widened to fp64."""
+    kr = float(np.float32(keep_ratio_f32))
+    return int(math.floor(kr * float(n_vis) + 0.5))
+
+
+def _clamp(x: float, lo: float, hi: float) -> float:
+    return min(max(x, lo), hi)
+
+
+def adaptive_ratios(S: Sequence[int], n: Sequence[int], r_base: float, alpha: float,
+                    relative: bool) -> List[float]:
+    """``r_i`` of paper §3.3.3 from fixed-point sums (fp64, one rounding per operation)."""
+    scale = 1.0 / float(2 ** FX_FRAC_BITS)
+    n_vis = sum(int(x) for x in n)
+    total = sum(int(x) for x in S)
+    ibar = [(float(int(S[i])) * scale) / float(int(n[i])) for i in range(len(n))]
+    ibar_avg = (float(total) * scale) / float(n_vis)
+    r = []
+    for i in range(len(n)):
+        if relative:
+            if ibar_avg == 0.0:
+                r.append(r_base)
+            else:
+                r.append(r_base * (1.0 + alpha * (ibar[i] / ibar_avg - 1.0)))
+        else:
+            r.append(r_base + alpha * (ibar[i] - ibar_avg))
+    return r
+
+
+def water_fill(r: Sequence[float], n: Sequence[int], B: int, r_min: float, r_max: float) -> float:
+    """Shift lambda with ``sum_i n_i * clamp(r_i + lambda, r_min, r_max) ~= B`` (64 bisection steps)."""
+
+    def F(lam: float) -> float:
+        acc = 0.0
+        for i in range(len(n)):  # image order, sequential
+            acc = acc + float(int(n[i])) * _clamp(r[i] + lam, r_min, r_max)
+        return acc
+
+    lo = r_min - max(r)
+    hi = r_max - min(r)
+    target = float(B)
+    for _ in range(BISECTION_STEPS):
+        mid = lo + (hi - lo) * 0.5
+        if F(mid) >= target:
+            hi = mid
+        else:
+            lo = mid
+    return hi
+
+
+def integer_budgets(r: Sequence[float], n: Sequence[int], B: int, lam: float,
+                    r_min: float, r_max: float) -> List[int]:
+    """Largest-remainder rounding of ``x_i = n_i * clamp(r_i + lambda)`` to a total of B."""
+    m = len(n)
+    x = [float(int(n[i])) * _clamp(r[i] + lam, r_min, r_max) for i in range(m)]
+    fl = [math.floor(v) for v in x]
+    frac = [x[i] - float(fl[i]) for i in range(m)]
+    k = [min(int(fl[i]), int(n[i])) for i in range(m)]
+    k = [max(v, 0) for v in k]
+    while sum(k) < B:
+        need = B - sum(k)
+        elig = [i for i in range(m) if k[i] < int(n[i])]
+        order = sorted(elig, key=lambda i: (-frac[i], i))
+        for i in order[:need]:
+            k[i] += 1
+    while sum(k) > B:
+        extra = sum(k) - B
+        elig = [i for i in range(m) if k[i] > 0]
+        order = sorted(elig, key=lambda i: (frac[i], -i))
+        for i in order[:extra]:
+            k[i] -= 1
+    return k
+
+
+def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
+             r_min: float = 0.05, r_max: float = 0.95, relative: bool = False) -> Dict[str, np.ndarray]:
+    """Per-image budgets ``k_i`` and the packed output offsets ``out_cu_seqlens``.
+
+    fp32 parameters (``keep_ratio``, ``alpha``, ``r_min``, ``r_max``) are widened to
+    fp64 exactly, as the device does. Returns a dict with ``budgets`` int32
+    [n_img], ``out_cu_seqlens`` int32 [R+1] and, for inspection, ``ratios`` and
+    ``lam`` per request.
+    """
+    R = len(layout.cu_seqlens) - 1
+    alpha = float(np.float32(alpha))
+    r_min = float(np.float32(r_min))
+    r_max = float(np.float32(r_max))
+    budgets = np.zeros(len(layout.img_len), dtype=np.int32)
+    out_cu = np.zeros(R + 1, dtype=np.int32)
+    ratios = np.zeros(len(layout.img_len), dtype=np.float64)
+    lams = np.zeros(R, dtype=np.float64)
+    for rq in range(R):
+        i0, i1 = int(layout.img_cu[rq]), int(layout.img_cu[rq + 1])
+        n = [int(v) for v in layout.img_len[i0:i1]]
+        n_vis = sum(n)
+        T_r = int(layout.cu_seqlens[rq + 1]) - int(layout.cu_seqlens[rq])
+        n_txt = T_r - n_vis
+        r_base = float(np.float32(keep_ratio[rq]))
+        B = global_budget(keep_ratio[rq], n_vis)
+        if i1 > i0:
+            Sr = [int(v) for v in S[i0:i1]]
+            r = adaptive_ratios(Sr, n, r_base, alpha, relative)
+            lam = water_fill(r, n, B, r_min, r_max)
+            k = integer_budgets(r, n, B, lam, r_min, r_max)
+            budgets[i0:i1] = k
+            ratios[i0:i1] = r
+            lams[rq] = lam
+        out_cu[rq + 1] = out_cu[rq] + B + n_txt
+    return {"budgets": budgets, "out_cu_seqlens": out_cu, "ratios": ratios, "lam": lams}
+
+
+# ----------------------------------------------------------------------------
+# Step 3: per-image top-k, text kept, ascending order (paper §3.1, §3.3.3)
+# ----------------------------------------------------------------------------
+def rank_key(score: float, pos: int):
+    """Sort key: score descending, position ascending; NaN below every number."""
+    if math.isnan(score):
+        return (1, 0.0, pos)
+    return (0, -score, pos)
+
+
+def select(layout, scores_f32: np.ndarray, budgets: np.ndarray) -> np.ndarray:
+    """Packed global indices of the kept tokens (int32), ascending within each request."""
+    sc = np.asarray(scores_f32, dtype=np.float32)
+    kept: List[int] = []
+    for r in range(len(layout.cu_seqlens) - 1):
+        a = int(layout.cu_seqlens[r])
+        b = int(layout.cu_seqlens[r + 1])
+        keep = ~_request_visual_local(layout, r)  # text always kept
+        for i in range(int(layout.img_cu[r]), int(layout.img_cu[r + 1])):
+            rows = _image_rows(layout, r, i)
+            order = sorted(rows.tolist(), key=lambda t: rank_key(float(sc[t]), t))
+            for t in order[:int(budgets[i])]:
+                keep[t - a] = True
+        kept.extend((np.nonzero(keep)[0] + a).tolist())
+    return np.asarray(kept, dtype=np.int32)
+
+
+# ----------------------------------------------------------------------------
+# Step 4: compaction (paper §3.1)
+# ----------------------------------------------------------------------------
+def compact(kept_idx: np.ndarray, rows: np.ndarray) -> np.ndarray:
+    """``out[j] = rows[kept_idx[j]]`` along axis 0 (any dtype, bit-exact)."""
+    return np.asarray(rows)[np.asarray(kept_idx, dtype=np.int64)]
+
+
+def compact_planes(kept_idx: np.ndarray, planes: np.ndarray) -> np.ndarray:
+    """Gather along the token axis of a [P, T] array (e.g. M-RoPE position ids)."""
+    return np.asarray(planes)[:, np.asarray(kept_idx, dtype=np.int64)]
+
+
+# ----------------------------------------------------------------------------
+# The whole stage
+# ----------------------------------------------------------------------------
+def prune(layout, *, criterion: str = "hidden_variation", keep_ratio, alpha: float = 1.0,
+          r_min: float = 0.05, r_max: float = 0.95, relative: Optional[bool] = None,
+          h_cur=None, h_prior=None, q=None, k=None, n_q_heads=None, n_kv_heads=None,
+          scale=None, lse=None, scores_f32=None, rows: Optional[Dict[str, np.ndarray]] = None,
+          planes: Optional[Dict[str, np.ndarray]] = None) -> Dict[str, np.ndarray]:
+    """score -> per-image sums -> budgets -> selection -> compaction.
+
+    ``scores_f32`` (optional) replaces step 1, to run steps 2-4 on given scores.
+    ``rows``: name -> [T, ...] arrays gathered along axis 0; ``planes``: name ->
+    [P, T] arrays gathered along axis 1. ``relative`` defaults to False for the
+    hidden-variation criterion and True for text attention.
+    """
+    if relative is None:
+        relative = criterion != "hidden_variation"
+    if scores_f32 is None:
+        if criterion == "hidden_variation":
+            s64 = score_hidden_variation(layout, h_cur, h_prior)
+        elif criterion == "text_attention":
+            s64 = score_text_attention(layout, q, k, n_q_heads, n_kv_heads, scale, lse=lse)
+        else:
+            raise ValueError(criterion)
+        scores_f32 = to_fp32(s64)
+    S = image_sums(layout, scores_f32)
+    alloc = allocate(layout, S, keep_ratio, alpha, r_min, r_max, relative)
+    kept = select(layout, scores_f32, alloc["budgets"])
+    out = {"scores": scores_f32, "img_sums": S, "budgets": alloc["budgets"],
+           "out_cu_seqlens": alloc["out_cu_seqlens"], "kept_idx": kept}
+    for name, arr in (rows or {}).items():
+        out[name] = compact(kept, arr)
+    for name, arr in (planes or {}).items():
+        out[name] = compact_planes(kept, arr)
+    return out

@@ -1,0 +1,85 @@
+"""Plant plausible mistakes in a copy of the oracle and check that a pin catches each.
+
+Each mutation edits the oracle's source text (a dropped term, a flipped sign, a
+wrong index, a transposed operand, a wrong mean), loads it as a fresh module and
+runs the pin tests of ``test_oracle_pins`` against it. At least one pin must
+fail. CPU only; the real oracle is untouched.
+"""
+import importlib.util
+import inspect
+import os
+import sys
+import types
+
+import pytest
+
+import tests.test_oracle_pins as pins
+from oracle import avtp_oracle
+
+SRC_PATH = inspect.getsourcefile(avtp_oracle)
+
+MUTATIONS = {
+    "ratio sign flipped": ("r.append(r_base + alpha * (ibar[i] - ibar_avg))",
+                           "r.append(r_base - alpha * (ibar[i] - ibar_avg))"),
+    "image-weighted mean": ("ibar_avg = (float(total) * scale) / float(n_vis)",
+                            "ibar_avg = sum(ibar) / len(ibar)"),
+    "GQA head mapping": ("g = h // (n_q_heads // n_kv_heads)", "g = h % n_kv_heads"),
+    "causal mask off by one": ("visible = keys[None, :] <= text_local[:, None]",
+                               "visible = keys[None, :] < text_local[:, None]"),
+    "logits transposed": ("z = float(scale) * (Qh @ Kg.T)",
+                          "z = float(scale) * (Kg @ Qh.T).T[:, ::-1]"),
+    "norm of wrong row": ("nb = np.sqrt(np.sum(b * b, axis=1))", "nb = np.sqrt(np.sum(a * a, axis=1))"),
+    "cosine not subtracted": ("out[rows] = 1.0 - cos", "out[rows] = cos"),
+    "query count dropped": ("out[a:b][vis] = acc[vis] / (n_q_heads * nq)", "out[a:b][vis] = acc[vis] / n_q_heads"),
+    "remainder tie to higher index": ("order = sorted(elig, key=lambda i: (-frac[i], i))",
+                                      "order = sorted(elig, key=lambda i: (-frac[i], -i))"),
+    "no clamp": ("return min(max(x, lo), hi)", "return x"),
+    "budget rounding floor": ("return int(math.floor(kr * float(n_vis) + 0.5))",
+                              "return int(math.floor(kr * float(n_vis)))"),
+    "ties by higher position": ("return (0, -score, pos)", "return (0, -score, -pos)"),
+    "NaN ranked high": ("return (1, 0.0, pos)", "return (-1, 0.0, pos)"),
+    "text dropped": ("keep = ~_request_visual_local(layout, r)  # text always kept",
+                     "keep = np.zeros(b - a, dtype=bool)"),
+    "fixed point truncates": ("return np.rint(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)",
+                              "return np.trunc(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)"),
+}
+
+PIN_TESTS = [name for name, fn in inspect.getmembers(pins, inspect.isfunction) if name.startswith("test_")]
+
+
+def _mutant(old, new):
+    src = open(SRC_PATH).read()
+    assert src.count(old) == 1, f"mutation anchor not found exactly once: {old!r}"
+    mod = types.ModuleType("avtp_oracle_mutant")
+    exec(compile(src.replace(old, new), "avtp_oracle_mutant", "exec"), mod.__dict__)
+    return mod
+
+
+def _run_pins(module, monkeypatch):
+    monkeypatch.setattr(pins, "O", module)
+    failures = []
+    for name in PIN_TESTS:
+        fn = getattr(pins, name)
+        params = getattr(fn, "pytestmark", [])
+        arg_sets = [()]
+        for mark in params:
+            if mark.name == "parametrize":
+                arg_sets = [v if isinstance(v, tuple) else (v,) for v in mark.args[1]]
+        for args in arg_sets:
+            try:
+                fn(*args)
+            except Exception:  # noqa: BLE001 - any failure counts as caught
+                failures.append(name)
+                break
+    return failures
+
+
+def test_unmutated_oracle_passes_every_pin(monkeypatch):
+    assert _run_pins(avtp_oracle, monkeypatch) == []
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_mutation_is_caught(name, monkeypatch):
+    old, new = MUTATIONS[name]
+    failures = _run_pins(_mutant(old, new), monkeypatch)
+    assert failures, f"no pin caught the planted mistake: {name}"

@@ -1,0 +1,381 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Nothing here compares the oracle with itself: each check uses a hand-derived
+value (tests/golden), a closed form, a library routine reached by a different
+route (scipy cosine distance, scipy softmax over the full square attention
+matrix with np.repeat for the grouped heads), brute-force enumeration, or an
+invariant the method must satisfy. CPU only.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.spatial.distance as ssd
+import scipy.special as ssp
+
+from oracle import avtp_oracle as O
+from paper_2608_26806_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _f(v):
+    return float(v) if not isinstance(v, str) else float(v.replace("inf", "inf"))
+
+
+def _bits(rows):
+    return synth.f32_to_bf16_bits(np.asarray(rows, dtype=np.float32))
+
+
+# ---------------------------------------------------------------- step 1A
+def test_hidden_variation_golden():
+    g = _load("hidden_variation.json")
+    for case in g["cases"]:
+        lay = synth.Layout.from_segments([[("i", 1)]])
+        I = O.score_hidden_variation(lay, _bits([case["h_cur"]]), _bits([case["h_prior"]]))
+        assert I[0] == pytest.approx(case["expected"], abs=1e-15), case["derivation"]
+
+
+def test_hidden_variation_matches_scipy_cosine_distance():
+    rng = np.random.default_rng(0)
+    lay = synth.Layout.from_segments([[("t", 3), ("i", 40), ("t", 2), ("i", 25)]])
+    T, D = lay.n_tokens, 96
+    hc = _bits(rng.standard_normal((T, D)))
+    hp = _bits(rng.standard_normal((T, D)) * 0.3 + synth.bf16_bits_to_f32(hc))
+    I = O.score_hidden_variation(lay, hc, hp)
+    vis = lay.visual_mask()
+    a = synth.bf16_bits_to_f32(hc).astype(np.float64)
+    b = synth.bf16_bits_to_f32(hp).astype(np.float64)
+    for t in range(T):
+        if vis[t]:
+            assert I[t] == pytest.approx(ssd.cosine(a[t], b[t]), rel=1e-12, abs=1e-14)
+        else:
+            assert I[t] == 0.0
+
+
+def test_hidden_variation_identity_and_opposite():
+    rng = np.random.default_rng(1)
+    lay = synth.Layout.from_segments([[("i", 16)]])
+    h = _bits(rng.standard_normal((16, 64)))
+    assert np.allclose(O.score_hidden_variation(lay, h, h), 0.0, atol=1e-15)
+    neg = (h ^ np.uint16(0x8000)).astype(np.uint16)  # bf16 negation flips the sign bit
+    assert np.allclose(O.score_hidden_variation(lay, h, neg), 2.0, atol=1e-15)
+
+
+# ---------------------------------------------------------------- step 1B
+def test_text_attention_golden():
+    g = _load("text_attention.json")
+    lay = synth.Layout.from_segments([[(k, n) for k, n in g["layout"]]])
+    q = _bits(g["q"]).reshape(-1, 1, 1)
+    k = _bits(g["k"]).reshape(-1, 1, 1)
+    s = O.score_text_attention(lay, q, k, 1, 1, g["scale"])
+    assert np.allclose(s, g["expected_scores"], rtol=1e-14, atol=1e-16), g["derivation"]
+
+
+def _brute_force_scores(lay, q, k, Hq, Hkv, scale):
+    """Full square causal attention per request via scipy softmax; GQA by np.repeat."""
+    out = np.zeros(lay.n_tokens)
+    vis_all = lay.visual_mask()
+    for r in range(lay.n_requests):
+        a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+        Q = synth.bf16_bits_to_f32(q[a:b]).astype(np.float64)          # [T, Hq, d]
+        K = synth.bf16_bits_to_f32(k[a:b]).astype(np.float64)          # [T, Hkv, d]
+        K = np.repeat(K, Hq // Hkv, axis=1)                            # head h -> kv h // (Hq/Hkv)
+        logits = np.einsum("qhd,khd->hqk", Q, K) * scale                # [Hq, T, T]
+        mask = np.tril(np.ones((b - a, b - a), dtype=bool))            # key <= query
+        logits = np.where(mask[None], logits, -np.inf)
+        P = ssp.softmax(logits, axis=-1)
+        text = ~vis_all[a:b]
+        nq = text.sum()
+        if nq == 0:
+            continue
+        s = P[:, text, :].sum(axis=(0, 1)) / (Hq * nq)
+        out[a:b][vis_all[a:b]] = s[vis_all[a:b]]
+    return out
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(4, 2), (4, 4), (6, 2)])
+def test_text_attention_matches_full_square_attention(Hq, Hkv):
+    wl = synth.make_custom([[("t", 5), ("i", 12), ("t", 3), ("i", 7), ("t", 4)], [("i", 9), ("t", 6)]],
+                           hidden=32, n_q_heads=Hq, n_kv_heads=Hkv, head_dim=16, seed=3, parts=("B",))
+    scale = wl.softmax_scale
+    s = O.score_text_attention(wl.layout, wl.q, wl.k, Hq, Hkv, scale)
+    ref = _brute_force_scores(wl.layout, wl.q, wl.k, Hq, Hkv, scale)
+    assert np.allclose(s, ref, rtol=1e-12, atol=1e-15)
+
+
+def test_tiny_config_matches_full_square_attention():
+    wl = synth.make_workload("tiny", parts=("B",))
+    s = O.score_text_attention(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale)
+    ref = _brute_force_scores(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale)
+    assert np.allclose(s, ref, rtol=1e-12, atol=1e-16)
+
+
+def test_softmax_rows_sum_to_one():
+    wl = synth.make_custom([[("t", 4), ("i", 20), ("t", 6)]], n_q_heads=4, n_kv_heads=2,
+                           head_dim=16, seed=5, parts=("B",))
+    for h in range(4):
+        z, text_local = O.attention_logits(wl.layout, wl.q, wl.k, 0, h, 4, 2, wl.softmax_scale)
+        lse = O.logsumexp_rows(z)
+        P = np.exp(z - lse[:, None])
+        assert np.allclose(P.sum(axis=1), 1.0, atol=1e-13)
+        # nothing leaks past the causal frontier
+        keys = np.arange(z.shape[1])
+        assert np.all(P[keys[None, :] > text_local[:, None]] == 0.0)
+
+
+def test_zero_queries_give_uniform_attention():
+    lay = synth.Layout.from_segments([[("t", 3), ("i", 5), ("t", 2), ("i", 4), ("t", 2)]])
+    T, Hq, Hkv, d = lay.n_tokens, 2, 1, 8
+    rng = np.random.default_rng(2)
+    q = np.zeros((T, Hq, d), dtype=np.uint16)              # bf16 +0
+    k = _bits(rng.standard_normal((T * Hkv * d))).reshape(T, Hkv, d)
+    s = O.score_text_attention(lay, q, k, Hq, Hkv, 0.25)
+    vis = lay.visual_mask()
+    text_pos = np.nonzero(~vis)[0]
+    for t in np.nonzero(vis)[0]:
+        # every text query q >= t spreads 1/(q+1) on each visible key
+        expect = sum(1.0 / (p + 1) for p in text_pos if p >= t) / len(text_pos)
+        assert s[t] == pytest.approx(expect, rel=1e-14)
+
+
+def test_single_visible_key_lse():
+    lay = synth.Layout.from_segments([[("t", 1), ("i", 3), ("t", 1)]])
+    rng = np.random.default_rng(4)
+    q = _bits(rng.standard_normal((5 * 2 * 8))).reshape(5, 2, 8)
+    k = _bits(rng.standard_normal((5 * 1 * 8))).reshape(5, 1, 8)
+    lse = O.text_lse(lay, q, k, 2, 1, 0.5)
+    for h in range(2):
+        z00 = 0.5 * float(np.dot(synth.bf16_bits_to_f32(q[0, h]).astype(np.float64),
+                                 synth.bf16_bits_to_f32(k[0, 0]).astype(np.float64)))
+        assert lse[h, 0] == pytest.approx(z00, abs=1e-14)  # log(exp(z)) = z: P = 1
+
+
+def test_supplied_lse_reproduces_scores():
+    wl = synth.make_custom([[("t", 6), ("i", 10), ("t", 2), ("i", 10), ("t", 5)]], seed=9, parts=("B",))
+    lse = O.text_lse(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale)
+    a = O.score_text_attention(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale)
+    b = O.score_text_attention(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale, lse=lse)
+    assert np.allclose(a, b, rtol=1e-13, atol=1e-16)
+    # a shifted normaliser scales every probability by exp(-shift)
+    c = O.score_text_attention(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale, lse=lse + math.log(2.0))
+    assert np.allclose(c, a / 2.0, rtol=1e-13, atol=1e-16)
+
+
+def test_request_without_text_scores_zero():
+    wl = synth.make_custom([[("i", 8), ("i", 8)]], seed=1, parts=("B",))
+    s = O.score_text_attention(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale)
+    assert np.all(s == 0.0)
+
+
+# ---------------------------------------------------------------- fixed point
+def test_fixed_point_values():
+    v = np.array([0.5, -0.25, np.nan, 2048.0, -np.inf, 2.0 ** -33, 3 * 2.0 ** -33, 0.0], dtype=np.float32)
+    fx = O.fixed_point(v)
+    assert fx.tolist() == [2 ** 31, -(2 ** 30), 0, 2 ** 42, -(2 ** 42), 0, 2, 0]
+
+
+# ---------------------------------------------------------------- step 2
+def _alloc_case(case):
+    lay = synth.Layout.from_segments([[(k, n) for k, n in case["layout"]]])
+    scores = np.zeros(lay.n_tokens, dtype=np.float32)
+    for i, v in enumerate(case["image_scores"]):
+        s = int(lay.img_start[i])
+        scores[s:s + int(lay.img_len[i])] = v
+    S = O.image_sums(lay, scores)
+    kr = np.array([case["keep_ratio"]], dtype=np.float32)
+    return lay, O.allocate(lay, S, kr, case["alpha"], 0.05, 0.95, case["relative"])
+
+
+def test_allocation_golden():
+    for case in _load("allocation.json")["cases"]:
+        lay, res = _alloc_case(case)
+        assert res["budgets"].tolist() == case["expected_budgets"], case["name"] + ": " + case["derivation"]
+        assert int(res["out_cu_seqlens"][-1]) == case["expected_out_len"], case["name"]
+
+
+def test_allocation_no_clamp_lambda_is_zero():
+    # token-weighted mean => sum_i n_i r_i = r_base N_vis: no shift needed when no clamp binds
+    case = _load("allocation.json")["cases"][0]
+    lay, res = _alloc_case(case)
+    assert abs(res["lam"][0]) < 1e-15
+    assert np.allclose(res["ratios"], [0.71875, 0.34375, 0.46875], rtol=0, atol=1e-15)
+
+
+def test_global_budget_rounding():
+    assert O.global_budget(np.float32(0.5), 3) == 2          # 1.5 + 0.5
+    assert O.global_budget(np.float32(0.25), 5832) == 1458
+    assert O.global_budget(np.float32(0.33), 9600) == 3168  # fp32 0.33 = 0.3300000131...
+    assert O.global_budget(np.float32(1.0), 7) == 7
+    assert O.global_budget(np.float32(0.125), 0) == 0
+
+
+def _random_alloc(rng, m, relative=False, alpha=1.0, kr=None):
+    n = rng.integers(1, 300, size=m)
+    segs = []
+    for v in n:
+        segs += [("t", int(rng.integers(0, 3))), ("i", int(v))]
+    lay = synth.Layout.from_segments([segs])
+    S = rng.integers(0, 2 ** 33, size=m).astype(np.int64) * n  # mean in [0, 2)
+    kr = np.array([rng.choice([0.05, 0.125, 0.25, 0.33, 0.5, 0.9]) if kr is None else kr], dtype=np.float32)
+    return lay, S, kr, O.allocate(lay, S, kr, alpha, 0.05, 0.95, relative)
+
+
+@pytest.mark.parametrize("relative", [False, True])
+def test_allocation_conserves_total_and_bounds(relative):
+    rng = np.random.default_rng(11)
+    for trial in range(60):
+        m = int(rng.integers(1, 20))
+        alpha = float(rng.choice([0.0, 1.0, 2.0, 5.0]))
+        lay, S, kr, res = _random_alloc(rng, m, relative, alpha)
+        n = lay.img_len.astype(np.int64)
+        B = O.global_budget(kr[0], int(n.sum()))
+        k = res["budgets"].astype(np.int64)
+        assert k.sum() == B
+        assert np.all(k >= 0) and np.all(k <= n)
+        r_min, r_max = float(np.float32(0.05)), float(np.float32(0.95))
+        assert np.all(k >= np.floor(r_min * n) - 1)
+        assert np.all(k <= np.floor(r_max * n) + 1)
+        T_txt = lay.n_tokens - int(n.sum())
+        assert int(res["out_cu_seqlens"][-1]) == B + T_txt
+
+
+def test_allocation_alpha_zero_is_uniform():
+    rng = np.random.default_rng(12)
+    for trial in range(30):
+        lay, S, kr, res = _random_alloc(rng, int(rng.integers(1, 12)), alpha=0.0)
+        n = lay.img_len.astype(np.float64)
+        target = float(kr[0]) * n * (O.global_budget(kr[0], int(n.sum())) / (float(kr[0]) * n.sum()))
+        assert np.all(np.abs(res["budgets"] - target) <= 1.0 + 1e-9)
+
+
+def test_identical_images_equal_budgets():
+    for m, kr in [(4, 0.5), (3, 0.33), (8, 0.125)]:
+        lay = synth.Layout.from_segments([[("t", 2)] + [("i", 96)] * m + [("t", 5)]])
+        S = np.full(m, 96 * 2 ** 30, dtype=np.int64)
+        res = O.allocate(lay, S, np.array([kr], dtype=np.float32), 1.0, 0.05, 0.95, False)
+        k = res["budgets"]
+        assert k.max() - k.min() <= 1
+        assert np.all(np.diff(k) <= 0)  # the extra tokens go to the lower image indices
+        B = O.global_budget(np.float32(kr), 96 * m)
+        if (B * 96) % (96 * m) == 0:
+            assert k.max() == k.min()
+
+
+def test_budgets_are_permutation_equivariant():
+    rng = np.random.default_rng(13)
+    for trial in range(25):
+        m = int(rng.integers(2, 10))
+        n = rng.integers(16, 200, size=m)
+        S = (rng.integers(1, 2 ** 32, size=m).astype(np.int64) * n)
+        perm = rng.permutation(m)
+        lay1 = synth.Layout.from_segments([[("i", int(v)) for v in n] + [("t", 3)]])
+        lay2 = synth.Layout.from_segments([[("i", int(v)) for v in n[perm]] + [("t", 3)]])
+        kr = np.array([0.3], dtype=np.float32)
+        k1 = O.allocate(lay1, S, kr, 1.0)["budgets"]
+        k2 = O.allocate(lay2, S[perm], kr, 1.0)["budgets"]
+        assert k2.tolist() == k1[perm].tolist()
+
+
+def test_more_importance_never_fewer_tokens():
+    rng = np.random.default_rng(14)
+    for trial in range(25):
+        m = int(rng.integers(2, 10))
+        n = rng.integers(16, 200, size=m)
+        S = (rng.integers(1, 2 ** 31, size=m).astype(np.int64) * n)
+        lay = synth.Layout.from_segments([[("i", int(v)) for v in n]])
+        kr = np.array([0.4], dtype=np.float32)
+        k1 = O.allocate(lay, S, kr, 2.0)["budgets"]
+        j = int(rng.integers(0, m))
+        S2 = S.copy()
+        S2[j] += int(n[j]) * 2 ** 29
+        k2 = O.allocate(lay, S2, kr, 2.0)["budgets"]
+        assert k2[j] >= k1[j]
+
+
+def test_relative_rule_is_proportional_to_image_mass():
+    # alpha = 1, relative: r_i = r_base * Ibar_i / Ibar_avg, so x_i = B * S_i / sum S
+    n = np.array([100, 300, 200])
+    S = np.array([100 * 2 ** 30, 300 * 2 ** 31, 200 * 3 * 2 ** 29], dtype=np.int64)
+    lay = synth.Layout.from_segments([[("i", 100), ("i", 300), ("i", 200)]])
+    res = O.allocate(lay, S, np.array([0.5], dtype=np.float32), 1.0, 0.0, 1.0, True)
+    B = 300
+    x = B * S / S.sum()
+    assert np.all(np.abs(res["budgets"] - x) < 1.0)
+
+
+# ---------------------------------------------------------------- step 3
+def test_selection_golden():
+    for case in _load("selection.json")["cases"]:
+        lay = synth.Layout.from_segments([[(k, n) for k, n in case["layout"]]])
+        sc = np.array([_f(v) for v in case["scores"]], dtype=np.float32)
+        kept = O.select(lay, sc, np.array(case["budgets"], dtype=np.int32))
+        assert kept.tolist() == case["expected_kept"], case["derivation"]
+
+
+def _dominates(sa, pa, sb, pb):
+    """True iff token a ranks strictly above token b: larger score, or equal score and lower position."""
+    na, nb = math.isnan(sa), math.isnan(sb)
+    if na and nb:
+        return pa < pb
+    if na:
+        return False
+    if nb:
+        return True
+    return sa > sb or (sa == sb and pa < pb)
+
+
+def test_selection_brute_force_small():
+    rng = np.random.default_rng(21)
+    pool = np.array([0.0, -0.0, 0.5, 0.5, 1.0, -1.0, np.nan, np.inf, -np.inf, 0.25], dtype=np.float32)
+    for trial in range(120):
+        n = int(rng.integers(1, 11))
+        sc_img = rng.choice(pool, size=n) if trial % 2 else rng.standard_normal(n).astype(np.float32)
+        lay = synth.Layout.from_segments([[("t", 1), ("i", n), ("t", 1)]])
+        sc = np.zeros(n + 2, dtype=np.float32)
+        sc[1:n + 1] = sc_img
+        for kk in range(n + 1):
+            kept = O.select(lay, sc, np.array([kk], dtype=np.int32))
+            # brute force: the unique k-subset whose every member ranks above every non-member
+            winners = []
+            for sub in itertools.combinations(range(1, n + 1), kk):
+                rest = [t for t in range(1, n + 1) if t not in sub]
+                if all(_dominates(float(sc[a]), a, float(sc[b]), b) for a in sub for b in rest):
+                    winners.append(sub)
+            assert len(winners) == 1
+            assert kept.tolist() == sorted([0, n + 1] + list(winners[0]))
+
+
+def test_selection_structure_on_tiny():
+    wl = synth.make_workload("tiny", parts=("A",))
+    res = O.prune(wl.layout, keep_ratio=wl.keep_ratio, h_cur=wl.h_cur, h_prior=wl.h_prior)
+    kept = res["kept_idx"]
+    assert np.all(np.diff(kept) > 0)
+    vis = wl.layout.visual_mask()
+    assert set(np.nonzero(~vis)[0].tolist()) <= set(kept.tolist())   # text never dropped
+    assert len(kept) == int(res["out_cu_seqlens"][-1])
+    assert int(res["budgets"].sum()) == O.global_budget(wl.keep_ratio[0], int(vis.sum()))
+    # image importance grows with the synthetic signal (0, 0.5, 1): so do the budgets
+    assert res["budgets"][0] < res["budgets"][1] < res["budgets"][2]
+
+
+# ---------------------------------------------------------------- step 4
+def test_compact_is_row_gather():
+    rng = np.random.default_rng(31)
+    rows = rng.integers(0, 2 ** 16, size=(50, 7), dtype=np.uint16)
+    planes = rng.integers(0, 2 ** 31, size=(3, 50), dtype=np.int64).astype(np.int32)
+    idx = np.array(sorted(rng.choice(50, size=17, replace=False)), dtype=np.int32)
+    out = O.compact(idx, rows)
+    outp = O.compact_planes(idx, planes)
+    for j, t in enumerate(idx):
+        assert out[j].tobytes() == rows[t].tobytes()
+        for p in range(3):
+            assert outp[p, j] == planes[p, t]
