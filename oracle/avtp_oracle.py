@@ -36,18 +36,24 @@ the design notes of the repository):
 * ``relative=1`` replaces the additive rule by ``r_i = r_base*(1 + alpha*(Ibar_i/Ibar_avg - 1))``
   (``r_base`` when ``Ibar_avg == 0``); criterion 1B's raw values are of order
   1/N, where the additive rule would leave every ratio at ``r_base``.
-* A shift lambda (water-fill) restores ``sum_i n_i * clamp(r_i + lambda)`` to ``B_r``
-  after clamping: 64 fp64 bisection steps on ``[r_min - max r, r_max - min r]``,
-  midpoint ``lo + (hi - lo) * 0.5``, move ``hi`` iff ``F(mid) >= B_r``, take ``hi``.
-* Integer budgets: ``x_i = n_i * clamp(r_i + lambda)``, ``k_i = min(floor(x_i), n_i)``,
-  then largest remainder (ties to the lower image index) until ``sum k_i = B_r``;
-  a surplus is removed from the smallest remainders (ties to the higher index).
+* Ratios go on a 2^-40 integer grid: ``R_i = rint(clamp(r_i, -2^20, 2^20) * 2^40)``,
+  and likewise ``R_min``, ``R_max`` from the fp32 clamps.
+* A shift lambda (water-fill) restores the clamped total: lambda is the smallest
+  grid value with ``G(lambda) = sum_i n_i * clamp(R_i + lambda, R_min, R_max) >= B_r * 2^40``
+  on ``[R_min - max R, R_max - min R]`` (an end of that range if none inside
+  qualifies). G is exact integer arithmetic, so lambda is a definition, not the
+  output of one particular search.
+* Integer budgets: ``x_i = n_i * clamp(R_i + lambda)`` (2^-40 token units),
+  ``k_i = min(floor(x_i), n_i)``, then largest remainder (ties to the lower image
+  index) until ``sum k_i = B_r``; a surplus is removed from the smallest
+  remainders (ties to the higher index).
 * Top-k order: score descending, position ascending; NaN ranks below -inf;
   -0 equals +0.
 
-All floating-point steps of the budget rule are single fp64 operations in a
-fixed order (Python floats: no fused multiply-add), so a correct device
-implementation that rounds each operation to nearest reproduces them exactly.
+The only floating-point steps of the budget rule are the few fp64 operations of
+the ratio formula, each rounded once (Python floats: no fused multiply-add);
+everything after them is exact integer arithmetic. A device implementation that
+rounds each of those operations to nearest reproduces every budget exactly.
 """
 from __future__ import annotations
 
@@ -59,7 +65,8 @@ import numpy as np
 FX_FRAC_BITS = 32
 FX_SCORE_LIMIT = 1024.0  # |score| is clamped to 2^10 before the fixed-point conversion
 NORM_EPS = 1e-8
-BISECTION_STEPS = 64
+RATIO_FRAC_BITS = 40     # ratios, shifts and kept masses live on a 2^-40 integer grid
+RATIO_LIMIT = 2.0 ** 20  # ratios are saturated to +-2^20 before going on the grid
 
 
 # ----------------------------------------------------------------------------
@@ -218,7 +225,7 @@ def global_budget(keep_ratio_f32: float, n_vis: int) -> int:
     return int(math.floor(kr * float(n_vis) + 0.5))
 
 
-def _clamp(x: float, lo: float, hi: float) -> float:
+def _clamp(x, lo, hi):
     return min(max(x, lo), hi)
 
 
@@ -242,36 +249,47 @@ def adaptive_ratios(S: Sequence[int], n: Sequence[int], r_base: float, alpha: fl
     return r
 
 
-def water_fill(r: Sequence[float], n: Sequence[int], B: int, r_min: float, r_max: float) -> float:
-    """Shift lambda with ``sum_i n_i * clamp(r_i + lambda, r_min, r_max) ~= B`` (64 bisection steps)."""
+def ratio_to_grid(r: float) -> int:
+    """A ratio on the 2^-40 grid: ``rint(clamp(r, -2^20, 2^20) * 2^40)`` (exact integer)."""
+    r = _clamp(r, -RATIO_LIMIT, RATIO_LIMIT)
+    return int(np.rint(r * float(2 ** RATIO_FRAC_BITS)))
 
-    def F(lam: float) -> float:
-        acc = 0.0
-        for i in range(len(n)):  # image order, sequential
-            acc = acc + float(int(n[i])) * _clamp(r[i] + lam, r_min, r_max)
-        return acc
 
-    lo = r_min - max(r)
-    hi = r_max - min(r)
-    target = float(B)
-    for _ in range(BISECTION_STEPS):
-        mid = lo + (hi - lo) * 0.5
-        if F(mid) >= target:
+def kept_mass(R: Sequence[int], n: Sequence[int], lam: int, R_min: int, R_max: int) -> int:
+    """``G(lambda) = sum_i n_i * clamp(R_i + lambda, R_min, R_max)`` in 2^-40 token units (exact)."""
+    return sum(int(n[i]) * _clamp(int(R[i]) + lam, R_min, R_max) for i in range(len(n)))
+
+
+def water_fill(R: Sequence[int], n: Sequence[int], B: int, R_min: int, R_max: int) -> int:
+    """The smallest grid shift lambda with ``G(lambda) >= B * 2^40``, searched in
+    ``[R_min - max R, R_max - min R]`` (the ends when no point inside qualifies).
+
+    G is non-decreasing in lambda, so integer bisection finds it exactly.
+    """
+    target = int(B) << RATIO_FRAC_BITS
+    lo = R_min - max(R)
+    hi = R_max - min(R)
+    if kept_mass(R, n, lo, R_min, R_max) >= target:
+        return lo
+    if kept_mass(R, n, hi, R_min, R_max) < target:
+        return hi
+    while hi - lo > 1:  # invariant: G(lo) < target <= G(hi)
+        mid = (lo + hi) // 2
+        if kept_mass(R, n, mid, R_min, R_max) >= target:
             hi = mid
         else:
             lo = mid
     return hi
 
 
-def integer_budgets(r: Sequence[float], n: Sequence[int], B: int, lam: float,
-                    r_min: float, r_max: float) -> List[int]:
-    """Largest-remainder rounding of ``x_i = n_i * clamp(r_i + lambda)`` to a total of B."""
+def integer_budgets(R: Sequence[int], n: Sequence[int], B: int, lam: int,
+                    R_min: int, R_max: int) -> List[int]:
+    """Largest-remainder rounding of ``x_i = n_i * clamp(R_i + lambda)`` to a total of B."""
     m = len(n)
-    x = [float(int(n[i])) * _clamp(r[i] + lam, r_min, r_max) for i in range(m)]
-    fl = [math.floor(v) for v in x]
-    frac = [x[i] - float(fl[i]) for i in range(m)]
-    k = [min(int(fl[i]), int(n[i])) for i in range(m)]
-    k = [max(v, 0) for v in k]
+    one = 1 << RATIO_FRAC_BITS
+    x = [int(n[i]) * _clamp(int(R[i]) + lam, R_min, R_max) for i in range(m)]
+    frac = [v % one for v in x]
+    k = [min(v // one, int(n[i])) for i, v in enumerate(x)]
     while sum(k) < B:
         need = B - sum(k)
         elig = [i for i in range(m) if k[i] < int(n[i])]
@@ -315,11 +333,13 @@ def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
         if i1 > i0:
             Sr = [int(v) for v in S[i0:i1]]
             r = adaptive_ratios(Sr, n, r_base, alpha, relative)
-            lam = water_fill(r, n, B, r_min, r_max)
-            k = integer_budgets(r, n, B, lam, r_min, r_max)
+            R = [ratio_to_grid(v) for v in r]
+            R_min, R_max = ratio_to_grid(r_min), ratio_to_grid(r_max)
+            lam = water_fill(R, n, B, R_min, R_max)
+            k = integer_budgets(R, n, B, lam, R_min, R_max)
             budgets[i0:i1] = k
             ratios[i0:i1] = r
-            lams[rq] = lam
+            lams[rq] = lam / float(2 ** RATIO_FRAC_BITS)
         out_cu[rq + 1] = out_cu[rq] + B + n_txt
     return {"budgets": budgets, "out_cu_seqlens": out_cu, "ratios": ratios, "lam": lams}
 

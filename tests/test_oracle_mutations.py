@@ -34,6 +34,8 @@ MUTATIONS = {
     "remainder tie to higher index": ("order = sorted(elig, key=lambda i: (-frac[i], i))",
                                       "order = sorted(elig, key=lambda i: (-frac[i], -i))"),
     "no clamp": ("return min(max(x, lo), hi)", "return x"),
+    "water-fill takes the last short shift": ("    return hi\n\n\ndef integer_budgets", "    return lo\n\n\ndef integer_budgets"),
+    "remainder from the wrong end": ("frac = [v % one for v in x]", "frac = [one - 1 - v % one for v in x]"),
     "budget rounding floor": ("return int(math.floor(kr * float(n_vis) + 0.5))",
                               "return int(math.floor(kr * float(n_vis)))"),
     "ties by higher position": ("return (0, -score, pos)", "return (0, -score, -pos)"),
