@@ -1,0 +1,491 @@
+"""Benchmark of the AVTP pruning stage on GB300.
+
+One step = one avtp_prune call (validate -> score -> allocate -> select ->
+compact) over the Qwen3-VL-8B-shaped multi-image request: 16 images of
+256..1024 visual tokens, 256 text tokens, hidden 4096, M-RoPE position ids
+(3 planes), keep ratio 0.33, criterion = hidden-state variation (paper §3.3.1).
+Inputs are synthetic and resident in HBM before the timed region; L2 is flushed
+(256 MiB write) before every timed step, outside the step's own events.
+
+Prints one JSON line. ``--impl reference`` times the fp64 CPU oracle on the
+host instead (the reference arm of this build: the paper ships no code).
+
+Multi-GPU (torchrun): every rank runs an independent replica of the workload
+(the stage shards by request with no exchange); ``value`` sums all ranks'
+visual tokens over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "pruning-stage latency (µs) and visual tokens/s on 1 GB300; % of HBM roofline"
+UNIT = "visual tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+STEP_NAMES = ("validate", "score", "allocate", "select", "compact")
+SCORE_KERNELS = {"hidden_variation": ["k_score_hvar"], "text_attention": ["k_attn_lse", "k_attn_mass",
+                                                                         "k_attn_finalize"]}
+
+
+# ---------------------------------------------------------------- helpers
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def reduce_max(value: float, world: int, device=None) -> float:
+    """Max over ranks (timing only; not on the data path)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+
+
+class ClockSampler:
+    """Samples SM clock and throttle reasons with nvidia-smi while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, period_ms: int = 50):
+        self.gpu_index = gpu_index
+        self.period_ms = period_ms
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-i",
+                 str(self.gpu_index), "-lms", str(self.period_ms)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(self.period_ms / 1000.0 * 2)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread is not None:
+            self.thread.join(timeout=5)
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for _, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, flag in zip(names, parts[4:8]):
+                if flag.lower() in ("active", "1", "0x1"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def kernel_source_sha(names):
+    csrc = os.path.join(ROOT, "paper_2608_26806_gb300", "csrc")
+    h = hashlib.sha256()
+    for fn in sorted(os.listdir(csrc)):
+        if fn.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, fn), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on the current sources."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    e = d.get(f"{kernel}@{workload}")
+    if not e or e.get("source_sha") != kernel_source_sha(None):
+        return None
+    return float(e["dram_bytes_per_launch"])
+
+
+# ---------------------------------------------------------------- workload accounting
+def stage_accounting(wl, criterion, n_kept):
+    lay = wl.layout
+    n_vis = int(lay.n_visual_per_request().sum())
+    n_txt = lay.n_tokens - n_vis
+    D = wl.hidden
+    pos_bytes = wl.pos_planes * 4
+    gather = n_kept * D * 2 * 2 + n_kept * pos_bytes * 2  # read + write of every kept row
+    if criterion == "hidden_variation":
+        score_bytes = 2 * n_vis * D * 2
+        # compulsory: both visual rows once, text rows once (kept), kept rows written, positions
+        stage_bytes = score_bytes + n_txt * D * 2 + n_kept * D * 2 + n_kept * pos_bytes * 2
+        flops = 0
+    else:
+        Hq, Hkv, d = wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+        score_bytes = lay.n_tokens * Hkv * d * 2 + n_txt * Hq * d * 2
+        stage_bytes = score_bytes + n_txt * D * 2 + n_kept * D * 2 + n_kept * pos_bytes * 2
+        flops = 0
+        vis = lay.visual_mask()
+        for r in range(lay.n_requests):
+            a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+            v = vis[a:b]
+            text_pos = np.nonzero(~v)[0]
+            vis_prefix = np.concatenate([[0], np.cumsum(v)])
+            for p in text_pos:
+                flops += 2 * Hq * d * (p + 1)              # pass 1: every visible key
+                flops += 2 * Hq * d * int(vis_prefix[p + 1])  # pass 2: visible visual keys
+    return {"n_vis": n_vis, "n_txt": n_txt, "score_bytes": score_bytes, "stage_bytes": stage_bytes,
+            "gather_bytes": gather, "flops": flops}
+
+
+# ---------------------------------------------------------------- our arm
+def run_ours(args, world, rank, local):
+    import torch
+
+    from paper_2608_26806_gb300 import avtp, synth
+
+    import __graft_entry__
+
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    __graft_entry__.build()
+    crit = args.criterion
+    parts = ("A", "pos") if crit == "hidden_variation" else ("A", "B", "pos")
+    wl = synth.make_workload(args.config, parts=parts)
+    lay = wl.layout
+
+    def bf16(x):
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    L = avtp.Layout.from_host(lay.cu_seqlens, lay.img_cu, lay.img_start, lay.img_len, device=dev)
+    h_cur, h_prior = bf16(wl.h_cur), bf16(wl.h_prior)
+    pos = torch.from_numpy(wl.pos).to(dev)
+    kr = torch.from_numpy(wl.keep_ratio).to(dev)
+    score_tensors = dict(h_cur=h_cur, h_prior=h_prior)
+    if crit == "text_attention":
+        score_tensors = dict(q=bf16(wl.q), k=bf16(wl.k), softmax_scale=wl.softmax_scale)
+    call = avtp.PruneCall(L, crit, keep_ratio=kr, keep_ratio_host=wl.keep_ratio, rows={"hidden": h_cur},
+                          planes={"pos": pos}, **score_tensors)
+    n_kept = call.buffers.n_kept
+    acct = stage_accounting(wl, crit, n_kept)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    K, W = args.steps, args.warmup
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(K)]
+    for evs in events:  # create the driver events before they are handed to the library
+        for e in evs:
+            e.record(stream)
+    for _ in range(W):
+        flush.zero_()
+        call.run(stream)
+    torch.cuda.synchronize()
+    st = avtp.read_device_status(call.buffers.workspace)
+    if st != avtp.OK:
+        raise RuntimeError(f"device status after warm-up: {avtp.status_string(st)}")
+
+    sampler = ClockSampler(torch.cuda.current_device()) if not args.no_clocks else None
+    barrier(world)
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
+    for i in range(K):
+        flush.zero_()
+        call.run(stream, step_events=events[i])
+    torch.cuda.synchronize()
+    clocks = sampler.stop() if sampler else None
+    barrier(world)
+    step_ms = [events[i][0].elapsed_time(events[i][5]) for i in range(K)]
+    per_step = {name: [events[i][j].elapsed_time(events[i][j + 1]) for i in range(K)]
+                for j, name in enumerate(STEP_NAMES)}
+    total_ms = sum(step_ms)
+    total_ms_max = reduce_max(total_ms, world, dev)
+
+    # end to end through the public API: pinned host inputs -> device -> prune -> host outputs
+    e2e = run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp)
+
+    if rank != 0:
+        return None
+    hbm, bf16_tf, peak_kind = measured_peaks()
+    score_ms = statistics.mean(per_step["score"])
+    dominant = SCORE_KERNELS[crit][0] if crit == "hidden_variation" else "k_attn_mass"
+    if crit == "hidden_variation":
+        achieved = acct["score_bytes"] / (score_ms * 1e-3) / 1e9
+        roof = {"bound": "hbm", "kernel": dominant, "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(achieved / hbm, 4), "peak_kind": peak_kind,
+                "algorithmic_bytes_per_launch": acct["score_bytes"],
+                "avg_launch_us": round(score_ms * 1e3, 2),
+                "traffic": recorded_traffic(dominant, args.config)}
+    else:
+        achieved = acct["flops"] / (score_ms * 1e-3) / 1e12
+        roof = {"bound": "tensor", "kernel": "score (lse + mass + finalize)", "achieved": round(achieved, 2),
+                "peak": bf16_tf, "unit": "TFLOP/s", "frac": round(achieved / bf16_tf, 4), "peak_kind": peak_kind,
+                "algorithmic_flops_per_launch": acct["flops"], "avg_launch_us": round(score_ms * 1e3, 2),
+                "traffic": None}
+    ms_step = total_ms_max / K
+    stage_gbs = acct["stage_bytes"] / (ms_step * 1e-3) / 1e9
+    value = acct["n_vis"] * K * world / (total_ms_max * 1e-3)
+    srt = sorted(step_ms)
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": round(ms_step, 5), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.config, "criterion": crit, "global_batch": lay.n_requests,
+                   "seq_len": lay.n_tokens, "visual_tokens": acct["n_vis"], "kept_tokens": n_kept,
+                   "hidden": wl.hidden, "images": lay.n_images, "keep_ratio": float(wl.keep_ratio[0]),
+                   "parallelism": f"replicas{world}", "l2": "flushed: 256 MiB write before every timed step"},
+        "latency_us": {"p50": round(srt[len(srt) // 2] * 1e3, 2), "p90": round(srt[int(len(srt) * 0.9)] * 1e3, 2),
+                       "mean": round(statistics.mean(step_ms) * 1e3, 2)},
+        "steps_us": {k: round(statistics.mean(v) * 1e3, 2) for k, v in per_step.items()},
+        "stage_roofline": {"bound": "hbm", "algorithmic_bytes": acct["stage_bytes"],
+                           "achieved": round(stage_gbs, 1), "peak": hbm, "unit": "GB/s",
+                           "frac": round(stage_gbs / hbm, 4), "peak_kind": peak_kind},
+        "roofline": roof,
+        "e2e": e2e,
+        "gpu_launches": K * (5 if crit == "hidden_variation" else (7 if crit == "text_attention" else 5)),
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, crit, args.cpu_seconds)
+    return line
+
+
+def run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp):
+    """Same metric through the public API with host buffers: H2D inputs, prune, D2H outputs, all timed."""
+    b = call.buffers
+    host_in = {"h_cur": torch.from_numpy(np.ascontiguousarray(wl.h_cur).view(np.int16)).pin_memory(),
+               "pos": torch.from_numpy(wl.pos).pin_memory()}
+    if crit == "hidden_variation":
+        host_in["h_prior"] = torch.from_numpy(np.ascontiguousarray(wl.h_prior).view(np.int16)).pin_memory()
+    else:
+        host_in["q"] = torch.from_numpy(np.ascontiguousarray(wl.q).view(np.int16)).pin_memory()
+        host_in["k"] = torch.from_numpy(np.ascontiguousarray(wl.k).view(np.int16)).pin_memory()
+    for name in ("cu_seqlens", "img_cu", "img_start", "img_len"):
+        host_in["lay_" + name] = torch.from_numpy(L.host[name].copy()).pin_memory()
+    host_in["keep_ratio"] = torch.from_numpy(wl.keep_ratio.copy()).pin_memory()
+    # device destinations: the very tensors the prepared call reads
+    dev_dst = {"h_cur": call._keep_alive[1]["hidden"], "pos": call._keep_alive[2]["pos"],
+               "lay_cu_seqlens": L.cu_seqlens, "lay_img_cu": L.img_cu, "lay_img_start": L.img_start,
+               "lay_img_len": L.img_len, "keep_ratio": call._keep_alive[0]}
+    st = call._keep_alive[3]
+    if crit == "hidden_variation":
+        dev_dst["h_prior"] = st["h_prior"]
+    else:
+        dev_dst["q"], dev_dst["k"] = st["q"], st["k"]
+    outs = [b.kept_idx[:b.n_kept], b.budgets, b.out_cu_seqlens] + list(b.outputs.values())
+    host_out = [torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs]
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+    d2h = sum(o.numel() * o.element_size() for o in outs)
+    steps = max(3, min(50, args.e2e_steps))
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def one():
+        for k, h in host_in.items():
+            dst = dev_dst[k]
+            dst.view(torch.int16 if dst.dtype == torch.bfloat16 else dst.dtype).copy_(
+                h.view(torch.int16) if dst.dtype == torch.bfloat16 else h, non_blocking=True)
+        call.run(stream)
+        for o, h in zip(outs, host_out):
+            h.copy_(o, non_blocking=True)
+
+    for _ in range(3):
+        one()
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for _ in range(steps):
+        one()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / steps
+    n_vis = int(wl.layout.n_visual_per_request().sum())
+    return {"value": round(n_vis / (ms * 1e-3), 1), "unit": UNIT, "ms_per_step": round(ms, 4),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
+
+
+# ---------------------------------------------------------------- CPU oracle (baseline / reference arm)
+def _sub_workload(wl, n_images):
+    """The first n_images images of request 0 with their surrounding text: a bounded sample."""
+    from paper_2608_26806_gb300 import synth
+
+    lay = wl.layout
+    i_end = min(n_images, int(lay.img_cu[1]))
+    if i_end < int(lay.img_cu[1]):
+        end_tok = int(lay.img_start[i_end])  # stop before the next image
+    else:
+        end_tok = int(lay.cu_seqlens[1])
+    sub = synth.Layout(cu_seqlens=np.array([0, end_tok], dtype=np.int32), img_cu=np.array([0, i_end], dtype=np.int32),
+                       img_start=lay.img_start[:i_end].copy(), img_len=lay.img_len[:i_end].copy())
+    t = {k: v[:end_tok] for k, v in wl.tensors.items() if k in ("h_cur", "h_prior", "q", "k")}
+    if "pos" in wl.tensors:
+        t["pos"] = wl.tensors["pos"][:, :end_tok]
+    return sub, t
+
+
+def _oracle_step(O, sub, t, wl, crit):
+    kw = dict(keep_ratio=wl.keep_ratio[:1], rows={"hidden": t["h_cur"]}, planes={"pos": t["pos"]})
+    if crit == "hidden_variation":
+        return O.prune(sub, h_cur=t["h_cur"], h_prior=t["h_prior"], **kw)
+    return O.prune(sub, criterion="text_attention", q=t["q"], k=t["k"], n_q_heads=wl.n_q_heads,
+                   n_kv_heads=wl.n_kv_heads, scale=wl.softmax_scale, **kw)
+
+
+def _oracle_threads():
+    try:
+        import threadpoolctl
+
+        info = threadpoolctl.threadpool_info()
+        return max([int(i.get("num_threads", 1)) for i in info] or [1])
+    except Exception:  # noqa: BLE001
+        return 1
+
+
+def cpu_baseline(wl, crit, seconds):
+    from oracle import avtp_oracle as O
+
+    lay = wl.layout
+    n_img = int(lay.img_cu[1])
+    sub, t = _sub_workload(wl, n_img)
+    t0 = time.perf_counter()
+    done_tokens = 0
+    runs = 0
+    while True:
+        _oracle_step(O, sub, t, wl, crit)
+        runs += 1
+        done_tokens += int(sub.img_len.sum())
+        if time.perf_counter() - t0 > seconds or runs >= 3:
+            break
+    el = time.perf_counter() - t0
+    cores = 1 if crit == "hidden_variation" else _oracle_threads()
+    return {"value": round(done_tokens / el, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{runs} full pass(es) of the oracle pipeline over request 0 ({n_img} images, "
+                      f"{int(sub.img_len.sum())} visual tokens), criterion {crit}, {el:.1f} s"}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return None
+    from oracle import avtp_oracle as O
+    from paper_2608_26806_gb300 import synth
+
+    crit = args.criterion
+    parts = ("A", "pos") if crit == "hidden_variation" else ("A", "B", "pos")
+    wl = synth.make_workload(args.config, parts=parts)
+    n_img = int(wl.layout.img_cu[1])
+    # size each step's sample so that warm-up + timed steps stay within ~2 minutes
+    sub, t = _sub_workload(wl, 1)
+    t0 = time.perf_counter()
+    _oracle_step(O, sub, t, wl, crit)
+    per_img = max(time.perf_counter() - t0, 1e-3)
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    k_img = int(max(1, min(n_img, budget // per_img)))
+    sub, t = _sub_workload(wl, k_img)
+    for _ in range(args.warmup):
+        _oracle_step(O, sub, t, wl, crit)
+    times = []
+    for _ in range(args.steps):
+        s = time.perf_counter()
+        _oracle_step(O, sub, t, wl, crit)
+        times.append(time.perf_counter() - s)
+    toks = int(sub.img_len.sum())
+    total = sum(times)
+    value = toks * args.steps / total
+    cores = 1 if crit == "hidden_variation" else _oracle_threads()
+    sample = (f"each step: the oracle's full pipeline on the first {k_img} of {n_img} images of the "
+              f"{args.config} request ({toks} visual tokens), criterion {crit}")
+    return {"impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.config, "criterion": crit, "parallelism": "host cores"},
+            "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="qwen3_vl_8b")
+    ap.add_argument("--criterion", default="hidden_variation", choices=["hidden_variation", "text_attention"])
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world, rank, local = dist_env()
+    if args.impl == "reference":
+        line = run_reference(args, world, rank)
+    else:
+        line = run_ours(args, world, rank, local)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    if world > 1 and args.impl == "ours":
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

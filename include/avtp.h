@@ -1,0 +1,218 @@
+/*
+ * avtp.h -- C ABI of the AVTP pruning stage on one NVIDIA GB300 (sm_103a).
+ *
+ * AVTP (Adaptive Visual Token Pruning for multi-image LVLMs) prunes visual tokens
+ * once, at a chosen decoder layer, in four steps:
+ *   1. score every visual token              (paper §3.3.1; attention variant §3.3.2)
+ *   2. allocate per-image keep budgets       (paper §3.3.3 mean + adaptive ratio, App. A.2 clamps)
+ *   3. keep each image's top-k tokens, keep all text, emit ascending positions
+ *                                            (paper §3.1 subsequence, §3.3.3)
+ *   4. compact the kept rows into a varlen-packed batch (paper §3.1, E_pruned = p(E_v))
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Pointers named as device pointers must point to GPU memory of the current
+ *   device; the library reads and writes them only from kernels launched on the
+ *   given stream. Host scalars are passed by value or in the argument structs.
+ * - The caller owns every buffer. The library never allocates or frees memory:
+ *   scratch lives in a caller-provided workspace of avtp_workspace_size() bytes,
+ *   256-byte aligned. A workspace may be reused by calls that do not overlap on
+ *   the GPU; calls that overlap need separate workspaces.
+ * - All compute calls are asynchronous on `stream` (NULL = legacy default stream).
+ *   Only avtp_read_device_status() synchronises.
+ * - Errors the host can see (null pointers, bad sizes, misalignment, a workspace
+ *   that is too small) are returned before anything is launched. Errors only the
+ *   device can see (a span outside its request, an out-of-range keep ratio, a
+ *   kept index outside [0, T)) are recorded in the workspace's status word; the
+ *   affected kernels then skip their work (no trap, no out-of-bounds access) and
+ *   avtp_read_device_status() returns the code.
+ * - bf16 tensors are row-major with a contiguous last dimension; their base
+ *   pointers and row strides must be multiples of 16 bytes.
+ * - Layout: varlen-packed requests. Request r owns packed tokens
+ *   [cu_seqlens[r], cu_seqlens[r+1]). Its images are entries img_cu[r] ..
+ *   img_cu[r+1]-1 of img_start/img_len; a span [img_start, img_start+img_len)
+ *   is request-local, at least 1 token long, and the spans of one request are
+ *   sorted and disjoint. Every token outside the spans is text and is always kept.
+ * - Limits: T < 2^31; at most 2^20 visual tokens and 4096 images per request.
+ */
+#ifndef AVTP_H_
+#define AVTP_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define AVTP_API __attribute__((visibility("default")))
+#else
+#define AVTP_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t / CUstream. */
+typedef struct CUstream_st* avtp_stream_t;
+
+typedef enum {
+  AVTP_OK = 0,
+  AVTP_ERR_INVALID_ARG = 1,   /* null pointer, negative size, bad enum              */
+  AVTP_ERR_UNSUPPORTED = 2,   /* head_dim not 64/128, misaligned rows, Hq % Hkv != 0 */
+  AVTP_ERR_RANGE = 3,         /* a size above the documented limits                  */
+  AVTP_ERR_CUDA = 4,          /* a CUDA runtime call failed (launch, copy)           */
+  AVTP_ERR_TIMEOUT = 5,       /* a bounded device wait gave up (reserved)            */
+  AVTP_ERR_DEVICE_INPUT = 6,  /* device-side data failed validation                  */
+  AVTP_ERR_WORKSPACE = 7      /* workspace null, misaligned or too small             */
+} avtp_status_t;
+
+typedef enum {
+  /* I_v = 1 - cos(h^l_v, h^prior_v): hidden-state variation (paper §3.3.1). */
+  AVTP_CRIT_HIDDEN_VARIATION = 0,
+  /* Mean over heads and text queries of the causal softmax probability that a
+   * text query puts on each visual key (the per-token form of the attention
+   * quantity of paper §3.3.2). Never materialises the attention matrix. */
+  AVTP_CRIT_TEXT_ATTENTION = 1
+} avtp_criterion_t;
+
+typedef struct {
+  int32_t n_requests;         /* R >= 1 (host scalar)                         */
+  int32_t n_images;           /* total images over all requests, >= 0 (host)  */
+  int64_t n_tokens;           /* T = cu_seqlens[R] (host)                     */
+  const int32_t* cu_seqlens;  /* device [R+1], cu_seqlens[0] = 0, non-decreasing */
+  const int32_t* img_cu;      /* device [R+1], img_cu[0] = 0, img_cu[R] = n_images */
+  const int32_t* img_start;   /* device [n_images], request-local first token */
+  const int32_t* img_len;     /* device [n_images], >= 1                      */
+} avtp_layout_t;
+
+typedef struct {
+  avtp_criterion_t criterion;
+  /* AVTP_CRIT_HIDDEN_VARIATION: h_cur = hidden state at the pruning layer,
+   * h_prior = hidden state after the previous pruning (or the input embedding
+   * for the first pruning layer), paper §3.3.1. bf16 [T, hidden]; row strides
+   * in elements. hidden must be a multiple of 8. */
+  const void* h_cur;
+  const void* h_prior;
+  int32_t hidden;
+  int64_t h_cur_stride;
+  int64_t h_prior_stride;
+  /* AVTP_CRIT_TEXT_ATTENTION: q bf16 [T, n_q_heads, head_dim] (only text rows
+   * are read), k bf16 [T, n_kv_heads, head_dim]; token strides in elements.
+   * Query head h reads KV head h / (n_q_heads / n_kv_heads). Logits are
+   * softmax_scale * q.k. head_dim must be 64 or 128. */
+  const void* q;
+  const void* k;
+  int32_t n_q_heads;
+  int32_t n_kv_heads;
+  int32_t head_dim;
+  int64_t q_stride;
+  int64_t k_stride;
+  float softmax_scale;
+  /* Optional fp32 [n_q_heads, T] (row stride lse_stride elements): the natural-log
+   * log-sum-exp of the scaled causal logits of each text query, as kept by a
+   * FlashAttention-style forward pass. NULL: the library computes it. */
+  const float* lse;
+  int64_t lse_stride;
+} avtp_score_args_t;
+
+typedef struct {
+  const float* keep_ratio;  /* device [R]: base keep ratio r_base of each request, in [0, 1] */
+  float alpha;              /* variance control alpha of paper §3.3.3, in [0, 1024]; paper uses 1.0 */
+  float r_min;              /* ratio clamps of App. A.2: 0 <= r_min <= r_max <= 1; paper uses 0.05 */
+  float r_max;              /*                                                        and 0.95 */
+  int32_t relative;         /* 0: r_i = r_base + alpha*(Ibar_i - Ibar_avg) (paper §3.3.3)
+                             * 1: r_i = r_base*(1 + alpha*(Ibar_i/Ibar_avg - 1)), for scores of
+                             *    order 1/N such as the text-attention criterion */
+} avtp_alloc_args_t;
+
+/* One set of rows to gather: out[j] = in[kept_idx[j]] for j in [0, n_kept).
+ * Device pointers; sizes and strides in bytes. Any row size works; rows whose
+ * size, strides and pointers are 16-byte multiples take the vectorised path. */
+typedef struct {
+  const void* in;
+  void* out;
+  int64_t row_bytes;
+  int64_t in_stride;
+  int64_t out_stride;
+} avtp_rows_t;
+
+#define AVTP_MAX_ROW_SETS 8
+
+/* Bytes of workspace the calls below need for this layout and scoring setup
+ * (score_args may be NULL when no scoring call will use the workspace).
+ * Returns AVTP_OK and writes *bytes, or an error for invalid arguments. */
+AVTP_API avtp_status_t avtp_workspace_size(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
+                                  size_t* bytes);
+
+/* Step 1 (paper §3.3.1 / §3.3.2). Writes scores[t] (device fp32 [T]) for every
+ * visual token t; entries at text positions are left unchanged. Also writes
+ * img_sums (device int64 [n_images]), the fixed-point per-image sums
+ * S_i = sum_{t in V_i} rint(fx(scores[t]) * 2^32), fx mapping NaN to 0 and
+ * clamping to +-2^10; being integers, they do not depend on summation order. */
+AVTP_API avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_args_t* args, float* scores,
+                         int64_t* img_sums, void* workspace, size_t workspace_bytes, avtp_stream_t stream);
+
+/* Step 2 (paper §3.3.3, App. A.2). From img_sums (device int64 [n_images]) writes
+ * budgets (device int32 [n_images]) and out_cu_seqlens (device int32 [R+1]),
+ * the packed offsets of the pruned batch. Per request: B_r = floor(r_base*N_vis+0.5);
+ * Ibar_i = S_i/2^32/n_i; Ibar_avg = sum S/2^32/N_vis; r_i by the rule above
+ * (fp64, each operation rounded once); R_i = rint(clamp(r_i,+-2^20)*2^40);
+ * lambda = smallest integer with sum n_i*clamp(R_i+lambda, R_min, R_max) >= B_r*2^40;
+ * k_i = min(floor(x_i/2^40), n_i) with x_i = n_i*clamp(R_i+lambda), then
+ * largest remainder (ties to the lower index) until sum k_i = B_r. */
+AVTP_API avtp_status_t avtp_allocate(const avtp_layout_t* layout, const int64_t* img_sums, const avtp_alloc_args_t* args,
+                            int32_t* budgets, int32_t* out_cu_seqlens, void* workspace, size_t workspace_bytes,
+                            avtp_stream_t stream);
+
+/* Step 3 (paper §3.1, §3.3.3). Keeps, in every image i, the budgets[i] visual
+ * tokens ranked highest by (score descending, position ascending; NaN lowest,
+ * -0 == +0), plus every text token, and writes their packed positions to
+ * kept_idx (device int32, capacity n_kept >= out_cu_seqlens[R]) in ascending
+ * order. scores: device fp32 [T]; budgets: device int32 [n_images], each in
+ * [0, img_len]; out_cu_seqlens: device int32 [R+1] as written by avtp_allocate.
+ * A request whose budgets and offsets disagree, or that would write past
+ * n_kept, is skipped and recorded as AVTP_ERR_DEVICE_INPUT. */
+AVTP_API avtp_status_t avtp_select(const avtp_layout_t* layout, const float* scores, const int32_t* budgets,
+                          const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, void* workspace,
+                          size_t workspace_bytes, avtp_stream_t stream);
+
+/* Step 4 (paper §3.1). For each of the n_sets row sets (at most AVTP_MAX_ROW_SETS):
+ * out[j] = in[kept_idx[j]] for j < n_kept. Indices outside [0, n_tokens) are
+ * skipped and recorded as AVTP_ERR_DEVICE_INPUT. Position ids with P planes
+ * (M-RoPE) are passed as P row sets of one element each. */
+AVTP_API avtp_status_t avtp_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
+                           int32_t n_sets, void* workspace, size_t workspace_bytes, avtp_stream_t stream);
+
+/* Steps 1-4 fused on one stream. Outputs as in the single steps; scores and
+ * img_sums may be NULL (then kept in the workspace). n_kept must equal
+ * avtp_kept_count_host() for this layout and these keep ratios.
+ * step_events (optional, NULL to skip): 6 cudaEvent_t handles recorded on
+ * `stream` before the first kernel and after each step (validation, score,
+ * allocate, select, compact), for per-step timing. */
+AVTP_API avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
+                         const avtp_alloc_args_t* alloc_args, float* scores, int64_t* img_sums, int32_t* budgets,
+                         int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, const avtp_rows_t* sets,
+                         int32_t n_sets, void* workspace, size_t workspace_bytes, void* const* step_events,
+                         avtp_stream_t stream);
+
+/* Host-side size of the pruned batch: sum_r floor(keep_ratio[r]*N_vis,r + 0.5) + N_txt,r.
+ * Host arrays: cu_seqlens [R+1], img_cu [R+1], img_len [n_images], keep_ratio [R].
+ * Returns the count, or -1 for invalid arguments. */
+AVTP_API int64_t avtp_kept_count_host(const int32_t* cu_seqlens, const int32_t* img_cu, const int32_t* img_len,
+                             const float* keep_ratio, int32_t n_requests);
+
+/* Waits for `stream`, then reads the workspace's device status word into *out
+ * (an avtp_status_t value; AVTP_OK if no device-side error was recorded since the
+ * last entry point reset it). */
+AVTP_API avtp_status_t avtp_read_device_status(const void* workspace, avtp_stream_t stream, int32_t* out);
+
+/* Static English text for a status code. */
+AVTP_API const char* avtp_status_string(int32_t status);
+
+/* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
+AVTP_API int32_t avtp_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AVTP_H_ */

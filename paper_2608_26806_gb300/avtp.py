@@ -1,0 +1,390 @@
+"""Thin Python binding of the AVTP C ABI (``include/avtp.h``).
+
+Argument marshalling only: every step of the pruning stage runs in the CUDA
+kernels of ``libavtp.so``. torch supplies device memory and streams. There is
+no CPU fallback: if the library is missing or a call fails, this module raises.
+
+Function names follow the C ABI (``score``, ``allocate``, ``select``,
+``compact``, ``prune``, ``workspace_size``, ``kept_count_host``,
+``read_device_status``); each takes torch tensors and calls the entry point of
+the same name.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_float, c_int, c_int32, c_int64, c_size_t, c_void_p
+from dataclasses import dataclass
+from typing import Dict, Iterable, List, Optional, Sequence, Tuple
+
+import numpy as np
+import torch
+
+from . import build as _build
+
+OK = 0
+ERR_INVALID_ARG = 1
+ERR_UNSUPPORTED = 2
+ERR_RANGE = 3
+ERR_CUDA = 4
+ERR_TIMEOUT = 5
+ERR_DEVICE_INPUT = 6
+ERR_WORKSPACE = 7
+
+CRIT_HIDDEN_VARIATION = 0
+CRIT_TEXT_ATTENTION = 1
+MAX_ROW_SETS = 8
+
+_CRITERIA = {"hidden_variation": CRIT_HIDDEN_VARIATION, "text_attention": CRIT_TEXT_ATTENTION}
+
+
+class AVTPError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = int(code)
+        super().__init__(f"{where}: {status_string(code)} (status {code})")
+
+
+# ---------------------------------------------------------------- C structs
+class _Layout(ctypes.Structure):
+    _fields_ = [("n_requests", c_int32), ("n_images", c_int32), ("n_tokens", c_int64),
+                ("cu_seqlens", c_void_p), ("img_cu", c_void_p), ("img_start", c_void_p), ("img_len", c_void_p)]
+
+
+class _ScoreArgs(ctypes.Structure):
+    _fields_ = [("criterion", c_int), ("h_cur", c_void_p), ("h_prior", c_void_p), ("hidden", c_int32),
+                ("h_cur_stride", c_int64), ("h_prior_stride", c_int64), ("q", c_void_p), ("k", c_void_p),
+                ("n_q_heads", c_int32), ("n_kv_heads", c_int32), ("head_dim", c_int32), ("q_stride", c_int64),
+                ("k_stride", c_int64), ("softmax_scale", c_float), ("lse", c_void_p), ("lse_stride", c_int64)]
+
+
+class _AllocArgs(ctypes.Structure):
+    _fields_ = [("keep_ratio", c_void_p), ("alpha", c_float), ("r_min", c_float), ("r_max", c_float),
+                ("relative", c_int32)]
+
+
+class _Rows(ctypes.Structure):
+    _fields_ = [("in_", c_void_p), ("out", c_void_p), ("row_bytes", c_int64), ("in_stride", c_int64),
+                ("out_stride", c_int64)]
+
+
+# ---------------------------------------------------------------- library
+_LIB = None
+
+# name -> (restype, argtypes); every symbol the header declares
+SIGNATURES = {
+    "avtp_workspace_size": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(c_size_t)]),
+    "avtp_score": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "avtp_allocate": (c_int, [POINTER(_Layout), c_void_p, POINTER(_AllocArgs), c_void_p, c_void_p, c_void_p,
+                              c_size_t, c_void_p]),
+    "avtp_select": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
+                            c_void_p]),
+    "avtp_compact": (c_int, [c_void_p, c_int64, c_int64, POINTER(_Rows), c_int32, c_void_p, c_size_t, c_void_p]),
+    "avtp_prune": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(_AllocArgs), c_void_p, c_void_p, c_void_p,
+                           c_void_p, c_void_p, c_int64, POINTER(_Rows), c_int32, c_void_p, c_size_t,
+                           POINTER(c_void_p), c_void_p]),
+    "avtp_kept_count_host": (c_int64, [c_void_p, c_void_p, c_void_p, c_void_p, c_int32]),
+    "avtp_read_device_status": (c_int, [c_void_p, c_void_p, POINTER(c_int32)]),
+    "avtp_status_string": (ctypes.c_char_p, [c_int32]),
+    "avtp_version": (c_int32, []),
+}
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def load() -> ctypes.CDLL:
+    """Load libavtp.so (built by ``__graft_entry__.build()``); raise if it is missing."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = library_path()
+    if not os.path.exists(path):
+        if os.environ.get("AVTP_AUTOBUILD") == "1":
+            _build.build()
+        else:
+            raise RuntimeError(f"libavtp.so is not built ({path}); run __graft_entry__.build() first")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _LIB = lib
+    return lib
+
+
+def status_string(code: int) -> str:
+    return load().avtp_status_string(int(code)).decode()
+
+
+def _check(code: int, where: str) -> None:
+    if code != OK:
+        raise AVTPError(code, where)
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else int(t.data_ptr())
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
+
+
+# ---------------------------------------------------------------- layout
+@dataclass
+class Layout:
+    """A varlen-packed multi-image layout on the device (int32 tensors) plus host copies."""
+    cu_seqlens: torch.Tensor
+    img_cu: torch.Tensor
+    img_start: torch.Tensor
+    img_len: torch.Tensor
+    host: Dict[str, np.ndarray]
+
+    @staticmethod
+    def from_host(cu_seqlens, img_cu, img_start, img_len, device="cuda") -> "Layout":
+        host = {k: np.ascontiguousarray(np.asarray(v, dtype=np.int32))
+                for k, v in dict(cu_seqlens=cu_seqlens, img_cu=img_cu, img_start=img_start, img_len=img_len).items()}
+        dev = {k: torch.from_numpy(v.copy()).to(device) for k, v in host.items()}
+        return Layout(host=host, **dev)
+
+    @property
+    def n_requests(self) -> int:
+        return int(self.host["cu_seqlens"].shape[0] - 1)
+
+    @property
+    def n_images(self) -> int:
+        return int(self.host["img_len"].shape[0])
+
+    @property
+    def n_tokens(self) -> int:
+        return int(self.host["cu_seqlens"][-1])
+
+    def c(self) -> _Layout:
+        return _Layout(self.n_requests, self.n_images, self.n_tokens, _ptr(self.cu_seqlens), _ptr(self.img_cu),
+                       _ptr(self.img_start) if self.n_images else None, _ptr(self.img_len) if self.n_images else None)
+
+
+def _score_args(criterion, h_cur=None, h_prior=None, q=None, k=None, softmax_scale=None, lse=None) -> _ScoreArgs:
+    a = _ScoreArgs()
+    a.criterion = _CRITERIA[criterion] if isinstance(criterion, str) else int(criterion)
+    if a.criterion == CRIT_HIDDEN_VARIATION:
+        for t in (h_cur, h_prior):
+            if t is None or t.dtype != torch.bfloat16 or t.dim() != 2 or t.stride(1) != 1:
+                raise ValueError("h_cur / h_prior must be bf16 [T, hidden] with a contiguous last dim")
+        a.h_cur, a.h_prior = _ptr(h_cur), _ptr(h_prior)
+        a.hidden = h_cur.shape[1]
+        a.h_cur_stride, a.h_prior_stride = h_cur.stride(0), h_prior.stride(0)
+    else:
+        for t in (q, k):
+            if t is None or t.dtype != torch.bfloat16 or t.dim() != 3 or t.stride(2) != 1 or t.stride(1) != t.shape[2]:
+                raise ValueError("q / k must be bf16 [T, heads, head_dim] with contiguous heads")
+        a.q, a.k = _ptr(q), _ptr(k)
+        a.n_q_heads, a.n_kv_heads, a.head_dim = q.shape[1], k.shape[1], q.shape[2]
+        a.q_stride, a.k_stride = q.stride(0), k.stride(0)
+        a.softmax_scale = float(softmax_scale if softmax_scale is not None else q.shape[2] ** -0.5)
+        if lse is not None:
+            if lse.dtype != torch.float32 or lse.dim() != 2 or lse.stride(1) != 1:
+                raise ValueError("lse must be fp32 [Hq, T] with a contiguous last dim")
+            a.lse, a.lse_stride = _ptr(lse), lse.stride(0)
+    return a
+
+
+def _alloc_args(keep_ratio: torch.Tensor, alpha=1.0, r_min=0.05, r_max=0.95, relative=False) -> _AllocArgs:
+    if keep_ratio.dtype != torch.float32 or not keep_ratio.is_cuda:
+        raise ValueError("keep_ratio must be a float32 CUDA tensor [R]")
+    return _AllocArgs(_ptr(keep_ratio), float(alpha), float(r_min), float(r_max), 1 if relative else 0)
+
+
+def _row_sets(rows: Sequence[Tuple[torch.Tensor, torch.Tensor]]) -> Tuple[ctypes.Array, int]:
+    """(in, out) pairs gathered along dim 0: row j of out = row kept_idx[j] of in."""
+    arr = (_Rows * MAX_ROW_SETS)()
+    if len(rows) > MAX_ROW_SETS:
+        raise ValueError(f"at most {MAX_ROW_SETS} row sets")
+    for i, (src, dst) in enumerate(rows):
+        es = src.element_size()
+        row_elems = int(np.prod(src.shape[1:])) if src.dim() > 1 else 1
+        if src.dim() > 1 and not src[0].is_contiguous():
+            raise ValueError("each row must be contiguous")
+        arr[i] = _Rows(_ptr(src), _ptr(dst), row_elems * es, src.stride(0) * es, dst.stride(0) * es)
+    return arr, len(rows)
+
+
+def workspace_size(layout: Layout, criterion=None, **score_tensors) -> int:
+    lay = layout.c()
+    sa = _score_args(criterion, **score_tensors) if criterion is not None else None
+    out = c_size_t()
+    _check(load().avtp_workspace_size(ctypes.byref(lay), ctypes.byref(sa) if sa is not None else None,
+                                      ctypes.byref(out)), "avtp_workspace_size")
+    return int(out.value)
+
+
+def new_workspace(nbytes: int, device="cuda") -> torch.Tensor:
+    """A caller-owned workspace (torch allocations are 256-byte aligned)."""
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+# ---------------------------------------------------------------- entry points
+def score(layout: Layout, criterion, *, h_cur=None, h_prior=None, q=None, k=None, softmax_scale=None, lse=None,
+          scores=None, img_sums=None, workspace=None, stream=None):
+    """avtp_score: per-token scores (fp32 [T], text entries untouched) and fixed-point per-image sums."""
+    dev = layout.cu_seqlens.device
+    sa = _score_args(criterion, h_cur, h_prior, q, k, softmax_scale, lse)
+    if scores is None:
+        scores = torch.zeros(layout.n_tokens, dtype=torch.float32, device=dev)
+    if img_sums is None:
+        img_sums = torch.empty(max(layout.n_images, 1), dtype=torch.int64, device=dev)
+    if workspace is None:
+        workspace = new_workspace(workspace_size(layout, criterion, h_cur=h_cur, h_prior=h_prior, q=q, k=k,
+                                                 softmax_scale=softmax_scale, lse=lse), dev)
+    lay = layout.c()
+    _check(load().avtp_score(ctypes.byref(lay), ctypes.byref(sa), _ptr(scores), _ptr(img_sums), _ptr(workspace),
+                             workspace.numel(), _stream(stream)), "avtp_score")
+    return scores, img_sums[:layout.n_images]
+
+
+def allocate(layout: Layout, img_sums: torch.Tensor, keep_ratio: torch.Tensor, alpha=1.0, r_min=0.05, r_max=0.95,
+             relative=False, budgets=None, out_cu_seqlens=None, workspace=None, stream=None):
+    """avtp_allocate: per-image budgets (int32 [n_images]) and out_cu_seqlens (int32 [R+1])."""
+    dev = layout.cu_seqlens.device
+    aa = _alloc_args(keep_ratio, alpha, r_min, r_max, relative)
+    if budgets is None:
+        budgets = torch.empty(max(layout.n_images, 1), dtype=torch.int32, device=dev)
+    if out_cu_seqlens is None:
+        out_cu_seqlens = torch.empty(layout.n_requests + 1, dtype=torch.int32, device=dev)
+    if workspace is None:
+        workspace = new_workspace(workspace_size(layout), dev)
+    lay = layout.c()
+    _check(load().avtp_allocate(ctypes.byref(lay), _ptr(img_sums), ctypes.byref(aa), _ptr(budgets),
+                                _ptr(out_cu_seqlens), _ptr(workspace), workspace.numel(), _stream(stream)),
+           "avtp_allocate")
+    return budgets[:layout.n_images], out_cu_seqlens
+
+
+def select(layout: Layout, scores: torch.Tensor, budgets: torch.Tensor, out_cu_seqlens: torch.Tensor, n_kept: int,
+           kept_idx=None, workspace=None, stream=None):
+    """avtp_select: ascending packed positions of the kept tokens (int32 [n_kept])."""
+    dev = layout.cu_seqlens.device
+    if kept_idx is None:
+        kept_idx = torch.empty(max(int(n_kept), 1), dtype=torch.int32, device=dev)
+    if workspace is None:
+        workspace = new_workspace(workspace_size(layout), dev)
+    lay = layout.c()
+    _check(load().avtp_select(ctypes.byref(lay), _ptr(scores), _ptr(budgets), _ptr(out_cu_seqlens), _ptr(kept_idx),
+                              int(n_kept), _ptr(workspace), workspace.numel(), _stream(stream)), "avtp_select")
+    return kept_idx[:int(n_kept)]
+
+
+def compact(kept_idx: torch.Tensor, n_tokens: int, rows: Sequence[Tuple[torch.Tensor, torch.Tensor]],
+            workspace=None, stream=None) -> None:
+    """avtp_compact: for each (in, out) pair, out[j] = in[kept_idx[j]] along dim 0."""
+    dev = kept_idx.device
+    if workspace is None:
+        workspace = new_workspace(256, dev)
+    sets, n = _row_sets(rows)
+    _check(load().avtp_compact(_ptr(kept_idx), kept_idx.numel(), int(n_tokens), sets, n, _ptr(workspace),
+                               workspace.numel(), _stream(stream)), "avtp_compact")
+
+
+def kept_count_host(layout_host: Dict[str, np.ndarray], keep_ratio: np.ndarray) -> int:
+    """avtp_kept_count_host: sum_r floor(r_base*N_vis + 0.5) + N_txt over requests."""
+    h = {k: np.ascontiguousarray(np.asarray(layout_host[k], dtype=np.int32))
+         for k in ("cu_seqlens", "img_cu", "img_len")}
+    kr = np.ascontiguousarray(np.asarray(keep_ratio, dtype=np.float32))
+    img_len = h["img_len"] if h["img_len"].size else np.zeros(1, dtype=np.int32)
+    n = load().avtp_kept_count_host(h["cu_seqlens"].ctypes.data, h["img_cu"].ctypes.data, img_len.ctypes.data,
+                                    kr.ctypes.data, int(h["cu_seqlens"].shape[0] - 1))
+    if n < 0:
+        raise AVTPError(ERR_INVALID_ARG, "avtp_kept_count_host")
+    return int(n)
+
+
+def read_device_status(workspace: torch.Tensor, stream=None) -> int:
+    out = c_int32()
+    _check(load().avtp_read_device_status(_ptr(workspace), _stream(stream), ctypes.byref(out)),
+           "avtp_read_device_status")
+    return int(out.value)
+
+
+@dataclass
+class PruneBuffers:
+    """Every buffer one avtp_prune call touches, allocated once for a fixed layout."""
+    scores: torch.Tensor
+    img_sums: torch.Tensor
+    budgets: torch.Tensor
+    out_cu_seqlens: torch.Tensor
+    kept_idx: torch.Tensor
+    workspace: torch.Tensor
+    outputs: Dict[str, torch.Tensor]
+    n_kept: int
+
+
+def prune_buffers(layout: Layout, keep_ratio_host: np.ndarray, criterion, score_tensors: Dict[str, torch.Tensor],
+                  rows: Dict[str, torch.Tensor], planes: Dict[str, torch.Tensor]) -> PruneBuffers:
+    dev = layout.cu_seqlens.device
+    n_kept = kept_count_host(layout.host, keep_ratio_host)
+    outputs = {}
+    for name, src in rows.items():
+        outputs[name] = torch.empty((n_kept,) + tuple(src.shape[1:]), dtype=src.dtype, device=dev)
+    for name, src in planes.items():
+        outputs[name] = torch.empty((src.shape[0], n_kept), dtype=src.dtype, device=dev)
+    ws = new_workspace(workspace_size(layout, criterion, **score_tensors), dev)
+    return PruneBuffers(
+        scores=torch.zeros(layout.n_tokens, dtype=torch.float32, device=dev),
+        img_sums=torch.empty(max(layout.n_images, 1), dtype=torch.int64, device=dev),
+        budgets=torch.empty(max(layout.n_images, 1), dtype=torch.int32, device=dev),
+        out_cu_seqlens=torch.empty(layout.n_requests + 1, dtype=torch.int32, device=dev),
+        kept_idx=torch.empty(max(n_kept, 1), dtype=torch.int32, device=dev),
+        workspace=ws, outputs=outputs, n_kept=n_kept)
+
+
+class PruneCall:
+    """A prepared avtp_prune call: C structs built once, then launched with ``run()``.
+
+    ``rows``: name -> [T, ...] tensors gathered along dim 0; ``planes``: name ->
+    [P, T] tensors (e.g. M-RoPE position ids) gathered along dim 1.
+    """
+
+    def __init__(self, layout: Layout, criterion, *, keep_ratio: torch.Tensor, keep_ratio_host: np.ndarray,
+                 alpha=1.0, r_min=0.05, r_max=0.95, relative=None, rows: Optional[Dict[str, torch.Tensor]] = None,
+                 planes: Optional[Dict[str, torch.Tensor]] = None, buffers: Optional[PruneBuffers] = None,
+                 **score_tensors):
+        rows = rows or {}
+        planes = planes or {}
+        if relative is None:
+            crit = _CRITERIA[criterion] if isinstance(criterion, str) else int(criterion)
+            relative = crit == CRIT_TEXT_ATTENTION
+        self.layout = layout
+        self.buffers = buffers or prune_buffers(layout, keep_ratio_host, criterion, score_tensors, rows, planes)
+        b = self.buffers
+        self._lay = layout.c()
+        self._sa = _score_args(criterion, **score_tensors)
+        self._aa = _alloc_args(keep_ratio, alpha, r_min, r_max, relative)
+        pairs: List[Tuple[torch.Tensor, torch.Tensor]] = []
+        for name, src in rows.items():
+            pairs.append((src, b.outputs[name]))
+        for name, src in planes.items():
+            for p in range(src.shape[0]):
+                pairs.append((src[p], b.outputs[name][p]))
+        self._sets, self._n_sets = _row_sets(pairs)
+        self._keep_alive = (keep_ratio, rows, planes, score_tensors)
+
+    def run(self, stream=None, step_events: Optional[Sequence] = None) -> PruneBuffers:
+        b = self.buffers
+        ev = None
+        if step_events is not None:
+            ev = (c_void_p * 6)(*[int(e.cuda_event) if hasattr(e, "cuda_event") else int(e) for e in step_events])
+        _check(load().avtp_prune(ctypes.byref(self._lay), ctypes.byref(self._sa), ctypes.byref(self._aa),
+                                 _ptr(b.scores), _ptr(b.img_sums), _ptr(b.budgets), _ptr(b.out_cu_seqlens),
+                                 _ptr(b.kept_idx), b.n_kept, self._sets, self._n_sets, _ptr(b.workspace),
+                                 b.workspace.numel(), ev, _stream(stream)), "avtp_prune")
+        return b
+
+
+def prune(layout: Layout, criterion, *, keep_ratio: torch.Tensor, keep_ratio_host: np.ndarray, alpha=1.0,
+          r_min=0.05, r_max=0.95, relative=None, rows=None, planes=None, stream=None, **score_tensors) -> PruneBuffers:
+    """avtp_prune: score -> allocate -> select -> compact in one call on one stream."""
+    call = PruneCall(layout, criterion, keep_ratio=keep_ratio, keep_ratio_host=keep_ratio_host, alpha=alpha,
+                     r_min=r_min, r_max=r_max, relative=relative, rows=rows, planes=planes, **score_tensors)
+    return call.run(stream)

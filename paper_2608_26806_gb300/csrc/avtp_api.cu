@@ -1,0 +1,306 @@
+// C ABI of the AVTP pruning stage: argument validation, workspace plan and the
+// launch sequence of every entry point. Kernels live in k_*.cu.
+#include <math.h>
+#include <string.h>
+
+#include "avtp_internal.cuh"
+
+namespace avtp {
+
+int attn_q_tile(int Hq, int Hkv);
+
+namespace {
+
+constexpr size_t kAlign = 256;
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+avtp_status_t from_cuda(cudaError_t e) { return e == cudaSuccess ? AVTP_OK : AVTP_ERR_CUDA; }
+
+avtp_status_t check_layout(const avtp_layout_t* L) {
+  if (L == nullptr) return AVTP_ERR_INVALID_ARG;
+  if (L->n_requests < 1 || L->n_images < 0 || L->n_tokens < 0) return AVTP_ERR_INVALID_ARG;
+  if (L->n_tokens > 0x7fffffffLL || L->n_images > 0x7fffffff - L->n_requests) return AVTP_ERR_RANGE;
+  if (L->cu_seqlens == nullptr || L->img_cu == nullptr) return AVTP_ERR_INVALID_ARG;
+  if (L->n_images > 0 && (L->img_start == nullptr || L->img_len == nullptr)) return AVTP_ERR_INVALID_ARG;
+  return AVTP_OK;
+}
+
+avtp_status_t check_score_args(const avtp_layout_t* L, const avtp_score_args_t* a) {
+  if (a == nullptr) return AVTP_ERR_INVALID_ARG;
+  if (a->criterion == AVTP_CRIT_HIDDEN_VARIATION) {
+    if (a->h_cur == nullptr || a->h_prior == nullptr) return AVTP_ERR_INVALID_ARG;
+    if (a->hidden < 8 || a->hidden % 8 != 0) return AVTP_ERR_UNSUPPORTED;
+    if (a->h_cur_stride < a->hidden || a->h_prior_stride < a->hidden) return AVTP_ERR_INVALID_ARG;
+    if (a->h_cur_stride % 8 != 0 || a->h_prior_stride % 8 != 0) return AVTP_ERR_UNSUPPORTED;
+    if (!aligned16(a->h_cur) || !aligned16(a->h_prior)) return AVTP_ERR_UNSUPPORTED;
+    return AVTP_OK;
+  }
+  if (a->criterion == AVTP_CRIT_TEXT_ATTENTION) {
+    if (a->q == nullptr || a->k == nullptr) return AVTP_ERR_INVALID_ARG;
+    if (a->head_dim != 64 && a->head_dim != 128) return AVTP_ERR_UNSUPPORTED;
+    if (a->n_q_heads < 1 || a->n_kv_heads < 1) return AVTP_ERR_INVALID_ARG;
+    if (a->n_q_heads % a->n_kv_heads != 0) return AVTP_ERR_UNSUPPORTED;
+    if (a->n_q_heads / a->n_kv_heads > kAttnRowTile) return AVTP_ERR_UNSUPPORTED;
+    if (a->q_stride < static_cast<int64_t>(a->n_q_heads) * a->head_dim ||
+        a->k_stride < static_cast<int64_t>(a->n_kv_heads) * a->head_dim)
+      return AVTP_ERR_INVALID_ARG;
+    if (a->q_stride % 8 != 0 || a->k_stride % 8 != 0) return AVTP_ERR_UNSUPPORTED;
+    if (!aligned16(a->q) || !aligned16(a->k)) return AVTP_ERR_UNSUPPORTED;
+    if (!(a->softmax_scale > 0.f) || !isfinite(a->softmax_scale)) return AVTP_ERR_INVALID_ARG;
+    if (a->lse != nullptr && a->lse_stride < L->n_tokens) return AVTP_ERR_INVALID_ARG;
+    return AVTP_OK;
+  }
+  return AVTP_ERR_INVALID_ARG;
+}
+
+avtp_status_t check_alloc_args(const avtp_alloc_args_t* a) {
+  if (a == nullptr || a->keep_ratio == nullptr) return AVTP_ERR_INVALID_ARG;
+  if (!(a->alpha >= 0.f && a->alpha <= 1024.f)) return AVTP_ERR_INVALID_ARG;
+  if (!(a->r_min >= 0.f && a->r_min <= a->r_max && a->r_max <= 1.f)) return AVTP_ERR_INVALID_ARG;
+  if (a->relative != 0 && a->relative != 1) return AVTP_ERR_INVALID_ARG;
+  return AVTP_OK;
+}
+
+avtp_status_t check_sets(const avtp_rows_t* sets, int32_t n_sets) {
+  if (n_sets < 0 || n_sets > AVTP_MAX_ROW_SETS) return AVTP_ERR_INVALID_ARG;
+  if (n_sets > 0 && sets == nullptr) return AVTP_ERR_INVALID_ARG;
+  for (int i = 0; i < n_sets; ++i) {
+    const avtp_rows_t& s = sets[i];
+    if (s.in == nullptr || s.out == nullptr) return AVTP_ERR_INVALID_ARG;
+    if (s.row_bytes < 1 || s.in_stride < s.row_bytes || s.out_stride < s.row_bytes) return AVTP_ERR_INVALID_ARG;
+  }
+  return AVTP_OK;
+}
+
+avtp_status_t check_ws(void* ws, size_t ws_bytes, const WsPlan& p) {
+  if (ws == nullptr || (reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return AVTP_ERR_WORKSPACE;
+  if (ws_bytes < p.total) return AVTP_ERR_WORKSPACE;
+  return AVTP_OK;
+}
+
+avtp_status_t record(void* const* events, int i, cudaStream_t s) {
+  if (events == nullptr || events[i] == nullptr) return AVTP_OK;
+  return from_cuda(cudaEventRecord(static_cast<cudaEvent_t>(events[i]), s));
+}
+
+}  // namespace
+
+WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
+  WsPlan p{};
+  const size_t R = static_cast<size_t>(L.n_requests), NI = static_cast<size_t>(L.n_images);
+  const size_t T = static_cast<size_t>(L.n_tokens);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes);
+    return at;
+  };
+  p.status = take(sizeof(DevStatus));
+  p.vis_cu = take((NI + 1) * 4);
+  p.img_req = take(NI * 4 + 4);
+  p.req_budget = take(R * 4);
+  p.img_sums = take(NI * 8 + 8);
+  p.scores = take(T * 4 + 4);
+  if (sa != nullptr && sa->criterion == AVTP_CRIT_TEXT_ATTENTION) {
+    p.text_idx = take(T * 4 + 4);
+    p.text_cu = take((R + 1) * 4);
+    p.qtile_cu = take((R + 1) * 4);
+    p.ktile_cu = take((NI + 1) * 4);
+    p.lse = (sa->lse == nullptr) ? take(static_cast<size_t>(sa->n_q_heads) * T * 4 + 4) : 0;
+    p.partial = take(static_cast<size_t>(sa->n_kv_heads) * T * 4 + 4);
+  }
+  p.total = off;
+  return p;
+}
+
+int device_sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
+
+}  // namespace avtp
+
+using namespace avtp;
+
+extern "C" {
+
+avtp_status_t avtp_workspace_size(const avtp_layout_t* layout, const avtp_score_args_t* score_args, size_t* bytes) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if (bytes == nullptr) return AVTP_ERR_INVALID_ARG;
+  if (score_args != nullptr && (st = check_score_args(layout, score_args)) != AVTP_OK) return st;
+  *bytes = plan_workspace(*layout, score_args).total;
+  return AVTP_OK;
+}
+
+static avtp_status_t score_impl(const avtp_layout_t* L, const avtp_score_args_t* a, float* scores,
+                                int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s) {
+  if (a->criterion == AVTP_CRIT_HIDDEN_VARIATION) return from_cuda(launch_score_hvar(*L, *a, scores, img_sums, ws, p, s));
+  return from_cuda(launch_score_attn(*L, *a, scores, img_sums, ws, p, s));
+}
+
+avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_args_t* args, float* scores,
+                         int64_t* img_sums, void* workspace, size_t workspace_bytes, avtp_stream_t stream) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if ((st = check_score_args(layout, args)) != AVTP_OK) return st;
+  if (scores == nullptr || img_sums == nullptr) return AVTP_ERR_INVALID_ARG;
+  const WsPlan p = plan_workspace(*layout, args);
+  if ((st = check_ws(workspace, workspace_bytes, p)) != AVTP_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PrepArgs pa{};
+  pa.L = *layout;
+  pa.zero_img_sums = img_sums;
+  pa.build_text_tiles = args->criterion == AVTP_CRIT_TEXT_ATTENTION;
+  pa.q_tile = pa.build_text_tiles ? attn_q_tile(args->n_q_heads, args->n_kv_heads) : 1;
+  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
+  return score_impl(layout, args, scores, img_sums, workspace, p, s);
+}
+
+avtp_status_t avtp_allocate(const avtp_layout_t* layout, const int64_t* img_sums, const avtp_alloc_args_t* args,
+                            int32_t* budgets, int32_t* out_cu_seqlens, void* workspace, size_t workspace_bytes,
+                            avtp_stream_t stream) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if ((st = check_alloc_args(args)) != AVTP_OK) return st;
+  if ((layout->n_images > 0 && (img_sums == nullptr || budgets == nullptr)) || out_cu_seqlens == nullptr)
+    return AVTP_ERR_INVALID_ARG;
+  const WsPlan p = plan_workspace(*layout, nullptr);
+  if ((st = check_ws(workspace, workspace_bytes, p)) != AVTP_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PrepArgs pa{};
+  pa.L = *layout;
+  pa.keep_ratio = args->keep_ratio;
+  pa.out_cu_seqlens = out_cu_seqlens;
+  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
+  return from_cuda(launch_allocate(*layout, img_sums, *args, budgets, workspace, p, s));
+}
+
+avtp_status_t avtp_select(const avtp_layout_t* layout, const float* scores, const int32_t* budgets,
+                          const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, void* workspace,
+                          size_t workspace_bytes, avtp_stream_t stream) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if (out_cu_seqlens == nullptr || n_kept < 0 || (n_kept > 0 && kept_idx == nullptr)) return AVTP_ERR_INVALID_ARG;
+  if (layout->n_images > 0 && (scores == nullptr || budgets == nullptr)) return AVTP_ERR_INVALID_ARG;
+  const WsPlan p = plan_workspace(*layout, nullptr);
+  if ((st = check_ws(workspace, workspace_bytes, p)) != AVTP_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PrepArgs pa{};
+  pa.L = *layout;
+  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
+  return from_cuda(launch_select(*layout, scores, budgets, out_cu_seqlens, kept_idx, n_kept, workspace, p, s));
+}
+
+avtp_status_t avtp_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
+                           int32_t n_sets, void* workspace, size_t workspace_bytes, avtp_stream_t stream) {
+  avtp_status_t st = check_sets(sets, n_sets);
+  if (st != AVTP_OK) return st;
+  if (n_kept < 0 || n_tokens < 0 || (n_kept > 0 && kept_idx == nullptr)) return AVTP_ERR_INVALID_ARG;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1)) != 0 ||
+      workspace_bytes < sizeof(DevStatus))
+    return AVTP_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  WsPlan p{};
+  p.status = 0;
+  if ((st = from_cuda(cudaMemsetAsync(workspace, 0, sizeof(DevStatus), s))) != AVTP_OK) return st;
+  return from_cuda(launch_compact(kept_idx, n_kept, n_tokens, sets, n_sets, workspace, p, s));
+}
+
+avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
+                         const avtp_alloc_args_t* alloc_args, float* scores, int64_t* img_sums, int32_t* budgets,
+                         int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, const avtp_rows_t* sets,
+                         int32_t n_sets, void* workspace, size_t workspace_bytes, void* const* step_events,
+                         avtp_stream_t stream) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if ((st = check_score_args(layout, score_args)) != AVTP_OK) return st;
+  if ((st = check_alloc_args(alloc_args)) != AVTP_OK) return st;
+  if ((st = check_sets(sets, n_sets)) != AVTP_OK) return st;
+  if (out_cu_seqlens == nullptr || n_kept < 0 || (n_kept > 0 && kept_idx == nullptr)) return AVTP_ERR_INVALID_ARG;
+  if (layout->n_images > 0 && budgets == nullptr) return AVTP_ERR_INVALID_ARG;
+  const WsPlan p = plan_workspace(*layout, score_args);
+  if ((st = check_ws(workspace, workspace_bytes, p)) != AVTP_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  float* sc = scores != nullptr ? scores : ws_at<float>(workspace, p.scores);
+  int64_t* sums = img_sums != nullptr ? img_sums : ws_at<int64_t>(workspace, p.img_sums);
+
+  if ((st = record(step_events, 0, s)) != AVTP_OK) return st;
+  PrepArgs pa{};
+  pa.L = *layout;
+  pa.keep_ratio = alloc_args->keep_ratio;
+  pa.out_cu_seqlens = out_cu_seqlens;
+  pa.zero_img_sums = sums;
+  pa.build_text_tiles = score_args->criterion == AVTP_CRIT_TEXT_ATTENTION;
+  pa.q_tile = pa.build_text_tiles ? attn_q_tile(score_args->n_q_heads, score_args->n_kv_heads) : 1;
+  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
+  if ((st = record(step_events, 1, s)) != AVTP_OK) return st;
+  if ((st = score_impl(layout, score_args, sc, sums, workspace, p, s)) != AVTP_OK) return st;
+  if ((st = record(step_events, 2, s)) != AVTP_OK) return st;
+  if ((st = from_cuda(launch_allocate(*layout, sums, *alloc_args, budgets, workspace, p, s))) != AVTP_OK) return st;
+  if ((st = record(step_events, 3, s)) != AVTP_OK) return st;
+  if ((st = from_cuda(launch_select(*layout, sc, budgets, out_cu_seqlens, kept_idx, n_kept, workspace, p, s))) !=
+      AVTP_OK)
+    return st;
+  if ((st = record(step_events, 4, s)) != AVTP_OK) return st;
+  if ((st = from_cuda(launch_compact(kept_idx, n_kept, layout->n_tokens, sets, n_sets, workspace, p, s))) != AVTP_OK)
+    return st;
+  return record(step_events, 5, s);
+}
+
+int64_t avtp_kept_count_host(const int32_t* cu_seqlens, const int32_t* img_cu, const int32_t* img_len,
+                             const float* keep_ratio, int32_t n_requests) {
+  if (cu_seqlens == nullptr || img_cu == nullptr || keep_ratio == nullptr || n_requests < 1) return -1;
+  if (img_cu[n_requests] > 0 && img_len == nullptr) return -1;
+  int64_t total = 0;
+  for (int r = 0; r < n_requests; ++r) {
+    int64_t nvis = 0;
+    if (img_cu[r + 1] < img_cu[r] || cu_seqlens[r + 1] < cu_seqlens[r]) return -1;
+    for (int i = img_cu[r]; i < img_cu[r + 1]; ++i) nvis += img_len[i];
+    const float kr = keep_ratio[r];
+    if (!(kr >= 0.f && kr <= 1.f)) return -1;
+    // floor(kr * N + 0.5) with each operation rounded once (built with FMA contraction off)
+    volatile double prod = static_cast<double>(kr) * static_cast<double>(nvis);
+    const double x = prod + 0.5;
+    total += static_cast<int64_t>(floor(x)) + (static_cast<int64_t>(cu_seqlens[r + 1]) - cu_seqlens[r] - nvis);
+  }
+  return total;
+}
+
+avtp_status_t avtp_read_device_status(const void* workspace, avtp_stream_t stream, int32_t* out) {
+  if (workspace == nullptr || out == nullptr) return AVTP_ERR_INVALID_ARG;
+  DevStatus h{};
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemcpyAsync(&h, workspace, sizeof(h), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return AVTP_ERR_CUDA;
+  *out = h.code;
+  return AVTP_OK;
+}
+
+const char* avtp_status_string(int32_t status) {
+  switch (status) {
+    case AVTP_OK: return "ok";
+    case AVTP_ERR_INVALID_ARG: return "invalid argument";
+    case AVTP_ERR_UNSUPPORTED: return "unsupported configuration";
+    case AVTP_ERR_RANGE: return "size outside the supported range";
+    case AVTP_ERR_CUDA: return "CUDA runtime error";
+    case AVTP_ERR_TIMEOUT: return "device wait timed out";
+    case AVTP_ERR_DEVICE_INPUT: return "device data failed validation";
+    case AVTP_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    default: return "unknown status";
+  }
+}
+
+int32_t avtp_version(void) { return 100; }
+
+}  // extern "C"

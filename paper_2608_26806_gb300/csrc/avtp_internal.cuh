@@ -1,0 +1,126 @@
+// Internal declarations shared by the AVTP CUDA translation units.
+// Nothing here is part of the C ABI; see include/avtp.h for that.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "avtp.h"
+
+namespace avtp {
+
+// ---------------------------------------------------------------- limits
+constexpr int kMaxImagesPerRequest = 4096;
+constexpr int kMaxVisualPerRequest = 1 << 20;
+constexpr int kFxFracBits = 32;          // per-token fixed point of the per-image sums
+constexpr float kFxScoreLimit = 1024.f;  // |score| clamp before the fixed-point conversion
+constexpr int kRatioFracBits = 40;       // ratio grid of the budget rule
+constexpr double kRatioLimit = 1048576.0;  // ratios saturate at +-2^20 before the grid
+
+// Tiles of the text-attention criterion (CUDA-core path).
+constexpr int kAttnKeyTile = 64;     // visual keys per pass-2 tile
+constexpr int kAttnRowTile = 64;     // (head, query) rows per tile
+constexpr int kAttnQTile = 16;       // text queries per pass-1 tile (x heads per group <= 64 rows)
+
+// ---------------------------------------------------------------- status
+// First word of every workspace. code: first error recorded (0 = none);
+// layout_ok: set by the validation kernel when the layout may be used.
+struct DevStatus {
+  int32_t code;
+  int32_t layout_ok;
+  int32_t detail;  // index of the first offending item, for debugging
+  int32_t pad;
+};
+
+__device__ __forceinline__ void record_error(DevStatus* st, int32_t code, int32_t detail) {
+  if (atomicCAS(&st->code, 0, code) == 0) st->detail = detail;
+}
+
+// ---------------------------------------------------------------- workspace
+struct WsPlan {
+  size_t status;      // DevStatus
+  size_t vis_cu;      // int32 [n_img + 1]: exclusive prefix of img_len over all images
+  size_t img_req;     // int32 [n_img]: request of each image
+  size_t req_budget;  // int32 [R]: B_r
+  size_t img_sums;    // int64 [n_img]: used by avtp_prune when the caller passes NULL
+  size_t scores;      // float [T]: used by avtp_prune when the caller passes NULL
+  size_t text_idx;    // int32 [T]: packed position of each text ordinal (criterion B)
+  size_t text_cu;     // int32 [R + 1]: text ordinals per request (criterion B)
+  size_t qtile_cu;    // int32 [R + 1]: pass-1 query tiles per request (criterion B)
+  size_t ktile_cu;    // int32 [n_img + 1]: pass-2 key tiles per image (criterion B)
+  size_t lse;         // float [Hq * T]: per (head, text query) log2-domain LSE (criterion B)
+  size_t partial;     // float [Hkv * T]: per (KV group, visual key) probability sums (criterion B)
+  size_t total;
+};
+
+WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa);
+
+template <typename T>
+__host__ __device__ __forceinline__ T* ws_at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+// ---------------------------------------------------------------- small device helpers
+__device__ __forceinline__ int64_t fixed_point_score(float s) {
+  // rint(fx(s) * 2^32); fx: NaN -> 0, clamp to [-2^10, 2^10]. The product is exact.
+  if (isnan(s)) return 0;
+  s = fminf(fmaxf(s, -kFxScoreLimit), kFxScoreLimit);
+  return __double2ll_rn(static_cast<double>(s) * 4294967296.0);
+}
+
+// Order-preserving key: larger score -> larger key; NaN -> 0 (below -inf); -0 == +0.
+__device__ __forceinline__ uint32_t rank_key(float s) {
+  if (isnan(s)) return 0u;
+  uint32_t b = __float_as_uint(s);
+  if (b == 0x80000000u) b = 0u;
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Largest r in [0, n) with a[r] <= v, for non-decreasing a[0..n] with a[0] <= v.
+__device__ __forceinline__ int upper_index(const int32_t* a, int n, int64_t v) {
+  int lo = 0, hi = n;  // a[lo] <= v; answer in [lo, hi)
+  while (hi - lo > 1) {
+    int mid = (lo + hi) >> 1;
+    if (static_cast<int64_t>(a[mid]) <= v) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
+template <typename T>
+__device__ __forceinline__ T warp_sum(T v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// ---------------------------------------------------------------- launchers (one per kernel)
+struct PrepArgs {
+  avtp_layout_t L;
+  const float* keep_ratio;   // NULL: no budgets / out_cu_seqlens
+  int32_t* out_cu_seqlens;   // NULL: not written
+  int64_t* zero_img_sums;    // NULL: not zeroed
+  int build_text_tiles;      // criterion B bookkeeping
+  int q_tile;                // text queries per pass-1 tile (criterion B)
+};
+cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s);
+
+cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
+                              int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s);
+
+cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
+                              int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s);
+
+cudaError_t launch_allocate(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
+                            int32_t* budgets, void* ws, const WsPlan& p, cudaStream_t s);
+
+cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int32_t* budgets,
+                          const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, void* ws,
+                          const WsPlan& p, cudaStream_t s);
+
+cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
+                           int n_sets, void* ws, const WsPlan& p, cudaStream_t s);
+
+int device_sm_count();
+
+}  // namespace avtp

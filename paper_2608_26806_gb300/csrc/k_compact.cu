@@ -1,0 +1,137 @@
+// Step 4: compaction, out[j] = in[kept_idx[j]] for every row set (paper §3.1:
+// E_pruned = p(E_v), the kept tokens as a dense, varlen-packed batch).
+//
+// Large rows (hidden states, K/V rows): one warp per row, 16-byte vector loads
+// and stores, several in flight per lane. Small rows (position ids, one element
+// per plane): one thread per row. All row sets go in one launch; the block index
+// range is split between the sets on the host.
+#include "avtp_internal.cuh"
+
+namespace avtp {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kRowsPerWarp = 1;
+constexpr int kUnroll = 4;
+
+struct RowSetDev {
+  const char* in;
+  char* out;
+  int64_t row_bytes;
+  int64_t in_stride;
+  int64_t out_stride;
+  int32_t unit;            // widest power-of-two access (1..16) dividing pointers, strides and row size
+  int32_t warp_per_row;    // 1: vector path, one warp per row; 0: one thread per row
+  int32_t rows_per_block;
+  int32_t block_begin;
+};
+
+struct CompactParams {
+  RowSetDev set[AVTP_MAX_ROW_SETS];
+  int32_t n_sets;
+};
+
+template <int U>
+struct UnitType;
+template <> struct UnitType<16> { using T = uint4; };
+template <> struct UnitType<8> { using T = uint2; };
+template <> struct UnitType<4> { using T = uint32_t; };
+template <> struct UnitType<2> { using T = uint16_t; };
+template <> struct UnitType<1> { using T = uint8_t; };
+
+template <int U>
+__device__ __forceinline__ void copy_row_thread(const char* src, char* dst, int64_t bytes) {
+  using T = typename UnitType<U>::T;
+  const T* s = reinterpret_cast<const T*>(src);
+  T* d = reinterpret_cast<T*>(dst);
+  for (int64_t u = 0; u < bytes / U; ++u) d[u] = s[u];
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_compact(CompactParams P, const int32_t* __restrict__ kept_idx, int64_t n_kept, int64_t n_tokens, DevStatus* st) {
+  const int b = blockIdx.x;
+  int si = 0;
+  while (si + 1 < P.n_sets && b >= P.set[si + 1].block_begin) ++si;
+  const RowSetDev S = P.set[si];
+  const int64_t row0 = static_cast<int64_t>(b - S.block_begin) * S.rows_per_block;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (S.warp_per_row) {
+    const int64_t n16 = S.row_bytes >> 4;
+    for (int rr = 0; rr < kRowsPerWarp; ++rr) {
+      const int64_t j = row0 + static_cast<int64_t>(rr) * kWarps + warp;
+      if (j >= n_kept) break;
+      const int64_t t = kept_idx[j];
+      if (t < 0 || t >= n_tokens) {
+        if (lane == 0) record_error(st, AVTP_ERR_DEVICE_INPUT, static_cast<int32_t>(j));
+        continue;
+      }
+      const uint4* src = reinterpret_cast<const uint4*>(S.in + t * S.in_stride);
+      uint4* dst = reinterpret_cast<uint4*>(S.out + j * S.out_stride);
+      int64_t c = lane;
+      for (; c + 32 * (kUnroll - 1) < n16; c += 32 * kUnroll) {
+        uint4 v[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) v[u] = __ldcs(src + c + 32 * u);
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) __stcs(dst + c + 32 * u, v[u]);
+      }
+      for (; c < n16; c += 32) __stcs(dst + c, __ldcs(src + c));
+    }
+  } else {
+    const int64_t j = row0 + threadIdx.x;
+    if (threadIdx.x >= S.rows_per_block || j >= n_kept) return;
+    const int64_t t = kept_idx[j];
+    if (t < 0 || t >= n_tokens) {
+      record_error(st, AVTP_ERR_DEVICE_INPUT, static_cast<int32_t>(j));
+      return;
+    }
+    const char* src = S.in + t * S.in_stride;
+    char* dst = S.out + j * S.out_stride;
+    switch (S.unit) {
+      case 16: copy_row_thread<16>(src, dst, S.row_bytes); break;
+      case 8: copy_row_thread<8>(src, dst, S.row_bytes); break;
+      case 4: copy_row_thread<4>(src, dst, S.row_bytes); break;
+      case 2: copy_row_thread<2>(src, dst, S.row_bytes); break;
+      default: copy_row_thread<1>(src, dst, S.row_bytes); break;
+    }
+  }
+}
+
+int access_unit(const avtp_rows_t& s) {
+  const uint64_t bits = reinterpret_cast<uint64_t>(s.in) | reinterpret_cast<uint64_t>(s.out) |
+                        static_cast<uint64_t>(s.row_bytes) | static_cast<uint64_t>(s.in_stride) |
+                        static_cast<uint64_t>(s.out_stride);
+  for (int u = 16; u > 1; u >>= 1)
+    if ((bits & static_cast<uint64_t>(u - 1)) == 0) return u;
+  return 1;
+}
+
+}  // namespace
+
+cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
+                           int n_sets, void* ws, const WsPlan& p, cudaStream_t s) {
+  if (n_kept == 0 || n_sets == 0) return cudaSuccess;
+  CompactParams P{};
+  P.n_sets = n_sets;
+  int64_t blocks = 0;
+  for (int i = 0; i < n_sets; ++i) {
+    RowSetDev& d = P.set[i];
+    d.in = static_cast<const char*>(sets[i].in);
+    d.out = static_cast<char*>(sets[i].out);
+    d.row_bytes = sets[i].row_bytes;
+    d.in_stride = sets[i].in_stride;
+    d.out_stride = sets[i].out_stride;
+    d.unit = access_unit(sets[i]);
+    d.warp_per_row = (d.unit == 16 && d.row_bytes >= 256) ? 1 : 0;
+    d.rows_per_block = d.warp_per_row ? kWarps * kRowsPerWarp : kThreads;
+    d.block_begin = static_cast<int32_t>(blocks);
+    blocks += (n_kept + d.rows_per_block - 1) / d.rows_per_block;
+  }
+  if (blocks > 0x7fffffff) return cudaErrorInvalidConfiguration;
+  k_compact<<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(P, kept_idx, n_kept, n_tokens,
+                                                              ws_at<DevStatus>(ws, p.status));
+  return cudaGetLastError();
+}
+
+}  // namespace avtp

@@ -1,0 +1,183 @@
+// Layout validation and per-call bookkeeping, run once at the start of every
+// entry point that reads the layout. One CTA: the layout arrays are small
+// (requests and images, not tokens), except the optional text index list.
+//
+// Writes into the workspace: the status word, vis_cu (visual-token prefix over
+// all images), img_req (request of each image), and optionally the global
+// budgets B_r = floor(r_base * N_vis + 0.5) (paper §3.3.3 base keep ratio),
+// out_cu_seqlens, and the text-query bookkeeping of the attention criterion.
+#include "avtp_internal.cuh"
+
+namespace avtp {
+namespace {
+
+constexpr int kPrepThreads = 1024;
+
+// Block-wide exclusive scan of value(i), i in [0, n): out[i] = sum_{j<i}, out[n] = total.
+template <typename T, typename F>
+__device__ T block_exclusive_scan(int n, F value, T* out, T* s_warp) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  T carry = 0;
+  for (int base = 0; base < n; base += blockDim.x) {
+    const int i = base + threadIdx.x;
+    const T v = (i < n) ? value(i) : T(0);
+    T x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      T y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) s_warp[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+      T w = (lane < nwarps) ? s_warp[lane] : T(0);
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        T y = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += y;
+      }
+      s_warp[lane] = w;
+    }
+    __syncthreads();
+    const T warp_prefix = (warp > 0) ? s_warp[warp - 1] : T(0);
+    if (i < n) out[i] = carry + warp_prefix + x - v;
+    const T chunk_total = s_warp[nwarps - 1];
+    __syncthreads();
+    carry += chunk_total;
+  }
+  if (threadIdx.x == 0) out[n] = carry;
+  __syncthreads();
+  return carry;
+}
+
+__global__ void __launch_bounds__(kPrepThreads)
+k_prep(PrepArgs a, DevStatus* st, int32_t* vis_cu, int32_t* img_req, int32_t* req_budget, int32_t* text_idx,
+       int32_t* text_cu, int32_t* qtile_cu, int32_t* ktile_cu, int q_tile) {
+  __shared__ int s_err, s_detail;
+  __shared__ int32_t s_warp[32];
+  const int tid = threadIdx.x;
+  const int R = a.L.n_requests, NI = a.L.n_images;
+  const int64_t T = a.L.n_tokens;
+  const int32_t* cu = a.L.cu_seqlens;
+  const int32_t* icu = a.L.img_cu;
+  const int32_t* ist = a.L.img_start;
+  const int32_t* iln = a.L.img_len;
+  if (tid == 0) { s_err = 0; s_detail = -1; }
+  __syncthreads();
+  auto fail = [&](int code, int detail) {
+    if (atomicCAS(&s_err, 0, code) == 0) s_detail = detail;
+  };
+
+  // Phase 0: offsets arrays.
+  if (tid == 0) {
+    if (cu[0] != 0 || static_cast<int64_t>(cu[R]) != T || icu[0] != 0 || icu[R] != NI) fail(AVTP_ERR_DEVICE_INPUT, -1);
+  }
+  for (int r = tid; r < R; r += blockDim.x) {
+    if (cu[r + 1] < cu[r] || icu[r + 1] < icu[r]) fail(AVTP_ERR_DEVICE_INPUT, r);
+    else if (icu[r + 1] - icu[r] > kMaxImagesPerRequest) fail(AVTP_ERR_RANGE, r);
+  }
+  __syncthreads();
+
+  // Phase 1: image spans (inside their request, >= 1 token, sorted, disjoint).
+  if (s_err == 0) {
+    for (int i = tid; i < NI; i += blockDim.x) {
+      const int r = upper_index(icu, R, i);
+      const int64_t Tr = static_cast<int64_t>(cu[r + 1]) - cu[r];
+      const int64_t s0 = ist[i], n0 = iln[i];
+      bool bad = n0 < 1 || s0 < 0 || s0 + n0 > Tr;
+      if (!bad && i > icu[r]) bad = s0 < static_cast<int64_t>(ist[i - 1]) + iln[i - 1];
+      if (bad) fail(AVTP_ERR_DEVICE_INPUT, i);
+      img_req[i] = r;
+    }
+  }
+  __syncthreads();
+
+  if (s_err == 0) {
+    // Phase 2: visual prefix over all images.
+    block_exclusive_scan<int32_t>(NI, [&](int i) { return iln[i]; }, vis_cu, s_warp);
+    for (int r = tid; r < R; r += blockDim.x) {
+      if (vis_cu[icu[r + 1]] - vis_cu[icu[r]] > kMaxVisualPerRequest) fail(AVTP_ERR_RANGE, r);
+    }
+    __syncthreads();
+  }
+
+  if (s_err == 0 && a.keep_ratio != nullptr) {
+    // Phase 3: global budgets B_r and the packed offsets of the pruned batch.
+    for (int r = tid; r < R; r += blockDim.x) {
+      const float kr = a.keep_ratio[r];
+      const int32_t nvis = vis_cu[icu[r + 1]] - vis_cu[icu[r]];
+      if (!(kr >= 0.f && kr <= 1.f)) {
+        fail(AVTP_ERR_DEVICE_INPUT, r);
+        req_budget[r] = 0;
+      } else {
+        const double x = __dadd_rn(__dmul_rn(static_cast<double>(kr), static_cast<double>(nvis)), 0.5);
+        req_budget[r] = static_cast<int32_t>(floor(x));
+      }
+    }
+    __syncthreads();
+    if (a.out_cu_seqlens != nullptr) {
+      block_exclusive_scan<int32_t>(
+          R,
+          [&](int r) {
+            const int32_t nvis = vis_cu[icu[r + 1]] - vis_cu[icu[r]];
+            return req_budget[r] + (cu[r + 1] - cu[r] - nvis);
+          },
+          a.out_cu_seqlens, s_warp);
+    }
+  }
+
+  if (s_err == 0 && a.build_text_tiles) {
+    // Phase 4: text ordinals. Text ordinal of packed token t = t - (visual tokens before t).
+    for (int r = tid; r <= R; r += blockDim.x) text_cu[r] = cu[r] - vis_cu[icu[r]];
+    __syncthreads();
+    const int lane = tid & 31, warp = tid >> 5, nwarps = blockDim.x >> 5;
+    for (int run = warp; run < NI + R; run += nwarps) {
+      int r, p0, p1, base;
+      if (run < NI) {  // text after image `run`, up to the next image or the request end
+        const int i = run;
+        r = img_req[i];
+        const int Tr = cu[r + 1] - cu[r];
+        p0 = ist[i] + iln[i];
+        p1 = (i + 1 < icu[r + 1]) ? ist[i + 1] : Tr;
+        base = text_cu[r] + p0 - (vis_cu[i + 1] - vis_cu[icu[r]]);
+      } else {  // text before the first image of request r
+        r = run - NI;
+        const int Tr = cu[r + 1] - cu[r];
+        p0 = 0;
+        p1 = (icu[r] < icu[r + 1]) ? ist[icu[r]] : Tr;
+        base = text_cu[r];
+      }
+      for (int p = p0 + lane; p < p1; p += 32) text_idx[base + (p - p0)] = cu[r] + p;
+    }
+    __syncthreads();
+    block_exclusive_scan<int32_t>(
+        R, [&](int r) { return (text_cu[r + 1] - text_cu[r] + q_tile - 1) / q_tile; }, qtile_cu, s_warp);
+    block_exclusive_scan<int32_t>(
+        NI, [&](int i) { return (iln[i] + kAttnKeyTile - 1) / kAttnKeyTile; }, ktile_cu, s_warp);
+  }
+
+  if (s_err == 0 && a.zero_img_sums != nullptr) {
+    for (int i = tid; i < NI; i += blockDim.x) a.zero_img_sums[i] = 0;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    st->code = s_err;
+    st->detail = s_detail;
+    st->layout_ok = (s_err == 0) ? 1 : 0;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s) {
+  const int q_tile = a.q_tile > 0 ? a.q_tile : 1;
+  k_prep<<<1, kPrepThreads, 0, s>>>(a, ws_at<DevStatus>(ws, p.status), ws_at<int32_t>(ws, p.vis_cu),
+                                    ws_at<int32_t>(ws, p.img_req), ws_at<int32_t>(ws, p.req_budget),
+                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.text_idx) : nullptr,
+                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.text_cu) : nullptr,
+                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.qtile_cu) : nullptr,
+                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr, q_tile);
+  return cudaGetLastError();
+}
+
+}  // namespace avtp

@@ -1,0 +1,158 @@
+"""C ABI checks that need no GPU: the library loads, exports every symbol that
+include/avtp.h declares, and its host-side logic (argument validation, output
+sizing, status strings) behaves as documented. No call here reaches a kernel:
+every invalid-argument path returns before the first CUDA call.
+"""
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+from oracle import avtp_oracle as O
+from paper_2608_26806_gb300 import avtp, synth
+from tests.gpu_util import ensure_built
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "avtp.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return ensure_built()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"AVTP_API\s+[\w\s\*]+?\b(avtp_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_stage_entry_points():
+    names = declared_functions()
+    for required in ("avtp_score", "avtp_allocate", "avtp_select", "avtp_compact", "avtp_prune"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", avtp.library_path()], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\bT\s+(avtp_\w+)", out))
+    for name in declared_functions():
+        assert name in exported, name
+        assert hasattr(lib, name)
+        assert name in avtp.SIGNATURES  # the binding wraps each one
+
+
+def test_status_strings(lib):
+    assert avtp.status_string(avtp.OK) == "ok"
+    assert "workspace" in avtp.status_string(avtp.ERR_WORKSPACE)
+    assert avtp.status_string(12345) == "unknown status"
+    assert lib.avtp_version() >= 100
+
+
+def test_kept_count_matches_oracle_budget_rule(lib):
+    rng = np.random.default_rng(17)
+    for _ in range(50):
+        R = int(rng.integers(1, 6))
+        reqs = []
+        for _ in range(R):
+            segs = [("t", int(rng.integers(0, 50)))]
+            for _ in range(int(rng.integers(0, 10))):
+                segs += [("i", int(rng.integers(1, 2000))), ("t", int(rng.integers(0, 4)))]
+            reqs.append(segs)
+        lay = synth.Layout.from_segments(reqs)
+        kr = rng.choice(np.array([0.0, 0.05, 0.125, 0.25, 0.33, 0.5, 0.7, 1.0], dtype=np.float32), size=R)
+        host = dict(cu_seqlens=lay.cu_seqlens, img_cu=lay.img_cu, img_len=lay.img_len)
+        expect = 0
+        vis = lay.n_visual_per_request()
+        for r in range(R):
+            T_r = int(lay.cu_seqlens[r + 1] - lay.cu_seqlens[r])
+            expect += O.global_budget(kr[r], int(vis[r])) + T_r - int(vis[r])
+        assert avtp.kept_count_host(host, kr) == expect
+
+
+def test_kept_count_rejects_bad_ratio(lib):
+    host = dict(cu_seqlens=np.array([0, 10]), img_cu=np.array([0, 1]), img_len=np.array([5]))
+    with pytest.raises(avtp.AVTPError):
+        avtp.kept_count_host(host, np.array([1.5], dtype=np.float32))
+
+
+FAKE = 0x7f0000000000  # a 256-aligned address that is never dereferenced on these paths
+
+
+def _layout(n_req=1, n_img=1, T=100):
+    return avtp._Layout(n_req, n_img, T, FAKE, FAKE, FAKE, FAKE)
+
+
+def _hv_args(hidden=64):
+    a = avtp._ScoreArgs()
+    a.criterion = avtp.CRIT_HIDDEN_VARIATION
+    a.h_cur = a.h_prior = FAKE
+    a.hidden, a.h_cur_stride, a.h_prior_stride = hidden, hidden, hidden
+    return a
+
+
+def _attn_args(d=128, hq=32, hkv=8):
+    a = avtp._ScoreArgs()
+    a.criterion = avtp.CRIT_TEXT_ATTENTION
+    a.q = a.k = FAKE
+    a.n_q_heads, a.n_kv_heads, a.head_dim = hq, hkv, d
+    a.q_stride, a.k_stride = hq * d, hkv * d
+    a.softmax_scale = d ** -0.5
+    return a
+
+
+def _score(lib, lay, args, ws_bytes=1 << 30, ws=FAKE):
+    return lib.avtp_score(ctypes.byref(lay), ctypes.byref(args), FAKE, FAKE, ws, ws_bytes, None)
+
+
+def test_host_validation_of_score_arguments(lib):
+    assert lib.avtp_score(None, ctypes.byref(_hv_args()), FAKE, FAKE, FAKE, 1 << 30, None) == avtp.ERR_INVALID_ARG
+    assert _score(lib, _layout(n_req=0), _hv_args()) == avtp.ERR_INVALID_ARG
+    assert _score(lib, _layout(T=-1), _hv_args()) == avtp.ERR_INVALID_ARG
+    assert _score(lib, _layout(T=1 << 31), _hv_args()) == avtp.ERR_RANGE
+    assert _score(lib, _layout(), _hv_args(hidden=60)) == avtp.ERR_UNSUPPORTED
+    assert _score(lib, _layout(), _attn_args(d=96)) == avtp.ERR_UNSUPPORTED
+    assert _score(lib, _layout(), _attn_args(hq=30, hkv=8)) == avtp.ERR_UNSUPPORTED
+    assert _score(lib, _layout(), _attn_args(hq=128, hkv=1)) == avtp.ERR_UNSUPPORTED  # group > 64 rows
+    bad = _attn_args()
+    bad.softmax_scale = float("nan")
+    assert _score(lib, _layout(), bad) == avtp.ERR_INVALID_ARG
+    misaligned = _hv_args()
+    misaligned.h_cur = FAKE + 8
+    assert _score(lib, _layout(), misaligned) == avtp.ERR_UNSUPPORTED
+    assert _score(lib, _layout(), _hv_args(), ws_bytes=512) == avtp.ERR_WORKSPACE
+    assert _score(lib, _layout(), _hv_args(), ws=FAKE + 16) == avtp.ERR_WORKSPACE
+    crit = _hv_args()
+    crit.criterion = 7
+    assert _score(lib, _layout(), crit) == avtp.ERR_INVALID_ARG
+
+
+def test_host_validation_of_alloc_and_compact_arguments(lib):
+    lay = _layout()
+    for alpha, r_min, r_max in [(float("nan"), 0.05, 0.95), (-1.0, 0.05, 0.95), (2048.0, 0.05, 0.95),
+                                (1.0, 0.5, 0.4), (1.0, -0.1, 0.9), (1.0, 0.1, 1.5)]:
+        aa = avtp._AllocArgs(FAKE, alpha, r_min, r_max, 0)
+        assert lib.avtp_allocate(ctypes.byref(lay), FAKE, ctypes.byref(aa), FAKE, FAKE, FAKE, 1 << 30,
+                                 None) == avtp.ERR_INVALID_ARG
+    rows = (avtp._Rows * 9)()
+    for i in range(9):
+        rows[i] = avtp._Rows(FAKE, FAKE, 16, 16, 16)
+    assert lib.avtp_compact(FAKE, 10, 100, rows, 9, FAKE, 1 << 20, None) == avtp.ERR_INVALID_ARG
+    rows[0] = avtp._Rows(FAKE, FAKE, 32, 16, 32)  # stride shorter than the row
+    assert lib.avtp_compact(FAKE, 10, 100, rows, 1, FAKE, 1 << 20, None) == avtp.ERR_INVALID_ARG
+    rows[0] = avtp._Rows(FAKE, FAKE, 16, 16, 16)
+    assert lib.avtp_compact(FAKE, 10, 100, rows, 1, None, 1 << 20, None) == avtp.ERR_WORKSPACE
+    assert lib.avtp_compact(FAKE, -1, 100, rows, 1, FAKE, 1 << 20, None) == avtp.ERR_INVALID_ARG
+
+
+def test_workspace_size_grows_with_attention_bookkeeping(lib):
+    lay = _layout(n_req=2, n_img=5, T=10000)
+    a = ctypes.c_size_t()
+    b = ctypes.c_size_t()
+    assert lib.avtp_workspace_size(ctypes.byref(lay), ctypes.byref(_hv_args()), ctypes.byref(a)) == avtp.OK
+    assert lib.avtp_workspace_size(ctypes.byref(lay), ctypes.byref(_attn_args()), ctypes.byref(b)) == avtp.OK
+    assert b.value > a.value >= 10000 * 4
+    assert a.value % 256 == 0 and b.value % 256 == 0

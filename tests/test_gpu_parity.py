@@ -1,0 +1,317 @@
+"""GPU parity: every step of the pruning stage, through the C ABI, against the fp64 oracle.
+
+Scores: rel 1e-3 / abs 1e-5 (bf16 inputs, fp32 accumulation). Budgets, kept
+indices and compacted rows: bit-exact when both sides are fed the same fp32
+scores. End to end, index sets may differ only at near-ties of the oracle's
+scores.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import avtp_oracle as O
+from paper_2608_26806_gb300 import avtp, synth
+from tests.gpu_util import (ATOL, RTOL, DevWorkload, assert_scores_close, bits_of, dev_layout, ensure_built,
+                            near_tie)
+
+pytestmark = pytest.mark.gpu
+
+CONFIGS = ["tiny", "llava_ov_7b", "qwen3_vl_8b", "internvl3_5_8b"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    ensure_built()
+
+
+_CACHE = {}
+
+
+def workload(name):
+    if name not in _CACHE:
+        wl = synth.make_workload(name)
+        _CACHE.clear()  # keep one large workload resident at a time
+        _CACHE[name] = (wl, DevWorkload(wl))
+    return _CACHE[name]
+
+
+def oracle_scores(wl, criterion):
+    if criterion == "hidden_variation":
+        return O.score_hidden_variation(wl.layout, wl.h_cur, wl.h_prior)
+    return O.score_text_attention(wl.layout, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
+
+
+# ---------------------------------------------------------------- step 1
+@pytest.mark.parametrize("name", CONFIGS)
+@pytest.mark.parametrize("criterion", ["hidden_variation", "text_attention"])
+def test_score_parity(name, criterion):
+    wl, dw = workload(name)
+    scores, sums = avtp.score(dw.L, criterion, **dw.score_tensors(criterion))
+    torch.cuda.synchronize()
+    got = scores.cpu().numpy()
+    ref = oracle_scores(wl, criterion)
+    vis = wl.layout.visual_mask()
+    assert_scores_close(got, ref, vis)
+    # the fixed-point per-image sums of the GPU's own scores are exact integers
+    assert np.array_equal(sums.cpu().numpy(), O.image_sums(wl.layout, got))
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen3_vl_8b"])
+def test_score_attention_with_supplied_lse(name):
+    wl, dw = workload(name)
+    lse = O.text_lse(wl.layout, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
+    lse_dev = torch.from_numpy(lse.astype(np.float32)).cuda()
+    scores, _ = avtp.score(dw.L, "text_attention", lse=lse_dev, **dw.score_tensors("text_attention"))
+    torch.cuda.synchronize()
+    ref = O.score_text_attention(wl.layout, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale,
+                                 lse=lse.astype(np.float32).astype(np.float64))
+    assert_scores_close(scores.cpu().numpy(), ref, wl.layout.visual_mask())
+
+
+# ---------------------------------------------------------------- step 2
+@pytest.mark.parametrize("name", CONFIGS)
+@pytest.mark.parametrize("relative", [False, True])
+def test_allocate_bit_exact_on_oracle_sums(name, relative):
+    wl, dw = workload(name)
+    crit = "text_attention" if relative else "hidden_variation"
+    s32 = O.to_fp32(oracle_scores(wl, crit))
+    S = O.image_sums(wl.layout, s32)
+    ref = O.allocate(wl.layout, S, wl.keep_ratio, 1.0, 0.05, 0.95, relative)
+    budgets, out_cu = avtp.allocate(dw.L, torch.from_numpy(S).cuda(), dw.keep_ratio, 1.0, 0.05, 0.95, relative)
+    torch.cuda.synchronize()
+    assert np.array_equal(budgets.cpu().numpy(), ref["budgets"])
+    assert np.array_equal(out_cu.cpu().numpy(), ref["out_cu_seqlens"])
+
+
+def test_allocate_bit_exact_random_strong_signal():
+    rng = np.random.default_rng(7)
+    for trial in range(40):
+        R = int(rng.integers(1, 5))
+        reqs = []
+        for _ in range(R):
+            segs = [("t", int(rng.integers(0, 5)))]
+            for _ in range(int(rng.integers(0, 40))):
+                segs += [("i", int(rng.integers(1, 700))), ("t", int(rng.integers(0, 3)))]
+            reqs.append(segs)
+        lay = synth.Layout.from_segments(reqs)
+        n = lay.img_len.astype(np.int64)
+        S = (rng.integers(-2 ** 33, 2 ** 34, size=lay.n_images) * n).astype(np.int64)
+        kr = rng.choice(np.array([0.05, 0.125, 0.25, 0.33, 0.5, 0.9, 1.0], dtype=np.float32), size=R)
+        alpha = float(rng.choice([0.0, 1.0, 2.0, 5.0, 100.0]))
+        relative = bool(trial % 2)
+        r_min, r_max = (0.05, 0.95) if trial % 3 else (0.0, 1.0)
+        ref = O.allocate(lay, S, kr, alpha, r_min, r_max, relative)
+        L = dev_layout(lay)
+        budgets, out_cu = avtp.allocate(L, torch.from_numpy(S).cuda(), torch.from_numpy(kr).cuda(), alpha, r_min,
+                                        r_max, relative)
+        torch.cuda.synchronize()
+        assert np.array_equal(budgets.cpu().numpy(), ref["budgets"]), trial
+        assert np.array_equal(out_cu.cpu().numpy(), ref["out_cu_seqlens"]), trial
+        assert avtp.kept_count_host(L.host, kr) == int(ref["out_cu_seqlens"][-1])
+
+
+# ---------------------------------------------------------------- step 3
+def _select_case(lay, scores_f32, budgets):
+    L = dev_layout(lay)
+    out_cu = np.zeros(lay.n_requests + 1, dtype=np.int32)
+    vis = lay.visual_mask()
+    for r in range(lay.n_requests):
+        a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+        kk = int(budgets[int(lay.img_cu[r]):int(lay.img_cu[r + 1])].sum())
+        out_cu[r + 1] = out_cu[r] + kk + int((~vis[a:b]).sum())
+    n_kept = int(out_cu[-1])
+    kept = avtp.select(L, torch.from_numpy(scores_f32).cuda(), torch.from_numpy(budgets.astype(np.int32)).cuda(),
+                       torch.from_numpy(out_cu).cuda(), n_kept)
+    torch.cuda.synchronize()
+    return kept.cpu().numpy()
+
+
+@pytest.mark.parametrize("name", CONFIGS)
+def test_select_bit_exact_on_oracle_scores(name):
+    wl, dw = workload(name)
+    s32 = O.to_fp32(oracle_scores(wl, "hidden_variation"))
+    ref = O.prune(wl.layout, keep_ratio=wl.keep_ratio, scores_f32=s32)
+    got = _select_case(wl.layout, s32, ref["budgets"])
+    assert np.array_equal(got, ref["kept_idx"])
+
+
+def test_select_edge_cases():
+    rng = np.random.default_rng(3)
+    pool = np.array([0.0, -0.0, 0.5, 0.5, 1.0, -1.0, np.nan, np.inf, -np.inf, 0.25], dtype=np.float32)
+    layouts = [
+        [[("i", 1), ("t", 2), ("i", 1)]],
+        [[("t", 7)], [("i", 5)], [("t", 3), ("i", 9)]],                 # request without images / without text
+        [[("i", 3000), ("t", 1), ("i", 1025), ("i", 1024)]],             # multi-tile images
+        [[("t", 2), ("i", 40), ("t", 5), ("i", 64)]] * 3,
+        [[("i", 2048)]],
+    ]
+    for li, segs in enumerate(layouts):
+        lay = synth.Layout.from_segments(segs)
+        for trial in range(6):
+            T = lay.n_tokens
+            if trial % 3 == 0:
+                sc = rng.choice(pool, size=T).astype(np.float32)            # heavy ties, NaN, inf
+            elif trial % 3 == 1:
+                sc = np.full(T, 0.25, dtype=np.float32)                        # all equal
+            else:
+                sc = rng.standard_normal(T).astype(np.float32)
+            n = lay.img_len
+            budgets = np.array([int(rng.integers(0, v + 1)) for v in n], dtype=np.int32)
+            if trial == 0:
+                budgets = n.copy()           # keep everything
+            if trial == 1:
+                budgets[:] = 0               # keep text only
+            ref = O.select(lay, sc, budgets)
+            got = _select_case(lay, sc, budgets)
+            assert np.array_equal(got, ref), (li, trial)
+
+
+# ---------------------------------------------------------------- step 4
+@pytest.mark.parametrize("row_shape,dtype", [((4096,), torch.bfloat16), ((8, 128), torch.bfloat16),
+                                             ((3,), torch.int16), ((5,), torch.uint8), ((1,), torch.int64),
+                                             ((24,), torch.float32)])
+def test_compact_bit_exact(row_shape, dtype):
+    g = torch.Generator().manual_seed(5)
+    T = 3001
+    if dtype.is_floating_point:
+        src = torch.randn((T,) + row_shape, generator=g).to(dtype)
+    else:
+        src = torch.randint(0, 100, (T,) + row_shape, generator=g).to(dtype)
+    idx = np.sort(np.random.default_rng(1).choice(T, size=1234, replace=False)).astype(np.int32)
+    src_d = src.cuda()
+    out_d = torch.empty((len(idx),) + row_shape, dtype=dtype, device="cuda")
+    avtp.compact(torch.from_numpy(idx).cuda(), T, [(src_d, out_d)])
+    torch.cuda.synchronize()
+    assert torch.equal(out_d.cpu(), src[torch.from_numpy(idx).long()])
+
+
+def test_compact_planes_and_strided_rows():
+    T = 777
+    pos = torch.arange(3 * T, dtype=torch.int32).reshape(3, T)
+    big = torch.randn(T, 3 * 256).to(torch.bfloat16)
+    view = big[:, 256:512]  # row stride 768 elements, row 256 elements
+    idx = torch.arange(0, T, 3, dtype=torch.int32)
+    pos_d, view_d = pos.cuda(), big.cuda()[:, 256:512]
+    out_pos = torch.empty((3, len(idx)), dtype=torch.int32, device="cuda")
+    out_v = torch.empty((len(idx), 256), dtype=torch.bfloat16, device="cuda")
+    avtp.compact(idx.cuda(), T, [(view_d, out_v)] + [(pos_d[p], out_pos[p]) for p in range(3)])
+    torch.cuda.synchronize()
+    assert torch.equal(out_v.cpu(), view[idx.long()])
+    assert torch.equal(out_pos.cpu(), pos[:, idx.long()])
+
+
+# ---------------------------------------------------------------- fused stage
+@pytest.mark.parametrize("name", CONFIGS)
+@pytest.mark.parametrize("criterion", ["hidden_variation", "text_attention"])
+def test_prune_end_to_end(name, criterion):
+    wl, dw = workload(name)
+    relative = criterion == "text_attention"
+    out = avtp.prune(dw.L, criterion, keep_ratio=dw.keep_ratio, keep_ratio_host=wl.keep_ratio,
+                     rows={"hidden": dw.t["h_cur"]}, planes={"pos": dw.t["pos"]}, **dw.score_tensors(criterion))
+    torch.cuda.synchronize()
+    assert avtp.read_device_status(out.workspace) == avtp.OK
+    vis = wl.layout.visual_mask()
+    got_scores = out.scores.cpu().numpy()
+    ref64 = oracle_scores(wl, criterion)
+    assert_scores_close(got_scores, ref64, vis)
+    # steps 2-4 fed the GPU's own scores: bit-exact
+    ref = O.prune(wl.layout, keep_ratio=wl.keep_ratio, scores_f32=got_scores, relative=relative,
+                  rows={"hidden": wl.h_cur}, planes={"pos": wl.pos})
+    assert np.array_equal(out.img_sums[:wl.layout.n_images].cpu().numpy(), ref["img_sums"])
+    assert np.array_equal(out.budgets[:wl.layout.n_images].cpu().numpy(), ref["budgets"])
+    assert np.array_equal(out.out_cu_seqlens.cpu().numpy(), ref["out_cu_seqlens"])
+    assert np.array_equal(out.kept_idx.cpu().numpy(), ref["kept_idx"])
+    assert np.array_equal(bits_of(out.outputs["hidden"]), ref["hidden"])
+    assert np.array_equal(out.outputs["pos"].cpu().numpy(), ref["pos"])
+    # against the oracle end to end: totals equal, budgets within one, swaps only at near-ties
+    own = O.prune(wl.layout, keep_ratio=wl.keep_ratio, scores_f32=O.to_fp32(ref64), relative=relative)
+    assert int(own["out_cu_seqlens"][-1]) == int(ref["out_cu_seqlens"][-1])
+    assert np.all(np.abs(own["budgets"].astype(int) - ref["budgets"].astype(int)) <= 1)
+    s_ref = O.to_fp32(ref64)
+    lay = wl.layout
+    got_set, own_set = set(ref["kept_idx"].tolist()), set(own["kept_idx"].tolist())
+    for r in range(lay.n_requests):
+        for i in range(int(lay.img_cu[r]), int(lay.img_cu[r + 1])):
+            if ref["budgets"][i] != own["budgets"][i]:
+                continue
+            s = int(lay.cu_seqlens[r]) + int(lay.img_start[i])
+            rows = range(s, s + int(lay.img_len[i]))
+            only_gpu = [t for t in rows if t in got_set and t not in own_set]
+            only_ref = [t for t in rows if t in own_set and t not in got_set]
+            assert len(only_gpu) == len(only_ref)
+            for a in only_gpu:
+                assert any(near_tie(float(s_ref[a]), float(s_ref[b])) for b in only_ref), (i, a)
+
+
+def test_prune_repeatable_and_deterministic():
+    wl, dw = workload("qwen3_vl_8b")
+    call = avtp.PruneCall(dw.L, "hidden_variation", keep_ratio=dw.keep_ratio, keep_ratio_host=wl.keep_ratio,
+                          rows={"hidden": dw.t["h_cur"]}, planes={"pos": dw.t["pos"]},
+                          **dw.score_tensors("hidden_variation"))
+    first = None
+    for _ in range(3):
+        b = call.run()
+        torch.cuda.synchronize()
+        snap = (b.scores.cpu().numpy().copy(), b.img_sums.cpu().numpy().copy(), b.kept_idx.cpu().numpy().copy())
+        if first is None:
+            first = snap
+        else:
+            for x, y in zip(first, snap):
+                assert np.array_equal(x, y)
+
+
+# ---------------------------------------------------------------- device-side validation
+def _status_after(fn):
+    ws = avtp.new_workspace(1 << 20)
+    fn(ws)
+    torch.cuda.synchronize()
+    return avtp.read_device_status(ws)
+
+
+def test_device_rejects_bad_spans():
+    h_cur = torch.randn(20, 64, device="cuda").to(torch.bfloat16)
+    for starts, lens in [([0, 10], [12, 5]),      # overlapping spans
+                         ([15], [10]),            # past the request end
+                         ([3], [0])]:             # empty image
+        L = avtp.Layout.from_host([0, 20], [0, len(starts)], starts, lens)
+        st = _status_after(lambda ws: avtp.score(L, "hidden_variation", h_cur=h_cur, h_prior=h_cur, workspace=ws))
+        assert st == avtp.ERR_DEVICE_INPUT
+
+
+def test_device_rejects_bad_keep_ratio_and_budgets():
+    L = avtp.Layout.from_host([0, 20], [0, 1], [2], [10])
+    sums = torch.zeros(1, dtype=torch.int64, device="cuda")
+    st = _status_after(lambda ws: avtp.allocate(L, sums, torch.tensor([1.5], device="cuda"), workspace=ws))
+    assert st == avtp.ERR_DEVICE_INPUT
+    scores = torch.zeros(20, device="cuda")
+    out_cu = torch.tensor([0, 30], dtype=torch.int32, device="cuda")
+    bad_budget = torch.tensor([11], dtype=torch.int32, device="cuda")
+    st = _status_after(lambda ws: avtp.select(L, scores, bad_budget, out_cu, 30, workspace=ws))
+    assert st == avtp.ERR_DEVICE_INPUT
+
+
+def test_device_rejects_out_of_range_kept_index():
+    src = torch.randn(10, 64, device="cuda").to(torch.bfloat16)
+    out = torch.zeros(3, 64, dtype=torch.bfloat16, device="cuda")
+    idx = torch.tensor([1, 10, 2], dtype=torch.int32, device="cuda")
+    st = _status_after(lambda ws: avtp.compact(idx, 10, [(src, out)], workspace=ws))
+    assert st == avtp.ERR_DEVICE_INPUT
+    assert torch.equal(out[0].cpu(), src[1].cpu()) and torch.equal(out[2].cpu(), src[2].cpu())
+
+
+def test_host_rejects_bad_arguments():
+    L = avtp.Layout.from_host([0, 20], [0, 1], [2], [10])
+    x = torch.randn(20, 60, device="cuda").to(torch.bfloat16)  # hidden 60: not a multiple of 8
+    with pytest.raises(avtp.AVTPError) as e:
+        avtp.score(L, "hidden_variation", h_cur=x, h_prior=x)
+    assert e.value.code == avtp.ERR_UNSUPPORTED
+    q = torch.randn(20, 4, 96, device="cuda").to(torch.bfloat16)  # head_dim 96
+    with pytest.raises(avtp.AVTPError) as e:
+        avtp.score(L, "text_attention", q=q, k=q[:, :2].contiguous())
+    assert e.value.code == avtp.ERR_UNSUPPORTED
+    with pytest.raises(avtp.AVTPError) as e:
+        avtp.score(L, "hidden_variation", h_cur=x[:, :56].contiguous(), h_prior=x[:, :56].contiguous(),
+                   workspace=avtp.new_workspace(256))
+    assert e.value.code == avtp.ERR_WORKSPACE
