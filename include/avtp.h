@@ -175,6 +175,29 @@ AVTP_API avtp_status_t avtp_select(const avtp_layout_t* layout, const float* sco
                           const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, void* workspace,
                           size_t workspace_bytes, avtp_stream_t stream);
 
+/* avtp_select without a workspace, for callers that cannot allocate device
+ * memory where they call it: for example an inference engine that reserves all
+ * free HBM for its KV-cache pool up front and gives plugins only their inputs
+ * and outputs, or code running where allocation calls are not allowed. The
+ * paper has no counterpart to this; it is a deployment convenience.
+ * Same inputs, outputs and result as avtp_select. The scratch (about 145 KiB)
+ * is a fixed device array inside the library, held by every GPU that loads
+ * the library until the process exits. Limits: at most
+ * AVTP_NOALLOC_MAX_IMAGES images and AVTP_NOALLOC_MAX_REQUESTS requests;
+ * larger layouts return AVTP_ERR_RANGE before anything is launched.
+ * The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress, which may load the library's GPU module); make that
+ * first call before any stream capture. All calls share the one array, so calls
+ * that overlap on the GPU race and must not be issued; calls ordered on one
+ * stream are fine, since each call rewrites the scratch it reads.
+ * device_status (optional device int32, NULL to skip) receives the device-side
+ * status word of this call (an avtp_status_t value). */
+#define AVTP_NOALLOC_MAX_IMAGES 16384
+#define AVTP_NOALLOC_MAX_REQUESTS 4096
+AVTP_API avtp_status_t avtp_select_noalloc(const avtp_layout_t* layout, const float* scores, const int32_t* budgets,
+                                           const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept,
+                                           int32_t* device_status, avtp_stream_t stream);
+
 /* Step 4 (paper §3.1). For each of the n_sets row sets (at most AVTP_MAX_ROW_SETS):
  * out[j] = in[kept_idx[j]] for j < n_kept. Indices outside [0, n_tokens) are
  * skipped and recorded as AVTP_ERR_DEVICE_INPUT. Position ids with P planes

@@ -82,6 +82,8 @@ SIGNATURES = {
     "avtp_prune": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(_AllocArgs), c_void_p, c_void_p, c_void_p,
                            c_void_p, c_void_p, c_int64, POINTER(_Rows), c_int32, c_void_p, c_size_t,
                            POINTER(c_void_p), c_void_p]),
+    "avtp_select_noalloc": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_void_p,
+                                    c_void_p]),
     "avtp_kept_count_host": (c_int64, [c_void_p, c_void_p, c_void_p, c_void_p, c_int32]),
     "avtp_read_device_status": (c_int, [c_void_p, c_void_p, POINTER(c_int32)]),
     "avtp_status_string": (ctypes.c_char_p, [c_int32]),
@@ -273,6 +275,21 @@ def select(layout: Layout, scores: torch.Tensor, budgets: torch.Tensor, out_cu_s
     lay = layout.c()
     _check(load().avtp_select(ctypes.byref(lay), _ptr(scores), _ptr(budgets), _ptr(out_cu_seqlens), _ptr(kept_idx),
                               int(n_kept), _ptr(workspace), workspace.numel(), _stream(stream)), "avtp_select")
+    return kept_idx[:int(n_kept)]
+
+
+def select_noalloc(layout: Layout, scores: torch.Tensor, budgets: torch.Tensor, out_cu_seqlens: torch.Tensor,
+                   kept_idx: torch.Tensor, n_kept: int, device_status: Optional[torch.Tensor] = None,
+                   stream=None) -> torch.Tensor:
+    """avtp_select_noalloc: avtp_select with the library's fixed scratch instead of a workspace.
+
+    For callers that cannot allocate device memory at the call site; ``kept_idx``
+    (int32, capacity >= n_kept) must be supplied by the caller.
+    """
+    lay = layout.c()
+    _check(load().avtp_select_noalloc(ctypes.byref(lay), _ptr(scores), _ptr(budgets), _ptr(out_cu_seqlens),
+                                      _ptr(kept_idx), int(n_kept), _ptr(device_status), _stream(stream)),
+           "avtp_select_noalloc")
     return kept_idx[:int(n_kept)]
 
 
