@@ -207,10 +207,13 @@ AVTP_API avtp_status_t avtp_compact(const int32_t* kept_idx, int64_t n_kept, int
 
 /* Steps 1-4 fused on one stream. Outputs as in the single steps; scores and
  * img_sums may be NULL (then kept in the workspace). n_kept must equal
- * avtp_kept_count_host() for this layout and these keep ratios.
- * step_events (optional, NULL to skip): 6 cudaEvent_t handles recorded on
- * `stream` before the first kernel and after each step (validation, score,
- * allocate, select, compact), for per-step timing. */
+ * avtp_kept_count_host() for this layout and these keep ratios. Steps 2 and 3
+ * run as one kernel here. The kernels are chained with programmatic dependent
+ * launch (set AVTP_PDL=0 in the environment to launch them plainly).
+ * step_events (optional, NULL to skip): 5 cudaEvent_t handles recorded on
+ * `stream` before the first kernel and after validation, scoring,
+ * allocation+selection and compaction, for per-step timing; recording them
+ * serialises the kernels, so leave it NULL when timing the whole call. */
 AVTP_API avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
                          const avtp_alloc_args_t* alloc_args, float* scores, int64_t* img_sums, int32_t* budgets,
                          int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, const avtp_rows_t* sets,

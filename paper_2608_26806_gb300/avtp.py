@@ -34,6 +34,7 @@ ERR_WORKSPACE = 7
 CRIT_HIDDEN_VARIATION = 0
 CRIT_TEXT_ATTENTION = 1
 MAX_ROW_SETS = 8
+N_STEP_EVENTS = 5
 
 _CRITERIA = {"hidden_variation": CRIT_HIDDEN_VARIATION, "text_attention": CRIT_TEXT_ATTENTION}
 
@@ -390,8 +391,11 @@ class PruneCall:
     def run(self, stream=None, step_events: Optional[Sequence] = None) -> PruneBuffers:
         b = self.buffers
         ev = None
-        if step_events is not None:
-            ev = (c_void_p * 6)(*[int(e.cuda_event) if hasattr(e, "cuda_event") else int(e) for e in step_events])
+        if step_events is not None:  # 5 events: start, after validation, scoring, allocation+selection, compaction
+            if len(step_events) != N_STEP_EVENTS:
+                raise ValueError(f"step_events needs {N_STEP_EVENTS} events")
+            ev = (c_void_p * N_STEP_EVENTS)(*[int(e.cuda_event) if hasattr(e, "cuda_event") else int(e)
+                                              for e in step_events])
         _check(load().avtp_prune(ctypes.byref(self._lay), ctypes.byref(self._sa), ctypes.byref(self._aa),
                                  _ptr(b.scores), _ptr(b.img_sums), _ptr(b.budgets), _ptr(b.out_cu_seqlens),
                                  _ptr(b.kept_idx), b.n_kept, self._sets, self._n_sets, _ptr(b.workspace),

@@ -1,6 +1,7 @@
 // C ABI of the AVTP pruning stage: argument validation, workspace plan and the
 // launch sequence of every entry point. Kernels live in k_*.cu.
 #include <math.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "avtp_internal.cuh"
@@ -113,6 +114,14 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
   }
   p.total = off;
   return p;
+}
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = getenv("AVTP_PDL");
+    return !(v != nullptr && v[0] == '0');
+  }();
+  return on;
 }
 
 int device_sm_count() {
@@ -246,15 +255,13 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   if ((st = record(step_events, 1, s)) != AVTP_OK) return st;
   if ((st = score_impl(layout, score_args, sc, sums, workspace, p, s)) != AVTP_OK) return st;
   if ((st = record(step_events, 2, s)) != AVTP_OK) return st;
-  if ((st = from_cuda(launch_allocate(*layout, sums, *alloc_args, budgets, workspace, p, s))) != AVTP_OK) return st;
-  if ((st = record(step_events, 3, s)) != AVTP_OK) return st;
-  if ((st = from_cuda(launch_select(*layout, sc, budgets, out_cu_seqlens, kept_idx, n_kept, workspace, p, s))) !=
-      AVTP_OK)
+  if ((st = from_cuda(launch_alloc_select(*layout, sums, *alloc_args, budgets, sc, out_cu_seqlens, kept_idx, n_kept,
+                                          workspace, p, s))) != AVTP_OK)
     return st;
-  if ((st = record(step_events, 4, s)) != AVTP_OK) return st;
+  if ((st = record(step_events, 3, s)) != AVTP_OK) return st;
   if ((st = from_cuda(launch_compact(kept_idx, n_kept, layout->n_tokens, sets, n_sets, workspace, p, s))) != AVTP_OK)
     return st;
-  return record(step_events, 5, s);
+  return record(step_events, 4, s);
 }
 
 int64_t avtp_kept_count_host(const int32_t* cu_seqlens, const int32_t* img_cu, const int32_t* img_len,

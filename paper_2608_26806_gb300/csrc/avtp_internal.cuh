@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "avtp.h"
 
 namespace avtp {
@@ -63,10 +65,27 @@ __host__ __device__ __forceinline__ T* ws_at(void* ws, size_t off) {
 
 // ---------------------------------------------------------------- small device helpers
 __device__ __forceinline__ int64_t fixed_point_score(float s) {
-  // rint(fx(s) * 2^32); fx: NaN -> 0, clamp to [-2^10, 2^10]. The product is exact.
+  // rint(fx(s) * 2^32) with fx: NaN -> 0, clamp to [-2^10, 2^10], rounding half to
+  // even. Done on the fp32 bits with integer operations (fp64 is scarce on this
+  // part): s = M * 2^e with a 24-bit integer M, so s * 2^32 = M * 2^(e + 32).
   if (isnan(s)) return 0;
   s = fminf(fmaxf(s, -kFxScoreLimit), kFxScoreLimit);
-  return __double2ll_rn(static_cast<double>(s) * 4294967296.0);
+  const uint32_t b = __float_as_uint(s);
+  const int biased = static_cast<int>((b >> 23) & 0xFFu);
+  if (biased == 0) return 0;  // zero or subnormal: |s * 2^32| < 2^-94
+  const int64_t M = static_cast<int64_t>((b & 0x7FFFFFu) | 0x800000u);
+  const int sh = biased - 127 - 23 + 32;  // s * 2^32 = M * 2^sh, sh <= 19 after the clamp
+  int64_t v;
+  if (sh >= 0) {
+    v = M << sh;
+  } else if (-sh > 25) {
+    v = 0;  // M * 2^sh < 1/2
+  } else {
+    const int rs = -sh;
+    const int64_t q = M >> rs, rem = M & ((int64_t(1) << rs) - 1), half = int64_t(1) << (rs - 1);
+    v = q + ((rem > half || (rem == half && (q & 1))) ? 1 : 0);
+  }
+  return (b >> 31) ? -v : v;
 }
 
 // Order-preserving key: larger score -> larger key; NaN -> 0 (below -inf); -0 == +0.
@@ -94,6 +113,36 @@ __device__ __forceinline__ T warp_sum(T v) {
   return v;
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// A kernel launched with programmatic stream serialization may start before the
+// kernel ahead of it in the stream has finished. It must call pdl_wait() before
+// it reads anything that kernel writes, and every thread calls it before exiting,
+// so that the completion of a grid implies the completion of all grids before it.
+// pdl_trigger() lets the next grid in the stream be scheduled. Without the launch
+// attribute both are no-ops.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// True unless the environment sets AVTP_PDL=0 (read once).
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl,
+                          Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  const bool use = pdl && pdl_enabled();
+  cfg.attrs = use ? attr : nullptr;
+  cfg.numAttrs = use ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 // ---------------------------------------------------------------- launchers (one per kernel)
 struct PrepArgs {
   avtp_layout_t L;
@@ -117,6 +166,11 @@ cudaError_t launch_allocate(const avtp_layout_t& L, const int64_t* img_sums, con
 cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int32_t* budgets,
                           const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, void* ws,
                           const WsPlan& p, cudaStream_t s);
+
+// Budget rule and selection in one kernel (the fused stage).
+cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
+                                int32_t* budgets, const float* scores, const int32_t* out_cu_seqlens,
+                                int32_t* kept_idx, int64_t n_kept, void* ws, const WsPlan& p, cudaStream_t s);
 
 cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
                            int n_sets, void* ws, const WsPlan& p, cudaStream_t s);

@@ -50,6 +50,8 @@ __device__ __forceinline__ void copy_row_thread(const char* src, char* dst, int6
 
 __global__ void __launch_bounds__(kThreads)
 k_compact(CompactParams P, const int32_t* __restrict__ kept_idx, int64_t n_kept, int64_t n_tokens, DevStatus* st) {
+  pdl_wait();  // kept_idx comes from the selection kernel
+  pdl_trigger();
   const int b = blockIdx.x;
   int si = 0;
   while (si + 1 < P.n_sets && b >= P.set[si + 1].block_begin) ++si;
@@ -129,9 +131,8 @@ cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_to
     blocks += (n_kept + d.rows_per_block - 1) / d.rows_per_block;
   }
   if (blocks > 0x7fffffff) return cudaErrorInvalidConfiguration;
-  k_compact<<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(P, kept_idx, n_kept, n_tokens,
-                                                              ws_at<DevStatus>(ws, p.status));
-  return cudaGetLastError();
+  return launch_kernel(k_compact, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0, s, /*pdl=*/true, P,
+                       kept_idx, n_kept, n_tokens, ws_at<DevStatus>(ws, p.status));
 }
 
 }  // namespace avtp

@@ -50,11 +50,20 @@ __device__ T block_exclusive_scan(int n, F value, T* out, T* s_warp) {
   return carry;
 }
 
+// Layout arrays are staged in shared memory when they fit. Kept small (10 KiB) so
+// that this one-CTA kernel can share an SM with a CTA of the scoring kernel,
+// which is launched while this kernel still runs.
+constexpr int kStageInts = 2560;
+
 __global__ void __launch_bounds__(kPrepThreads)
-k_prep(PrepArgs a, DevStatus* st, int32_t* vis_cu, int32_t* img_req, int32_t* req_budget, int32_t* text_idx,
+k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t* req_budget, int32_t* text_idx,
        int32_t* text_cu, int32_t* qtile_cu, int32_t* ktile_cu, int q_tile) {
   __shared__ int s_err, s_detail;
   __shared__ int32_t s_warp[32];
+  __shared__ int32_t s_stage[kStageInts];
+  // The first kernel of a call: it is launched after everything before it in the
+  // stream has finished, so the next kernel may be scheduled at once.
+  pdl_trigger();
   const int tid = threadIdx.x;
   const int R = a.L.n_requests, NI = a.L.n_images;
   const int64_t T = a.L.n_tokens;
@@ -62,6 +71,33 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* vis_cu, int32_t* img_req, int32_t* re
   const int32_t* icu = a.L.img_cu;
   const int32_t* ist = a.L.img_start;
   const int32_t* iln = a.L.img_len;
+  int32_t* vis_cu = g_vis_cu;
+  int32_t* img_req = g_img_req;
+  // Stage the small layout arrays in shared memory: one round trip to global
+  // memory instead of one per dependent step below.
+  const bool staged = 2 * static_cast<int64_t>(R) + 4 * static_cast<int64_t>(NI) + 3 <= kStageInts;
+  if (staged) {
+    int32_t* s_cu = s_stage;
+    int32_t* s_icu = s_cu + (R + 1);
+    int32_t* s_ist = s_icu + (R + 1);
+    int32_t* s_iln = s_ist + NI;
+    int32_t* s_vis = s_iln + NI;
+    int32_t* s_req = s_vis + (NI + 1);
+    for (int j = tid; j <= R; j += blockDim.x) {
+      s_cu[j] = cu[j];
+      s_icu[j] = icu[j];
+    }
+    for (int j = tid; j < NI; j += blockDim.x) {
+      s_ist[j] = ist[j];
+      s_iln[j] = iln[j];
+    }
+    cu = s_cu;
+    icu = s_icu;
+    ist = s_ist;
+    iln = s_iln;
+    vis_cu = s_vis;
+    img_req = s_req;
+  }
   if (tid == 0) { s_err = 0; s_detail = -1; }
   __syncthreads();
   auto fail = [&](int code, int detail) {
@@ -160,6 +196,10 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* vis_cu, int32_t* img_req, int32_t* re
     for (int i = tid; i < NI; i += blockDim.x) a.zero_img_sums[i] = 0;
   }
   __syncthreads();
+  if (staged && s_err == 0) {
+    for (int j = tid; j <= NI; j += blockDim.x) g_vis_cu[j] = vis_cu[j];
+    for (int j = tid; j < NI; j += blockDim.x) g_img_req[j] = img_req[j];
+  }
   if (tid == 0) {
     st->code = s_err;
     st->detail = s_detail;

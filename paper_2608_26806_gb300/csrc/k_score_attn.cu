@@ -56,6 +56,8 @@ k_attn_lse(const __nv_bfloat16* __restrict__ q, int64_t q_stride, const __nv_bfl
   extern __shared__ __align__(16) float sm[];
   __shared__ const __nv_bfloat16* s_rows[kRows];
   __shared__ int32_t s_rpos[kRows];
+  pdl_wait();
+  pdl_trigger();
   if (!st->layout_ok) return;
   const int b = blockIdx.x, g = blockIdx.y;
   if (b >= qtile_cu[R]) return;
@@ -164,6 +166,8 @@ k_attn_mass(const __nv_bfloat16* __restrict__ q, int64_t q_stride, const __nv_bf
   __shared__ const __nv_bfloat16* s_keys[kKT];
   __shared__ int32_t s_rpos[kRows];
   __shared__ float s_rlse[kRows];
+  pdl_wait();
+  pdl_trigger();
   if (!st->layout_ok) return;
   const int b = blockIdx.x, g = blockIdx.y;
   if (b >= ktile_cu[NI]) return;
@@ -249,6 +253,8 @@ k_attn_finalize(const float* __restrict__ partial, int Hq, int Hkv, int64_t T, c
                 const int32_t* __restrict__ img_start, const int32_t* __restrict__ vis_cu,
                 const int32_t* __restrict__ img_req, const int32_t* __restrict__ text_cu, int NI,
                 float* __restrict__ scores, int64_t* __restrict__ img_sums, const DevStatus* st) {
+  pdl_wait();
+  pdl_trigger();
   if (!st->layout_ok) return;
   const int n_vis = vis_cu[NI];
   for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < n_vis;
@@ -300,11 +306,11 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
     float* lse2 = ws_at<float>(ws, p.lse);
     const int64_t q_tiles = L.n_tokens / q_tile + L.n_requests;
     dim3 grid1(static_cast<unsigned>(q_tiles), static_cast<unsigned>(Hkv));
-    k_attn_lse<<<grid1, kThreads, smem, s>>>(static_cast<const __nv_bfloat16*>(sa.q), sa.q_stride,
-                                             static_cast<const __nv_bfloat16*>(sa.k), sa.k_stride, Hq, Hkv, d, c2,
-                                             L.cu_seqlens, L.n_requests, text_idx, text_cu,
-                                             ws_at<int32_t>(ws, p.qtile_cu), q_tile, lse2, L.n_tokens, st);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_kernel(k_attn_lse, grid1, dim3(kThreads), smem, s, /*pdl=*/true,
+                                  static_cast<const __nv_bfloat16*>(sa.q), sa.q_stride,
+                                  static_cast<const __nv_bfloat16*>(sa.k), sa.k_stride, Hq, Hkv, d, c2, L.cu_seqlens,
+                                  L.n_requests, text_idx, text_cu, ws_at<int32_t>(ws, p.qtile_cu), q_tile, lse2,
+                                  L.n_tokens, st);
     if (e != cudaSuccess) return e;
     lse = lse2;
     lse_stride = L.n_tokens;
@@ -317,20 +323,19 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   float* partial = ws_at<float>(ws, p.partial);
   const int64_t k_tiles = L.n_tokens / kKT + L.n_images;
   dim3 grid2(static_cast<unsigned>(k_tiles), static_cast<unsigned>(Hkv));
-  k_attn_mass<<<grid2, kThreads, smem, s>>>(static_cast<const __nv_bfloat16*>(sa.q), sa.q_stride,
-                                            static_cast<const __nv_bfloat16*>(sa.k), sa.k_stride, Hq, Hkv, d, c2,
-                                            L.cu_seqlens, L.img_start, L.img_len, ws_at<int32_t>(ws, p.img_req),
-                                            L.n_images, text_idx, text_cu, ws_at<int32_t>(ws, p.ktile_cu), q_tile, lse,
-                                            lse_stride, lse_mul, partial, L.n_tokens, st);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_kernel(k_attn_mass, grid2, dim3(kThreads), smem, s, /*pdl=*/true,
+                                static_cast<const __nv_bfloat16*>(sa.q), sa.q_stride,
+                                static_cast<const __nv_bfloat16*>(sa.k), sa.k_stride, Hq, Hkv, d, c2, L.cu_seqlens,
+                                L.img_start, L.img_len, ws_at<int32_t>(ws, p.img_req), L.n_images, text_idx, text_cu,
+                                ws_at<int32_t>(ws, p.ktile_cu), q_tile, lse, lse_stride, lse_mul, partial,
+                                L.n_tokens, st);
   if (e != cudaSuccess) return e;
   const int64_t want = (L.n_tokens + kThreads - 1) / kThreads;
   const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
   const int grid3 = static_cast<int>(want < cap ? want : cap);
-  k_attn_finalize<<<grid3, kThreads, 0, s>>>(partial, Hq, Hkv, L.n_tokens, L.cu_seqlens, L.img_start,
-                                             ws_at<int32_t>(ws, p.vis_cu), ws_at<int32_t>(ws, p.img_req), text_cu,
-                                             L.n_images, scores, img_sums, st);
-  return cudaGetLastError();
+  return launch_kernel(k_attn_finalize, dim3(grid3), dim3(kThreads), 0, s, /*pdl=*/true, partial, Hq, Hkv,
+                       L.n_tokens, L.cu_seqlens, L.img_start, ws_at<int32_t>(ws, p.vis_cu),
+                       ws_at<int32_t>(ws, p.img_req), text_cu, L.n_images, scores, img_sums, st);
 }
 
 }  // namespace avtp

@@ -1,18 +1,43 @@
-// Criterion A (paper §3.3.1): I_v = 1 - cos(h^l_v, h^prior_v) for every visual token,
-// plus the fixed-point per-image sums S_i used by the budget rule (§3.3.3).
+// Criterion A (paper §3.3.1): I_v = 1 - cos(h^l_v, h^prior_v) for every visual token.
 //
 // HBM-bound stream: each visual row of h_cur and h_prior is read once (2 x D x 2
-// bytes per token). One warp owns one row at a time and issues 16-byte loads,
-// several per lane in flight, accumulating dot, |a|^2 and |b|^2 in fp32.
-// h_prior is read with an L2 evict-first policy; h_cur with evict-last, because
-// the compaction step reads the kept h_cur rows again right after.
+// bytes per token). Rows are staged through shared memory by bulk asynchronous
+// copies (cp.async.bulk, completion on an mbarrier): every warp runs its own
+// 3-deep pipeline of row chunks (2 x 2 KiB), so about 12 KiB per warp and
+// 192 KiB per SM are in flight, independent of the register file. The warp then
+// accumulates dot, |a|^2 and |b|^2 in fp32 from shared memory.
+//
+// Work is split by visual ordinal: warp w of W takes a contiguous range of
+// visual tokens. Each CTA derives the ordinal -> (image, packed position) map
+// itself from the layout, staged in shared memory, so it needs nothing from the
+// validation kernel and runs alongside it (programmatic dependent launch). Every
+// position is checked to lie in [0, T) before a copy is issued, so a malformed
+// layout cannot make it read out of bounds; the validation kernel reports it.
+// Layouts too large to stage fall back to the validation kernel's prefix arrays.
+//
+// Per-image sums S_i = sum rint(fx(I) * 2^32) (integers, so any order gives the
+// same value) are accumulated per warp over runs of rows of the same image and
+// added to img_sums with one atomic per run. The validation kernel zeroes
+// img_sums, so the first atomic of a warp waits for it; with contiguous ranges
+// that is normally at the end of the warp's work, when it has long finished.
+//
+// L2 policy: h_prior evict-first, h_cur evict-last, because the compaction step
+// reads the kept h_cur rows again right after.
 #include "avtp_internal.cuh"
 
 namespace avtp {
 namespace {
 
-constexpr int kThreads = 512;
-constexpr int kUnroll = 4;  // 16-byte loads per lane per tensor in flight
+constexpr int kWarps = 16;                // warps per CTA, each with its own pipeline
+constexpr int kThreads = kWarps * 32;
+constexpr int kSlots = 3;                 // pipeline depth per warp
+constexpr int kChunkElems = 1024;         // bf16 per tensor per slot (2 KiB)
+constexpr int kChunkBytes = kChunkElems * 2;
+constexpr int kSlotBytes = 2 * kChunkBytes;
+constexpr size_t kSmemBytes = static_cast<size_t>(kWarps) * kSlots * kSlotBytes;  // 192 KiB
+constexpr uint32_t kMaxSpins = 1u << 22;  // bounded mbarrier wait
+constexpr int kStageImages = 2048;        // layouts up to this many images are staged in shared memory
+constexpr int kStageRequests = 512;
 
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
@@ -24,79 +49,272 @@ __device__ __forceinline__ uint64_t policy_evict_last() {
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
-__device__ __forceinline__ uint4 ld_stream(const void* ptr, uint64_t pol) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(ptr), "l"(pol));
-  return v;
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile(
+      "{\n\t.reg .b64 st;\n\t"
+      "mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}" ::"r"(smem_addr(bar)),
+      "r"(bytes)
+      : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::
+          "r"(smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
+      : "memory");
 }
 
-__device__ __forceinline__ void accum8(const uint4& a, const uint4& b, float& dot, float& na, float& nb) {
-  const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
-  const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const float2 fa = __bfloat1622float2(pa[j]);
-    const float2 fb = __bfloat1622float2(pb[j]);
-    dot = fmaf(fa.x, fb.x, dot);
-    dot = fmaf(fa.y, fb.y, dot);
-    na = fmaf(fa.x, fa.x, na);
-    na = fmaf(fa.y, fa.y, na);
-    nb = fmaf(fb.x, fb.x, nb);
-    nb = fmaf(fb.y, fb.y, nb);
+// Ordinal -> packed position map: image i covers visual ordinals [vcu[i], vcu[i+1])
+// and starts at packed position gstart[i].
+struct VisMap {
+  const int32_t* vcu;     // [NI + 1]
+  const int32_t* gstart;  // [NI] (staged) or nullptr (then cu[req[i]] + ist[i])
+  const int32_t* req;     // [NI] (unstaged path)
+  const int32_t* cu;
+  const int32_t* ist;
+  int NI;
+  int64_t n_vis;
+  __device__ int64_t position(int64_t v, int& img) const {
+    if (!(vcu[img] <= v && v < vcu[img + 1])) img = upper_index(vcu, NI, v);
+    const int64_t start = gstart ? gstart[img] : static_cast<int64_t>(cu[req[img]]) + ist[img];
+    return start + (v - vcu[img]);
   }
+};
+
+// Exclusive scan over n values of a shared array, in place, by the whole block; out[n] = total.
+__device__ void block_scan_inplace(int32_t* a, int n, int32_t* s_warp) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int per = (n + kThreads - 1) / kThreads;
+  const int b0 = threadIdx.x * per, b1 = min(n, b0 + per);
+  int32_t sum = 0;
+  for (int j = b0; j < b1; ++j) sum += a[j];
+  int32_t x = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int32_t y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) s_warp[warp] = x;
+  __syncthreads();
+  int32_t pre = 0, tot = 0;
+  for (int w = 0; w < kWarps; ++w) {
+    pre += (w < warp) ? s_warp[w] : 0;
+    tot += s_warp[w];
+  }
+  int32_t run = pre + x - sum;
+  __syncthreads();
+  for (int j = b0; j < b1; ++j) {
+    const int32_t v = a[j];
+    a[j] = run;
+    run += v;
+  }
+  if (threadIdx.x == 0) a[n] = tot;
+  __syncthreads();
 }
 
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 1)
 k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const __nv_bfloat16* __restrict__ h_prior,
-             int64_t prior_stride, int D, const int32_t* __restrict__ cu, const int32_t* __restrict__ img_start,
-             const int32_t* __restrict__ vis_cu, const int32_t* __restrict__ img_req, int n_img,
-             float* __restrict__ scores, int64_t* __restrict__ img_sums, const DevStatus* st) {
-  if (!st->layout_ok) return;
-  const int lane = threadIdx.x & 31;
-  const int warps_per_block = blockDim.x >> 5;
-  const int64_t gwarp = static_cast<int64_t>(blockIdx.x) * warps_per_block + (threadIdx.x >> 5);
-  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * warps_per_block;
-  const int n_vis = vis_cu[n_img];
+             int64_t prior_stride, int D, const int32_t* __restrict__ cu, int R, const int32_t* __restrict__ icu,
+             const int32_t* __restrict__ ist, const int32_t* __restrict__ iln, int NI, int64_t T,
+             const int32_t* __restrict__ prep_vis_cu, const int32_t* __restrict__ prep_img_req,
+             float* __restrict__ scores, int64_t* __restrict__ img_sums, DevStatus* st) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  __shared__ uint64_t bars[kWarps][kSlots];
+  __shared__ int32_t s_vcu[kStageImages + 1];
+  __shared__ int32_t s_gstart[kStageImages];
+  __shared__ int32_t s_icu[kStageRequests + 1];
+  __shared__ int32_t s_warp[kWarps];
+  pdl_trigger();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  unsigned char* wbuf = smem + static_cast<size_t>(warp) * kSlots * kSlotBytes;
+  uint64_t* wbar = bars[warp];
+  if (lane == 0) {
+    for (int s = 0; s < kSlots; ++s) mbar_init(&wbar[s], 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+
+  // ---- ordinal map
+  VisMap map;
+  map.cu = cu;
+  map.ist = ist;
+  map.NI = NI;
+  const bool staged = NI <= kStageImages && R <= kStageRequests;
+  if (staged) {
+    for (int j = threadIdx.x; j <= R; j += kThreads) s_icu[j] = min(max(icu[j], 0), NI);
+    for (int j = threadIdx.x; j < NI; j += kThreads) s_vcu[j] = max(iln[j], 0);
+    __syncthreads();
+    block_scan_inplace(s_vcu, NI, s_warp);
+    for (int j = threadIdx.x; j < NI; j += kThreads) {
+      const int r = upper_index(s_icu, R, j);  // request of image j
+      s_gstart[j] = cu[r] + ist[j];
+    }
+    __syncthreads();
+    map.vcu = s_vcu;
+    map.gstart = s_gstart;
+    map.req = nullptr;
+    map.n_vis = s_vcu[NI];
+  } else {
+    pdl_wait();  // use the validation kernel's prefix arrays
+    if (!st->layout_ok) return;
+    map.vcu = prep_vis_cu;
+    map.gstart = nullptr;
+    map.req = prep_img_req;
+    map.n_vis = prep_vis_cu[NI];
+    __syncwarp();
+  }
   const uint64_t pol_first = policy_evict_first();
   const uint64_t pol_last = policy_evict_last();
-  int img = 0;  // cached image of the previous row (rows visited in increasing order)
-  for (int64_t v = gwarp; v < n_vis; v += nwarps) {
-    if (!(vis_cu[img] <= v && v < vis_cu[img + 1])) img = upper_index(vis_cu, n_img, v);
-    const int r = img_req[img];
-    const int64_t t = static_cast<int64_t>(cu[r]) + img_start[img] + (v - vis_cu[img]);
-    const char* pa = reinterpret_cast<const char*>(h_cur + t * cur_stride);
-    const char* pb = reinterpret_cast<const char*>(h_prior + t * prior_stride);
-    float dot = 0.f, na = 0.f, nb = 0.f;
-    const int nvec = D >> 3;  // 16-byte vectors per row
-    int c = lane;
-    for (; c + 32 * (kUnroll - 1) < nvec; c += 32 * kUnroll) {
-      uint4 a[kUnroll], b[kUnroll];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        a[u] = ld_stream(pa + 16 * static_cast<int64_t>(c + 32 * u), pol_last);
-        b[u] = ld_stream(pb + 16 * static_cast<int64_t>(c + 32 * u), pol_first);
-      }
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) accum8(a[u], b[u], dot, na, nb);
-    }
-    for (; c < nvec; c += 32) {
-      const uint4 a = ld_stream(pa + 16 * static_cast<int64_t>(c), pol_last);
-      const uint4 b = ld_stream(pb + 16 * static_cast<int64_t>(c), pol_first);
-      accum8(a, b, dot, na, nb);
-    }
-    dot = warp_sum(dot);
-    na = warp_sum(na);
-    nb = warp_sum(nb);
+  const int n_chunks = (D + kChunkElems - 1) / kChunkElems;
+  const int64_t n_items = min(max(map.n_vis, int64_t(0)), T);  // visual ordinals (never more than T)
+  const int64_t n_warps = static_cast<int64_t>(gridDim.x) * kWarps;
+  const int64_t per_warp = (n_items + n_warps - 1) / n_warps;
+  const int64_t w0 = (static_cast<int64_t>(blockIdx.x) * kWarps + warp) * per_warp;  // this warp's range
+  const int64_t w1 = min(n_items, w0 + per_warp);
+
+  int64_t issue_v = w0;
+  int issue_chunk = 0;
+  int issue_img = 0;
+  int64_t issue_t = issue_v < w1 ? map.position(issue_v, issue_img) : 0;
+
+  auto issue_valid = [&]() { return issue_v < w1; };
+  auto advance_issue = [&]() {
+    if (++issue_chunk < n_chunks) return;
+    issue_chunk = 0;
+    ++issue_v;
+    if (issue_v < w1) issue_t = map.position(issue_v, issue_img);
+  };
+  auto issue_one = [&](int slot) {
+    const int e0 = issue_chunk * kChunkElems;
+    const int ne = min(kChunkElems, D - e0);
+    const uint32_t bytes = static_cast<uint32_t>(ne) * 2u;
+    unsigned char* dst = wbuf + static_cast<size_t>(slot) * kSlotBytes;
+    // a position outside [0, T) only comes from a malformed layout: read row 0 instead
+    const int64_t t = (issue_t >= 0 && issue_t < T) ? issue_t : 0;
     if (lane == 0) {
-      const float den = fmaxf(sqrtf(na), 1e-8f) * fmaxf(sqrtf(nb), 1e-8f);
-      const float I = 1.f - dot / den;
-      scores[t] = I;
-      atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + img),
-                static_cast<unsigned long long>(fixed_point_score(I)));
+      // order this warp's earlier shared-memory reads of the slot before the async-proxy writes
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_expect_tx(&wbar[slot], 2u * bytes);
+      bulk_g2s(dst, h_cur + t * cur_stride + e0, bytes, &wbar[slot], pol_last);
+      bulk_g2s(dst + kChunkBytes, h_prior + t * prior_stride + e0, bytes, &wbar[slot], pol_first);
+    }
+  };
+
+  __syncwarp();
+  uint32_t phase_bits = 0;  // bit s: parity to wait for on slot s
+  int in_flight = 0;
+  int slot_issue = 0;
+  for (; in_flight < kSlots && issue_valid(); ++in_flight) {
+    issue_one(slot_issue);
+    slot_issue = (slot_issue + 1) % kSlots;
+    advance_issue();
+  }
+  bool timed_out = false;
+  bool waited = false;  // the validation kernel (which zeroes img_sums) is known to be done
+  float dot = 0.f, na = 0.f, nb = 0.f;
+  int slot_take = 0;
+  int64_t take_v = w0;
+  int take_chunk = 0;
+  int take_img = 0;
+  int run_img = -1;     // image of the current run of rows (lane 0's view)
+  int64_t run_sum = 0;  // its fixed-point sum so far
+  auto flush_run = [&]() {
+    if (!waited) {
+      pdl_wait();
+      waited = true;
+    }
+    if (lane == 0 && run_img >= 0)
+      atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + run_img), static_cast<unsigned long long>(run_sum));
+  };
+  while (in_flight > 0) {
+    const uint32_t parity = (phase_bits >> slot_take) & 1u;
+    // warp-uniform bounded wait: a completed phase stays visible, so every lane gets there
+    uint32_t spins = 0;
+    while (!__all_sync(0xffffffffu, mbar_try_wait(&wbar[slot_take], parity))) {
+      if (++spins >= kMaxSpins) { timed_out = true; break; }
+    }
+    if (timed_out) break;
+    phase_bits ^= 1u << slot_take;
+    const int e0 = take_chunk * kChunkElems;
+    const int ne = min(kChunkElems, D - e0);
+    const uint4* a = reinterpret_cast<const uint4*>(wbuf + static_cast<size_t>(slot_take) * kSlotBytes);
+    const uint4* b = reinterpret_cast<const uint4*>(wbuf + static_cast<size_t>(slot_take) * kSlotBytes + kChunkBytes);
+    for (int c = lane; c < (ne >> 3); c += 32) {
+      const uint4 va = a[c], vb = b[c];
+      const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&va);
+      const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&vb);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float2 fa = __bfloat1622float2(pa[j]);
+        const float2 fb = __bfloat1622float2(pb[j]);
+        dot = fmaf(fa.x, fb.x, dot);
+        dot = fmaf(fa.y, fb.y, dot);
+        na = fmaf(fa.x, fa.x, na);
+        na = fmaf(fa.y, fa.y, na);
+        nb = fmaf(fb.x, fb.x, nb);
+        nb = fmaf(fb.y, fb.y, nb);
+      }
+    }
+    __syncwarp();
+    --in_flight;
+    const bool row_done = take_chunk == n_chunks - 1;
+    // refill the slot just consumed
+    if (issue_valid()) {
+      issue_one(slot_take);
+      advance_issue();
+      ++in_flight;
+    }
+    slot_take = (slot_take + 1) % kSlots;
+    if (row_done) {
+      const float d = warp_sum(dot), x = warp_sum(na), y = warp_sum(nb);
+      dot = na = nb = 0.f;
+      const int64_t t = map.position(take_v, take_img);
+      const bool inside = t >= 0 && t < T;
+      const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
+      const float I = 1.f - d / den;
+      if (lane == 0 && inside) scores[t] = I;
+      // run-length accumulation of the per-image sums (take_img is uniform over the warp)
+      if (take_img != run_img) {
+        if (run_img >= 0) flush_run();
+        run_img = take_img;
+        run_sum = 0;
+      }
+      if (inside) run_sum += fixed_point_score(I);
+      take_chunk = 0;
+      ++take_v;
+    } else {
+      ++take_chunk;
     }
   }
+  if (!timed_out && run_img >= 0) flush_run();
+  if (timed_out) {
+    // drain: give the copies still in flight a bounded chance to land before the CTA exits
+    for (int k = 0; k < kSlots; ++k) {
+      const uint32_t parity = (phase_bits >> k) & 1u;
+      for (uint32_t spins = 0; spins < kMaxSpins && !__all_sync(0xffffffffu, mbar_try_wait(&wbar[k], parity));
+           ++spins) {
+      }
+    }
+    pdl_wait();  // the validation kernel resets the status word: record after it
+    if (lane == 0) record_error(st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));
+  }
+  pdl_wait();  // completion of this grid implies completion of the one before it
 }
 
 }  // namespace
@@ -104,15 +322,23 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
 cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
                               int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s) {
   if (L.n_images == 0 || L.n_tokens == 0) return cudaSuccess;
-  const int warps_per_block = kThreads / 32;
-  const int64_t want = (L.n_tokens + warps_per_block - 1) / warps_per_block;
-  const int64_t cap = static_cast<int64_t>(device_sm_count()) * 2;  // 2 x 512 threads per SM
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_score_hvar, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kSmemBytes));
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int64_t want = (L.n_tokens + kWarps - 1) / kWarps;
+  const int64_t cap = static_cast<int64_t>(device_sm_count());  // one 192 KiB CTA per SM
   const int grid = static_cast<int>(want < cap ? want : cap);
-  k_score_hvar<<<grid, kThreads, 0, s>>>(
-      static_cast<const __nv_bfloat16*>(sa.h_cur), sa.h_cur_stride, static_cast<const __nv_bfloat16*>(sa.h_prior),
-      sa.h_prior_stride, sa.hidden, L.cu_seqlens, L.img_start, ws_at<int32_t>(ws, p.vis_cu),
-      ws_at<int32_t>(ws, p.img_req), L.n_images, scores, img_sums, ws_at<DevStatus>(ws, p.status));
-  return cudaGetLastError();
+  cudaError_t e = launch_kernel(k_score_hvar, dim3(grid), dim3(kThreads), kSmemBytes, s, /*pdl=*/true,
+                                static_cast<const __nv_bfloat16*>(sa.h_cur), sa.h_cur_stride,
+                                static_cast<const __nv_bfloat16*>(sa.h_prior), sa.h_prior_stride, sa.hidden,
+                                L.cu_seqlens, L.n_requests, L.img_cu, L.img_start, L.img_len, L.n_images, L.n_tokens,
+                                ws_at<int32_t>(ws, p.vis_cu), ws_at<int32_t>(ws, p.img_req), scores, img_sums,
+                                ws_at<DevStatus>(ws, p.status));
+  return e;
 }
 
 }  // namespace avtp

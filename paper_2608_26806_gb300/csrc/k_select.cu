@@ -2,180 +2,503 @@
 // (paper §3.1: the pruned sequence is an order-preserving subsequence; §3.3.3:
 // image i keeps its k_i most important tokens).
 //
-// One CTA per image, plus one CTA per request for the text before its first image.
-// Ranking: order-preserving 32-bit keys (score descending; NaN lowest; -0 == +0),
-// ties by lower position. A 4-pass 8-bit radix select finds the k-th key K*;
-// tokens above K* are kept, and of those equal to K* the first (by position)
-// k - #{key > K*}. Kept positions are written in order with block-wide scans.
-// The CTA also writes the text run that follows its image.
-#include "avtp_internal.cuh"
+// One CTA (8 warps) per image, plus one per request for the text before its
+// first image. Ranking uses order-preserving 32-bit keys (score descending, NaN
+// lowest, -0 == +0) with ties to the lower position. A radix select finds the
+// k-th key K*: the passes start below the highest bit in which the image's keys
+// differ, use 8-bit digits with per-warp sub-histograms (no contention between
+// warps), and stop as soon as the chosen digit's candidates are all kept. Tokens
+// above K* are kept, and of those equal to K* the first k - #{key > K*} by
+// position; kept positions are written in order after two block scans. The CTA
+// also writes the text run that follows its image.
+//
+// Two kernels: k_select takes the budgets as input (avtp_select); k_alloc_select
+// runs the budget rule of avtp_alloc.cuh for the image's request in warp 0 while
+// warps 1-7 stage the keys and build the first histogram, then selects
+// (avtp_prune). Everything that needs only the call's inputs is done before the
+// kernel waits for the scoring kernel, so it overlaps the scoring.
+#include "avtp_alloc.cuh"
 
 namespace avtp {
 namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kItems = 4;
-constexpr int kTile = kThreads * kItems;
+constexpr int kPer = 8;                   // keys per thread in a tile
+constexpr int kKeyCap = kThreads * kPer;  // keys staged in shared memory (2048)
+constexpr unsigned kFull = 0xffffffffu;
 
-// Exclusive block scan of one int per thread; returns the block total via *total.
-__device__ __forceinline__ int block_excl_scan(int v, int* s_warp, int* total) {
+struct SelectArgs {
+  const int32_t* cu;
+  const int32_t* icu;
+  const int32_t* ist;
+  const int32_t* iln;
+  int R;
+  int NI;
+  int64_t T;
+  const float* scores;
+  const int32_t* out_cu;
+  int32_t* kept_idx;
+  int64_t n_kept;
+  const int32_t* vis_cu;
+  const int32_t* img_req;
+  DevStatus* st;
+};
+
+struct SelShared {
+  __align__(16) uint32_t keys[kKeyCap];
+  int hist[kWarps][256];
+  int wsum[kWarps];
+  uint32_t wmin[kWarps], wmax[kWarps];
+  int digit, above, count;
+  // hand-over from the warps of the fused kernel
+  uint32_t kmin, kmax;
+  int k, before, total, alloc_ok, vis_before, n_vis;
+};
+
+// Named barrier for warps 1..7 (224 threads) while warp 0 runs the budget rule.
+__device__ __forceinline__ void bar_workers() { asm volatile("bar.sync 1, 224;" ::: "memory"); }
+
+// Inclusive scan of v over the block in thread order; the block total goes to *total.
+// Out of line: called several times per kernel, so its code is fetched once.
+__device__ __noinline__ int block_incl_scan(int v, int* wsum, int* total) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int x = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    const int y = __shfl_up_sync(kFull, x, o);
     if (lane >= o) x += y;
   }
-  __syncthreads();
-  if (lane == 31) s_warp[warp] = x;
+  __syncthreads();  // wsum may still be read by a previous scan
+  if (lane == 31) wsum[warp] = x;
   __syncthreads();
   int pre = 0, tot = 0;
 #pragma unroll
   for (int w = 0; w < kWarps; ++w) {
-    const int t = s_warp[w];
-    pre += (w < warp) ? t : 0;
+    const int t = wsum[w];
+    pre += w < warp ? t : 0;
     tot += t;
   }
   *total = tot;
-  return pre + x - v;
+  return pre + x;
 }
 
-__device__ __forceinline__ int block_sum_int(int v, int* s_warp) {
+struct KeySource {
+  const float* sc;
+  const uint32_t* staged;  // nullptr: read from global
+  __device__ __forceinline__ uint32_t operator()(int j) const { return staged ? staged[j] : rank_key(sc[j]); }
+};
+
+// One histogram pass over the candidates (key & mask) == prefix, digit = (key >> shift) & dmask,
+// into the calling warp's sub-histogram (cleared by the caller). Threads take keys tid, tid+nthreads, ...
+__device__ __noinline__ void hist_pass(const KeySource& key_at, int n, uint32_t mask, uint32_t prefix, int shift,
+                                          uint32_t dmask, int* my_hist, int tid, int nthreads) {
+  for (int j = tid; j < n; j += nthreads) {
+    const uint32_t key = key_at(j);
+    if ((key & mask) == prefix) atomicAdd(&my_hist[(key >> shift) & dmask], 1);
+  }
+}
+
+// From the sub-histograms, the digit holding the `remaining`-th largest candidate.
+// All threads call; the answer is left in sh.digit / sh.above / sh.count.
+__device__ __noinline__ void choose_digit(SelShared& sh, int remaining) {
+  const int d = 255 - static_cast<int>(threadIdx.x);  // thread order = descending digits
+  int c = 0;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) c += sh.hist[w][d];
   int tot;
-  block_excl_scan(v, s_warp, &tot);
-  return tot;
+  const int incl = block_incl_scan(c, sh.wsum, &tot);
+  const int excl = incl - c;
+  if (excl < remaining && remaining <= incl) {
+    sh.digit = d;
+    sh.above = excl;
+    sh.count = c;
+  }
+  __syncthreads();
+}
+
+__device__ __forceinline__ int highest_differing_bit(uint32_t kmin, uint32_t kmax) {
+  return kmin == kmax ? -1 : 31 - __clz(kmin ^ kmax);
+}
+__device__ __forceinline__ uint32_t shared_bits_mask(int top) {
+  return top < 0 ? 0xffffffffu : (top == 31 ? 0u : ~((2u << top) - 1u));
+}
+
+// Keep the top k of the n tokens whose scores start at sc (packed position t0), in
+// ascending position order, at kept_idx[base ...]. kmin/kmax: range of the keys.
+// With first_pass_done the sub-histograms already hold the first pass.
+__device__ void block_select(const float* __restrict__ sc, int n, int k, int64_t t0, int64_t base,
+                             int32_t* __restrict__ kept_idx, SelShared& sh, bool keys_staged, uint32_t kmin,
+                             uint32_t kmax, bool first_pass_done) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (k >= n) {
+    for (int j = tid; j < n; j += kThreads) kept_idx[base + j] = static_cast<int32_t>(t0 + j);
+    return;
+  }
+  if (k <= 0) return;
+  const KeySource key_at{sc, keys_staged ? sh.keys : nullptr};
+  const int top = highest_differing_bit(kmin, kmax);
+  uint32_t mask = shared_bits_mask(top);
+  uint32_t prefix = kmin & mask;
+  int remaining = k;
+  bool have_hist = first_pass_done;
+  for (int hi = top; hi >= 0; hi -= 8) {
+    const int shift = hi >= 7 ? hi - 7 : 0;
+    const uint32_t dmask = (2u << (hi - shift)) - 1u;
+    if (!have_hist) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) sh.hist[warp][lane * 8 + q] = 0;
+      __syncwarp();
+      hist_pass(key_at, n, mask, prefix, shift, dmask, sh.hist[warp], tid, kThreads);
+    }
+    have_hist = false;
+    __syncthreads();
+    choose_digit(sh, remaining);
+    prefix |= static_cast<uint32_t>(sh.digit) << shift;
+    mask |= dmask << shift;
+    remaining -= sh.above;
+    const bool done = remaining == sh.count;  // every candidate left is kept
+    __syncthreads();                          // sh.digit/above/count and the histograms are reused
+    if (done) break;
+  }
+  // kept: (key & mask) > prefix, or (key & mask) == prefix among the first `remaining` by position
+  const uint32_t kstar = prefix;
+  const int need_eq = remaining;
+
+  // ---- ordered write: tiles of kKeyCap positions, thread t owns kPer consecutive ones
+  int eq_carry = 0, out_carry = 0;
+  for (int b0 = 0; b0 < n; b0 += kKeyCap) {
+    uint32_t key[kPer];
+    int n_eq = 0;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      const int j = b0 + tid * kPer + q;
+      key[q] = j < n ? (key_at(j) & mask) : 0u;
+      n_eq += (j < n && key[q] == kstar) ? 1 : 0;
+    }
+    int eq_tot;
+    int eq_rank = eq_carry + block_incl_scan(n_eq, sh.wsum, &eq_tot) - n_eq;
+    uint32_t keep_bits = 0;
+    int n_keep = 0;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      const int j = b0 + tid * kPer + q;
+      bool kp = false;
+      if (j < n) {
+        if (key[q] > kstar) {
+          kp = true;
+        } else if (key[q] == kstar) {
+          kp = eq_rank < need_eq;
+          ++eq_rank;
+        }
+      }
+      keep_bits |= (kp ? 1u : 0u) << q;
+      n_keep += kp ? 1 : 0;
+    }
+    int keep_tot;
+    int o = out_carry + block_incl_scan(n_keep, sh.wsum, &keep_tot) - n_keep;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      if ((keep_bits >> q) & 1u) kept_idx[base + o++] = static_cast<int32_t>(t0 + b0 + tid * kPer + q);
+    }
+    eq_carry += eq_tot;
+    out_carry += keep_tot;
+  }
+}
+
+// Stage the image's keys (when they fit) and find their range; all threads call.
+__device__ void stage_and_range(const float* __restrict__ sc, int n, bool stage, SelShared& sh, uint32_t* kmin_out,
+                                uint32_t* kmax_out) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t lo = 0xffffffffu, hi = 0u;
+  if (stage) {
+    uint32_t v[kPer];
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {  // all loads in flight at once
+      const int j = tid + q * kThreads;
+      v[q] = j < n ? rank_key(sc[j]) : 0u;
+    }
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      const int j = tid + q * kThreads;
+      if (j < n) {
+        sh.keys[j] = v[q];
+        lo = min(lo, v[q]);
+        hi = max(hi, v[q]);
+      }
+    }
+  } else {
+    for (int j = tid; j < n; j += kThreads) {
+      const uint32_t key = rank_key(sc[j]);
+      lo = min(lo, key);
+      hi = max(hi, key);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = min(lo, __shfl_xor_sync(kFull, lo, o));
+    hi = max(hi, __shfl_xor_sync(kFull, hi, o));
+  }
+  if (lane == 0) {
+    sh.wmin[warp] = lo;
+    sh.wmax[warp] = hi;
+  }
+  __syncthreads();
+  lo = sh.wmin[0];
+  hi = sh.wmax[0];
+#pragma unroll
+  for (int w = 1; w < kWarps; ++w) {
+    lo = min(lo, sh.wmin[w]);
+    hi = max(hi, sh.wmax[w]);
+  }
+  *kmin_out = lo;
+  *kmax_out = hi;
+}
+
+// Text before the first image of request r (the whole request if it has none).
+__device__ void leading_text(const SelectArgs& a, int r) {
+  const int Tr = a.cu[r + 1] - a.cu[r];
+  const int first = (a.icu[r] < a.icu[r + 1]) ? a.ist[a.icu[r]] : Tr;
+  const int64_t base = a.out_cu[r];
+  if (base < 0 || base + first > a.out_cu[r + 1] || static_cast<int64_t>(a.out_cu[r + 1]) > a.n_kept) {
+    if (threadIdx.x == 0) record_error(a.st, AVTP_ERR_DEVICE_INPUT, r);
+    return;
+  }
+  for (int p = threadIdx.x; p < first; p += kThreads) a.kept_idx[base + p] = a.cu[r] + p;
 }
 
 __global__ void __launch_bounds__(kThreads)
-k_select(const int32_t* __restrict__ cu, const int32_t* __restrict__ icu, const int32_t* __restrict__ ist,
-         const int32_t* __restrict__ iln, int R, int NI, const float* __restrict__ scores,
-         const int32_t* __restrict__ budgets, const int32_t* __restrict__ out_cu, int32_t* __restrict__ kept_idx,
-         int64_t n_kept, const int32_t* __restrict__ vis_cu, const int32_t* __restrict__ img_req, DevStatus* st) {
-  __shared__ int s_hist[256];
-  __shared__ int s_warp[kWarps];
-  __shared__ int s_digit, s_above;
-  if (!st->layout_ok) return;
-  const int tid = threadIdx.x;
+k_select(SelectArgs a, const int32_t* __restrict__ budgets) {
+  __shared__ SelShared sh;
+  pdl_wait();
+  pdl_trigger();
+  if (!a.st->layout_ok) return;
   const int b = blockIdx.x;
-
-  if (b >= NI) {  // text before the first image of request r (the whole request if it has none)
-    const int r = b - NI;
-    const int Tr = cu[r + 1] - cu[r];
-    const int first = (icu[r] < icu[r + 1]) ? ist[icu[r]] : Tr;
-    const int64_t base = out_cu[r];
-    if (base < 0 || base + first > out_cu[r + 1] || static_cast<int64_t>(out_cu[r + 1]) > n_kept) {
-      if (tid == 0) record_error(st, AVTP_ERR_DEVICE_INPUT, r);
-      return;
-    }
-    for (int p = tid; p < first; p += kThreads) kept_idx[base + p] = cu[r] + p;
+  if (b >= a.NI) {
+    leading_text(a, b - a.NI);
     return;
   }
-
   const int i = b;
-  const int r = img_req[i];
-  const int i0 = icu[r], i1 = icu[r + 1];
-  // kept tokens of earlier images of this request, and the request's total; validate budgets
+  const int r = a.img_req[i];
+  const int i0 = a.icu[r], i1 = a.icu[r + 1];
   int before = 0, total = 0, bad = 0;
-  for (int j = i0 + tid; j < i1; j += kThreads) {
+  for (int j = i0 + threadIdx.x; j < i1; j += kThreads) {
     const int kj = budgets[j];
-    bad |= (kj < 0 || kj > iln[j]);
+    bad |= (kj < 0 || kj > a.iln[j]);
     total += kj;
     before += (j < i) ? kj : 0;
   }
-  before = block_sum_int(before, s_warp);
-  total = block_sum_int(total, s_warp);
-  bad = block_sum_int(bad, s_warp);
-  const int Tr = cu[r + 1] - cu[r];
-  const int ntxt = Tr - (vis_cu[i1] - vis_cu[i0]);
-  if (bad || out_cu[r] < 0 || out_cu[r + 1] - out_cu[r] != total + ntxt ||
-      static_cast<int64_t>(out_cu[r + 1]) > n_kept) {
-    if (tid == 0) record_error(st, AVTP_ERR_DEVICE_INPUT, i);
+  int sb, st, sbad;
+  block_incl_scan(before, sh.wsum, &sb);
+  block_incl_scan(total, sh.wsum, &st);
+  block_incl_scan(bad, sh.wsum, &sbad);
+  if (sbad) {
+    if (threadIdx.x == 0) record_error(a.st, AVTP_ERR_DEVICE_INPUT, i);
     return;
   }
-  const int s0 = ist[i], n = iln[i], k = budgets[i];
-  const int64_t base = static_cast<int64_t>(out_cu[r]) + (s0 - (vis_cu[i] - vis_cu[i0])) + before;
-  const int64_t t0 = static_cast<int64_t>(cu[r]) + s0;  // packed position of the image's first token
-  const float* sc = scores + t0;
+  const int Tr = a.cu[r + 1] - a.cu[r];
+  const int ntxt = Tr - (a.vis_cu[i1] - a.vis_cu[i0]);
+  if (a.out_cu[r] < 0 || a.out_cu[r + 1] - a.out_cu[r] != st + ntxt ||
+      static_cast<int64_t>(a.out_cu[r + 1]) > a.n_kept) {
+    if (threadIdx.x == 0) record_error(a.st, AVTP_ERR_DEVICE_INPUT, i);
+    return;
+  }
+  const int s0 = a.ist[i], n = a.iln[i], k = budgets[i];
+  const int64_t base = static_cast<int64_t>(a.out_cu[r]) + (s0 - (a.vis_cu[i] - a.vis_cu[i0])) + sb;
+  const int64_t t0 = static_cast<int64_t>(a.cu[r]) + s0;
+  const bool stage = n <= kKeyCap;
+  uint32_t kmin, kmax;
+  stage_and_range(a.scores + t0, n, stage, sh, &kmin, &kmax);
+  block_select(a.scores + t0, n, k, t0, base, a.kept_idx, sh, stage, kmin, kmax, false);
+  const int e = s0 + n;
+  const int nxt = (i + 1 < i1) ? a.ist[i + 1] : Tr;
+  for (int p = e + threadIdx.x; p < nxt; p += kThreads) a.kept_idx[base + k + (p - e)] = a.cu[r] + p;
+}
 
-  if (k == n) {
-    for (int j = tid; j < n; j += kThreads) kept_idx[base + j] = static_cast<int32_t>(t0 + j);
-  } else if (k > 0) {
-    // ---- radix select of the k-th largest key
-    uint32_t prefix = 0, mask = 0;
-    int remaining = k;
-    for (int shift = 24; shift >= 0; shift -= 8) {
-      s_hist[tid] = 0;  // kThreads == 256 bins
-      __syncthreads();
-      for (int base_j = 0; base_j < n; base_j += kTile) {
-#pragma unroll
-        for (int it = 0; it < kItems; ++it) {
-          const int j = base_j + tid * kItems + it;
-          if (j < n) {
-            const uint32_t key = rank_key(sc[j]);
-            if ((key & mask) == prefix) atomicAdd(&s_hist[(key >> shift) & 255u], 1);
-          }
-        }
-      }
-      __syncthreads();
-      // thread t looks at digit 255 - t; inclusive prefix = count with digit >= 255 - t
-      const int c = s_hist[255 - tid];
-      int tot;
-      const int excl = block_excl_scan(c, s_warp, &tot);
-      if (excl < remaining && remaining <= excl + c) {
-        s_digit = 255 - tid;
-        s_above = excl;
-      }
-      __syncthreads();
-      prefix |= static_cast<uint32_t>(s_digit) << shift;
-      mask |= 0xFFu << shift;
-      remaining -= s_above;
-      __syncthreads();
-    }
-    const uint32_t kstar = prefix;
-    const int need_eq = remaining;  // tokens equal to K* to keep, lowest positions first
-    // ---- ordered write
-    int eq_carry = 0, out_carry = 0;
-    for (int base_j = 0; base_j < n; base_j += kTile) {
-      uint32_t key[kItems];
-      int n_eq = 0;
-#pragma unroll
-      for (int it = 0; it < kItems; ++it) {
-        const int j = base_j + tid * kItems + it;
-        key[it] = (j < n) ? rank_key(sc[j]) : 0u;
-        n_eq += (j < n && key[it] == kstar) ? 1 : 0;
-      }
-      int eq_tot;
-      int eq_rank = eq_carry + block_excl_scan(n_eq, s_warp, &eq_tot);
-      bool keep[kItems];
-      int n_keep = 0;
-#pragma unroll
-      for (int it = 0; it < kItems; ++it) {
-        const int j = base_j + tid * kItems + it;
-        bool kp = false;
-        if (j < n) {
-          if (key[it] > kstar) kp = true;
-          else if (key[it] == kstar) { kp = eq_rank < need_eq; ++eq_rank; }
-        }
-        keep[it] = kp;
-        n_keep += kp ? 1 : 0;
-      }
-      int keep_tot;
-      int o = out_carry + block_excl_scan(n_keep, s_warp, &keep_tot);
-#pragma unroll
-      for (int it = 0; it < kItems; ++it) {
-        const int j = base_j + tid * kItems + it;
-        if (keep[it]) kept_idx[base + o++] = static_cast<int32_t>(t0 + j);
-      }
-      eq_carry += eq_tot;
-      out_carry += keep_tot;
+struct AllocParams {
+  const int64_t* img_sums;
+  const float* keep_ratio;
+  float alpha, r_min, r_max;
+  int relative;
+  int32_t* budgets;  // output: each CTA writes its own image's budget
+  int m_cap;
+};
+
+__global__ void __launch_bounds__(kThreads)
+k_alloc_select(SelectArgs a, AllocParams ap) {
+  extern __shared__ __align__(16) unsigned char dsmem[];  // budget scratch for requests of > 32 images
+  __shared__ SelShared sh;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int b = blockIdx.x;
+  const WarpAllocSmem wsm = carve_warp_alloc(dsmem, ap.m_cap);
+
+  // ---- set-up from the call's inputs only, overlapped with the scoring kernel.
+  // The layout is not validated yet, so every index is clamped; nothing here is
+  // used unless the validation kernel accepts the layout.
+  int r = 0, i0 = 0, m = 0, li = 0;
+  int32_t s0 = 0, n = 0, nxt = 0, Tr = 0;
+  int64_t t0 = 0;
+  if (b < a.NI) {
+    r = upper_index(a.icu, a.R, b);
+    i0 = min(max(a.icu[r], 0), a.NI);
+    const int i1 = min(max(a.icu[r + 1], i0), a.NI);
+    m = min(i1 - i0, ap.m_cap);
+    if (m > 0) {
+      li = min(max(b - i0, 0), m - 1);
+      Tr = a.cu[r + 1] - a.cu[r];
+      s0 = a.ist[i0 + li];
+      n = a.iln[i0 + li];
+      nxt = (li + 1 < m) ? a.ist[i0 + li + 1] : Tr;
+      t0 = static_cast<int64_t>(a.cu[r]) + s0;
     }
   }
+  // warp 0: the request's sizes and the scalars of the budget rule
+  int32_t N = 0, n_lane = 0, vis_before = 0;
+  int64_t B = 0, Rmin = 0, Rmax = 0;
+  float kr = 0.f;
+  if (warp == 0 && b < a.NI) {
+    int64_t nsum = 0, nbefore = 0;
+    for (int j = lane; j < m; j += 32) {
+      const int32_t nj = a.iln[i0 + j];
+      if (m > 32) wsm.n[j] = nj;
+      else n_lane = nj;
+      nsum += nj;
+      nbefore += j < li ? nj : 0;
+    }
+    N = static_cast<int32_t>(warp_sum(nsum));
+    vis_before = static_cast<int32_t>(warp_sum(nbefore));
+    kr = ap.keep_ratio[r];
+    // B_r = floor(r_base * N_vis + 0.5), each operation rounded once
+    B = static_cast<int64_t>(floor(__dadd_rn(__dmul_rn(static_cast<double>(kr), static_cast<double>(N)), 0.5)));
+    Rmin = ratio_grid(ap.r_min);
+    Rmax = ratio_grid(ap.r_max);
+  }
 
-  // ---- the text run after this image
+  // ---- wait for the scores and per-image sums (and, through them, the validation)
+  pdl_wait();
+  pdl_trigger();
+  if (!a.st->layout_ok) return;
+  if (b >= a.NI) {
+    leading_text(a, b - a.NI);
+    return;
+  }
+  const int i = b;
+  const float* sc = a.scores + t0;
+  const bool stage = n <= kKeyCap;
+  if (warp == 0) {
+    // ---- the budget rule, one warp
+    bool ok;
+    int k, before, total;
+    if (m <= 32) {
+      const int64_t S = lane < m ? ap.img_sums[i0 + lane] : 0;
+      int32_t K;
+      ok = warp_allocate32(m, S, n_lane, B, N, kr, ap.alpha, Rmin, Rmax, ap.relative, &K);
+      k = __shfl_sync(kFull, K, li);
+      before = warp_sum(lane < li ? K : 0);
+      total = warp_sum(lane < m ? K : 0);
+    } else {
+      for (int j = lane; j < m; j += 32) wsm.X[j] = ap.img_sums[i0 + j];
+      __syncwarp();
+      ok = warp_allocate(wsm, m, B, N, kr, ap.alpha, Rmin, Rmax, ap.relative);
+      int bs = 0, ts = 0;
+      for (int j = lane; j < m; j += 32) {
+        ts += wsm.K[j];
+        bs += j < li ? wsm.K[j] : 0;
+      }
+      before = warp_sum(bs);
+      total = warp_sum(ts);
+      k = wsm.K[li];
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) sh.hist[0][lane * 8 + q] = 0;  // warp 0 takes no part in the first pass
+    if (lane == 0) {
+      sh.k = k;
+      sh.before = before;
+      sh.total = total;
+      sh.alloc_ok = ok ? 1 : 0;
+      sh.vis_before = vis_before;
+      sh.n_vis = N;
+    }
+  } else {
+    // ---- warps 1..7: stage the keys, find their range, build the first histogram
+    const int wt = tid - 32;
+    uint32_t lo = 0xffffffffu, hi = 0u;
+    for (int j = wt; j < n; j += kThreads - 32) {
+      const uint32_t key = rank_key(sc[j]);
+      if (stage) sh.keys[j] = key;
+      lo = min(lo, key);
+      hi = max(hi, key);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      lo = min(lo, __shfl_xor_sync(kFull, lo, o));
+      hi = max(hi, __shfl_xor_sync(kFull, hi, o));
+    }
+    if (lane == 0) {
+      sh.wmin[warp] = lo;
+      sh.wmax[warp] = hi;
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) sh.hist[warp][lane * 8 + q] = 0;
+    bar_workers();  // ranges published, keys staged, sub-histograms cleared
+    lo = sh.wmin[1];
+    hi = sh.wmax[1];
+#pragma unroll
+    for (int w = 2; w < kWarps; ++w) {
+      lo = min(lo, sh.wmin[w]);
+      hi = max(hi, sh.wmax[w]);
+    }
+    const int top = highest_differing_bit(lo, hi);
+    if (top >= 0) {
+      const uint32_t mask = shared_bits_mask(top);
+      const int shift = top >= 7 ? top - 7 : 0;
+      const uint32_t dmask = (2u << (top - shift)) - 1u;
+      hist_pass(KeySource{sc, stage ? sh.keys : nullptr}, n, mask, lo & mask, shift, dmask, sh.hist[warp], wt,
+                kThreads - 32);
+    }
+    if (tid == 32) {
+      sh.kmin = lo;
+      sh.kmax = hi;
+    }
+  }
+  __syncthreads();
+  const uint32_t kmin = sh.kmin, kmax = sh.kmax;
+  const int k = sh.k, before = sh.before, total = sh.total, vis_b = sh.vis_before, Nv = sh.n_vis;
+  const bool alloc_ok = sh.alloc_ok != 0;
+  if (!alloc_ok) {
+    if (tid == 0) record_error(a.st, AVTP_ERR_RANGE, r);
+    return;
+  }
+  if (tid == 0) ap.budgets[i] = k;
+  const int32_t out_lo = a.out_cu[r], out_hi = a.out_cu[r + 1];
+  if (out_lo < 0 || out_hi - out_lo != total + (Tr - Nv) || static_cast<int64_t>(out_hi) > a.n_kept) {
+    if (tid == 0) record_error(a.st, AVTP_ERR_DEVICE_INPUT, i);
+    return;
+  }
+  const int64_t base = static_cast<int64_t>(out_lo) + (s0 - vis_b) + before;
+  block_select(sc, n, k, t0, base, a.kept_idx, sh, stage, kmin, kmax, kmin != kmax);
   const int e = s0 + n;
-  const int nxt = (i + 1 < i1) ? ist[i + 1] : Tr;
-  for (int p = e + tid; p < nxt; p += kThreads) kept_idx[base + k + (p - e)] = cu[r] + p;
+  for (int p = e + tid; p < nxt; p += kThreads) a.kept_idx[base + k + (p - e)] = a.cu[r] + p;
+}
+
+SelectArgs make_args(const avtp_layout_t& L, const float* scores, const int32_t* out_cu_seqlens, int32_t* kept_idx,
+                     int64_t n_kept, void* ws, const WsPlan& p) {
+  SelectArgs a;
+  a.cu = L.cu_seqlens;
+  a.icu = L.img_cu;
+  a.ist = L.img_start;
+  a.iln = L.img_len;
+  a.R = L.n_requests;
+  a.NI = L.n_images;
+  a.T = L.n_tokens;
+  a.scores = scores;
+  a.out_cu = out_cu_seqlens;
+  a.kept_idx = kept_idx;
+  a.n_kept = n_kept;
+  a.vis_cu = ws_at<int32_t>(ws, p.vis_cu);
+  a.img_req = ws_at<int32_t>(ws, p.img_req);
+  a.st = ws_at<DevStatus>(ws, p.status);
+  return a;
 }
 
 }  // namespace
@@ -183,11 +506,33 @@ k_select(const int32_t* __restrict__ cu, const int32_t* __restrict__ icu, const 
 cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int32_t* budgets,
                           const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, void* ws,
                           const WsPlan& p, cudaStream_t s) {
-  const int grid = L.n_images + L.n_requests;
-  k_select<<<grid, kThreads, 0, s>>>(L.cu_seqlens, L.img_cu, L.img_start, L.img_len, L.n_requests, L.n_images, scores,
-                                      budgets, out_cu_seqlens, kept_idx, n_kept, ws_at<int32_t>(ws, p.vis_cu),
-                                      ws_at<int32_t>(ws, p.img_req), ws_at<DevStatus>(ws, p.status));
-  return cudaGetLastError();
+  const SelectArgs a = make_args(L, scores, out_cu_seqlens, kept_idx, n_kept, ws, p);
+  return launch_kernel(k_select, dim3(L.n_images + L.n_requests), dim3(kThreads), 0, s, /*pdl=*/true, a, budgets);
+}
+
+cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
+                                int32_t* budgets, const float* scores, const int32_t* out_cu_seqlens,
+                                int32_t* kept_idx, int64_t n_kept, void* ws, const WsPlan& p, cudaStream_t s) {
+  const SelectArgs a = make_args(L, scores, out_cu_seqlens, kept_idx, n_kept, ws, p);
+  AllocParams ap;
+  ap.img_sums = img_sums;
+  ap.keep_ratio = aa.keep_ratio;
+  ap.alpha = aa.alpha;
+  ap.r_min = aa.r_min;
+  ap.r_max = aa.r_max;
+  ap.relative = aa.relative;
+  ap.budgets = budgets;
+  ap.m_cap = L.n_images < kMaxImagesPerRequest ? L.n_images : kMaxImagesPerRequest;
+  if (ap.m_cap < 1) ap.m_cap = 1;
+  // the budget scratch is only used for requests of more than 32 images
+  const size_t smem = ap.m_cap > 32 ? warp_alloc_smem_bytes(ap.m_cap) : 0;
+  if (smem > 16 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(k_alloc_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  return launch_kernel(k_alloc_select, dim3(L.n_images + L.n_requests), dim3(kThreads), smem, s, /*pdl=*/true, a,
+                       ap);
 }
 
 }  // namespace avtp
