@@ -32,12 +32,15 @@ the design notes of the repository):
   fp32-rounded score, with ``fx`` mapping NaN to 0 and clamping to +-2^10, so that
   every summation order gives the same integer.
 * ``Ibar_avg`` is the token-weighted mean ``sum_i S_i / 2^32 / N_vis``.
+* The adaptive ratios are computed in exact integer arithmetic on a 2^-40 grid:
+  means through fixed-point reciprocals ``floor(2^62 / n)``, fp32 alpha and
+  r_base decomposed exactly, one rounding (nearest, ties upward) per product
+  (see ``adaptive_ratio_grid``).
 * The global budget is ``B_r = floor(keep_ratio_r * N_vis_r + 0.5)``.
 * ``relative=1`` replaces the additive rule by ``r_i = r_base*(1 + alpha*(Ibar_i/Ibar_avg - 1))``
   (``r_base`` when ``Ibar_avg == 0``); criterion 1B's raw values are of order
   1/N, where the additive rule would leave every ratio at ``r_base``.
-* Ratios go on a 2^-40 integer grid: ``R_i = rint(clamp(r_i, -2^20, 2^20) * 2^40)``,
-  and likewise ``R_min``, ``R_max`` from the fp32 clamps.
+* The clamps go on the same grid: ``R_min = rint(r_min * 2^40)``, ``R_max`` likewise.
 * A shift lambda (water-fill) restores the clamped total: lambda is the smallest
   grid value with ``G(lambda) = sum_i n_i * clamp(R_i + lambda, R_min, R_max) >= B_r * 2^40``
   on ``[R_min - max R, R_max - min R]`` (an end of that range if none inside
@@ -50,15 +53,14 @@ the design notes of the repository):
 * Top-k order: score descending, position ascending; NaN ranks below -inf;
   -0 equals +0.
 
-The only floating-point steps of the budget rule are the few fp64 operations of
-the ratio formula, each rounded once (Python floats: no fused multiply-add);
-everything after them is exact integer arithmetic. A device implementation that
-rounds each of those operations to nearest reproduces every budget exactly.
+Apart from the fp64 global budget (``kr * N + 0.5``, exact for fp32 ratios and
+N < 2^29) the budget rule is exact integer arithmetic, so a device implementation
+of the same integer steps reproduces every budget exactly.
 """
 from __future__ import annotations
 
 import math
-from typing import Dict, List, Optional, Sequence
+from typing import Dict, List, Optional, Sequence, Tuple
 
 import numpy as np
 
@@ -67,6 +69,7 @@ FX_SCORE_LIMIT = 1024.0  # |score| is clamped to 2^10 before the fixed-point con
 NORM_EPS = 1e-8
 RATIO_FRAC_BITS = 40     # ratios, shifts and kept masses live on a 2^-40 integer grid
 RATIO_LIMIT = 2.0 ** 20  # ratios are saturated to +-2^20 before going on the grid
+RECIP_BITS = 62          # per-image means are taken with floor(2^62 / n) reciprocals
 
 
 # ----------------------------------------------------------------------------
@@ -229,24 +232,67 @@ def _clamp(x, lo, hi):
     return min(max(x, lo), hi)
 
 
-def adaptive_ratios(S: Sequence[int], n: Sequence[int], r_base: float, alpha: float,
-                    relative: bool) -> List[float]:
-    """``r_i`` of paper §3.3.3 from fixed-point sums (fp64, one rounding per operation)."""
-    scale = 1.0 / float(2 ** FX_FRAC_BITS)
-    n_vis = sum(int(x) for x in n)
+def reciprocal(n: int) -> int:
+    """``floor(2^62 / n)``: the fixed-point reciprocal the per-image means are taken with."""
+    return (1 << RECIP_BITS) // int(n)
+
+
+def round_shift(x: int, s: int) -> int:
+    """``x / 2^s`` rounded to nearest with ties upward (``floor(x / 2^s + 1/2)``); s <= 0 shifts left."""
+    if s <= 0:
+        return x << (-s)
+    return (x + (1 << (s - 1))) >> s
+
+
+def fp32_parts(v) -> Tuple[int, int]:
+    """Exact decomposition of an fp32 value as ``M * 2^E`` with an integer ``|M| < 2^24``."""
+    f = float(np.float32(v))
+    if f == 0.0:
+        return 0, 0
+    m, e = math.frexp(f)  # f = m * 2^e with 0.5 <= |m| < 1
+    return int(m * (1 << 24)), e - 24
+
+
+def _sat(x: int, lim: int) -> int:
+    return min(max(x, -lim), lim)
+
+
+def adaptive_ratio_grid(S: Sequence[int], n: Sequence[int], r_base_f32, alpha_f32,
+                        relative: bool) -> List[int]:
+    """The adaptive keep ratios of paper §3.3.3 on the 2^-40 grid, in exact integers.
+
+    Means of the fixed-point sums (units of 2^-32), through reciprocals:
+      ``Ibar_i = round(S_i * floor(2^62 / n_i) / 2^62)``, ``Ibar_avg = round(sum S * floor(2^62 / N) / 2^62)``.
+    Additive rule: ``r_i = r_base + alpha * (Ibar_i - Ibar_avg)``, i.e.
+      ``R_i = R_base + round(alpha * (Ibar_i - Ibar_avg) * 2^8)``.
+    Relative rule: ``r_i = r_base * (1 + alpha * (Ibar_i / Ibar_avg - 1))``, i.e.
+      ``R_i = R_base + round(r_base * alpha * q_i)`` with the ratio on the 2^-40 grid
+      ``q_i = sgn(Ibar_avg) * round((Ibar_i - Ibar_avg) * floor(2^62 / |Ibar_avg|) / 2^22)``
+      saturated to +-2^60, and ``R_i = R_base`` when ``Ibar_avg == 0``.
+    ``R_base = rint(r_base * 2^40)``; fp32 alpha and r_base enter as exact ``M * 2^E``;
+    every product is exact and rounded once; ``R_i`` saturates to +-2^60.
+    """
+    N = sum(int(x) for x in n)
     total = sum(int(x) for x in S)
-    ibar = [(float(int(S[i])) * scale) / float(int(n[i])) for i in range(len(n))]
-    ibar_avg = (float(total) * scale) / float(n_vis)
-    r = []
+    ibar = [round_shift(int(S[i]) * reciprocal(int(n[i])), RECIP_BITS) for i in range(len(n))]
+    avg = round_shift(total * reciprocal(N), RECIP_BITS)
+    Rb = ratio_to_grid(float(np.float32(r_base_f32)))
+    A, E = fp32_parts(alpha_f32)
+    Bm, Be = fp32_parts(r_base_f32)
+    lim = 1 << 60
+    R = []
     for i in range(len(n)):
-        if relative:
-            if ibar_avg == 0.0:
-                r.append(r_base)
-            else:
-                r.append(r_base * (1.0 + alpha * (ibar[i] / ibar_avg - 1.0)))
+        d = ibar[i] - avg
+        if not relative:
+            delta = round_shift(A * d, -(E + 8))
+        elif avg == 0:
+            delta = 0
         else:
-            r.append(r_base + alpha * (ibar[i] - ibar_avg))
-    return r
+            sgn = 1 if avg > 0 else -1
+            q = _sat(sgn * round_shift(d * ((1 << RECIP_BITS) // abs(avg)), RECIP_BITS - RATIO_FRAC_BITS), lim)
+            delta = round_shift(Bm * A * q, -(Be + E))
+        R.append(_sat(Rb + delta, lim))
+    return R
 
 
 def ratio_to_grid(r: float) -> int:
@@ -332,8 +378,8 @@ def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
         B = global_budget(keep_ratio[rq], n_vis)
         if i1 > i0:
             Sr = [int(v) for v in S[i0:i1]]
-            r = adaptive_ratios(Sr, n, r_base, alpha, relative)
-            R = [ratio_to_grid(v) for v in r]
+            R = adaptive_ratio_grid(Sr, n, r_base, alpha, relative)
+            r = [v / float(1 << RATIO_FRAC_BITS) for v in R]
             R_min, R_max = ratio_to_grid(r_min), ratio_to_grid(r_max)
             lam = water_fill(R, n, B, R_min, R_max)
             k = integer_budgets(R, n, B, lam, R_min, R_max)

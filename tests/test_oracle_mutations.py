@@ -19,10 +19,12 @@ from oracle import avtp_oracle
 SRC_PATH = inspect.getsourcefile(avtp_oracle)
 
 MUTATIONS = {
-    "ratio sign flipped": ("r.append(r_base + alpha * (ibar[i] - ibar_avg))",
-                           "r.append(r_base - alpha * (ibar[i] - ibar_avg))"),
-    "image-weighted mean": ("ibar_avg = (float(total) * scale) / float(n_vis)",
-                            "ibar_avg = sum(ibar) / len(ibar)"),
+    "ratio sign flipped": ("delta = round_shift(A * d, -(E + 8))", "delta = round_shift(-A * d, -(E + 8))"),
+    "ratio off by a factor of two": ("delta = round_shift(A * d, -(E + 8))", "delta = round_shift(A * d, -(E + 9))"),
+    "image-weighted mean": ("avg = round_shift(total * reciprocal(N), RECIP_BITS)", "avg = sum(ibar) // len(ibar)"),
+    "relative rule ignores the sign of the mean": ("sgn = 1 if avg > 0 else -1", "sgn = 1"),
+    "relative rule drops r_base": ("delta = round_shift(Bm * A * q, -(Be + E))",
+                                   "delta = round_shift(A * q, -E)"),
     "GQA head mapping": ("g = h // (n_q_heads // n_kv_heads)", "g = h % n_kv_heads"),
     "causal mask off by one": ("visible = keys[None, :] <= text_local[:, None]",
                                "visible = keys[None, :] < text_local[:, None]"),

@@ -312,6 +312,34 @@ def test_relative_rule_is_proportional_to_image_mass():
     assert np.all(np.abs(res["budgets"] - x) < 1.0)
 
 
+@pytest.mark.parametrize("relative", [False, True])
+def test_ratios_match_the_real_formula(relative):
+    # Section 3.3.3 in exact rationals: Ibar_i = S_i / (2^32 n_i), Ibar_avg = sum S / (2^32 N),
+    # r_i = r_base + alpha (Ibar_i - Ibar_avg)  or  r_base (1 + alpha (Ibar_i / Ibar_avg - 1)).
+    # The integer grid must agree to well below one token; means of either sign.
+    from fractions import Fraction as F
+    rng = np.random.default_rng(15)
+    for trial in range(80):
+        m = int(rng.integers(1, 12))
+        n = rng.integers(1, 5000, size=m)
+        sign = -1 if trial % 3 == 0 else 1
+        mean = rng.uniform(0.1, 2.0, size=m)
+        S = (sign * np.rint(mean * 2.0 ** 32) * n).astype(np.int64) + rng.integers(-n, n + 1)
+        alpha = float(np.float32(rng.choice([0.0, 0.3, 1.0, 2.0, 5.0])))
+        kr = np.float32(rng.choice([0.05, 0.125, 0.33, 0.5, 0.9]))
+        lay = synth.Layout.from_segments([[("t", 1)] + [("i", int(v)) for v in n]])
+        res = O.allocate(lay, S, np.array([kr], dtype=np.float32), alpha, 0.0, 1.0, relative)
+        N = int(n.sum())
+        avg = F(int(S.sum()), 2 ** 32 * N)
+        for i in range(m):
+            ib = F(int(S[i]), 2 ** 32 * int(n[i]))
+            if relative:
+                exact = F(float(kr)) * (1 + F(alpha) * (ib / avg - 1))
+            else:
+                exact = F(float(kr)) + F(alpha) * (ib - avg)
+            assert abs(float(F(res["ratios"][i]) - exact)) < 2.0 ** -24, (trial, i, relative)
+
+
 # ---------------------------------------------------------------- step 3
 def test_selection_golden():
     for case in _load("selection.json")["cases"]:
