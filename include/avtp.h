@@ -115,7 +115,9 @@ typedef struct {
 } avtp_score_args_t;
 
 typedef struct {
-  const float* keep_ratio;  /* device [R]: base keep ratio r_base of each request, in [0, 1] */
+  const float* keep_ratio;  /* device [R]: base keep ratio r_base of each request, within
+                             * [r_min, r_max] (else AVTP_ERR_DEVICE_INPUT: no shift of the
+                             * ratios could meet both the clamps and the request's budget) */
   float alpha;              /* variance control alpha of paper §3.3.3, in [0, 1024]; paper uses 1.0 */
   float r_min;              /* ratio clamps of App. A.2: 0 <= r_min <= r_max <= 1; paper uses 0.05 */
   float r_max;              /*                                                        and 0.95 */
@@ -154,11 +156,19 @@ AVTP_API avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_
 /* Step 2 (paper §3.3.3, App. A.2). From img_sums (device int64 [n_images]) writes
  * budgets (device int32 [n_images]) and out_cu_seqlens (device int32 [R+1]),
  * the packed offsets of the pruned batch. Per request: B_r = floor(r_base*N_vis+0.5);
- * Ibar_i = S_i/2^32/n_i; Ibar_avg = sum S/2^32/N_vis; r_i by the rule above
- * (fp64, each operation rounded once); R_i = rint(clamp(r_i,+-2^20)*2^40);
+ * the ratios r_i of the rule above are taken in exact integers on a 2^-40 grid:
+ * Ibar_i = round(S_i*floor(2^62/n_i)/2^62) and Ibar_avg likewise with sum S and
+ * N_vis (units of 2^-32); R_i = rint(r_base*2^40) + round(alpha*(Ibar_i-Ibar_avg)*2^8),
+ * or for the relative rule + round(r_base*alpha*q_i) with
+ * q_i = sgn(Ibar_avg)*round((Ibar_i-Ibar_avg)*floor(2^62/|Ibar_avg|)/2^22);
+ * fp32 alpha, r_base exact, one rounding (nearest, ties up) per product, R_i
+ * saturated to +-2^60;
  * lambda = smallest integer with sum n_i*clamp(R_i+lambda, R_min, R_max) >= B_r*2^40;
  * k_i = min(floor(x_i/2^40), n_i) with x_i = n_i*clamp(R_i+lambda), then
- * largest remainder (ties to the lower index) until sum k_i = B_r. */
+ * largest remainder (ties to the lower index) until sum k_i = B_r.
+ * Every |img_sums[i]| must be at most img_len[i]*2^42 (avtp_score's sums are);
+ * otherwise the request's budgets are not written and the call reports
+ * AVTP_ERR_DEVICE_INPUT. */
 AVTP_API avtp_status_t avtp_allocate(const avtp_layout_t* layout, const int64_t* img_sums, const avtp_alloc_args_t* args,
                             int32_t* budgets, int32_t* out_cu_seqlens, void* workspace, size_t workspace_bytes,
                             avtp_stream_t stream);

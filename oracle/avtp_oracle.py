@@ -70,6 +70,7 @@ NORM_EPS = 1e-8
 RATIO_FRAC_BITS = 40     # ratios, shifts and kept masses live on a 2^-40 integer grid
 RATIO_LIMIT = 2.0 ** 20  # ratios are saturated to +-2^20 before going on the grid
 RECIP_BITS = 62          # per-image means are taken with floor(2^62 / n) reciprocals
+SUM_MAGNITUDE_BITS = 42  # |S_i| <= n_i * 2^42: scores clamped to +-2^10, 32 fraction bits
 
 
 # ----------------------------------------------------------------------------
@@ -355,10 +356,12 @@ def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
              r_min: float = 0.05, r_max: float = 0.95, relative: bool = False) -> Dict[str, np.ndarray]:
     """Per-image budgets ``k_i`` and the packed output offsets ``out_cu_seqlens``.
 
-    fp32 parameters (``keep_ratio``, ``alpha``, ``r_min``, ``r_max``) are widened to
-    fp64 exactly, as the device does. Returns a dict with ``budgets`` int32
-    [n_img], ``out_cu_seqlens`` int32 [R+1] and, for inspection, ``ratios`` and
-    ``lam`` per request.
+    fp32 parameters (``keep_ratio``, ``alpha``, ``r_min``, ``r_max``) enter exactly.
+    The sums must satisfy ``|S_i| <= n_i * 2^42`` (every fixed-point score is within
+    +-2^42), and every keep ratio must lie within the clamps ``[r_min, r_max]`` (else
+    no ratio shift meets both the clamps and the global budget); otherwise ValueError. Returns a dict with ``budgets`` int32
+    [n_img], ``out_cu_seqlens`` int32 [R+1] and, for inspection, ``ratios`` (on the
+    grid, before the clamps) and ``lam`` per request.
     """
     R = len(layout.cu_seqlens) - 1
     alpha = float(np.float32(alpha))
@@ -375,14 +378,19 @@ def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
         T_r = int(layout.cu_seqlens[rq + 1]) - int(layout.cu_seqlens[rq])
         n_txt = T_r - n_vis
         r_base = float(np.float32(keep_ratio[rq]))
+        if not (r_min <= r_base <= r_max):
+            raise ValueError(f"request {rq}: keep ratio {r_base} outside the clamps [{r_min}, {r_max}]")
         B = global_budget(keep_ratio[rq], n_vis)
         if i1 > i0:
             Sr = [int(v) for v in S[i0:i1]]
-            R = adaptive_ratio_grid(Sr, n, r_base, alpha, relative)
-            r = [v / float(1 << RATIO_FRAC_BITS) for v in R]
+            for j in range(len(n)):
+                if abs(Sr[j]) > n[j] << SUM_MAGNITUDE_BITS:
+                    raise ValueError(f"image {i0 + j}: |S_i| exceeds n_i * 2^{SUM_MAGNITUDE_BITS}")
+            Rg = adaptive_ratio_grid(Sr, n, r_base, alpha, relative)
+            r = [v / float(1 << RATIO_FRAC_BITS) for v in Rg]
             R_min, R_max = ratio_to_grid(r_min), ratio_to_grid(r_max)
-            lam = water_fill(R, n, B, R_min, R_max)
-            k = integer_budgets(R, n, B, lam, R_min, R_max)
+            lam = water_fill(Rg, n, B, R_min, R_max)
+            k = integer_budgets(Rg, n, B, lam, R_min, R_max)
             budgets[i0:i1] = k
             ratios[i0:i1] = r
             lams[rq] = lam / float(2 ** RATIO_FRAC_BITS)

@@ -1,13 +1,16 @@
 // Per-request budget rule (paper §3.3.3 adaptive keep ratio, App. A.2 clamps),
-// computed by ONE WARP from values staged in that warp's shared memory.
+// computed by ONE WARP, in exact integer arithmetic on a 2^-40 ratio grid.
 //
-// fp64 part (one rounding per operation, explicit _rn intrinsics, no FMA):
-//   Ibar_i   = (S_i * 2^-32) / n_i
-//   Ibar_avg = (sum_i S_i * 2^-32) / N_vis
-//   r_i      = r_base + alpha * (Ibar_i - Ibar_avg)              (relative = 0)
-//            = r_base * (1 + alpha * (Ibar_i / Ibar_avg - 1))     (relative = 1; r_base if Ibar_avg == 0)
-// exact integer part on the 2^-40 grid:
-//   R_i = rint(clamp(r_i, +-2^20) * 2^40), R_min, R_max likewise,
+// Ratios (S_i in units of 2^-32, each product exact, rounded once to nearest, ties up):
+//   Ibar_i   = round(S_i * floor(2^62 / n_i) / 2^62)
+//   Ibar_avg = round(sum_i S_i * floor(2^62 / N_vis) / 2^62)
+//   R_i = R_base + round(alpha * (Ibar_i - Ibar_avg) * 2^8)                       (relative = 0)
+//   R_i = R_base + round(r_base * alpha * q_i),                                    (relative = 1)
+//         q_i = sgn(Ibar_avg) * round((Ibar_i - Ibar_avg) * floor(2^62 / |Ibar_avg|) / 2^22),
+//         saturated to +-2^60 (R_i = R_base when Ibar_avg == 0)
+//   with R_base = rint(r_base * 2^40), fp32 alpha and r_base taken as exact M * 2^E,
+//   and R_i saturated to +-2^60. R_min, R_max = rint(r_min * 2^40), rint(r_max * 2^40).
+// Water-fill and rounding:
 //   G(l) = sum_i n_i * clamp(R_i + l, R_min, R_max),
 //   lambda = min { l in [R_min - max R, R_max - min R] : G(l) >= B * 2^40 } (an end of the range if none),
 //   x_i = n_i * clamp(R_i + lambda), k_i = min(x_i >> 40, n_i), then largest remainder.
@@ -19,8 +22,9 @@
 // Beyond that a 32-way multisection gives the same lambda.
 //
 // Everything is warp-synchronous (shuffles and __syncwarp only): on this part a
-// block-wide barrier or a dependent fp64 operation costs far more than the
-// arithmetic, so the rule is kept to one warp and a short fp64 chain.
+// block-wide barrier or a dependent fp64 operation or division costs far more
+// than the arithmetic, so the reciprocals are taken before the sums are known
+// and the rest is integer multiplies and shifts.
 #pragma once
 
 #include "avtp_internal.cuh"
@@ -73,31 +77,100 @@ __device__ __forceinline__ WarpAllocSmem carve_warp_alloc(unsigned char* base, i
 // The grid values of the clamps, rint(r * 2^40) (exact for fp32 inputs >= 2^-17).
 __device__ __forceinline__ int64_t ratio_grid(float r) { return __double2ll_rn(static_cast<double>(r) * 0x1p40); }
 
+constexpr int kRecipBits = 62;
+constexpr int64_t kGridSat = int64_t(1) << 60;   // ratios saturate here on the grid
+constexpr int kSumMagnitudeBits = 42;            // |S_i| <= n_i * 2^42 (scores clamped to +-2^10)
+
+// floor(2^62 / n) for n >= 1 (0 for n <= 0, which only unused lanes pass).
+__device__ __forceinline__ int64_t recip62(int64_t n) {
+  return n > 0 ? static_cast<int64_t>((uint64_t(1) << kRecipBits) / static_cast<uint64_t>(n)) : 0;
+}
+
+// floor(x / 2^s + 1/2) for 1 <= s, saturated to +-lim.
+__device__ __forceinline__ int64_t round_shift_sat(__int128 x, int s, int64_t lim) {
+  if (s > 120) return 0;  // every x passed here is below 2^110 in magnitude
+  const __int128 y = (x + (static_cast<__int128>(1) << (s - 1))) >> s;
+  return y > lim ? lim : (y < -lim ? -lim : static_cast<int64_t>(y));
+}
+
+// The fp32 value v as M * 2^E exactly, |M| < 2^24.
+__device__ __forceinline__ void fp32_parts(float v, int64_t* M, int* E) {
+  const uint32_t b = __float_as_uint(v);
+  const int e8 = (b >> 23) & 0xff;
+  const int64_t mag = (b & 0x7fffff) | (e8 ? 0x800000 : 0);
+  *M = (b >> 31) ? -mag : mag;
+  *E = e8 ? e8 - 150 : -149;
+}
+
+// The parts of the ratio rule that do not depend on the sums. alpha in [0, 1024]
+// and r_base in [0, 1] (validated before any launch) keep `shift` >= 5.
+struct RatioRule {
+  int64_t Rb;    // rint(r_base * 2^40)
+  int64_t coef;  // alpha (additive) or r_base * alpha (relative) is coef * 2^-shift on the grid
+  int shift;
+  int relative;
+};
+
+__device__ __forceinline__ RatioRule make_ratio_rule(float r_base, float alpha, int relative) {
+  RatioRule q;
+  q.Rb = ratio_grid(r_base);
+  int64_t A, Bm;
+  int E, Be;
+  fp32_parts(alpha, &A, &E);
+  fp32_parts(r_base, &Bm, &Be);
+  q.relative = relative;
+  if (relative) {
+    q.coef = A * Bm;
+    q.shift = -(E + Be);
+  } else {
+    q.coef = A;
+    q.shift = -(E + kRatioFracBits - kFxFracBits);
+  }
+  return q;
+}
+
+// Ibar on the 2^-32 grid: round(S * floor(2^62 / n) / 2^62), exact for |S| <= n * 2^42.
+__device__ __forceinline__ int64_t grid_mean(int64_t S, int64_t inv_n) {
+  return round_shift_sat(static_cast<__int128>(S) * inv_n, kRecipBits, INT64_MAX);
+}
+
+// R_i from Ibar_i, Ibar_avg and (relative rule only) floor(2^62 / |Ibar_avg|).
+__device__ __forceinline__ int64_t grid_ratio(const RatioRule& q, int64_t ibar, int64_t avg, int64_t inv_avg) {
+  const int64_t d = ibar - avg;
+  int64_t delta;
+  if (!q.relative) {
+    delta = round_shift_sat(static_cast<__int128>(q.coef) * d, q.shift, kGridSat * 2);
+  } else if (avg == 0) {
+    delta = 0;
+  } else {
+    int64_t t = round_shift_sat(static_cast<__int128>(d) * inv_avg, kRecipBits - kRatioFracBits, kGridSat);
+    t = avg > 0 ? t : -t;
+    delta = round_shift_sat(static_cast<__int128>(q.coef) * t, q.shift, kGridSat * 2);
+  }
+  return clamp64(q.Rb + delta, -kGridSat, kGridSat);
+}
+
 // All 32 lanes call with identical scalars. sm.X[j] = S_j and sm.n[j] = n_j for j < m on entry.
-// Returns false if the rounding loop did not converge (never expected).
-static __device__ __noinline__ bool warp_allocate(const WarpAllocSmem& sm, int m, int64_t B, int32_t N, float r_base_f, float alpha_f,
+// Returns AVTP_OK, AVTP_ERR_DEVICE_INPUT for a sum beyond n_j * 2^42, or AVTP_ERR_RANGE
+// if the rounding loop did not converge (never expected).
+static __device__ __noinline__ int warp_allocate(const WarpAllocSmem& sm, int m, int64_t B, int32_t N, float r_base_f, float alpha_f,
                               int64_t Rmin, int64_t Rmax, int relative) {
   const int lane = threadIdx.x & 31;
-  // ---- fp64 ratio formula
+  // ---- ratios on the grid
   int64_t part = 0;
-  for (int j = lane; j < m; j += 32) part += sm.X[j];
-  const int64_t total = warp_sum(part);
-  const double kScale = 0x1p-32;
-  const double ibar_avg = __ddiv_rn(__dmul_rn(__ll2double_rn(total), kScale), static_cast<double>(N));
-  const double rb = static_cast<double>(r_base_f);
-  const double al = static_cast<double>(alpha_f);
+  bool bad = false;
+  for (int j = lane; j < m; j += 32) {
+    const int64_t S = sm.X[j], lim = static_cast<int64_t>(sm.n[j]) << kSumMagnitudeBits;
+    bad |= S > lim || S < -lim;
+    part += S;
+  }
+  if (__any_sync(0xffffffffu, bad)) return AVTP_ERR_DEVICE_INPUT;
+  const int64_t avg = grid_mean(warp_sum(part), recip62(N));
+  const int64_t inv_avg = (relative && avg != 0) ? recip62(avg > 0 ? avg : -avg) : 0;
+  const RatioRule rule = make_ratio_rule(r_base_f, alpha_f, relative);
   int64_t mx = INT64_MIN, mn = INT64_MAX;
   for (int j = lane; j < m; j += 32) {
-    const double ibar = __ddiv_rn(__dmul_rn(__ll2double_rn(sm.X[j]), kScale), static_cast<double>(sm.n[j]));
-    double rr;
-    if (relative) {
-      rr = (ibar_avg == 0.0) ? rb
-                             : __dmul_rn(rb, __dadd_rn(1.0, __dmul_rn(al, __dsub_rn(__ddiv_rn(ibar, ibar_avg), 1.0))));
-    } else {
-      rr = __dadd_rn(rb, __dmul_rn(al, __dsub_rn(ibar, ibar_avg)));
-    }
-    rr = fmin(fmax(rr, -kRatioLimit), kRatioLimit);
-    const int64_t g = __double2ll_rn(rr * 0x1p40);  // exact power-of-two scaling
+    const int64_t g = grid_ratio(rule, grid_mean(sm.X[j], recip62(sm.n[j])), avg, inv_avg);
     sm.R[j] = g;
     mx = g > mx ? g : mx;
     mn = g < mn ? g : mn;
@@ -184,7 +257,7 @@ static __device__ __noinline__ bool warp_allocate(const WarpAllocSmem& sm, int m
     int64_t ks = 0;
     for (int j = lane; j < m; j += 32) ks += sm.K[j];
     const int64_t D = B - warp_sum(ks);
-    if (D == 0) return true;
+    if (D == 0) return AVTP_OK;
     // decide every image from the same snapshot of K (sm.R is free by now), then apply
     for (int j = lane; j < m; j += 32) {
       int dec = 0;
@@ -205,7 +278,7 @@ static __device__ __noinline__ bool warp_allocate(const WarpAllocSmem& sm, int m
     for (int j = lane; j < m; j += 32) sm.K[j] += static_cast<int32_t>(sm.R[j]);
     __syncwarp();
   }
-  return false;
+  return AVTP_ERR_RANGE;
 }
 
 // lambda from the breakpoints, for warp_allocate32 when a clamp binds near the
@@ -255,34 +328,24 @@ static __device__ __noinline__ int64_t breakpoint_lambda32(int m, int64_t R, int
 }
 
 // The same rule for requests of at most 32 images, held in registers: lane j owns
-// image j (S_j, n_j in; its budget out). Identical results to warp_allocate.
+// image j (S_j, n_j in; its budget out). Identical results and status to warp_allocate.
+// inv_n = floor(2^62 / n_j) and inv_N = floor(2^62 / N) come from the caller, which
+// can take them before the sums are ready; after that no division is left on the
+// common path.
 // Fast path for lambda: without clamps G is linear with slope N, so the smallest
 // solution is lambda0 = ceil((B * 2^40 - sum n_i R_i) / N); when no clamp binds
 // at lambda0 - 1 or lambda0, G is that line on [lambda0 - 1, lambda0] and
 // lambda0 is exact. Otherwise the breakpoints decide.
-inline __device__ bool warp_allocate32(int m, int64_t S, int32_t n, int64_t B, int32_t N, float r_base_f,
-                                       float alpha_f, int64_t Rmin, int64_t Rmax, int relative, int32_t* k_out) {
+inline __device__ int warp_allocate32(int m, int64_t S, int32_t n, int64_t inv_n, int64_t B, int32_t N, int64_t inv_N,
+                                       const RatioRule& rule, int64_t Rmin, int64_t Rmax, int32_t* k_out) {
   const int lane = threadIdx.x & 31;
   const bool has = lane < m;
-  // ---- fp64 ratio formula
-  const int64_t total = warp_sum(has ? S : int64_t(0));
-  const double kScale = 0x1p-32;
-  const double ibar_avg = __ddiv_rn(__dmul_rn(__ll2double_rn(total), kScale), static_cast<double>(N));
-  const double rb = static_cast<double>(r_base_f);
-  const double al = static_cast<double>(alpha_f);
-  int64_t R = 0;
-  if (has) {
-    const double ibar = __ddiv_rn(__dmul_rn(__ll2double_rn(S), kScale), static_cast<double>(n));
-    double rr;
-    if (relative) {
-      rr = (ibar_avg == 0.0) ? rb
-                             : __dmul_rn(rb, __dadd_rn(1.0, __dmul_rn(al, __dsub_rn(__ddiv_rn(ibar, ibar_avg), 1.0))));
-    } else {
-      rr = __dadd_rn(rb, __dmul_rn(al, __dsub_rn(ibar, ibar_avg)));
-    }
-    rr = fmin(fmax(rr, -kRatioLimit), kRatioLimit);
-    R = __double2ll_rn(rr * 0x1p40);
-  }
+  // ---- ratios on the grid
+  const int64_t lim = static_cast<int64_t>(n) << kSumMagnitudeBits;
+  if (__any_sync(0xffffffffu, has && (S > lim || S < -lim))) return AVTP_ERR_DEVICE_INPUT;
+  const int64_t avg = grid_mean(warp_sum(has ? S : int64_t(0)), inv_N);
+  const int64_t inv_avg = (rule.relative && avg != 0) ? recip62(avg > 0 ? avg : -avg) : 0;
+  const int64_t R = has ? grid_ratio(rule, grid_mean(S, inv_n), avg, inv_avg) : 0;
   const int64_t mx = warp_max64(has ? R : INT64_MIN);
   const int64_t mn = warp_min64(has ? R : INT64_MAX);
   const int64_t target = B << kRatioFracBits;
@@ -313,7 +376,7 @@ inline __device__ bool warp_allocate32(int m, int64_t S, int32_t n, int64_t B, i
     const int64_t D = B - warp_sum(static_cast<int64_t>(K));
     if (D == 0) {
       *k_out = K;
-      return true;
+      return AVTP_OK;
     }
     const bool elig = has && (D > 0 ? K < n : K > 0);
     // remainders are below 2^40: split them so each shuffle moves 32 bits
@@ -333,7 +396,7 @@ inline __device__ bool warp_allocate32(int m, int64_t S, int32_t n, int64_t B, i
     if (elig && rank < (D > 0 ? D : -D)) K += D > 0 ? 1 : -1;
   }
   *k_out = K;
-  return false;
+  return AVTP_ERR_RANGE;
 }
 
 }  // namespace avtp

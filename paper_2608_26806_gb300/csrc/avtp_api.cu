@@ -189,6 +189,8 @@ avtp_status_t avtp_allocate(const avtp_layout_t* layout, const int64_t* img_sums
   PrepArgs pa{};
   pa.L = *layout;
   pa.keep_ratio = args->keep_ratio;
+  pa.r_min = args->r_min;
+  pa.r_max = args->r_max;
   pa.out_cu_seqlens = out_cu_seqlens;
   if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
   return from_cuda(launch_allocate(*layout, img_sums, *args, budgets, workspace, p, s));
@@ -247,6 +249,8 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   PrepArgs pa{};
   pa.L = *layout;
   pa.keep_ratio = alloc_args->keep_ratio;
+  pa.r_min = alloc_args->r_min;
+  pa.r_max = alloc_args->r_max;
   pa.out_cu_seqlens = out_cu_seqlens;
   pa.zero_img_sums = sums;
   pa.build_text_tiles = score_args->criterion == AVTP_CRIT_TEXT_ATTENTION;

@@ -147,6 +147,7 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
 struct PrepArgs {
   avtp_layout_t L;
   const float* keep_ratio;   // NULL: no budgets / out_cu_seqlens
+  float r_min, r_max;        // each keep ratio must lie in [r_min, r_max]
   int32_t* out_cu_seqlens;   // NULL: not written
   int64_t* zero_img_sums;    // NULL: not zeroed
   int build_text_tiles;      // criterion B bookkeeping

@@ -31,9 +31,10 @@ k_allocate(const int32_t* __restrict__ img_cu, const int32_t* __restrict__ img_l
   }
   __syncwarp();
   const int32_t N = vis_cu[i0 + m] - vis_cu[i0];
-  if (!warp_allocate(sm, m, req_budget[r], N, keep_ratio[r], alpha, ratio_grid(r_min), ratio_grid(r_max),
-                     relative)) {
-    if (lane == 0) record_error(st, AVTP_ERR_RANGE, r);
+  const int err = warp_allocate(sm, m, req_budget[r], N, keep_ratio[r], alpha, ratio_grid(r_min), ratio_grid(r_max),
+                                relative);
+  if (err != AVTP_OK) {
+    if (lane == 0) record_error(st, err, r);
     return;
   }
   for (int j = lane; j < m; j += 32) budgets[i0 + j] = sm.K[j];

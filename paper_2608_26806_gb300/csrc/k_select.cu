@@ -53,7 +53,7 @@ struct SelShared {
   int digit, above, count;
   // hand-over from the warps of the fused kernel
   uint32_t kmin, kmax;
-  int k, before, total, alloc_ok, vis_before, n_vis;
+  int k, before, total, alloc_err, vis_before, n_vis;
 };
 
 // Named barrier for warps 1..7 (224 threads) while warp 0 runs the budget rule.
@@ -354,8 +354,9 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
   }
   // warp 0: the request's sizes and the scalars of the budget rule
   int32_t N = 0, n_lane = 0, vis_before = 0;
-  int64_t B = 0, Rmin = 0, Rmax = 0;
+  int64_t B = 0, Rmin = 0, Rmax = 0, inv_n = 0, inv_N = 0;
   float kr = 0.f;
+  RatioRule rule{};
   if (warp == 0 && b < a.NI) {
     int64_t nsum = 0, nbefore = 0;
     for (int j = lane; j < m; j += 32) {
@@ -372,6 +373,9 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
     B = static_cast<int64_t>(floor(__dadd_rn(__dmul_rn(static_cast<double>(kr), static_cast<double>(N)), 0.5)));
     Rmin = ratio_grid(ap.r_min);
     Rmax = ratio_grid(ap.r_max);
+    rule = make_ratio_rule(kr, ap.alpha, ap.relative);
+    inv_N = recip62(N);
+    inv_n = recip62(n_lane);
   }
 
   // ---- wait for the scores and per-image sums (and, through them, the validation)
@@ -387,19 +391,19 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
   const bool stage = n <= kKeyCap;
   if (warp == 0) {
     // ---- the budget rule, one warp
-    bool ok;
+    int err;
     int k, before, total;
     if (m <= 32) {
       const int64_t S = lane < m ? ap.img_sums[i0 + lane] : 0;
       int32_t K;
-      ok = warp_allocate32(m, S, n_lane, B, N, kr, ap.alpha, Rmin, Rmax, ap.relative, &K);
+      err = warp_allocate32(m, S, n_lane, inv_n, B, N, inv_N, rule, Rmin, Rmax, &K);
       k = __shfl_sync(kFull, K, li);
       before = warp_sum(lane < li ? K : 0);
       total = warp_sum(lane < m ? K : 0);
     } else {
       for (int j = lane; j < m; j += 32) wsm.X[j] = ap.img_sums[i0 + j];
       __syncwarp();
-      ok = warp_allocate(wsm, m, B, N, kr, ap.alpha, Rmin, Rmax, ap.relative);
+      err = warp_allocate(wsm, m, B, N, kr, ap.alpha, Rmin, Rmax, ap.relative);
       int bs = 0, ts = 0;
       for (int j = lane; j < m; j += 32) {
         ts += wsm.K[j];
@@ -415,7 +419,7 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
       sh.k = k;
       sh.before = before;
       sh.total = total;
-      sh.alloc_ok = ok ? 1 : 0;
+      sh.alloc_err = err;
       sh.vis_before = vis_before;
       sh.n_vis = N;
     }
@@ -464,9 +468,8 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
   __syncthreads();
   const uint32_t kmin = sh.kmin, kmax = sh.kmax;
   const int k = sh.k, before = sh.before, total = sh.total, vis_b = sh.vis_before, Nv = sh.n_vis;
-  const bool alloc_ok = sh.alloc_ok != 0;
-  if (!alloc_ok) {
-    if (tid == 0) record_error(a.st, AVTP_ERR_RANGE, r);
+  if (sh.alloc_err != AVTP_OK) {
+    if (tid == 0) record_error(a.st, sh.alloc_err, r);
     return;
   }
   if (tid == 0) ap.budgets[i] = k;

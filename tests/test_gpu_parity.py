@@ -98,10 +98,11 @@ def test_allocate_bit_exact_random_strong_signal():
         lay = synth.Layout.from_segments(reqs)
         n = lay.img_len.astype(np.int64)
         S = (rng.integers(-2 ** 33, 2 ** 34, size=lay.n_images) * n).astype(np.int64)
-        kr = rng.choice(np.array([0.05, 0.125, 0.25, 0.33, 0.5, 0.9, 1.0], dtype=np.float32), size=R)
+        r_min, r_max = (0.05, 0.95) if trial % 3 else (0.0, 1.0)
+        choices = [0.05, 0.125, 0.25, 0.33, 0.5, 0.9] + ([0.95] if trial % 3 else [0.0, 1.0])
+        kr = rng.choice(np.array(choices, dtype=np.float32), size=R)
         alpha = float(rng.choice([0.0, 1.0, 2.0, 5.0, 100.0]))
         relative = bool(trial % 2)
-        r_min, r_max = (0.05, 0.95) if trial % 3 else (0.0, 1.0)
         ref = O.allocate(lay, S, kr, alpha, r_min, r_max, relative)
         L = dev_layout(lay)
         budgets, out_cu = avtp.allocate(L, torch.from_numpy(S).cuda(), torch.from_numpy(kr).cuda(), alpha, r_min,
@@ -110,6 +111,80 @@ def test_allocate_bit_exact_random_strong_signal():
         assert np.array_equal(budgets.cpu().numpy(), ref["budgets"]), trial
         assert np.array_equal(out_cu.cpu().numpy(), ref["out_cu_seqlens"]), trial
         assert avtp.kept_count_host(L.host, kr) == int(ref["out_cu_seqlens"][-1])
+
+
+def test_allocate_bit_exact_extreme_sums_and_alphas():
+    # sums at the +-n * 2^42 bound, means of either sign or zero, alpha from tiny to the
+    # 1024 limit, both rules: the integer ratio grid must match the oracle to the bit
+    rng = np.random.default_rng(8)
+    alphas = [0.0, 2.0 ** -60, 1e-7, 0.3, 1.0, 37.5, 1024.0]
+    for trial in range(42):
+        R = int(rng.integers(1, 4))
+        reqs = [[("t", 2)] + [("i", int(rng.integers(1, 3000))) for _ in range(int(rng.integers(1, 45)))]
+                for _ in range(R)]
+        lay = synth.Layout.from_segments(reqs)
+        n = lay.img_len.astype(np.int64)
+        kind = trial % 6
+        if kind == 0:
+            S = rng.choice([-1, 1], size=lay.n_images) * (n << 42)
+        elif kind == 1:
+            S = -(rng.integers(0, 2 ** 33, size=lay.n_images) * n)
+        elif kind == 2:
+            S = np.zeros(lay.n_images, dtype=np.int64)
+        elif kind == 3:
+            S = rng.integers(-2 ** 20, 2 ** 20, size=lay.n_images)  # means of a few 2^-32 units
+        else:
+            S = rng.integers(0, 2 ** 34, size=lay.n_images) * n + rng.integers(-n, n + 1)
+        S = np.asarray(S, dtype=np.int64)
+        r_min, r_max = (0.0, 1.0) if trial % 2 else (0.05, 0.95)
+        kr = rng.choice(np.array([r_min, 0.05, 0.33, 0.5, r_max], dtype=np.float32), size=R)
+        alpha = alphas[trial % len(alphas)]
+        relative = bool((trial // 6) % 2)
+        ref = O.allocate(lay, S, kr, alpha, r_min, r_max, relative)
+        L = dev_layout(lay)
+        budgets, out_cu = avtp.allocate(L, torch.from_numpy(S).cuda(), torch.from_numpy(kr).cuda(), alpha, r_min,
+                                        r_max, relative)
+        torch.cuda.synchronize()
+        assert np.array_equal(budgets.cpu().numpy(), ref["budgets"]), trial
+        assert np.array_equal(out_cu.cpu().numpy(), ref["out_cu_seqlens"]), trial
+
+
+def test_allocate_rejects_sums_beyond_bound():
+    L = avtp.Layout.from_host([0, 30], [0, 2], [0, 12], [10, 10])
+    kr = torch.tensor([0.5], device="cuda")
+    for bad in ([(10 << 42) + 1, 0], [0, -(10 << 42) - 1]):
+        sums = torch.tensor(bad, dtype=torch.int64, device="cuda")
+        st = _status_after(lambda ws: avtp.allocate(L, sums, kr, workspace=ws))
+        assert st == avtp.ERR_DEVICE_INPUT
+    with pytest.raises(ValueError):
+        O.allocate(synth.Layout.from_segments([[("i", 10), ("t", 2), ("i", 10)]]),
+                   np.array([(10 << 42) + 1, 0], dtype=np.int64), np.array([0.5], dtype=np.float32))
+
+
+@pytest.mark.parametrize("alpha", [0.0, 1e-7, 0.3, 5.0, 1024.0])
+@pytest.mark.parametrize("relative", [False, True])
+def test_prune_fused_budget_rule_across_alphas(alpha, relative):
+    # requests of <= 32 images take the register path of the fused kernel, larger ones
+    # the shared-memory path; both must equal the oracle fed the same scores
+    rng = np.random.default_rng(9)
+    reqs = []
+    for m in (1, 5, 32, 33, 70):
+        segs = [("t", 3)]
+        for _ in range(m):
+            segs += [("i", int(rng.integers(1, 120))), ("t", int(rng.integers(0, 2)))]
+        reqs.append(segs)
+    wl = synth.make_custom(reqs, keep_ratio=0.3, parts=("A", "pos"))
+    dw = DevWorkload(wl)
+    out = avtp.prune(dw.L, "hidden_variation", keep_ratio=dw.keep_ratio, keep_ratio_host=wl.keep_ratio,
+                     alpha=alpha, relative=relative, planes={"pos": dw.t["pos"]},
+                     **dw.score_tensors("hidden_variation"))
+    torch.cuda.synchronize()
+    assert avtp.read_device_status(out.workspace) == avtp.OK
+    got = out.scores.cpu().numpy()
+    ref = O.prune(wl.layout, keep_ratio=wl.keep_ratio, scores_f32=got, alpha=alpha, relative=relative,
+                  planes={"pos": wl.pos})
+    assert np.array_equal(out.budgets[:wl.layout.n_images].cpu().numpy(), ref["budgets"])
+    assert np.array_equal(out.kept_idx.cpu().numpy(), ref["kept_idx"])
 
 
 # ---------------------------------------------------------------- step 3
@@ -283,8 +358,9 @@ def test_device_rejects_bad_spans():
 def test_device_rejects_bad_keep_ratio_and_budgets():
     L = avtp.Layout.from_host([0, 20], [0, 1], [2], [10])
     sums = torch.zeros(1, dtype=torch.int64, device="cuda")
-    st = _status_after(lambda ws: avtp.allocate(L, sums, torch.tensor([1.5], device="cuda"), workspace=ws))
-    assert st == avtp.ERR_DEVICE_INPUT
+    for kr in (1.5, 0.01, 0.96):  # above 1, below r_min = 0.05, above r_max = 0.95
+        st = _status_after(lambda ws: avtp.allocate(L, sums, torch.tensor([kr], device="cuda"), workspace=ws))
+        assert st == avtp.ERR_DEVICE_INPUT
     scores = torch.zeros(20, device="cuda")
     out_cu = torch.tensor([0, 30], dtype=torch.int32, device="cuda")
     bad_budget = torch.tensor([11], dtype=torch.int32, device="cuda")

@@ -218,6 +218,20 @@ def test_global_budget_rounding():
     assert O.global_budget(np.float32(0.125), 0) == 0
 
 
+def test_allocation_rejects_ratio_outside_clamps_and_oversized_sums():
+    # App. A.2: with r_base below r_min (above r_max) every shifted ratio is clamped up
+    # (down) and the kept total would exceed (fall short of) the global budget
+    lay = synth.Layout.from_segments([[("i", 40), ("t", 3), ("i", 60)]])
+    S = np.array([40 * 2 ** 31, 60 * 2 ** 30], dtype=np.int64)
+    for kr in (0.0, 0.04, 0.96, 1.0):
+        with pytest.raises(ValueError):
+            O.allocate(lay, S, np.array([kr], dtype=np.float32), 1.0, 0.05, 0.95)
+    for kr in (0.05, 0.95):
+        O.allocate(lay, S, np.array([kr], dtype=np.float32), 1.0, 0.05, 0.95)
+    with pytest.raises(ValueError):
+        O.allocate(lay, np.array([(40 << 42) + 1, 0], dtype=np.int64), np.array([0.5], dtype=np.float32))
+
+
 def _random_alloc(rng, m, relative=False, alpha=1.0, kr=None):
     n = rng.integers(1, 300, size=m)
     segs = []
