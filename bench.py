@@ -178,6 +178,19 @@ class L2Flush:
 
 
 # ---------------------------------------------------------------- workload accounting
+def stage_roofline(acct, ms_step, hbm_gbs, bf16_tflops, peak_kind):
+    """The slower of the stage's compulsory bytes at HBM bandwidth and its FLOPs at the
+    bf16 tensor peak, as a fraction of the measured step time."""
+    t_hbm = acct["stage_bytes"] / (hbm_gbs * 1e9)
+    t_tensor = acct["flops"] / (bf16_tflops * 1e12)
+    out = {"bound": "hbm" if t_hbm >= t_tensor else "tensor", "algorithmic_bytes": acct["stage_bytes"],
+           "algorithmic_flops": acct["flops"], "bound_us": round(max(t_hbm, t_tensor) * 1e6, 2),
+           "achieved_gbs": round(acct["stage_bytes"] / (ms_step * 1e-3) / 1e9, 1), "peak_gbs": hbm_gbs,
+           "peak_tflops": bf16_tflops, "frac": round(max(t_hbm, t_tensor) / (ms_step * 1e-3), 4),
+           "peak_kind": peak_kind}
+    return out
+
+
 def stage_accounting(wl, criterion, n_kept):
     lay = wl.layout
     n_vis = int(lay.n_visual_per_request().sum())
@@ -204,8 +217,8 @@ def stage_accounting(wl, criterion, n_kept):
             for p in text_pos:
                 flops += 2 * Hq * d * (p + 1)              # pass 1: every visible key
                 flops += 2 * Hq * d * int(vis_prefix[p + 1])  # pass 2: visible visual keys
-    return {"n_vis": n_vis, "n_txt": n_txt, "score_bytes": score_bytes, "stage_bytes": stage_bytes,
-            "gather_bytes": gather, "flops": flops}
+    return {"n_vis": n_vis, "n_txt": n_txt, "score_bytes": int(score_bytes), "stage_bytes": int(stage_bytes),
+            "gather_bytes": int(gather), "flops": int(flops)}
 
 
 # ---------------------------------------------------------------- our arm
@@ -309,7 +322,6 @@ def run_ours(args, world, rank, local):
                 "algorithmic_flops_per_launch": acct["flops"], "avg_launch_us": round(score_ms * 1e3, 2),
                 "traffic": None}
     ms_step = total_ms_max / K
-    stage_gbs = acct["stage_bytes"] / (ms_step * 1e-3) / 1e9
     value = acct["n_vis"] * K * world / (total_ms_max * 1e-3)
     srt = sorted(step_ms)
     line = {
@@ -324,9 +336,7 @@ def run_ours(args, world, rank, local):
                        "mean": round(statistics.mean(step_ms) * 1e3, 2)},
         "steps_us": {k: round(statistics.mean(v) * 1e3, 2) for k, v in per_step.items()},
         "serialized_step_us": round(statistics.mean(serial_ms) * 1e3, 2),
-        "stage_roofline": {"bound": "hbm", "algorithmic_bytes": acct["stage_bytes"],
-                           "achieved": round(stage_gbs, 1), "peak": hbm, "unit": "GB/s",
-                           "frac": round(stage_gbs / hbm, 4), "peak_kind": peak_kind},
+        "stage_roofline": stage_roofline(acct, ms_step, hbm, bf16_tf, peak_kind),
         "roofline": roof,
         "e2e": e2e,
         "gpu_launches": K * (4 if crit == "hidden_variation" else 6),

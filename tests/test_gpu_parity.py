@@ -320,6 +320,43 @@ def test_prune_end_to_end(name, criterion):
                 assert any(near_tie(float(s_ref[a]), float(s_ref[b])) for b in only_ref), (i, a)
 
 
+def test_prune_fused_selection_ties_nan_and_sizes():
+    # image sizes around every sort size of the fused kernel (256, 512, 1024) and past it
+    # (radix path); rows with h_cur == h_prior score within a few ulps of 0 (many exact
+    # ties), rows with an inf entry score NaN, duplicated rows give equal scores at
+    # distant positions
+    sizes = [1, 7, 255, 256, 257, 511, 512, 513, 1023, 1024, 1025, 2100]
+    reqs = [[("t", 5)] + sum([[("i", n), ("t", 2)] for n in sizes[:6]], []),
+            [("t", 1)] + sum([[("i", n), ("t", 1)] for n in sizes[6:]], [])]
+    wl = synth.make_custom(reqs, keep_ratio=0.4, parts=("A", "pos"))
+    rng = np.random.default_rng(21)
+    h_cur, h_prior = wl.tensors["h_cur"].copy(), wl.tensors["h_prior"].copy()
+    vis = np.flatnonzero(wl.layout.visual_mask())
+    same = rng.choice(vis, size=len(vis) // 5, replace=False)
+    h_cur[same] = h_prior[same]
+    nan_rows = rng.choice(np.setdiff1d(vis, same), size=40, replace=False)
+    h_cur[nan_rows, 3] = 0x7F80  # +inf in bf16
+    free = np.setdiff1d(vis, np.concatenate([same, nan_rows]))
+    dup_src = rng.choice(vis, size=200)
+    dup_dst = rng.choice(free, size=200, replace=False)
+    h_cur[dup_dst], h_prior[dup_dst] = h_cur[dup_src], h_prior[dup_src]
+    wl.tensors["h_cur"], wl.tensors["h_prior"] = h_cur, h_prior
+    dw = DevWorkload(wl)
+    for kr in (0.05, 0.4, 0.95):
+        krs = np.full(wl.layout.n_requests, kr, dtype=np.float32)
+        out = avtp.prune(dw.L, "hidden_variation", keep_ratio=torch.from_numpy(krs).cuda(), keep_ratio_host=krs,
+                         planes={"pos": dw.t["pos"]}, **dw.score_tensors("hidden_variation"))
+        torch.cuda.synchronize()
+        assert avtp.read_device_status(out.workspace) == avtp.OK
+        got = out.scores.cpu().numpy()
+        # equal rows score 1 - cos within a few fp32 ulps of 0: many exact ties
+        assert np.isnan(got[nan_rows]).all() and (np.abs(got[same]) < 1e-6).all()
+        ref = O.prune(wl.layout, keep_ratio=krs, scores_f32=got, planes={"pos": wl.pos})
+        assert np.array_equal(out.budgets[:wl.layout.n_images].cpu().numpy(), ref["budgets"])
+        assert np.array_equal(out.kept_idx.cpu().numpy(), ref["kept_idx"]), kr
+        assert np.array_equal(out.outputs["pos"].cpu().numpy(), ref["pos"])
+
+
 def test_prune_repeatable_and_deterministic():
     wl, dw = workload("qwen3_vl_8b")
     call = avtp.PruneCall(dw.L, "hidden_variation", keep_ratio=dw.keep_ratio, keep_ratio_host=wl.keep_ratio,
