@@ -112,6 +112,11 @@ typedef struct {
    * FlashAttention-style forward pass. NULL: the library computes it. */
   const float* lse;
   int64_t lse_stride;
+  /* Optional upper bound on the number of text tokens in the whole batch, used
+   * only to size the workspace of AVTP_CRIT_TEXT_ATTENTION (it holds the text
+   * queries repacked by KV group). 0: n_tokens. A batch with more text tokens
+   * than this reports AVTP_ERR_RANGE. */
+  int64_t max_text_tokens;
 } avtp_score_args_t;
 
 typedef struct {

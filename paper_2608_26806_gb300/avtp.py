@@ -55,7 +55,8 @@ class _ScoreArgs(ctypes.Structure):
     _fields_ = [("criterion", c_int), ("h_cur", c_void_p), ("h_prior", c_void_p), ("hidden", c_int32),
                 ("h_cur_stride", c_int64), ("h_prior_stride", c_int64), ("q", c_void_p), ("k", c_void_p),
                 ("n_q_heads", c_int32), ("n_kv_heads", c_int32), ("head_dim", c_int32), ("q_stride", c_int64),
-                ("k_stride", c_int64), ("softmax_scale", c_float), ("lse", c_void_p), ("lse_stride", c_int64)]
+                ("k_stride", c_int64), ("softmax_scale", c_float), ("lse", c_void_p), ("lse_stride", c_int64),
+                ("max_text_tokens", c_int64)]
 
 
 class _AllocArgs(ctypes.Structure):
@@ -164,13 +165,19 @@ class Layout:
     def n_tokens(self) -> int:
         return int(self.host["cu_seqlens"][-1])
 
+    @property
+    def n_text(self) -> int:
+        return self.n_tokens - int(self.host["img_len"].astype(np.int64).sum())
+
     def c(self) -> _Layout:
         return _Layout(self.n_requests, self.n_images, self.n_tokens, _ptr(self.cu_seqlens), _ptr(self.img_cu),
                        _ptr(self.img_start) if self.n_images else None, _ptr(self.img_len) if self.n_images else None)
 
 
-def _score_args(criterion, h_cur=None, h_prior=None, q=None, k=None, softmax_scale=None, lse=None) -> _ScoreArgs:
+def _score_args(criterion, h_cur=None, h_prior=None, q=None, k=None, softmax_scale=None, lse=None,
+                max_text_tokens=0) -> _ScoreArgs:
     a = _ScoreArgs()
+    a.max_text_tokens = int(max_text_tokens)
     a.criterion = _CRITERIA[criterion] if isinstance(criterion, str) else int(criterion)
     if a.criterion == CRIT_HIDDEN_VARIATION:
         for t in (h_cur, h_prior):
@@ -216,7 +223,7 @@ def _row_sets(rows: Sequence[Tuple[torch.Tensor, torch.Tensor]]) -> Tuple[ctypes
 
 def workspace_size(layout: Layout, criterion=None, **score_tensors) -> int:
     lay = layout.c()
-    sa = _score_args(criterion, **score_tensors) if criterion is not None else None
+    sa = _score_args(criterion, max_text_tokens=layout.n_text, **score_tensors) if criterion is not None else None
     out = c_size_t()
     _check(load().avtp_workspace_size(ctypes.byref(lay), ctypes.byref(sa) if sa is not None else None,
                                       ctypes.byref(out)), "avtp_workspace_size")
@@ -233,7 +240,7 @@ def score(layout: Layout, criterion, *, h_cur=None, h_prior=None, q=None, k=None
           scores=None, img_sums=None, workspace=None, stream=None):
     """avtp_score: per-token scores (fp32 [T], text entries untouched) and fixed-point per-image sums."""
     dev = layout.cu_seqlens.device
-    sa = _score_args(criterion, h_cur, h_prior, q, k, softmax_scale, lse)
+    sa = _score_args(criterion, h_cur, h_prior, q, k, softmax_scale, lse, max_text_tokens=layout.n_text)
     if scores is None:
         scores = torch.zeros(layout.n_tokens, dtype=torch.float32, device=dev)
     if img_sums is None:
@@ -377,7 +384,7 @@ class PruneCall:
         self.buffers = buffers or prune_buffers(layout, keep_ratio_host, criterion, score_tensors, rows, planes)
         b = self.buffers
         self._lay = layout.c()
-        self._sa = _score_args(criterion, **score_tensors)
+        self._sa = _score_args(criterion, max_text_tokens=layout.n_text, **score_tensors)
         self._aa = _alloc_args(keep_ratio, alpha, r_min, r_max, relative)
         pairs: List[Tuple[torch.Tensor, torch.Tensor]] = []
         for name, src in rows.items():

@@ -8,8 +8,6 @@
 
 namespace avtp {
 
-int attn_q_tile(int Hq, int Hkv);
-
 namespace {
 
 constexpr size_t kAlign = 256;
@@ -43,7 +41,9 @@ avtp_status_t check_score_args(const avtp_layout_t* L, const avtp_score_args_t* 
     if (a->head_dim != 64 && a->head_dim != 128) return AVTP_ERR_UNSUPPORTED;
     if (a->n_q_heads < 1 || a->n_kv_heads < 1) return AVTP_ERR_INVALID_ARG;
     if (a->n_q_heads % a->n_kv_heads != 0) return AVTP_ERR_UNSUPPORTED;
-    if (a->n_q_heads / a->n_kv_heads > kAttnRowTile) return AVTP_ERR_UNSUPPORTED;
+    if (a->n_q_heads / a->n_kv_heads > kAttnMaxGroupHeads) return AVTP_ERR_UNSUPPORTED;
+    if (a->max_text_tokens < 0) return AVTP_ERR_INVALID_ARG;
+    if (attn_plan(*L, *a).rows > 0x7fffffffLL) return AVTP_ERR_RANGE;
     if (a->q_stride < static_cast<int64_t>(a->n_q_heads) * a->head_dim ||
         a->k_stride < static_cast<int64_t>(a->n_kv_heads) * a->head_dim)
       return AVTP_ERR_INVALID_ARG;
@@ -88,6 +88,22 @@ avtp_status_t record(void* const* events, int i, cudaStream_t s) {
 
 }  // namespace
 
+AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa) {
+  AttnPlan a{};
+  const int64_t T = L.n_tokens;
+  a.G = sa.n_kv_heads > 0 ? sa.n_q_heads / sa.n_kv_heads : 1;
+  a.max_text = (sa.max_text_tokens > 0 && sa.max_text_tokens < T) ? sa.max_text_tokens : T;
+  a.rows = a.max_text * a.G;
+  // every request's row tiles: ceil(rows_r / M) <= rows_r / M + 1
+  a.n_qtiles_max = a.rows / kAttnTileM + L.n_requests + 1;
+  // chunks of at least T / kAttnMaxChunks keys, so that a row tile has at most kAttnMaxChunks
+  int64_t ck = (T + kAttnMaxChunks - 1) / kAttnMaxChunks;
+  ck = (ck + kAttnTileN - 1) / kAttnTileN * kAttnTileN;
+  a.chunk_keys = static_cast<int>(ck > kAttnMinChunkKeys ? ck : kAttnMinChunkKeys);
+  a.p1_items_max = a.n_qtiles_max * kAttnMaxChunks;
+  return a;
+}
+
 WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
   WsPlan p{};
   const size_t R = static_cast<size_t>(L.n_requests), NI = static_cast<size_t>(L.n_images);
@@ -105,12 +121,18 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
   p.img_sums = take(NI * 8 + 8);
   p.scores = take(T * 4 + 4);
   if (sa != nullptr && sa->criterion == AVTP_CRIT_TEXT_ATTENTION) {
+    const AttnPlan a = attn_plan(L, *sa);
+    const size_t Hkv = static_cast<size_t>(sa->n_kv_heads), rows = static_cast<size_t>(a.rows);
     p.text_idx = take(T * 4 + 4);
     p.text_cu = take((R + 1) * 4);
     p.qtile_cu = take((R + 1) * 4);
+    p.p1_cu = take((static_cast<size_t>(a.n_qtiles_max) + 1) * 4);
+    p.p1_cnt = take(Hkv * static_cast<size_t>(a.n_qtiles_max) * 4);
     p.ktile_cu = take((NI + 1) * 4);
-    p.lse = (sa->lse == nullptr) ? take(static_cast<size_t>(sa->n_q_heads) * T * 4 + 4) : 0;
-    p.partial = take(static_cast<size_t>(sa->n_kv_heads) * T * 4 + 4);
+    p.qt = take(Hkv * rows * static_cast<size_t>(sa->head_dim) * 2 + 16);
+    p.lse_rows = take(Hkv * rows * 4 + 4);
+    p.p1_part = (sa->lse == nullptr) ? take(Hkv * static_cast<size_t>(a.p1_items_max) * kAttnTileM * 8) : 0;
+    p.partial = take(Hkv * T * 4 + 4);
   }
   p.total = off;
   return p;
@@ -170,7 +192,10 @@ avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_args_t* a
   pa.L = *layout;
   pa.zero_img_sums = img_sums;
   pa.build_text_tiles = args->criterion == AVTP_CRIT_TEXT_ATTENTION;
-  pa.q_tile = pa.build_text_tiles ? attn_q_tile(args->n_q_heads, args->n_kv_heads) : 1;
+  if (pa.build_text_tiles) {
+    pa.attn = attn_plan(*layout, *args);
+    pa.Hkv = args->n_kv_heads;
+  }
   if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
   return score_impl(layout, args, scores, img_sums, workspace, p, s);
 }
@@ -254,7 +279,10 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   pa.out_cu_seqlens = out_cu_seqlens;
   pa.zero_img_sums = sums;
   pa.build_text_tiles = score_args->criterion == AVTP_CRIT_TEXT_ATTENTION;
-  pa.q_tile = pa.build_text_tiles ? attn_q_tile(score_args->n_q_heads, score_args->n_kv_heads) : 1;
+  if (pa.build_text_tiles) {
+    pa.attn = attn_plan(*layout, *score_args);
+    pa.Hkv = score_args->n_kv_heads;
+  }
   if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
   if ((st = record(step_events, 1, s)) != AVTP_OK) return st;
   if ((st = score_impl(layout, score_args, sc, sums, workspace, p, s)) != AVTP_OK) return st;

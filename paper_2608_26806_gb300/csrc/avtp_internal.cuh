@@ -20,10 +20,13 @@ constexpr float kFxScoreLimit = 1024.f;  // |score| clamp before the fixed-point
 constexpr int kRatioFracBits = 40;       // ratio grid of the budget rule
 constexpr double kRatioLimit = 1048576.0;  // ratios saturate at +-2^20 before the grid
 
-// Tiles of the text-attention criterion (CUDA-core path).
-constexpr int kAttnKeyTile = 64;     // visual keys per pass-2 tile
-constexpr int kAttnRowTile = 64;     // (head, query) rows per tile
-constexpr int kAttnQTile = 16;       // text queries per pass-1 tile (x heads per group <= 64 rows)
+// Tiles of the text-attention criterion (tensor-core path). Rows are (text query, head
+// of the KV group) pairs, G = Hq / Hkv of them per text query, in text order.
+constexpr int kAttnTileM = 128;          // MMA M: rows of a pass-1 tile, keys of a pass-2 tile
+constexpr int kAttnTileN = 256;          // MMA N: keys per pass-1 step, rows per pass-2 step
+constexpr int kAttnMinChunkKeys = 512;   // pass-1 work item: one row tile against a chunk of keys
+constexpr int kAttnMaxChunks = 64;       // chunks per row tile at most (the chunk grows with T)
+constexpr int kAttnMaxGroupHeads = 128;  // Hq / Hkv at most
 
 // ---------------------------------------------------------------- status
 // First word of every workspace. code: first error recorded (0 = none);
@@ -47,14 +50,30 @@ struct WsPlan {
   size_t req_budget;  // int32 [R]: B_r
   size_t img_sums;    // int64 [n_img]: used by avtp_prune when the caller passes NULL
   size_t scores;      // float [T]: used by avtp_prune when the caller passes NULL
-  size_t text_idx;    // int32 [T]: packed position of each text ordinal (criterion B)
-  size_t text_cu;     // int32 [R + 1]: text ordinals per request (criterion B)
-  size_t qtile_cu;    // int32 [R + 1]: pass-1 query tiles per request (criterion B)
-  size_t ktile_cu;    // int32 [n_img + 1]: pass-2 key tiles per image (criterion B)
-  size_t lse;         // float [Hq * T]: per (head, text query) log2-domain LSE (criterion B)
-  size_t partial;     // float [Hkv * T]: per (KV group, visual key) probability sums (criterion B)
+  // criterion B (text attention); "rows" = rows per KV group = max_text * G
+  size_t text_idx;    // int32 [T]: packed position of each text ordinal
+  size_t text_cu;     // int32 [R + 1]: text ordinals per request
+  size_t qtile_cu;    // int32 [R + 1]: pass-1 row tiles per request
+  size_t p1_cu;       // int32 [n_qtiles_max + 1]: pass-1 work items (key chunks) per row tile
+  size_t p1_cnt;      // int32 [Hkv * n_qtiles_max]: finished chunks per (group, row tile)
+  size_t ktile_cu;    // int32 [n_img + 1]: pass-2 key tiles per image
+  size_t qt;          // bf16 [Hkv, rows, d]: the text queries, packed by KV group
+  size_t lse_rows;    // float [Hkv, rows]: log2-domain LSE of every row
+  size_t p1_part;     // float2 [Hkv * p1_items_max * 128]: per-chunk (max, sum) of every row
+  size_t partial;     // float [Hkv * T]: per (KV group, visual key) probability sums
   size_t total;
 };
+
+// Sizes of the text-attention bookkeeping that the host fixes before launch.
+struct AttnPlan {
+  int G;                 // query heads per KV group
+  int64_t max_text;      // text tokens of the whole batch, at most
+  int64_t rows;          // rows per KV group: max_text * G
+  int64_t n_qtiles_max;  // pass-1 row tiles, at most
+  int chunk_keys;        // keys per pass-1 work item
+  int64_t p1_items_max;  // pass-1 work items per KV group, at most
+};
+AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa);
 
 WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa);
 
@@ -150,8 +169,9 @@ struct PrepArgs {
   float r_min, r_max;        // each keep ratio must lie in [r_min, r_max]
   int32_t* out_cu_seqlens;   // NULL: not written
   int64_t* zero_img_sums;    // NULL: not zeroed
-  int build_text_tiles;      // criterion B bookkeeping
-  int q_tile;                // text queries per pass-1 tile (criterion B)
+  int build_text_tiles;      // criterion B bookkeeping, sized by `attn`
+  AttnPlan attn;
+  int Hkv;
 };
 cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s);
 

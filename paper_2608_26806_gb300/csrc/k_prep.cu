@@ -57,7 +57,7 @@ constexpr int kStageInts = 2560;
 
 __global__ void __launch_bounds__(kPrepThreads)
 k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t* req_budget, int32_t* text_idx,
-       int32_t* text_cu, int32_t* qtile_cu, int32_t* ktile_cu, int q_tile) {
+       int32_t* text_cu, int32_t* qtile_cu, int32_t* p1_cu, int32_t* p1_cnt, int32_t* ktile_cu) {
   __shared__ int s_err, s_detail;
   __shared__ int32_t s_warp[32];
   __shared__ int32_t s_stage[kStageInts];
@@ -186,10 +186,30 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
       for (int p = p0 + lane; p < p1; p += 32) text_idx[base + (p - p0)] = cu[r] + p;
     }
     __syncthreads();
-    block_exclusive_scan<int32_t>(
-        R, [&](int r) { return (text_cu[r + 1] - text_cu[r] + q_tile - 1) / q_tile; }, qtile_cu, s_warp);
-    block_exclusive_scan<int32_t>(
-        NI, [&](int i) { return (iln[i] + kAttnKeyTile - 1) / kAttnKeyTile; }, ktile_cu, s_warp);
+    const int G = a.attn.G;
+    if (tid == 0 && static_cast<int64_t>(text_cu[R]) > a.attn.max_text) fail(AVTP_ERR_RANGE, -1);
+    __syncthreads();
+    if (s_err == 0) {
+      // pass 1: row tiles of kAttnTileM (text query, head) rows per request, then key chunks per tile
+      block_exclusive_scan<int32_t>(
+          R, [&](int r) { return ((text_cu[r + 1] - text_cu[r]) * G + kAttnTileM - 1) / kAttnTileM; }, qtile_cu,
+          s_warp);
+      const int nq = qtile_cu[R];
+      const int ck = a.attn.chunk_keys;
+      block_exclusive_scan<int32_t>(
+          nq,
+          [&](int t) {
+            const int r = upper_index(qtile_cu, R, t);
+            const int row_end = min(text_cu[r] * G + (t - qtile_cu[r] + 1) * kAttnTileM, text_cu[r + 1] * G);
+            const int pmax = text_idx[(row_end - 1) / G] - cu[r];  // request-local position of the last query
+            return (pmax + ck) / ck;
+          },
+          p1_cu, s_warp);
+      for (int j = tid; j < a.Hkv * nq; j += blockDim.x) p1_cnt[j] = 0;
+      // pass 2: key tiles of kAttnTileM visual keys per image
+      block_exclusive_scan<int32_t>(
+          NI, [&](int i) { return (iln[i] + kAttnTileM - 1) / kAttnTileM; }, ktile_cu, s_warp);
+    }
   }
 
   if (s_err == 0 && a.zero_img_sums != nullptr) {
@@ -210,13 +230,15 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
 }  // namespace
 
 cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s) {
-  const int q_tile = a.q_tile > 0 ? a.q_tile : 1;
+  const bool b = a.build_text_tiles != 0;
   k_prep<<<1, kPrepThreads, 0, s>>>(a, ws_at<DevStatus>(ws, p.status), ws_at<int32_t>(ws, p.vis_cu),
                                     ws_at<int32_t>(ws, p.img_req), ws_at<int32_t>(ws, p.req_budget),
-                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.text_idx) : nullptr,
-                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.text_cu) : nullptr,
-                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.qtile_cu) : nullptr,
-                                    a.build_text_tiles ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr, q_tile);
+                                    b ? ws_at<int32_t>(ws, p.text_idx) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.text_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.qtile_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.p1_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.p1_cnt) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr);
   return cudaGetLastError();
 }
 

@@ -116,7 +116,7 @@ def test_host_validation_of_score_arguments(lib):
     assert _score(lib, _layout(), _hv_args(hidden=60)) == avtp.ERR_UNSUPPORTED
     assert _score(lib, _layout(), _attn_args(d=96)) == avtp.ERR_UNSUPPORTED
     assert _score(lib, _layout(), _attn_args(hq=30, hkv=8)) == avtp.ERR_UNSUPPORTED
-    assert _score(lib, _layout(), _attn_args(hq=128, hkv=1)) == avtp.ERR_UNSUPPORTED  # group > 64 rows
+    assert _score(lib, _layout(), _attn_args(hq=256, hkv=1)) == avtp.ERR_UNSUPPORTED  # more than 128 heads per KV group
     bad = _attn_args()
     bad.softmax_scale = float("nan")
     assert _score(lib, _layout(), bad) == avtp.ERR_INVALID_ARG
