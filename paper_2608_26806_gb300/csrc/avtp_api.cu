@@ -127,7 +127,6 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
     p.text_cu = take((R + 1) * 4);
     p.qtile_cu = take((R + 1) * 4);
     p.p1_cu = take((static_cast<size_t>(a.n_qtiles_max) + 1) * 4);
-    p.p1_cnt = take(Hkv * static_cast<size_t>(a.n_qtiles_max) * 4);
     p.ktile_cu = take((NI + 1) * 4);
     p.qt = take(Hkv * rows * static_cast<size_t>(sa->head_dim) * 2 + 16);
     p.lse_rows = take(Hkv * rows * 4 + 4);
@@ -194,7 +193,6 @@ avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_args_t* a
   pa.build_text_tiles = args->criterion == AVTP_CRIT_TEXT_ATTENTION;
   if (pa.build_text_tiles) {
     pa.attn = attn_plan(*layout, *args);
-    pa.Hkv = args->n_kv_heads;
   }
   if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
   return score_impl(layout, args, scores, img_sums, workspace, p, s);
@@ -281,7 +279,6 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   pa.build_text_tiles = score_args->criterion == AVTP_CRIT_TEXT_ATTENTION;
   if (pa.build_text_tiles) {
     pa.attn = attn_plan(*layout, *score_args);
-    pa.Hkv = score_args->n_kv_heads;
   }
   if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
   if ((st = record(step_events, 1, s)) != AVTP_OK) return st;

@@ -55,11 +55,10 @@ struct WsPlan {
   size_t text_cu;     // int32 [R + 1]: text ordinals per request
   size_t qtile_cu;    // int32 [R + 1]: pass-1 row tiles per request
   size_t p1_cu;       // int32 [n_qtiles_max + 1]: pass-1 work items (key chunks) per row tile
-  size_t p1_cnt;      // int32 [Hkv * n_qtiles_max]: finished chunks per (group, row tile)
   size_t ktile_cu;    // int32 [n_img + 1]: pass-2 key tiles per image
   size_t qt;          // bf16 [Hkv, rows, d]: the text queries, packed by KV group
   size_t lse_rows;    // float [Hkv, rows]: log2-domain LSE of every row
-  size_t p1_part;     // float2 [Hkv * p1_items_max * 128]: per-chunk (max, sum) of every row
+  size_t p1_part;     // float2 [Hkv * n_qtiles_max][128][kAttnMaxChunks]: per-chunk (max, sum) of every row
   size_t partial;     // float [Hkv * T]: per (KV group, visual key) probability sums
   size_t total;
 };
@@ -171,7 +170,6 @@ struct PrepArgs {
   int64_t* zero_img_sums;    // NULL: not zeroed
   int build_text_tiles;      // criterion B bookkeeping, sized by `attn`
   AttnPlan attn;
-  int Hkv;
 };
 cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s);
 

@@ -57,7 +57,7 @@ constexpr int kStageInts = 2560;
 
 __global__ void __launch_bounds__(kPrepThreads)
 k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t* req_budget, int32_t* text_idx,
-       int32_t* text_cu, int32_t* qtile_cu, int32_t* p1_cu, int32_t* p1_cnt, int32_t* ktile_cu) {
+       int32_t* text_cu, int32_t* qtile_cu, int32_t* p1_cu, int32_t* ktile_cu) {
   __shared__ int s_err, s_detail;
   __shared__ int32_t s_warp[32];
   __shared__ int32_t s_stage[kStageInts];
@@ -205,7 +205,6 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
             return (pmax + ck) / ck;
           },
           p1_cu, s_warp);
-      for (int j = tid; j < a.Hkv * nq; j += blockDim.x) p1_cnt[j] = 0;
       // pass 2: key tiles of kAttnTileM visual keys per image
       block_exclusive_scan<int32_t>(
           NI, [&](int i) { return (iln[i] + kAttnTileM - 1) / kAttnTileM; }, ktile_cu, s_warp);
@@ -237,7 +236,6 @@ cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream
                                     b ? ws_at<int32_t>(ws, p.text_cu) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.qtile_cu) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.p1_cu) : nullptr,
-                                    b ? ws_at<int32_t>(ws, p.p1_cnt) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr);
   return cudaGetLastError();
 }

@@ -10,8 +10,9 @@
 // Pass 1 (skipped when the caller supplies FlashAttention's LSE): a work item is one
 // tile of 128 rows of a request against one chunk of its keys; S = Q_rows K^T runs on
 // the tensor cores (tcgen05.mma, 128 x 256 per step, fp32 accumulator in TMEM) and the
-// epilogue warps keep an online (max, sum) per row. The last item of a tile merges
-// the chunks into lse2.
+// epilogue warps keep an online (max, sum) per row; k_attn_merge then combines the
+// chunks of every row into lse2 (a separate kernel: merging inside pass 1, in
+// whichever item finished a tile last, piled the merges onto a few CTAs).
 // Pass 2: a work item is one tile of 128 visual keys of an image; S^T = K_tile Qt^T
 // over the rows of every text query after the image (all of them see every key of
 // the image), 256 rows per step; each epilogue thread owns one key and sums
@@ -19,11 +20,14 @@
 // Finalize: sum the KV groups in a fixed order (deterministic), divide, and add the
 // fixed-point per-image sums.
 //
-// Both passes are persistent (one CTA per SM). Warps 0-3 are the epilogue (warp w
-// reads TMEM lanes 32w..32w+31), warp 4 issues the TMA loads, warp 5 owns TMEM and
-// issues the MMAs. Shared memory: the item's A tile (128 rows x d) and two stages of
+// Both passes are persistent (one CTA per SM). Warps 0-7 are the epilogue (warp w
+// reads TMEM lanes 32(w%4)..+31, columns 128(w/4)..+127 of each step), warp 8 issues
+// the TMA loads, warp 9 owns TMEM and issues the MMAs. Shared memory: two stages of
+// A tiles (128 rows x d, so the next item's tile loads during this one) and two of
 // B tiles (256 rows x d); TMEM: two 256-column accumulators, so the epilogue of one
-// step overlaps the MMA of the next.
+// step overlaps the MMA of the next. The epilogue keeps four independent partial
+// sums (and maxima) per thread: with two warps per scheduler there is little else
+// to hide the latency of a dependent chain.
 #include <cudaTypedefs.h>
 
 #include "avtp_tc.cuh"
@@ -33,18 +37,20 @@ namespace {
 
 constexpr int kM = kAttnTileM;   // 128
 constexpr int kN = kAttnTileN;   // 256
-constexpr int kThreads = 192;
-constexpr int kEpiThreads = 128;
+constexpr int kEpiWarps = 8;     // warps 0-7: epilogue
+constexpr int kTmaWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kThreads = 320;
 constexpr uint32_t kTmemCols = 2 * kN;
 constexpr float kLog2e = 1.4426950408889634f;
 
-// Shared memory for head_dim d: A tile, then two B stages, 1024-byte aligned.
+// Shared memory for head_dim d: two A stages, then two B stages, 1024-byte aligned.
 __host__ __device__ constexpr size_t a_bytes(int d) { return static_cast<size_t>(kM) * d * 2; }
 __host__ __device__ constexpr size_t b_bytes(int d) { return static_cast<size_t>(kN) * d * 2; }
-__host__ __device__ constexpr size_t tc_smem_bytes(int d) { return 1024 + a_bytes(d) + 2 * b_bytes(d); }
+__host__ __device__ constexpr size_t tc_smem_bytes(int d) { return 1024 + 2 * a_bytes(d) + 2 * b_bytes(d); }
 
 struct Sync {
-  uint64_t a_full, a_empty;
+  uint64_t a_full[2], a_empty[2];
   uint64_t b_full[2], b_empty[2];
   uint64_t acc_full[2], acc_empty[2];
   uint64_t drain;
@@ -66,10 +72,9 @@ struct AttnArgs {
   const int32_t* text_cu;
   const int32_t* qtile_cu;
   const int32_t* p1_cu;
-  int32_t* p1_cnt;
   const int32_t* ktile_cu;
   float* lse_rows;        // [Hkv, rows]
-  float2* p1_part;        // [Hkv * p1_items_max * 128]
+  float2* p1_part;        // [Hkv * n_qtiles_max][128 rows][kAttnMaxChunks]
   float* partial;         // [Hkv, T]
   int64_t rows;           // rows per group
   int64_t p1_items_max;
@@ -78,7 +83,7 @@ struct AttnArgs {
   DevStatus* st;
 };
 
-__device__ __forceinline__ void bar_epi() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+__device__ __forceinline__ void bar_epi() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
 // ---------------------------------------------------------------- work items
 struct P1Item {
@@ -131,49 +136,45 @@ __device__ __forceinline__ P2Item p2_item(const AttnArgs& a, int n_per_group, in
 }
 
 // ---------------------------------------------------------------- the persistent kernel
-// PASS 1: A = Qt rows (map qa, box 64 x 128), B = key tiles (map kb, box 64 x 256).
-// PASS 2: A = key tile (map ka, box 64 x 128), B = Qt rows (map qb, box 64 x 256).
+// PASS 1: A = Qt rows (box 64 x 128), B = key tiles (box 64 x 256).
+// PASS 2: A = key tile (box 64 x 128), B = Qt rows (box 64 x 256).
+// Epilogue warp w reads TMEM lane quadrant w % 4 and column half w / 4 of each step.
 template <int PASS>
 __global__ void __launch_bounds__(kThreads, 1)
 k_attn_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, AttnArgs a) {
   extern __shared__ unsigned char smem_raw[];
   __shared__ Sync sy;
-  __shared__ float s_lse[2][kN];
-  __shared__ int s_last;
+  __shared__ __align__(16) float s_lse[2][kN];
+  __shared__ float2 s_mrg[2][kM];
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  unsigned char* sA = smem;
-  unsigned char* sB[2] = {smem + a_bytes(a.d), smem + a_bytes(a.d) + b_bytes(a.d)};
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int d = a.d;
+  unsigned char* sA[2] = {smem, smem + a_bytes(d)};
+  unsigned char* sB[2] = {smem + 2 * a_bytes(d), smem + 2 * a_bytes(d) + b_bytes(d)};
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t atomA = kM * 128, atomB = kN * 128;  // bytes per 64-element atom column
 
   pdl_wait();
   pdl_trigger();
   if (!a.st->layout_ok) return;
-  int n_per_group;
-  if (PASS == 1) {
-    n_per_group = a.p1_cu[a.qtile_cu[a.R]];
-  } else {
-    n_per_group = a.ktile_cu[a.NI];
-  }
+  const int n_per_group = (PASS == 1) ? a.p1_cu[a.qtile_cu[a.R]] : a.ktile_cu[a.NI];
   const int n_items = n_per_group * a.Hkv;
   if (static_cast<int>(blockIdx.x) >= n_items) return;
 
   if (threadIdx.x == 0) {
-    tc::mbar_init(&sy.a_full, 1);
-    tc::mbar_init(&sy.a_empty, 1);
     for (int s = 0; s < 2; ++s) {
+      tc::mbar_init(&sy.a_full[s], 1);
+      tc::mbar_init(&sy.a_empty[s], 1);
       tc::mbar_init(&sy.b_full[s], 1);
       tc::mbar_init(&sy.b_empty[s], 1);
       tc::mbar_init(&sy.acc_full[s], 1);
-      tc::mbar_init(&sy.acc_empty[s], kEpiThreads / 32);
+      tc::mbar_init(&sy.acc_empty[s], kEpiWarps);
     }
     tc::mbar_init(&sy.drain, 1);
     sy.abort = 0;
     tc::fence_mbar_init();
   }
-  if (warp == 5) {
+  if (warp == kMmaWarp) {
     tc::tmem_alloc(&sy.tmem, kTmemCols);
     tc::tmem_relinquish();
   }
@@ -183,77 +184,75 @@ k_attn_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUte
   const uint32_t tmem = sy.tmem;
   volatile int* abort_flag = &sy.abort;
 
-  if (warp == 4) {
+  // B steps of an item (0: nothing to compute)
+  auto item_steps = [&](int id, int& a_y, int& a_z, int64_t& b0) {
+    if (PASS == 1) {
+      const P1Item it = p1_item(a, n_per_group, id);
+      a_y = static_cast<int>(it.row0);
+      a_z = it.g;
+      b0 = it.key0;
+      return (it.key_end - it.key0 + kN - 1) / kN;
+    }
+    const P2Item it = p2_item(a, n_per_group, id);
+    a_y = it.g;
+    a_z = it.kp0;
+    b0 = it.row_begin;
+    return it.row_end > it.row_begin ? static_cast<int>((it.row_end - it.row_begin + kN - 1) / kN) : 0;
+  };
+
+  if (warp == kTmaWarp) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       tc::tma_prefetch_map(&mapA);
       tc::tma_prefetch_map(&mapB);
       uint32_t na = 0, nb = 0;  // A loads and B loads issued so far
       for (int id = blockIdx.x; id < n_items && !*abort_flag; id += gridDim.x) {
-        int a_y, a_z, steps;
-        int64_t b0;  // first B row of the item (key position or row index)
-        if (PASS == 1) {
-          const P1Item it = p1_item(a, n_per_group, id);
-          a_y = static_cast<int>(it.row0);
-          a_z = it.g;
-          b0 = it.key0;
-          steps = (it.key_end - it.key0 + kN - 1) / kN;
-        } else {
-          const P2Item it = p2_item(a, n_per_group, id);
-          a_y = it.g;
-          a_z = it.kp0;
-          b0 = it.row_begin;
-          steps = it.row_end > it.row_begin ? static_cast<int>((it.row_end - it.row_begin + kN - 1) / kN) : 0;
-        }
+        int a_y, a_z;
+        int64_t b0;
+        const int steps = item_steps(id, a_y, a_z, b0);
         if (steps <= 0) continue;
-        if (na > 0 && !tc::mbar_wait(&sy.a_empty, (na - 1) & 1)) { *abort_flag = 1; break; }
-        tc::mbar_arrive_expect_tx(&sy.a_full, static_cast<uint32_t>(a_bytes(d)));
-        for (int ac = 0; ac < d / 64; ++ac) tc::tma_load_3d(sA + ac * atomA, &mapA, ac * 64, a_y, a_z, &sy.a_full);
+        const int sa = na & 1;
+        if (na >= 2 && !tc::mbar_wait(&sy.a_empty[sa], ((na >> 1) - 1) & 1)) { *abort_flag = 1; break; }
+        tc::mbar_arrive_expect_tx(&sy.a_full[sa], static_cast<uint32_t>(a_bytes(d)));
+        for (int ac = 0; ac < d / 64; ++ac) tc::tma_load_3d(sA[sa] + ac * atomA, &mapA, ac * 64, a_y, a_z, &sy.a_full[sa]);
         ++na;
         for (int st = 0; st < steps; ++st, ++nb) {
           const int s = nb & 1;
           if (nb >= 2 && !tc::mbar_wait(&sy.b_empty[s], ((nb >> 1) - 1) & 1)) { *abort_flag = 1; break; }
           tc::mbar_arrive_expect_tx(&sy.b_full[s], static_cast<uint32_t>(b_bytes(d)));
-          const int64_t y = b0 + static_cast<int64_t>(st) * kN;
+          const int y = static_cast<int>(b0 + static_cast<int64_t>(st) * kN);
           for (int ac = 0; ac < d / 64; ++ac) {
-            if (PASS == 1) {  // keys: map dims {d, Hkv, T}
-              tc::tma_load_3d(sB[s] + ac * atomB, &mapB, ac * 64, a_z, static_cast<int>(y), &sy.b_full[s]);
-            } else {          // rows: map dims {d, rows, Hkv}
-              tc::tma_load_3d(sB[s] + ac * atomB, &mapB, ac * 64, static_cast<int>(y), a_y, &sy.b_full[s]);
-            }
+            if (PASS == 1) tc::tma_load_3d(sB[s] + ac * atomB, &mapB, ac * 64, a_z, y, &sy.b_full[s]);  // {d, Hkv, T}
+            else tc::tma_load_3d(sB[s] + ac * atomB, &mapB, ac * 64, y, a_y, &sy.b_full[s]);            // {d, rows, Hkv}
           }
         }
       }
       // let the copies in flight land before the CTA may exit
-      if (na > 0) tc::mbar_wait(&sy.a_full, (na - 1) & 1);
+      for (uint32_t k = (na >= 2 ? na - 2 : 0); k < na; ++k) tc::mbar_wait(&sy.a_full[k & 1], (k >> 1) & 1);
       for (uint32_t k = (nb >= 2 ? nb - 2 : 0); k < nb; ++k) tc::mbar_wait(&sy.b_full[k & 1], (k >> 1) & 1);
     }
-  } else if (warp == 5) {
+  } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = tc::idesc_bf16(kM, kN);
       uint32_t na = 0, nb = 0;
       for (int id = blockIdx.x; id < n_items && !*abort_flag; id += gridDim.x) {
-        int steps;
-        if (PASS == 1) {
-          const P1Item it = p1_item(a, n_per_group, id);
-          steps = (it.key_end - it.key0 + kN - 1) / kN;
-        } else {
-          const P2Item it = p2_item(a, n_per_group, id);
-          steps = it.row_end > it.row_begin ? static_cast<int>((it.row_end - it.row_begin + kN - 1) / kN) : 0;
-        }
+        int a_y, a_z;
+        int64_t b0;
+        const int steps = item_steps(id, a_y, a_z, b0);
         if (steps <= 0) continue;
-        if (!tc::mbar_wait(&sy.a_full, na & 1)) { *abort_flag = 1; break; }
+        const int sa = na & 1;
+        if (!tc::mbar_wait(&sy.a_full[sa], (na >> 1) & 1)) { *abort_flag = 1; break; }
         for (int st = 0; st < steps; ++st, ++nb) {
           const int s = nb & 1;
           if (!tc::mbar_wait(&sy.b_full[s], (nb >> 1) & 1)) { *abort_flag = 1; break; }
           if (nb >= 2 && !tc::mbar_wait(&sy.acc_empty[s], ((nb >> 1) - 1) & 1)) { *abort_flag = 1; break; }
           tc::fence_after_sync();
-          tc::mma_rows(tmem + s * kN, tc::smem_u32(sA), atomA, tc::smem_u32(sB[s]), atomB, d, idesc);
+          tc::mma_rows(tmem + s * kN, tc::smem_u32(sA[sa]), atomA, tc::smem_u32(sB[s]), atomB, d, idesc);
           tc::mma_commit(&sy.b_empty[s]);
           tc::mma_commit(&sy.acc_full[s]);
         }
-        tc::mma_commit(&sy.a_empty);
+        tc::mma_commit(&sy.a_empty[sa]);
         ++na;
       }
       // every MMA issued has completed once this arrives
@@ -261,127 +260,188 @@ k_attn_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUte
       tc::mbar_wait(&sy.drain, 0);
     }
   } else {
-    // ------------------------------------------------------------ epilogue (128 threads)
-    const int etid = threadIdx.x;                       // 0..127 = TMEM lane
-    const uint32_t lane_addr = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    // ------------------------------------------------------------ epilogue (8 warps)
+    const int etid = threadIdx.x;               // 0 .. 255
+    const int quad = warp & 3, half = warp >> 2;
+    const int lrow = quad * 32 + lane;          // TMEM lane: row (pass 1) or key (pass 2) of the tile
+    const uint32_t taddr = tmem + (static_cast<uint32_t>(quad * 32) << 16) + half * (kN / 2);
+    const float c2 = a.c2;
+    // After a timeout (abort_flag) the epilogue keeps walking the same items and steps,
+    // skipping every wait and TMEM read, so that its named barriers still line up.
     uint32_t nb = 0;
-    for (int id = blockIdx.x; id < n_items && !*abort_flag; id += gridDim.x) {
+    int it_count = 0;
+    for (int id = blockIdx.x; id < n_items; id += gridDim.x, ++it_count) {
+      const int slot = it_count & 1;
       if (PASS == 1) {
         const P1Item it = p1_item(a, n_per_group, id);
         const int steps = (it.key_end - it.key0 + kN - 1) / kN;
-        const int64_t row = it.row0 + etid;
+        const int64_t row = it.row0 + lrow;
         const bool valid = row < it.row_end;
         const int qpos = valid ? a.text_idx[row / a.G] : -1;
-        // keys k0 + j with k0 + j <= min(qpos, key_end - 1) are visible to this row
+        // keys up to min(qpos, key_end - 1) are visible to this row
         const int last = min(qpos, it.key_end - 1);
-        float m = -INFINITY, l = 0.f;
+        float m = -INFINITY, l = 0.f;  // running max and sum, scaled (log2) domain
         for (int st = 0; st < steps; ++st, ++nb) {
           const int s = nb & 1;
-          if (!tc::mbar_wait_warp(&sy.acc_full[s], (nb >> 1) & 1)) { *abort_flag = 1; break; }
+          bool ok = !__any_sync(0xffffffffu, *abort_flag != 0);
+          if (ok && !tc::mbar_wait_warp(&sy.acc_full[s], (nb >> 1) & 1)) {
+            if (lane == 0) *abort_flag = 1;
+            ok = false;
+          }
           tc::fence_after_sync();
-          const int k0 = it.key0 + st * kN;
-          const int lim = last - k0;  // columns 0..lim are visible
+          const int k0 = it.key0 + st * kN + half * (kN / 2);  // key of this thread's first column
+          const int lim = last - k0;                            // columns 0..lim are visible
+          const bool all_visible = __all_sync(0xffffffffu, lim >= kN / 2 - 1);
+          const bool any_visible = __any_sync(0xffffffffu, lim >= 0);
+          if (ok && any_visible) {
 #pragma unroll 1
-          for (int p = 0; p < kN / 32; ++p) {
-            float v[32];
-            tc::tmem_ld32(lane_addr + s * kN + p * 32, v);
-            float pm = -INFINITY;
+            for (int p = 0; p < kN / 2 / 64; ++p) {
+              float v[64];
+              tc::tmem_ld64(taddr + s * kN + p * 64, v);
+              if (!all_visible) {
 #pragma unroll
-            for (int q = 0; q < 32; ++q) {
-              v[q] = (p * 32 + q <= lim) ? v[q] * a.c2 : -INFINITY;
-              pm = fmaxf(pm, v[q]);
-            }
-            const float mn = fmaxf(m, pm);
-            if (mn != -INFINITY) {
-              float sum = 0.f;
+                for (int q = 0; q < 64; ++q) v[q] = (p * 64 + q <= lim) ? v[q] : -INFINITY;
+              }
+              float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
 #pragma unroll
-              for (int q = 0; q < 32; ++q) sum += tc::ex2(v[q] - mn);
-              l = l * tc::ex2(m - mn) + sum;
-              m = mn;
+              for (int q = 4; q < 64; q += 4) {
+                mx0 = fmaxf(mx0, v[q]);
+                mx1 = fmaxf(mx1, v[q + 1]);
+                mx2 = fmaxf(mx2, v[q + 2]);
+                mx3 = fmaxf(mx3, v[q + 3]);
+              }
+              const float mn = fmaxf(m, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * c2);
+              if (mn != -INFINITY) {
+                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+                for (int q = 0; q < 64; q += 4) {
+                  s0 += tc::ex2(fmaf(v[q], c2, -mn));
+                  s1 += tc::ex2(fmaf(v[q + 1], c2, -mn));
+                  s2 += tc::ex2(fmaf(v[q + 2], c2, -mn));
+                  s3 += tc::ex2(fmaf(v[q + 3], c2, -mn));
+                }
+                l = l * tc::ex2(m - mn) + ((s0 + s1) + (s2 + s3));
+                m = mn;
+              }
             }
           }
           tc::fence_before_sync();
           __syncwarp();
           if (lane == 0) tc::mbar_arrive(&sy.acc_empty[s]);
         }
-        if (*abort_flag) break;
-        // this chunk's (max, sum) per row; the last chunk of the tile merges them
-        const int64_t slot = (static_cast<int64_t>(id) * kM + etid);
-        a.p1_part[slot] = make_float2(m, l);
-        __threadfence();
+        // the two column halves of a row meet here; this chunk's (max, sum) per row goes
+        // to [row tile][row][chunk] for k_attn_merge
+        if (half == 1) s_mrg[slot][lrow] = make_float2(m, l);
         bar_epi();
-        if (etid == 0) {
-          const int nq = a.qtile_cu[a.R];
-          const int nc = a.p1_cu[it.qt + 1] - a.p1_cu[it.qt];
-          const int prev = atomicAdd(&a.p1_cnt[it.g * nq + it.qt], 1);
-          s_last = (prev == nc - 1) ? 1 : 0;
-          if (s_last) a.p1_cnt[it.g * nq + it.qt] = 0;  // ready for the next call
-        }
-        bar_epi();
-        if (s_last) {
-          __threadfence();
-          const int nc = a.p1_cu[it.qt + 1] - a.p1_cu[it.qt];
-          const int id0 = it.g * n_per_group + a.p1_cu[it.qt];
-          float M = -INFINITY;
-          for (int c = 0; c < nc; ++c) M = fmaxf(M, __ldcg(&a.p1_part[(static_cast<int64_t>(id0) + c) * kM + etid]).x);
-          float L = 0.f;
-          if (M != -INFINITY) {
-            for (int c = 0; c < nc; ++c) {
-              const float2 ml = __ldcg(&a.p1_part[(static_cast<int64_t>(id0) + c) * kM + etid]);
-              if (ml.x != -INFINITY) L += ml.y * tc::ex2(ml.x - M);
-            }
-          }
-          if (valid) a.lse_rows[static_cast<int64_t>(it.g) * a.rows + row] = M + __log2f(L);
+        if (half == 0) {
+          const float2 o = s_mrg[slot][lrow];
+          const float M = fmaxf(m, o.x);
+          const float L = (M == -INFINITY) ? 0.f : l * tc::ex2(m - M) + o.y * tc::ex2(o.x - M);
+          const int64_t tile = static_cast<int64_t>(it.g) * a.qtile_cu[a.R] + it.qt;
+          a.p1_part[(tile * kM + lrow) * kAttnMaxChunks + it.chunk] = make_float2(M, L);
         }
       } else {
         const P2Item it = p2_item(a, n_per_group, id);
         const int steps =
             it.row_end > it.row_begin ? static_cast<int>((it.row_end - it.row_begin + kN - 1) / kN) : 0;
         const float* lse_g = a.lse_rows + static_cast<int64_t>(it.g) * a.rows;
-        float mass = 0.f;
+        // the rows' lse2 (+inf past the last row, which zeroes their terms); the next
+        // step's value is loaded while this step is processed
+        auto lse_of = [&](int st) {
+          const int64_t r = it.row_begin + static_cast<int64_t>(st) * kN + etid;
+          return (st < steps && r < it.row_end) ? lse_g[r] : INFINITY;
+        };
+        float lse_next = lse_of(0);
+        float m0 = 0.f, m1 = 0.f, m2 = 0.f, m3 = 0.f;
         for (int st = 0; st < steps; ++st, ++nb) {
           const int s = nb & 1;
-          // the rows' lse2 (+inf past the last row, which zeroes their terms)
-          const int64_t r0 = it.row_begin + static_cast<int64_t>(st) * kN;
-#pragma unroll
-          for (int h = 0; h < kN / kEpiThreads; ++h) {
-            const int j = etid + h * kEpiThreads;
-            s_lse[s][j] = (r0 + j < it.row_end) ? lse_g[r0 + j] : INFINITY;
-          }
+          s_lse[s][etid] = lse_next;
           bar_epi();
-          if (!tc::mbar_wait_warp(&sy.acc_full[s], (nb >> 1) & 1)) { *abort_flag = 1; break; }
+          lse_next = lse_of(st + 1);
+          bool ok = !__any_sync(0xffffffffu, *abort_flag != 0);
+          if (ok && !tc::mbar_wait_warp(&sy.acc_full[s], (nb >> 1) & 1)) {
+            if (lane == 0) *abort_flag = 1;
+            ok = false;
+          }
           tc::fence_after_sync();
 #pragma unroll 1
-          for (int p = 0; p < kN / 32; ++p) {
-            float v[32];
-            tc::tmem_ld32(lane_addr + s * kN + p * 32, v);
-            const float4* l4 = reinterpret_cast<const float4*>(&s_lse[s][p * 32]);
+          for (int p = 0; p < (ok ? kN / 2 / 64 : 0); ++p) {
+            float v[64];
+            tc::tmem_ld64(taddr + s * kN + p * 64, v);
+            const float4* l4 = reinterpret_cast<const float4*>(&s_lse[s][half * (kN / 2) + p * 64]);
 #pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4) {
+            for (int q4 = 0; q4 < 16; ++q4) {
               const float4 lv = l4[q4];
-              mass += tc::ex2(fmaf(v[4 * q4 + 0], a.c2, -lv.x));
-              mass += tc::ex2(fmaf(v[4 * q4 + 1], a.c2, -lv.y));
-              mass += tc::ex2(fmaf(v[4 * q4 + 2], a.c2, -lv.z));
-              mass += tc::ex2(fmaf(v[4 * q4 + 3], a.c2, -lv.w));
+              m0 += tc::ex2(fmaf(v[4 * q4 + 0], c2, -lv.x));
+              m1 += tc::ex2(fmaf(v[4 * q4 + 1], c2, -lv.y));
+              m2 += tc::ex2(fmaf(v[4 * q4 + 2], c2, -lv.z));
+              m3 += tc::ex2(fmaf(v[4 * q4 + 3], c2, -lv.w));
             }
           }
           tc::fence_before_sync();
           __syncwarp();
           if (lane == 0) tc::mbar_arrive(&sy.acc_empty[s]);
         }
-        if (*abort_flag) break;
-        if (etid < it.nk) a.partial[static_cast<int64_t>(it.g) * a.T + it.kp0 + etid] = mass;
+        const float mass = (m0 + m1) + (m2 + m3);
+        if (half == 1) s_mrg[slot][lrow].x = mass;
+        bar_epi();
+        if (half == 0 && lrow < it.nk)
+          a.partial[static_cast<int64_t>(it.g) * a.T + it.kp0 + lrow] = mass + s_mrg[slot][lrow].x;
       }
     }
   }
 
   tc::fence_before_sync();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kMmaWarp) {
     tc::fence_after_sync();
     tc::tmem_dealloc(tmem, kTmemCols);
   }
   if (threadIdx.x == 0 && sy.abort) record_error(a.st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));
+}
+
+// ---------------------------------------------------------------- pass-1 chunk merge
+// lse2 of every row: the log2-sum-exp2 merge of its chunks' (max, sum). One thread per
+// (KV group, row); a row's chunks are contiguous.
+__global__ void __launch_bounds__(256)
+k_attn_merge(AttnArgs a) {
+  pdl_wait();
+  pdl_trigger();
+  if (!a.st->layout_ok) return;
+  const int nq = a.qtile_cu[a.R];
+  const int64_t total = static_cast<int64_t>(a.Hkv) * nq * kM;
+  for (int64_t u = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; u < total;
+       u += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int lr = static_cast<int>(u % kM);
+    const int64_t tile = u / kM;
+    const int g = static_cast<int>(tile / nq), qt = static_cast<int>(tile - static_cast<int64_t>(g) * nq);
+    const int r = upper_index(a.qtile_cu, a.R, qt);
+    const int64_t row = static_cast<int64_t>(a.text_cu[r]) * a.G + static_cast<int64_t>(qt - a.qtile_cu[r]) * kM + lr;
+    if (row >= static_cast<int64_t>(a.text_cu[r + 1]) * a.G) continue;
+    const int nc = a.p1_cu[qt + 1] - a.p1_cu[qt];
+    const float4* src = reinterpret_cast<const float4*>(a.p1_part + u * kAttnMaxChunks);
+    float M = -INFINITY, L = 0.f;
+    auto merge = [&](float mc, float lc) {
+      const float Mn = fmaxf(M, mc);
+      if (Mn != -INFINITY) {
+        L = L * tc::ex2(M - Mn) + lc * tc::ex2(mc - Mn);
+        M = Mn;
+      }
+    };
+    const int n4 = (nc + 1) >> 1;  // a float4 holds two chunks
+    for (int c4 = 0; c4 < n4; c4 += 8) {
+      float4 buf[8];
+#pragma unroll
+      for (int w = 0; w < 8; ++w)
+        buf[w] = (c4 + w < n4) ? __ldg(src + c4 + w) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+#pragma unroll
+      for (int w = 0; w < 8; ++w) {
+        merge(buf[w].x, buf[w].y);
+        if (2 * (c4 + w) + 1 < nc) merge(buf[w].z, buf[w].w);
+      }
+    }
+    a.lse_rows[static_cast<int64_t>(g) * a.rows + row] = M + __log2f(L);
+  }
 }
 
 // ---------------------------------------------------------------- repacking of the text queries
@@ -500,7 +560,6 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   a.text_cu = ws_at<int32_t>(ws, p.text_cu);
   a.qtile_cu = ws_at<int32_t>(ws, p.qtile_cu);
   a.p1_cu = ws_at<int32_t>(ws, p.p1_cu);
-  a.p1_cnt = ws_at<int32_t>(ws, p.p1_cnt);
   a.ktile_cu = ws_at<int32_t>(ws, p.ktile_cu);
   a.lse_rows = ws_at<float>(ws, p.lse_rows);
   a.p1_part = sa.lse == nullptr ? ws_at<float2>(ws, p.p1_part) : nullptr;
@@ -537,6 +596,12 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   }
   if (sa.lse == nullptr) {
     cudaError_t e = launch_kernel(k_attn_tc<1>, dim3(sms), dim3(kThreads), smem, s, /*pdl=*/true, mq128, mk256, a);
+    if (e != cudaSuccess) return e;
+    const int64_t rows_max = static_cast<int64_t>(Hkv) * plan.n_qtiles_max * kM;
+    const int64_t cap = static_cast<int64_t>(sms) * 4;
+    const int64_t want = (rows_max + 255) / 256;
+    e = launch_kernel(k_attn_merge, dim3(static_cast<unsigned>(want < cap ? want : cap)), dim3(256), 0, s,
+                      /*pdl=*/true, a);
     if (e != cudaSuccess) return e;
   }
   cudaError_t e = launch_kernel(k_attn_tc<2>, dim3(sms), dim3(kThreads), smem, s, /*pdl=*/true, mk128, mq256, a);
