@@ -134,6 +134,18 @@ __device__ __forceinline__ int64_t grid_mean(int64_t S, int64_t inv_n) {
   return round_shift_sat(static_cast<__int128>(S) * inv_n, kRecipBits, INT64_MAX);
 }
 
+// ceil(a / N) for N >= 1 and |a| < 2^62, from inv_N = floor(2^62 / N): the product gives
+// the quotient to within one, which a multiply-back corrects (no division instruction).
+__device__ __forceinline__ int64_t ceil_div_recip(int64_t a, int64_t N, int64_t inv_N) {
+  const uint64_t u = static_cast<uint64_t>(a >= 0 ? a : -a);
+  uint64_t q = static_cast<uint64_t>((static_cast<unsigned __int128>(u) * static_cast<uint64_t>(inv_N)) >> kRecipBits);
+  uint64_t r = u - q * static_cast<uint64_t>(N);  // q <= floor(u / N) <= q + 2
+  if (r >= static_cast<uint64_t>(N)) { ++q; r -= static_cast<uint64_t>(N); }
+  if (r >= static_cast<uint64_t>(N)) { ++q; r -= static_cast<uint64_t>(N); }
+  // now q = floor(u / N), r = u mod N
+  return a >= 0 ? static_cast<int64_t>(q + (r != 0 ? 1 : 0)) : -static_cast<int64_t>(q);
+}
+
 // R_i from Ibar_i, Ibar_avg and (relative rule only) floor(2^62 / |Ibar_avg|).
 __device__ __forceinline__ int64_t grid_ratio(const RatioRule& q, int64_t ibar, int64_t avg, int64_t inv_avg) {
   const int64_t d = ibar - avg;
@@ -281,6 +293,25 @@ static __device__ __noinline__ int warp_allocate(const WarpAllocSmem& sm, int m,
   return AVTP_ERR_RANGE;
 }
 
+// The k-th largest (1 <= k <= 32) of the 32 lanes' values: a bitonic sort across the
+// warp (15 compare-exchange stages by shuffle), then one broadcast. Out of line and
+// rolled: it is fetched once per call from a cold instruction cache.
+static __device__ __noinline__ uint64_t warp_kth_largest(uint64_t v, int k) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll 1
+  for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll 1
+    for (int j = size >> 1; j > 0; j >>= 1) {
+      const uint64_t p = __shfl_xor_sync(0xffffffffu, v, j);
+      // descending overall: the lower lane of a pair keeps the larger value in blocks
+      // whose `size` bit is clear, the smaller one otherwise
+      const bool keep_max = ((lane & j) == 0) == ((lane & size) == 0);
+      v = keep_max ? (p > v ? p : v) : (p < v ? p : v);
+    }
+  }
+  return __shfl_sync(0xffffffffu, v, k - 1);
+}
+
 // lambda from the breakpoints, for warp_allocate32 when a clamp binds near the
 // unclamped solution. Out of line: it is the rare case, and its code is only
 // fetched when it runs.
@@ -329,6 +360,7 @@ static __device__ __noinline__ int64_t breakpoint_lambda32(int m, int64_t R, int
 
 // The same rule for requests of at most 32 images, held in registers: lane j owns
 // image j (S_j, n_j in; its budget out). Identical results and status to warp_allocate.
+// Out of line so that a warm-up call and the real one share the same code.
 // inv_n = floor(2^62 / n_j) and inv_N = floor(2^62 / N) come from the caller, which
 // can take them before the sums are ready; after that no division is left on the
 // common path.
@@ -336,8 +368,9 @@ static __device__ __noinline__ int64_t breakpoint_lambda32(int m, int64_t R, int
 // solution is lambda0 = ceil((B * 2^40 - sum n_i R_i) / N); when no clamp binds
 // at lambda0 - 1 or lambda0, G is that line on [lambda0 - 1, lambda0] and
 // lambda0 is exact. Otherwise the breakpoints decide.
-inline __device__ int warp_allocate32(int m, int64_t S, int32_t n, int64_t inv_n, int64_t B, int32_t N, int64_t inv_N,
-                                       const RatioRule& rule, int64_t Rmin, int64_t Rmax, int32_t* k_out) {
+static __device__ __noinline__ int warp_allocate32(int m, int64_t S, int32_t n, int64_t inv_n, int64_t B, int32_t N,
+                                                   int64_t inv_N, const RatioRule& rule, int64_t Rmin, int64_t Rmax,
+                                                   int32_t* k_out) {
   const int lane = threadIdx.x & 31;
   const bool has = lane < m;
   // ---- ratios on the grid
@@ -357,8 +390,8 @@ inline __device__ int warp_allocate32(int m, int64_t S, int32_t n, int64_t inv_n
   const int64_t kSafe = int64_t(1) << 42;  // keeps n * R and the sums inside int64
   if (mx <= kSafe && mn >= -kSafe) {
     const int64_t snr = warp_sum(nl * R);
-    const int64_t num = target - snr;  // smallest lam0 with snr + N * lam0 >= target
-    const int64_t lam0 = num >= 0 ? (num + N - 1) / N : -((-num) / N);
+    const int64_t num = target - snr;  // smallest lam0 with snr + N * lam0 >= target: ceil(num / N)
+    const int64_t lam0 = ceil_div_recip(num, N, inv_N);
     const bool ok = !has || (R + lam0 - 1 >= Rmin && R + lam0 <= Rmax);
     if (__all_sync(0xffffffffu, ok)) {
       lam = lam0;
@@ -379,21 +412,17 @@ inline __device__ int warp_allocate32(int m, int64_t S, int32_t n, int64_t inv_n
       return AVTP_OK;
     }
     const bool elig = has && (D > 0 ? K < n : K > 0);
-    // remainders are below 2^40: split them so each shuffle moves 32 bits
-    const uint32_t xh = static_cast<uint32_t>(X >> 20), xl = static_cast<uint32_t>(X & 0xFFFFF);
-    const unsigned elig_mask = __ballot_sync(0xffffffffu, elig);
-    int rank = 0;
-    // kept rolled: this code runs once per call from a cold instruction cache,
-    // where fetching unrolled code costs far more than the loop's latency
-#pragma unroll 1
-    for (int l = 0; l < m; ++l) {
-      const uint32_t h = __shfl_sync(0xffffffffu, xh, l), lo = __shfl_sync(0xffffffffu, xl, l);
-      const bool gt = h > xh || (h == xh && lo > xl), eq = h == xh && lo == xl;
-      // ahead of this lane: larger remainder (ties: lower index) when adding, the reverse when removing
-      const bool ahead = D > 0 ? (gt || (eq && l < lane)) : (!gt && !eq) || (eq && l > lane);
-      rank += (((elig_mask >> l) & 1u) && ahead) ? 1 : 0;
-    }
-    if (elig && rank < (D > 0 ? D : -D)) K += D > 0 ? 1 : -1;
+    // One unique key per eligible lane, larger = served first: adding, larger
+    // remainder then lower index; removing, smaller remainder then higher index.
+    // Remainders are below 2^40, so a key fits in 45 bits; ineligible lanes get 0.
+    const uint64_t rem = static_cast<uint64_t>(X);
+    const uint64_t key = !elig ? 0ull
+                         : (D > 0 ? (rem << 5) | static_cast<uint64_t>(31 - lane)
+                                  : (((uint64_t(1) << kRatioFracBits) - 1 - rem) << 5) | static_cast<uint64_t>(lane));
+    // the |D|-th largest key (0 when fewer lanes are eligible): every eligible lane at
+    // or above it moves by one
+    const uint64_t thr = warp_kth_largest(key, static_cast<int>(D > 0 ? (D < 32 ? D : 32) : (-D < 32 ? -D : 32)));
+    if (elig && key >= thr) K += D > 0 ? 1 : -1;
   }
   *k_out = K;
   return AVTP_ERR_RANGE;

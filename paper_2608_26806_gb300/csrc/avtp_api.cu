@@ -157,6 +157,12 @@ int device_sm_count() {
   return cached[dev];
 }
 
+int prune_reserve_sms(const avtp_layout_t& L) {
+  if (L.n_tokens > 32768 || L.n_images < 1) return 0;
+  const int64_t ctas = static_cast<int64_t>(L.n_images) + L.n_requests;
+  return static_cast<int>(ctas < 24 ? ctas : 24);
+}
+
 }  // namespace avtp
 
 using namespace avtp;
@@ -172,9 +178,11 @@ avtp_status_t avtp_workspace_size(const avtp_layout_t* layout, const avtp_score_
   return AVTP_OK;
 }
 
+
 static avtp_status_t score_impl(const avtp_layout_t* L, const avtp_score_args_t* a, float* scores,
-                                int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s) {
-  if (a->criterion == AVTP_CRIT_HIDDEN_VARIATION) return from_cuda(launch_score_hvar(*L, *a, scores, img_sums, ws, p, s));
+                                int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s, int reserve_sms = 0) {
+  if (a->criterion == AVTP_CRIT_HIDDEN_VARIATION)
+    return from_cuda(launch_score_hvar(*L, *a, scores, img_sums, ws, p, s, reserve_sms));
   return from_cuda(launch_score_attn(*L, *a, scores, img_sums, ws, p, s));
 }
 
@@ -282,10 +290,11 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   }
   if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
   if ((st = record(step_events, 1, s)) != AVTP_OK) return st;
-  if ((st = score_impl(layout, score_args, sc, sums, workspace, p, s)) != AVTP_OK) return st;
+  const int reserve = score_args->criterion == AVTP_CRIT_HIDDEN_VARIATION ? prune_reserve_sms(*layout) : 0;
+  if ((st = score_impl(layout, score_args, sc, sums, workspace, p, s, reserve)) != AVTP_OK) return st;
   if ((st = record(step_events, 2, s)) != AVTP_OK) return st;
   if ((st = from_cuda(launch_alloc_select(*layout, sums, *alloc_args, budgets, sc, out_cu_seqlens, kept_idx, n_kept,
-                                          workspace, p, s))) != AVTP_OK)
+                                          workspace, p, s, reserve))) != AVTP_OK)
     return st;
   if ((st = record(step_events, 3, s)) != AVTP_OK) return st;
   if ((st = from_cuda(launch_compact(kept_idx, n_kept, layout->n_tokens, sets, n_sets, workspace, p, s))) != AVTP_OK)

@@ -173,8 +173,9 @@ struct PrepArgs {
 };
 cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s);
 
+// reserve_sms: SMs left free for the next kernel of the fused stage (see prune_reserve_sms).
 cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
-                              int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s);
+                              int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s, int reserve_sms = 0);
 
 cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
                               int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s);
@@ -186,10 +187,19 @@ cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int
                           const int32_t* out_cu_seqlens, int32_t* kept_idx, int64_t n_kept, void* ws,
                           const WsPlan& p, cudaStream_t s);
 
-// Budget rule and selection in one kernel (the fused stage).
+// Budget rule and selection in one kernel (the fused stage). Its first warm_ctas CTAs
+// run the code once on made-up data before waiting for the scores (see prune_reserve_sms).
 cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
                                 int32_t* budgets, const float* scores, const int32_t* out_cu_seqlens,
-                                int32_t* kept_idx, int64_t n_kept, void* ws, const WsPlan& p, cudaStream_t s);
+                                int32_t* kept_idx, int64_t n_kept, void* ws, const WsPlan& p, cudaStream_t s,
+                                int warm_ctas = 0);
+
+// In avtp_prune with the hidden-variation criterion on a small batch, the scoring
+// kernel leaves this many SMs free so that the selection kernel's CTAs (one per image)
+// start while the scores stream in and warm their instruction caches; 0 otherwise.
+// On a request of about 10k tokens this trades about 1 us of scoring for about 3 us
+// of allocation and selection; on large batches the scoring time would grow instead.
+int prune_reserve_sms(const avtp_layout_t& L);
 
 cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
                            int n_sets, void* ws, const WsPlan& p, cudaStream_t s);

@@ -36,8 +36,11 @@ constexpr int kChunkBytes = kChunkElems * 2;
 constexpr int kSlotBytes = 2 * kChunkBytes;
 constexpr size_t kSmemBytes = static_cast<size_t>(kWarps) * kSlots * kSlotBytes;  // 192 KiB
 constexpr uint32_t kMaxSpins = 1u << 22;  // bounded mbarrier wait
-constexpr int kStageImages = 2048;        // layouts up to this many images are staged in shared memory
-constexpr int kStageRequests = 512;
+// Layouts up to this many images / requests are staged in shared memory. Kept small
+// (about 10 KiB with the barriers) so that a CTA of the selection kernel, launched
+// while this kernel still runs, fits on the same SM next to the 192-KiB pipeline.
+constexpr int kStageImages = 1024;
+constexpr int kStageRequests = 256;
 
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
@@ -79,6 +82,17 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
           "r"(smem_addr(dst)),
       "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
       : "memory");
+}
+
+// Two fp32 FMAs in one instruction (fma.rn.f32x2), each rounded as fmaf would be.
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
 }
 
 // Ordinal -> packed position map: image i covers visual ordinals [vcu[i], vcu[i+1])
@@ -227,7 +241,8 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   }
   bool timed_out = false;
   bool waited = false;  // the validation kernel (which zeroes img_sums) is known to be done
-  float dot = 0.f, na = 0.f, nb = 0.f;
+  // per lane: even and odd elements accumulate separately (one paired FMA each)
+  float2 dot2 = make_float2(0.f, 0.f), na2 = dot2, nb2 = dot2;
   int slot_take = 0;
   int64_t take_v = w0;
   int take_chunk = 0;
@@ -257,18 +272,16 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     const uint4* b = reinterpret_cast<const uint4*>(wbuf + static_cast<size_t>(slot_take) * kSlotBytes + kChunkBytes);
     for (int c = lane; c < (ne >> 3); c += 32) {
       const uint4 va = a[c], vb = b[c];
-      const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&va);
-      const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&vb);
+      const uint32_t* pa = reinterpret_cast<const uint32_t*>(&va);
+      const uint32_t* pb = reinterpret_cast<const uint32_t*>(&vb);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const float2 fa = __bfloat1622float2(pa[j]);
-        const float2 fb = __bfloat1622float2(pb[j]);
-        dot = fmaf(fa.x, fb.x, dot);
-        dot = fmaf(fa.y, fb.y, dot);
-        na = fmaf(fa.x, fa.x, na);
-        na = fmaf(fa.y, fa.y, na);
-        nb = fmaf(fb.x, fb.x, nb);
-        nb = fmaf(fb.y, fb.y, nb);
+        // a bf16 pair widens to two fp32 values by placing each in the high half of a word
+        const float2 fa = make_float2(__uint_as_float(pa[j] << 16), __uint_as_float(pa[j] & 0xffff0000u));
+        const float2 fb = make_float2(__uint_as_float(pb[j] << 16), __uint_as_float(pb[j] & 0xffff0000u));
+        dot2 = ffma2(fa, fb, dot2);
+        na2 = ffma2(fa, fa, na2);
+        nb2 = ffma2(fb, fb, nb2);
       }
     }
     __syncwarp();
@@ -282,8 +295,8 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     }
     slot_take = (slot_take + 1) % kSlots;
     if (row_done) {
-      const float d = warp_sum(dot), x = warp_sum(na), y = warp_sum(nb);
-      dot = na = nb = 0.f;
+      const float d = warp_sum(dot2.x + dot2.y), x = warp_sum(na2.x + na2.y), y = warp_sum(nb2.x + nb2.y);
+      dot2 = na2 = nb2 = make_float2(0.f, 0.f);
       const int64_t t = map.position(take_v, take_img);
       const bool inside = t >= 0 && t < T;
       const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
@@ -320,7 +333,7 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
 }  // namespace
 
 cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
-                              int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s) {
+                              int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s, int reserve_sms) {
   if (L.n_images == 0 || L.n_tokens == 0) return cudaSuccess;
   static bool attr_set = false;
   if (!attr_set) {
@@ -330,7 +343,9 @@ cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& s
     attr_set = true;
   }
   const int64_t want = (L.n_tokens + kWarps - 1) / kWarps;
-  const int64_t cap = static_cast<int64_t>(device_sm_count());  // one 192 KiB CTA per SM
+  // one 192 KiB CTA per SM, except the SMs left to the next kernel
+  int64_t cap = static_cast<int64_t>(device_sm_count()) - reserve_sms;
+  if (cap < 1) cap = 1;
   const int grid = static_cast<int>(want < cap ? want : cap);
   cudaError_t e = launch_kernel(k_score_hvar, dim3(grid), dim3(kThreads), kSmemBytes, s, /*pdl=*/true,
                                 static_cast<const __nv_bfloat16*>(sa.h_cur), sa.h_cur_stride,

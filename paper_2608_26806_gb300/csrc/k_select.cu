@@ -54,6 +54,8 @@ struct SelShared {
   // hand-over from the warps of the fused kernel
   uint32_t kmin, kmax;
   int k, before, total, alloc_err, vis_before, n_vis;
+  int ncand;      // candidates gathered from the chosen first-pass bucket
+  uint32_t thr;   // the k-th largest key, found among them
 };
 
 // Named barrier for warps 1..7 (224 threads) while warp 0 runs the budget rule.
@@ -206,6 +208,76 @@ __device__ void block_select(const float* __restrict__ sc, int n, int k, int64_t
   }
 }
 
+// Candidates of the chosen first-pass bucket ranked directly, when there are at most this many.
+constexpr int kCandCap = 256;
+
+// Finishes the selection from the first-pass histogram when the image's keys are staged:
+// the bucket holding the k-th largest key usually holds a few dozen keys, so they are
+// gathered and ranked against each other (one compare per pair), which gives the k-th
+// largest key thr directly. Then one block scan carries both the counts of keys above
+// thr and of keys equal to it (16 bits each), and the kept positions are written in
+// ascending order: every key above thr and the first k - #(key > thr) equal to it.
+// Returns false (having written nothing) when the bucket is too large; all threads call.
+// dry: compute everything but write nothing (warms the instruction cache).
+__device__ __noinline__ bool select_from_first_pass(int n, int k, int64_t t0, int64_t base,
+                                                    int32_t* __restrict__ kept_idx, SelShared& sh, uint32_t kmin,
+                                                    uint32_t kmax, bool dry) {
+  const int tid = threadIdx.x;
+  const int top = highest_differing_bit(kmin, kmax);
+  const uint32_t mask = shared_bits_mask(top);
+  const int shift = top >= 7 ? top - 7 : 0;
+  const uint32_t dmask = (2u << (top - shift)) - 1u;
+  choose_digit(sh, k);
+  const int c1 = sh.count, remaining = k - sh.above;
+  if (c1 > kCandCap) return false;
+  const uint32_t bmask = mask | (dmask << shift);
+  const uint32_t bval = (kmin & mask) | (static_cast<uint32_t>(sh.digit) << shift);
+  uint32_t* cand = reinterpret_cast<uint32_t*>(&sh.hist[1][0]);  // the histograms are dead now
+  for (int j = tid; j < n; j += kThreads) {
+    const uint32_t key = sh.keys[j];
+    if ((key & bmask) == bval) cand[atomicAdd(&sh.ncand, 1)] = key;
+  }
+  __syncthreads();
+  if (tid < c1) {
+    const uint32_t v = cand[tid];
+    int gt = 0, ge = 0;
+    for (int u = 0; u < c1; ++u) {
+      const uint32_t w = cand[u];
+      gt += w > v ? 1 : 0;
+      ge += w >= v ? 1 : 0;
+    }
+    if (gt < remaining && remaining <= ge) sh.thr = v;
+  }
+  __syncthreads();
+  const uint32_t thr = sh.thr;
+  // thread t owns positions t*kPer .. t*kPer + kPer - 1
+  const int j0 = tid * kPer;
+  uint32_t kk[kPer];
+  int gt = 0, eq = 0;
+#pragma unroll
+  for (int q = 0; q < kPer; ++q) {
+    kk[q] = j0 + q < n ? sh.keys[j0 + q] : 0u;
+    gt += (j0 + q < n && kk[q] > thr) ? 1 : 0;
+    eq += (j0 + q < n && kk[q] == thr) ? 1 : 0;
+  }
+  int tot;
+  const int packed = gt | (eq << 16);
+  const int pre = block_incl_scan(packed, sh.wsum, &tot) - packed;
+  const int need_eq = k - (tot & 0xffff);
+  int eq_rank = pre >> 16;
+  int o = (pre & 0xffff) + min(eq_rank, need_eq);
+#pragma unroll
+  for (int q = 0; q < kPer; ++q) {
+    if (j0 + q < n) {
+      bool kp = kk[q] > thr;
+      if (kk[q] == thr) kp = eq_rank++ < need_eq;
+      if (kp && !dry) kept_idx[base + o] = static_cast<int32_t>(t0 + j0 + q);
+      o += kp ? 1 : 0;
+    }
+  }
+  return true;
+}
+
 // Stage the image's keys (when they fit) and find their range; all threads call.
 __device__ void stage_and_range(const float* __restrict__ sc, int n, bool stage, SelShared& sh, uint32_t* kmin_out,
                                 uint32_t* kmax_out) {
@@ -322,6 +394,7 @@ struct AllocParams {
   int relative;
   int32_t* budgets;  // output: each CTA writes its own image's budget
   int m_cap;
+  int warm_ctas;     // CTAs below this index warm their instruction cache before the wait
 };
 
 __global__ void __launch_bounds__(kThreads)
@@ -376,6 +449,35 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
     rule = make_ratio_rule(kr, ap.alpha, ap.relative);
     inv_N = recip62(N);
     inv_n = recip62(n_lane);
+  }
+
+  // ---- warm the instruction cache. When the scoring kernel leaves SMs free
+  // (prune_reserve_sms), the first CTAs start while the scores stream in, so the budget
+  // rule and the selection run once on made-up data here, writing nothing to global
+  // memory; their code is then resident when the real data arrives (a cold fetch
+  // costs about 1 us per KiB, the L2 having been swept by the scoring kernel).
+  if (b < ap.warm_ctas && b < a.NI && m >= 1 && m <= 32) {
+    constexpr int kDryKeys = 1024;
+    if (warp == 0) {
+      const int64_t S = lane < m ? (static_cast<int64_t>(n_lane) << 30) : 0;
+      int32_t K = 0;
+      const int err = warp_allocate32(m, S, n_lane, inv_n, B, N, inv_N, rule, Rmin, Rmax, &K);
+      asm volatile("" ::"r"(K), "r"(err));
+#pragma unroll
+      for (int q = 0; q < 8; ++q) sh.hist[0][lane * 8 + q] = 0;
+    } else {
+      const int wt = tid - 32;
+      for (int j = wt; j < kDryKeys; j += kThreads - 32) sh.keys[j] = 0x3f800000u + static_cast<uint32_t>(j);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) sh.hist[warp][lane * 8 + q] = 0;
+      if (tid == 32) sh.ncand = 0;
+      bar_workers();
+      // keys 0x3f800000 .. +1023: the top differing bit is 9, digits are bits 2..9
+      hist_pass(KeySource{a.scores, sh.keys}, kDryKeys, ~0x3ffu, 0x3f800000u, 2, 0xffu, sh.hist[warp], wt, kThreads - 32);
+    }
+    __syncthreads();
+    select_from_first_pass(kDryKeys, kDryKeys / 2, 0, 0, a.kept_idx, sh, 0x3f800000u, 0x3f8003ffu, true);
+    __syncthreads();
   }
 
   // ---- wait for the scores and per-image sums (and, through them, the validation)
@@ -463,6 +565,7 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
     if (tid == 32) {
       sh.kmin = lo;
       sh.kmax = hi;
+      sh.ncand = 0;
     }
   }
   __syncthreads();
@@ -479,7 +582,9 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
     return;
   }
   const int64_t base = static_cast<int64_t>(out_lo) + (s0 - vis_b) + before;
-  block_select(sc, n, k, t0, base, a.kept_idx, sh, stage, kmin, kmax, kmin != kmax);
+  const bool fast = stage && kmin != kmax && k > 0 && k < n &&
+                    select_from_first_pass(n, k, t0, base, a.kept_idx, sh, kmin, kmax, false);
+  if (!fast) block_select(sc, n, k, t0, base, a.kept_idx, sh, stage, kmin, kmax, kmin != kmax);
   const int e = s0 + n;
   for (int p = e + tid; p < nxt; p += kThreads) a.kept_idx[base + k + (p - e)] = a.cu[r] + p;
 }
@@ -515,7 +620,8 @@ cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int
 
 cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
                                 int32_t* budgets, const float* scores, const int32_t* out_cu_seqlens,
-                                int32_t* kept_idx, int64_t n_kept, void* ws, const WsPlan& p, cudaStream_t s) {
+                                int32_t* kept_idx, int64_t n_kept, void* ws, const WsPlan& p, cudaStream_t s,
+                                int warm_ctas) {
   const SelectArgs a = make_args(L, scores, out_cu_seqlens, kept_idx, n_kept, ws, p);
   AllocParams ap;
   ap.img_sums = img_sums;
@@ -525,10 +631,20 @@ cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums,
   ap.r_max = aa.r_max;
   ap.relative = aa.relative;
   ap.budgets = budgets;
+  ap.warm_ctas = warm_ctas;
   ap.m_cap = L.n_images < kMaxImagesPerRequest ? L.n_images : kMaxImagesPerRequest;
   if (ap.m_cap < 1) ap.m_cap = 1;
   // the budget scratch is only used for requests of more than 32 images
   const size_t smem = ap.m_cap > 32 ? warp_alloc_smem_bytes(ap.m_cap) : 0;
+  static bool carveout_set = false;
+  if (!carveout_set) {
+    // same shared-memory configuration as the scoring kernels, so that a CTA of this
+    // kernel can start on an SM where a scoring CTA still runs
+    cudaError_t e = cudaFuncSetAttribute(k_alloc_select, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                         cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+    carveout_set = true;
+  }
   if (smem > 16 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(k_alloc_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
