@@ -159,8 +159,14 @@ int device_sm_count() {
 
 int prune_reserve_sms(const avtp_layout_t& L) {
   if (L.n_tokens > 32768 || L.n_images < 1) return 0;
+  const int64_t ctas = prune_warm_ctas(L);
+  return static_cast<int>((ctas + kSelectCtasPerSm - 1) / kSelectCtasPerSm);
+}
+
+int prune_warm_ctas(const avtp_layout_t& L) {
+  if (L.n_tokens > 32768 || L.n_images < 1) return 0;
   const int64_t ctas = static_cast<int64_t>(L.n_images) + L.n_requests;
-  return static_cast<int>(ctas < 24 ? ctas : 24);
+  return ctas <= kMaxWarmCtas ? static_cast<int>(ctas) : 0;
 }
 
 }  // namespace avtp
@@ -293,8 +299,9 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   const int reserve = score_args->criterion == AVTP_CRIT_HIDDEN_VARIATION ? prune_reserve_sms(*layout) : 0;
   if ((st = score_impl(layout, score_args, sc, sums, workspace, p, s, reserve)) != AVTP_OK) return st;
   if ((st = record(step_events, 2, s)) != AVTP_OK) return st;
+  const int warm = score_args->criterion == AVTP_CRIT_HIDDEN_VARIATION ? prune_warm_ctas(*layout) : 0;
   if ((st = from_cuda(launch_alloc_select(*layout, sums, *alloc_args, budgets, sc, out_cu_seqlens, kept_idx, n_kept,
-                                          workspace, p, s, reserve))) != AVTP_OK)
+                                          workspace, p, s, warm))) != AVTP_OK)
     return st;
   if ((st = record(step_events, 3, s)) != AVTP_OK) return st;
   if ((st = from_cuda(launch_compact(kept_idx, n_kept, layout->n_tokens, sets, n_sets, workspace, p, s))) != AVTP_OK)

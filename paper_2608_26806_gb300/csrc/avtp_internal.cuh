@@ -195,11 +195,16 @@ cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums,
                                 int warm_ctas = 0);
 
 // In avtp_prune with the hidden-variation criterion on a small batch, the scoring
-// kernel leaves this many SMs free so that the selection kernel's CTAs (one per image)
-// start while the scores stream in and warm their instruction caches; 0 otherwise.
-// On a request of about 10k tokens this trades about 1 us of scoring for about 3 us
-// of allocation and selection; on large batches the scoring time would grow instead.
+// kernel leaves prune_reserve_sms(L) SMs free so that the selection kernel's CTAs (one
+// per image, kSelectCtasPerSm of them fit on an SM) start while the scores stream in
+// and warm their instruction caches (prune_warm_ctas(L) of them run the code once on
+// made-up data first); 0 otherwise. Right after the scoring stream has swept L2 a cold
+// run of the budget rule and the selection takes several times longer. On large
+// batches the scoring time would grow instead.
+constexpr int kSelectCtasPerSm = 4;  // 256 threads, 64 registers, 16.5 KiB shared memory each
+constexpr int kMaxWarmCtas = 96;
 int prune_reserve_sms(const avtp_layout_t& L);
+int prune_warm_ctas(const avtp_layout_t& L);
 
 cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
                            int n_sets, void* ws, const WsPlan& p, cudaStream_t s);

@@ -1,8 +1,10 @@
 // Step 4: compaction, out[j] = in[kept_idx[j]] for every row set (paper §3.1:
 // E_pruned = p(E_v), the kept tokens as a dense, varlen-packed batch).
 //
-// Large rows (hidden states, K/V rows): one warp per row, 16-byte vector loads
-// and stores, several in flight per lane. Small rows (position ids, one element
+// Large rows (hidden states, K/V rows): one warp per row, 16-byte vector loads and
+// stores; a lane issues all its loads of an 8-KiB piece of the row before its first
+// store, so that a row costs one memory round trip (the kept rows are usually still in
+// L2: the scoring kernel reads h_cur with an evict-last policy). Small rows (position ids, one element
 // per plane): one thread per row. All row sets go in one launch; the block index
 // range is split between the sets on the host.
 #include "avtp_internal.cuh"
@@ -13,7 +15,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kRowsPerWarp = 1;
-constexpr int kUnroll = 4;
+constexpr int kUnroll = 16;  // 16 x 16 bytes per lane: 8 KiB per warp in flight
 
 struct RowSetDev {
   const char* in;
@@ -70,15 +72,19 @@ k_compact(CompactParams P, const int32_t* __restrict__ kept_idx, int64_t n_kept,
       }
       const uint4* src = reinterpret_cast<const uint4*>(S.in + t * S.in_stride);
       uint4* dst = reinterpret_cast<uint4*>(S.out + j * S.out_stride);
-      int64_t c = lane;
-      for (; c + 32 * (kUnroll - 1) < n16; c += 32 * kUnroll) {
+      for (int64_t c0 = 0; c0 < n16; c0 += 32 * kUnroll) {
         uint4 v[kUnroll];
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) v[u] = __ldcs(src + c + 32 * u);
+        for (int u = 0; u < kUnroll; ++u) {
+          const int64_t c = c0 + lane + 32 * u;
+          if (c < n16) v[u] = __ldcs(src + c);
+        }
 #pragma unroll
-        for (int u = 0; u < kUnroll; ++u) __stcs(dst + c + 32 * u, v[u]);
+        for (int u = 0; u < kUnroll; ++u) {
+          const int64_t c = c0 + lane + 32 * u;
+          if (c < n16) __stcs(dst + c, v[u]);
+        }
       }
-      for (; c < n16; c += 32) __stcs(dst + c, __ldcs(src + c));
     }
   } else {
     const int64_t j = row0 + threadIdx.x;
