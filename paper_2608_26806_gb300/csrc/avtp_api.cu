@@ -160,7 +160,8 @@ int device_sm_count() {
 int prune_reserve_sms(const avtp_layout_t& L) {
   if (L.n_tokens > 32768 || L.n_images < 1) return 0;
   const int64_t ctas = prune_warm_ctas(L);
-  return static_cast<int>((ctas + kSelectCtasPerSm - 1) / kSelectCtasPerSm);
+  const int per_sm = alloc_select_ctas_per_sm();
+  return static_cast<int>((ctas + per_sm - 1) / per_sm);
 }
 
 int prune_warm_ctas(const avtp_layout_t& L) {

@@ -196,13 +196,13 @@ cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums,
 
 // In avtp_prune with the hidden-variation criterion on a small batch, the scoring
 // kernel leaves prune_reserve_sms(L) SMs free so that the selection kernel's CTAs (one
-// per image, kSelectCtasPerSm of them fit on an SM) start while the scores stream in
+// per image, alloc_select_ctas_per_sm() of them fit on an SM) start while the scores stream in
 // and warm their instruction caches (prune_warm_ctas(L) of them run the code once on
 // made-up data first); 0 otherwise. Right after the scoring stream has swept L2 a cold
 // run of the budget rule and the selection takes several times longer. On large
 // batches the scoring time would grow instead.
-constexpr int kSelectCtasPerSm = 4;  // 256 threads, 64 registers, 16.5 KiB shared memory each
 constexpr int kMaxWarmCtas = 96;
+int alloc_select_ctas_per_sm();  // from the occupancy calculator (about 4: 256 threads, 64 registers)
 int prune_reserve_sms(const avtp_layout_t& L);
 int prune_warm_ctas(const avtp_layout_t& L);
 

@@ -618,6 +618,16 @@ cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int
   return launch_kernel(k_select, dim3(L.n_images + L.n_requests), dim3(kThreads), 0, s, /*pdl=*/true, a, budgets);
 }
 
+int alloc_select_ctas_per_sm() {
+  static int cached = 0;
+  if (cached == 0) {
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_alloc_select, kThreads, 0) != cudaSuccess || n < 1) n = 1;
+    cached = n;
+  }
+  return cached;
+}
+
 cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
                                 int32_t* budgets, const float* scores, const int32_t* out_cu_seqlens,
                                 int32_t* kept_idx, int64_t n_kept, void* ws, const WsPlan& p, cudaStream_t s,
