@@ -94,13 +94,12 @@ AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa) {
   a.G = sa.n_kv_heads > 0 ? sa.n_q_heads / sa.n_kv_heads : 1;
   a.max_text = (sa.max_text_tokens > 0 && sa.max_text_tokens < T) ? sa.max_text_tokens : T;
   a.rows = a.max_text * a.G;
-  // every request's row tiles: ceil(rows_r / M) <= rows_r / M + 1
-  a.n_qtiles_max = a.rows / kAttnTileM + L.n_requests + 1;
-  // chunks of at least T / kAttnMaxChunks keys, so that a row tile has at most kAttnMaxChunks
-  int64_t ck = (T + kAttnMaxChunks - 1) / kAttnMaxChunks;
-  ck = (ck + kAttnTileN - 1) / kAttnTileN * kAttnTileN;
-  a.chunk_keys = static_cast<int>(ck > kAttnMinChunkKeys ? ck : kAttnMinChunkKeys);
-  a.p1_items_max = a.n_qtiles_max * kAttnMaxChunks;
+  // every request's row blocks: ceil(rows_r / 256) <= rows_r / 256 + 1
+  a.n_blocks_max = a.rows / kAttnBlockRows + L.n_requests + 1;
+  // key tiles: sum_i ceil(n_i / 128) <= N_vis / 128 + n_img
+  a.n_ktiles_max = T / kAttnTileM + L.n_images + 1;
+  a.Hkv = sa.n_kv_heads;
+  a.grid = device_sm_count();
   return a;
 }
 
@@ -125,13 +124,17 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
     const size_t Hkv = static_cast<size_t>(sa->n_kv_heads), rows = static_cast<size_t>(a.rows);
     p.text_idx = take(T * 4 + 4);
     p.text_cu = take((R + 1) * 4);
-    p.qtile_cu = take((R + 1) * 4);
-    p.p1_cu = take((static_cast<size_t>(a.n_qtiles_max) + 1) * 4);
+    p.blk_cu = take((R + 1) * 4);
+    p.p1s_cu = take((static_cast<size_t>(a.n_blocks_max) + 1) * 4);
+    p.p2t_cu = take((static_cast<size_t>(a.n_blocks_max) + 1) * 4);
     p.ktile_cu = take((NI + 1) * 4);
+    p.meta = take(8 * 4);
     p.qt = take(Hkv * rows * static_cast<size_t>(sa->head_dim) * 2 + 16);
-    p.lse_rows = take(Hkv * rows * 4 + 4);
-    p.p1_part = (sa->lse == nullptr) ? take(Hkv * static_cast<size_t>(a.p1_items_max) * kAttnTileM * 8) : 0;
-    p.partial = take(Hkv * T * 4 + 4);
+    p.lse_rows = (sa->lse != nullptr) ? take(Hkv * rows * 4 + 4) : 0;
+    p.p1_part = (sa->lse == nullptr)
+                    ? take(Hkv * static_cast<size_t>(a.n_blocks_max) * kAttnBlockRows * kAttnMaxChunks * 8)
+                    : 0;
+    p.mass = take(static_cast<size_t>(a.n_ktiles_max) * kAttnTileM * 8);
   }
   p.total = off;
   return p;

@@ -21,12 +21,16 @@ constexpr int kRatioFracBits = 40;       // ratio grid of the budget rule
 constexpr double kRatioLimit = 1048576.0;  // ratios saturate at +-2^20 before the grid
 
 // Tiles of the text-attention criterion (tensor-core path). Rows are (text query, head
-// of the KV group) pairs, G = Hq / Hkv of them per text query, in text order.
-constexpr int kAttnTileM = 128;          // MMA M: rows of a pass-1 tile, keys of a pass-2 tile
-constexpr int kAttnTileN = 256;          // MMA N: keys per pass-1 step, rows per pass-2 step
-constexpr int kAttnMinChunkKeys = 512;   // pass-1 work item: one row tile against a chunk of keys
-constexpr int kAttnMaxChunks = 64;       // chunks per row tile at most (the chunk grows with T)
+// of the KV group) pairs, G = Hq / Hkv of them per text query, in text order. A request's
+// rows are cut into blocks of kAttnBlockRows; pass 1 runs a block as two MMA A tiles
+// against key tiles of kAttnTileN keys, pass 2 holds a block as the MMA B operand and
+// streams key tiles of kAttnTileM visual keys through it.
+constexpr int kAttnTileM = 128;          // MMA M: rows of a pass-1 A tile, keys of a pass-2 tile
+constexpr int kAttnTileN = 256;          // MMA N: keys per pass-1 step, rows of a pass-2 block
+constexpr int kAttnBlockRows = 256;      // rows per block (both passes)
+constexpr int kAttnMaxChunks = 64;       // pass-1 partial (max, sum) slots per row at most
 constexpr int kAttnMaxGroupHeads = 128;  // Hq / Hkv at most
+constexpr int kAttnMassFracBits = 40;    // fixed point of the per-key probability mass
 
 // ---------------------------------------------------------------- status
 // First word of every workspace. code: first error recorded (0 = none);
@@ -53,13 +57,15 @@ struct WsPlan {
   // criterion B (text attention); "rows" = rows per KV group = max_text * G
   size_t text_idx;    // int32 [T]: packed position of each text ordinal
   size_t text_cu;     // int32 [R + 1]: text ordinals per request
-  size_t qtile_cu;    // int32 [R + 1]: pass-1 row tiles per request
-  size_t p1_cu;       // int32 [n_qtiles_max + 1]: pass-1 work items (key chunks) per row tile
-  size_t ktile_cu;    // int32 [n_img + 1]: pass-2 key tiles per image
+  size_t blk_cu;      // int32 [R + 1]: row blocks per request
+  size_t p1s_cu;      // int32 [n_blocks_max + 1]: pass-1 key steps per row block
+  size_t p2t_cu;      // int32 [n_blocks_max + 1]: pass-2 key tiles per row block
+  size_t ktile_cu;    // int32 [n_img + 1]: key tiles per image
+  size_t meta;        // int32 [8]: F1, C1, F2, C2 (flat pass lengths per KV group, steps per CTA)
   size_t qt;          // bf16 [Hkv, rows, d]: the text queries, packed by KV group
-  size_t lse_rows;    // float [Hkv, rows]: log2-domain LSE of every row
-  size_t p1_part;     // float2 [Hkv * n_qtiles_max][128][kAttnMaxChunks]: per-chunk (max, sum) of every row
-  size_t partial;     // float [Hkv * T]: per (KV group, visual key) probability sums
+  size_t lse_rows;    // float [Hkv, rows]: log2-domain LSE of every row (supplied LSE only)
+  size_t p1_part;     // float2 [Hkv * n_blocks_max][256][kAttnMaxChunks]: per-CTA (max, sum) of every row
+  size_t mass;        // uint64 [n_ktiles_max][128]: fixed-point probability mass of every visual key, by key tile
   size_t total;
 };
 
@@ -68,9 +74,10 @@ struct AttnPlan {
   int G;                 // query heads per KV group
   int64_t max_text;      // text tokens of the whole batch, at most
   int64_t rows;          // rows per KV group: max_text * G
-  int64_t n_qtiles_max;  // pass-1 row tiles, at most
-  int chunk_keys;        // keys per pass-1 work item
-  int64_t p1_items_max;  // pass-1 work items per KV group, at most
+  int64_t n_blocks_max;  // row blocks of all requests, at most
+  int64_t n_ktiles_max;  // key tiles of all images, at most
+  int Hkv;               // KV groups
+  int grid;              // CTAs of the persistent tensor-core kernels (one per SM)
 };
 AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa);
 

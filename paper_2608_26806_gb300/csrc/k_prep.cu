@@ -57,8 +57,8 @@ constexpr int kStageInts = 2560;
 
 __global__ void __launch_bounds__(kPrepThreads)
 k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t* req_budget, int32_t* text_idx,
-       int32_t* text_cu, int32_t* qtile_cu, int32_t* p1_cu, int32_t* ktile_cu) {
-  __shared__ int s_err, s_detail;
+       int32_t* text_cu, int32_t* blk_cu, int32_t* p1s_cu, int32_t* p2t_cu, int32_t* ktile_cu, int32_t* meta) {
+  __shared__ int s_err, s_detail, s_max_steps;
   __shared__ int32_t s_warp[32];
   __shared__ int32_t s_stage[kStageInts];
   // The first kernel of a call: it is launched after everything before it in the
@@ -190,24 +190,61 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
     if (tid == 0 && static_cast<int64_t>(text_cu[R]) > a.attn.max_text) fail(AVTP_ERR_RANGE, -1);
     __syncthreads();
     if (s_err == 0) {
-      // pass 1: row tiles of kAttnTileM (text query, head) rows per request, then key chunks per tile
+      // Row blocks of kAttnBlockRows (text query, head) rows per request.
       block_exclusive_scan<int32_t>(
-          R, [&](int r) { return ((text_cu[r + 1] - text_cu[r]) * G + kAttnTileM - 1) / kAttnTileM; }, qtile_cu,
+          R, [&](int r) { return ((text_cu[r + 1] - text_cu[r]) * G + kAttnBlockRows - 1) / kAttnBlockRows; }, blk_cu,
           s_warp);
-      const int nq = qtile_cu[R];
-      const int ck = a.attn.chunk_keys;
-      block_exclusive_scan<int32_t>(
-          nq,
-          [&](int t) {
-            const int r = upper_index(qtile_cu, R, t);
-            const int row_end = min(text_cu[r] * G + (t - qtile_cu[r] + 1) * kAttnTileM, text_cu[r + 1] * G);
-            const int pmax = text_idx[(row_end - 1) / G] - cu[r];  // request-local position of the last query
-            return (pmax + ck) / ck;
-          },
-          p1_cu, s_warp);
-      // pass 2: key tiles of kAttnTileM visual keys per image
+      const int NB = blk_cu[R];
+      // Key tiles of kAttnTileM visual keys per image.
       block_exclusive_scan<int32_t>(
           NI, [&](int i) { return (iln[i] + kAttnTileM - 1) / kAttnTileM; }, ktile_cu, s_warp);
+      // Pass 2 of block b: the key tiles of every image that at least one of the block's
+      // queries follows. Images are sorted and the text ordinal of the first token after
+      // image i, o_first(i), does not decrease with i, so those images are a prefix.
+      auto p2_tiles = [&](int b) {
+        const int r = upper_index(blk_cu, R, b);
+        const int64_t R0 = static_cast<int64_t>(text_cu[r]) * G + static_cast<int64_t>(b - blk_cu[r]) * kAttnBlockRows;
+        const int64_t R1 = min(R0 + kAttnBlockRows, static_cast<int64_t>(text_cu[r + 1]) * G);
+        int lo = icu[r], hi = icu[r + 1];  // first image in [lo, hi) with o_first * G >= R1
+        while (lo < hi) {
+          const int i = (lo + hi) >> 1;
+          const int64_t o_first =
+              static_cast<int64_t>(text_cu[r]) + ist[i] + iln[i] - (vis_cu[i + 1] - vis_cu[icu[r]]);
+          if (o_first * G >= R1) hi = i; else lo = i + 1;
+        }
+        return ktile_cu[lo] - ktile_cu[icu[r]];
+      };
+      block_exclusive_scan<int32_t>(NB, p2_tiles, p2t_cu, s_warp);
+      // Pass 1 of block b: steps of kAttnTileN keys from the request's first token to its
+      // last query (none when pass 2 has nothing for the block).
+      if (tid == 0) s_max_steps = 0;
+      __syncthreads();
+      auto p1_steps = [&](int b) {
+        if (p2t_cu[b + 1] == p2t_cu[b]) return 0;
+        const int r = upper_index(blk_cu, R, b);
+        const int64_t R0 = static_cast<int64_t>(text_cu[r]) * G + static_cast<int64_t>(b - blk_cu[r]) * kAttnBlockRows;
+        const int64_t R1 = min(R0 + kAttnBlockRows, static_cast<int64_t>(text_cu[r + 1]) * G);
+        const int keys = text_idx[(R1 - 1) / G] - cu[r] + 1;
+        const int steps = (keys + kAttnTileN - 1) / kAttnTileN;
+        atomicMax(&s_max_steps, steps);
+        return steps;
+      };
+      block_exclusive_scan<int32_t>(NB, p1_steps, p1s_cu, s_warp);
+      if (tid == 0) {
+        // Each CTA of a persistent pass takes a contiguous run of C steps of the flat
+        // list (KV group, block, step). C1 also keeps a row's pass-1 partials within
+        // kAttnMaxChunks slots: a block of S steps meets at most (S - 1) / C1 + 2 CTAs.
+        const int64_t grid = a.attn.grid > 0 ? a.attn.grid : 1;
+        const int64_t F1 = p1s_cu[NB], F2 = p2t_cu[NB];
+        int64_t C1 = (a.attn.Hkv * F1 + grid - 1) / grid;
+        const int64_t c_min = (s_max_steps - 1 + kAttnMaxChunks - 3) / (kAttnMaxChunks - 2);
+        C1 = max(max(C1, c_min), static_cast<int64_t>(1));
+        const int64_t C2 = max((a.attn.Hkv * F2 + grid - 1) / grid, static_cast<int64_t>(1));
+        meta[0] = static_cast<int32_t>(F1);
+        meta[1] = static_cast<int32_t>(C1);
+        meta[2] = static_cast<int32_t>(F2);
+        meta[3] = static_cast<int32_t>(C2);
+      }
     }
   }
 
@@ -234,9 +271,11 @@ cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream
                                     ws_at<int32_t>(ws, p.img_req), ws_at<int32_t>(ws, p.req_budget),
                                     b ? ws_at<int32_t>(ws, p.text_idx) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.text_cu) : nullptr,
-                                    b ? ws_at<int32_t>(ws, p.qtile_cu) : nullptr,
-                                    b ? ws_at<int32_t>(ws, p.p1_cu) : nullptr,
-                                    b ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr);
+                                    b ? ws_at<int32_t>(ws, p.blk_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.p1s_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.p2t_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.meta) : nullptr);
   return cudaGetLastError();
 }
 

@@ -5,29 +5,31 @@
 //
 // Rows: for KV group g, row o*G + j is text query o (in text order over the batch)
 // with query head g*G + j. The text queries are first repacked by group into
-// Qt[g][row][d] (k_attn_pack), so that both passes read them with TMA boxes.
+// Qt[g][row][d] (k_attn_pack), so that both passes read them with TMA boxes. A
+// request's rows are cut into blocks of 256.
 //
-// Pass 1 (skipped when the caller supplies FlashAttention's LSE): a work item is one
-// tile of 128 rows of a request against one chunk of its keys; S = Q_rows K^T runs on
-// the tensor cores (tcgen05.mma, 128 x 256 per step, fp32 accumulator in TMEM) and the
-// epilogue warps keep an online (max, sum) per row; k_attn_merge then combines the
-// chunks of every row into lse2 (a separate kernel: merging inside pass 1, in
-// whichever item finished a tile last, piled the merges onto a few CTAs).
-// Pass 2: a work item is one tile of 128 visual keys of an image; S^T = K_tile Qt^T
-// over the rows of every text query after the image (all of them see every key of
-// the image), 256 rows per step; each epilogue thread owns one key and sums
-// exp2(z2 - lse2) over the rows.
-// Finalize: sum the KV groups in a fixed order (deterministic), divide, and add the
-// fixed-point per-image sums.
+// Pass 1, k_attn_lse (skipped when the caller supplies FlashAttention's LSE): a block
+// is held as two 128-row A tiles and every key tile of 256 keys, from the request's
+// first token to the block's last query, feeds two MMAs (128 x 256 x d each, one per
+// A tile, fp32 accumulators in TMEM). Each A tile has its own accumulator and its own
+// four epilogue warps, so one tile's epilogue overlaps the other tile's MMA and every
+// key byte brought to the SM serves 256 rows. The epilogue keeps an online (max, sum)
+// per row and leaves one partial per (row, CTA) behind.
+// Pass 2, k_attn_mass: a block is held as the MMA B operand (N = 256 rows) and the
+// tiles of 128 visual keys of every image that one of its queries follows stream
+// through it as A (M = 128 keys); the two accumulators alternate between the two
+// epilogue groups. A thread owns one key and sums exp2(z2 - lse2) over the block's
+// rows that see the key; lse2 comes from the pass-1 partials of the block (merged on
+// load) or from the supplied LSE. The per-key sums of all blocks and KV groups meet in
+// a 64-bit fixed-point accumulator (integer atomics: the result does not depend on
+// their order).
+// k_attn_finalize turns the accumulator into scores and the fixed-point image sums.
 //
-// Both passes are persistent (one CTA per SM). Warps 0-7 are the epilogue (warp w
-// reads TMEM lanes 32(w%4)..+31, columns 128(w/4)..+127 of each step), warp 8 issues
-// the TMA loads, warp 9 owns TMEM and issues the MMAs. Shared memory: two stages of
-// A tiles (128 rows x d, so the next item's tile loads during this one) and two of
-// B tiles (256 rows x d); TMEM: two 256-column accumulators, so the epilogue of one
-// step overlaps the MMA of the next. The epilogue keeps four independent partial
-// sums (and maxima) per thread: with two warps per scheduler there is little else
-// to hide the latency of a dependent chain.
+// Both passes are persistent: the flat list of (KV group, block, key step) is split
+// into equal contiguous runs, one per CTA (one CTA per SM). Warps 0-3 and 4-7 are the
+// two epilogue groups (warp w reads TMEM lanes 32(w%4)..+31 of accumulator w/4), warp 8
+// issues the TMA loads, warp 9 owns TMEM and issues the MMAs. TMEM holds the two
+// 256-column accumulators.
 #include <cudaTypedefs.h>
 
 #include "avtp_tc.cuh"
@@ -35,22 +37,33 @@
 namespace avtp {
 namespace {
 
-constexpr int kM = kAttnTileM;   // 128
-constexpr int kN = kAttnTileN;   // 256
-constexpr int kEpiWarps = 8;     // warps 0-7: epilogue
+constexpr int kM = kAttnTileM;        // 128
+constexpr int kN = kAttnTileN;        // 256
+constexpr int kBlk = kAttnBlockRows;  // 256
 constexpr int kTmaWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kThreads = 320;
+constexpr int kEpiWarps = 8;          // warps 0-7: epilogue
 constexpr uint32_t kTmemCols = 2 * kN;
+constexpr int kP2Stages = 4;          // key tiles in flight in pass 2
+constexpr int kMassWindow = 24;       // pass-2 steps whose key masses are held in shared memory between flushes
 constexpr float kLog2e = 1.4426950408889634f;
+// Flag of a key whose mass is not a finite number in [0, 256] (non-finite inputs). The
+// sum of its finite contributions stays below 2^62: at most 256 * 2^40 per (KV group,
+// block), fewer than 2^14 of them.
+constexpr unsigned long long kMassNotFinite = 1ull << 63;
 
-// Shared memory for head_dim d: two A stages, then two B stages, 1024-byte aligned.
+static_assert(kBlk == 2 * kM && kBlk == kN, "a block is two A tiles (pass 1) and one B operand (pass 2)");
+
+// Shared memory for head_dim d (1024-byte aligned tiles).
 __host__ __device__ constexpr size_t a_bytes(int d) { return static_cast<size_t>(kM) * d * 2; }
 __host__ __device__ constexpr size_t b_bytes(int d) { return static_cast<size_t>(kN) * d * 2; }
-__host__ __device__ constexpr size_t tc_smem_bytes(int d) { return 1024 + 2 * a_bytes(d) + 2 * b_bytes(d); }
+// pass 1: two A tiles (the block) + two key stages; pass 2: the block + kP2Stages key tiles
+__host__ __device__ constexpr size_t lse_smem_bytes(int d) { return 1024 + 2 * a_bytes(d) + 2 * b_bytes(d); }
+__host__ __device__ constexpr size_t mass_smem_bytes(int d) { return 1024 + b_bytes(d) + kP2Stages * a_bytes(d); }
 
 struct Sync {
-  uint64_t a_full[2], a_empty[2];
+  uint64_t a_full[kP2Stages], a_empty[kP2Stages];
   uint64_t b_full[2], b_empty[2];
   uint64_t acc_full[2], acc_empty[2];
   uint64_t drain;
@@ -67,104 +80,199 @@ struct AttnArgs {
   int NI;
   int64_t T;
   const int32_t* vis_cu;
-  const int32_t* img_req;
   const int32_t* text_idx;
   const int32_t* text_cu;
-  const int32_t* qtile_cu;
-  const int32_t* p1_cu;
+  const int32_t* blk_cu;
+  const int32_t* p1s_cu;
+  const int32_t* p2t_cu;
   const int32_t* ktile_cu;
-  float* lse_rows;        // [Hkv, rows]
-  float2* p1_part;        // [Hkv * n_qtiles_max][128 rows][kAttnMaxChunks]
-  float* partial;         // [Hkv, T]
-  int64_t rows;           // rows per group
-  int64_t p1_items_max;
-  int G, Hkv, d, chunk_keys;
-  float c2;               // softmax_scale * log2(e)
+  const int32_t* meta;           // F1, C1, F2, C2
+  const float* lse_rows;         // [Hkv, rows] (supplied LSE) or nullptr
+  float2* p1_part;               // [Hkv * NB][256 rows][kAttnMaxChunks]
+  unsigned long long* mass;      // [key tile][128] fixed point, 2^-kAttnMassFracBits
+  int64_t rows;
+  int G, Hkv, d;
+  float c2;                      // softmax_scale * log2(e)
   DevStatus* st;
 };
 
 __device__ __forceinline__ void bar_epi() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
-// ---------------------------------------------------------------- work items
-struct P1Item {
-  int g, qt, chunk;
-  int64_t row0;      // first row (within group g) of the tile
-  int64_t row_end;   // end of the request's rows, at most row0 + kM
-  int key0, key_end; // packed key positions of the chunk
+// A (KV group, row block) pair: rows [R0, R1) of group g belong to request r.
+struct Seg {
+  int g, b, r;
+  int64_t R0, R1;
 };
 
-__device__ __forceinline__ P1Item p1_item(const AttnArgs& a, int n_per_group, int id) {
-  P1Item it;
-  it.g = id / n_per_group;
-  const int rest = id - it.g * n_per_group;
-  const int nq = a.qtile_cu[a.R];
-  it.qt = upper_index(a.p1_cu, nq, rest);
-  it.chunk = rest - a.p1_cu[it.qt];
-  const int r = upper_index(a.qtile_cu, a.R, it.qt);
-  const int64_t rr0 = static_cast<int64_t>(a.text_cu[r]) * a.G, rr1 = static_cast<int64_t>(a.text_cu[r + 1]) * a.G;
-  it.row0 = rr0 + static_cast<int64_t>(it.qt - a.qtile_cu[r]) * kM;
-  it.row_end = min(it.row0 + kM, rr1);
-  const int pmax = a.text_idx[(it.row_end - 1) / a.G];
-  it.key0 = a.cu[r] + it.chunk * a.chunk_keys;
-  it.key_end = min(it.key0 + a.chunk_keys, pmax + 1);
-  return it;
+__device__ __forceinline__ Seg seg_of(const AttnArgs& a, int g, int b) {
+  Seg s;
+  s.g = g;
+  s.b = b;
+  s.r = upper_index(a.blk_cu, a.R, b);
+  s.R0 = static_cast<int64_t>(a.text_cu[s.r]) * a.G + static_cast<int64_t>(b - a.blk_cu[s.r]) * kBlk;
+  s.R1 = min(s.R0 + kBlk, static_cast<int64_t>(a.text_cu[s.r + 1]) * a.G);
+  return s;
 }
 
-struct P2Item {
-  int g, img;
-  int kp0, nk;           // packed position of the tile's first key, keys in the tile
-  int64_t row_begin, row_end;  // rows (within group g) of the text queries after the image
+// Walks a CTA's run of the flat list (KV group, block, entry) of a pass whose per-group
+// list has F entries with prefix cu over the NB blocks. Global memory is read only
+// when the walk enters a new block, so the single MMA-issuing and TMA-issuing threads
+// do not wait on dependent loads between steps.
+struct FlatCursor {
+  int g, b, j;  // KV group, block, entry within the block
+  int n;        // entries of block b
+  __device__ __forceinline__ void init(int64_t f, int F, const int32_t* cu, int NB) {
+    g = static_cast<int>(f / F);
+    const int fl = static_cast<int>(f - static_cast<int64_t>(g) * F);
+    b = upper_index(cu, NB, fl);
+    j = fl - cu[b];
+    n = cu[b + 1] - cu[b];
+  }
+  // Next entry; returns true when it lies in another block. Only called while another
+  // entry exists, so the loop over empty blocks ends.
+  __device__ __forceinline__ bool next(const int32_t* cu, int NB) {
+    if (++j < n) return false;
+    j = 0;
+    do {
+      if (++b == NB) {
+        b = 0;
+        ++g;
+      }
+      n = cu[b + 1] - cu[b];
+    } while (n == 0);
+    return true;
+  }
+  __device__ __forceinline__ bool last_of_block() const { return j + 1 == n; }
 };
 
-__device__ __forceinline__ P2Item p2_item(const AttnArgs& a, int n_per_group, int id) {
-  P2Item it;
-  it.g = id / n_per_group;
-  const int b = id - it.g * n_per_group;
-  const int i = upper_index(a.ktile_cu, a.NI, b);
-  const int r = a.img_req[i];
-  const int j = b - a.ktile_cu[i];
-  it.img = i;
-  it.kp0 = a.cu[r] + a.ist[i] + j * kM;
-  it.nk = min(kM, a.iln[i] - j * kM);
-  // text ordinal of the first token after the image: its request-local position minus the
-  // visual tokens before it, plus the request's first text ordinal
-  const int after = a.ist[i] + a.iln[i];
-  const int o_first = a.text_cu[r] + after - (a.vis_cu[i + 1] - a.vis_cu[a.icu[r]]);
-  it.row_begin = static_cast<int64_t>(o_first) * a.G;
-  it.row_end = static_cast<int64_t>(a.text_cu[r + 1]) * a.G;
-  return it;
+// Pass-2 key tiles of a block in order: tile j is tile jj of image i, the images of the
+// block's request in order. Image data is read when the walk enters a new image.
+struct TileCursor {
+  int i, jj;           // image, tile within the image
+  int kp0, nk, c0;     // first packed key, keys in the tile, first row of the block that sees it
+  int tile;            // key tile over all images (row of the mass accumulator)
+  int base, len, t0;   // packed position of the image's first key, its length, its first key tile
+  int64_t c0_img;      // o_first(i) * G - R0
+  __device__ __forceinline__ void load_image(const AttnArgs& a, const Seg& s) {
+    const int r = s.r;
+    base = a.cu[r] + a.ist[i];
+    len = a.iln[i];
+    t0 = a.ktile_cu[i];
+    const int64_t o_first =
+        static_cast<int64_t>(a.text_cu[r]) + a.ist[i] + len - (a.vis_cu[i + 1] - a.vis_cu[a.icu[r]]);
+    c0_img = o_first * a.G - s.R0;
+  }
+  __device__ __forceinline__ void fill() {
+    kp0 = base + jj * kM;
+    nk = min(kM, len - jj * kM);
+    tile = t0 + jj;
+    c0 = c0_img > 0 ? static_cast<int>(c0_img) : 0;
+  }
+  __device__ __forceinline__ void init(const AttnArgs& a, const Seg& s, int j) {
+    const int tile = a.ktile_cu[a.icu[s.r]] + j;
+    i = upper_index(a.ktile_cu, a.NI, tile);
+    jj = tile - a.ktile_cu[i];
+    load_image(a, s);
+    fill();
+  }
+  __device__ __forceinline__ void next(const AttnArgs& a, const Seg& s) {
+    if ((++jj) * kM >= len) {
+      ++i;
+      jj = 0;
+      load_image(a, s);
+    }
+    fill();
+  }
+};
+
+// ---------------------------------------------------------------- epilogue arithmetic
+// A warp's slice of an accumulator: its 32 TMEM lanes x kHalf columns, read as 32-column
+// chunks; chunk p+1 is loaded while chunk p is processed. MASKED = false is the common
+// case (every column visible to every lane): straight-line code without per-chunk
+// votes. The masked form handles the chunks [pb, pe) and keeps the columns c with
+// lo <= c < hi (per lane in pass 1, per CTA in pass 2).
+constexpr int kHalf = kN / 2;
+constexpr int kChunks = kHalf / 32;
+
+// Pass 1: online (max m, sum l) of exp2(c2 * z) over the visible columns of a row.
+template <bool MASKED>
+__device__ __forceinline__ void p1_slice(uint32_t taddr, int pe, int lim, float c2, float& m, float& l) {
+  uint32_t ra[32], rb[32];
+  auto chunk = [&](uint32_t(&r)[32], uint32_t(&nx)[32], int p) {
+    if (p + 1 < pe) tc::tmem_ld32_async(taddr + (p + 1) * 32, nx);
+    float v[32];
+#pragma unroll
+    for (int q = 0; q < 32; ++q) v[q] = __uint_as_float(r[q]);
+    if (MASKED) {
+#pragma unroll
+      for (int q = 0; q < 32; ++q) v[q] = (p * 32 + q <= lim) ? v[q] : -INFINITY;
+    }
+    float mx0 = fmaxf(v[0], v[1]), mx1 = fmaxf(v[2], v[3]);
+#pragma unroll
+    for (int q = 4; q < 32; q += 4) {
+      mx0 = fmaxf(mx0, fmaxf(v[q], v[q + 1]));
+      mx1 = fmaxf(mx1, fmaxf(v[q + 2], v[q + 3]));
+    }
+    const float mn = fmaxf(m, fmaxf(mx0, mx1) * c2);
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+    for (int q = 0; q < 32; q += 4) {
+      s0 += tc::ex2(fmaf(v[q], c2, -mn));
+      s1 += tc::ex2(fmaf(v[q + 1], c2, -mn));
+      s2 += tc::ex2(fmaf(v[q + 2], c2, -mn));
+      s3 += tc::ex2(fmaf(v[q + 3], c2, -mn));
+    }
+    // a row with nothing visible yet keeps (-inf, 0); exp2(-inf - -inf) would be NaN
+    if (mn != -INFINITY) {
+      l = l * tc::ex2(m - mn) + ((s0 + s1) + (s2 + s3));
+      m = mn;
+    }
+    if (p + 1 < pe) tc::tmem_wait(nx);
+  };
+  tc::tmem_ld32_async(taddr, ra);
+  tc::tmem_wait(ra);
+#pragma unroll
+  for (int p = 0; p < kChunks; p += 2) {
+    if (p < pe) chunk(ra, rb, p);
+    if (p + 1 < pe) chunk(rb, ra, p + 1);
+  }
 }
 
-// ---------------------------------------------------------------- the persistent kernel
-// PASS 1: A = Qt rows (box 64 x 128), B = key tiles (box 64 x 256).
-// PASS 2: A = key tile (box 64 x 128), B = Qt rows (box 64 x 256).
-// Epilogue warp w reads TMEM lane quadrant w % 4 and column half w / 4 of each step.
-template <int PASS>
-__global__ void __launch_bounds__(kThreads, 1)
-k_attn_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, AttnArgs a) {
-  extern __shared__ unsigned char smem_raw[];
-  __shared__ Sync sy;
-  __shared__ __align__(16) float s_lse[2][kN];
-  __shared__ float2 s_mrg[2][kM];
-  unsigned char* smem =
-      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  const int d = a.d;
-  unsigned char* sA[2] = {smem, smem + a_bytes(d)};
-  unsigned char* sB[2] = {smem + 2 * a_bytes(d), smem + 2 * a_bytes(d) + b_bytes(d)};
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t atomA = kM * 128, atomB = kN * 128;  // bytes per 64-element atom column
+// Pass 2: sum of exp2(c2 * z - lse2[c]) over the columns c of a key; a column that does
+// not see the key carries lse2 = +inf, which makes its term 0.
+__device__ __forceinline__ float p2_slice(uint32_t taddr, const float* lse, float c2) {
+  uint32_t ra[32], rb[32];
+  float m0 = 0.f, m1 = 0.f, m2 = 0.f, m3 = 0.f;
+  auto chunk = [&](uint32_t(&r)[32], uint32_t(&nx)[32], int p) {
+    if (p + 1 < kChunks) tc::tmem_ld32_async(taddr + (p + 1) * 32, nx);
+    const float4* l4 = reinterpret_cast<const float4*>(lse + p * 32);
+#pragma unroll
+    for (int q4 = 0; q4 < 8; ++q4) {
+      const float4 lv = l4[q4];
+      m0 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 0]), c2, -lv.x));
+      m1 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 1]), c2, -lv.y));
+      m2 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 2]), c2, -lv.z));
+      m3 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 3]), c2, -lv.w));
+    }
+    if (p + 1 < kChunks) tc::tmem_wait(nx);
+  };
+  tc::tmem_ld32_async(taddr, ra);
+  tc::tmem_wait(ra);
+#pragma unroll
+  for (int p = 0; p < kChunks; p += 2) {
+    chunk(ra, rb, p);
+    chunk(rb, ra, p + 1);
+  }
+  return (m0 + m1) + (m2 + m3);
+}
 
-  pdl_wait();
-  pdl_trigger();
-  if (!a.st->layout_ok) return;
-  const int n_per_group = (PASS == 1) ? a.p1_cu[a.qtile_cu[a.R]] : a.ktile_cu[a.NI];
-  const int n_items = n_per_group * a.Hkv;
-  if (static_cast<int>(blockIdx.x) >= n_items) return;
-
+__device__ __forceinline__ void setup_sync(Sync& sy, int warp) {
   if (threadIdx.x == 0) {
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kP2Stages; ++s) {
       tc::mbar_init(&sy.a_full[s], 1);
       tc::mbar_init(&sy.a_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       tc::mbar_init(&sy.b_full[s], 1);
       tc::mbar_init(&sy.b_empty[s], 1);
       tc::mbar_init(&sy.acc_full[s], 1);
@@ -181,54 +289,79 @@ k_attn_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUte
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
+}
+
+__device__ __forceinline__ void teardown(Sync& sy, int warp, uint32_t tmem, DevStatus* st) {
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, kTmemCols);
+  }
+  if (threadIdx.x == 0 && sy.abort) record_error(st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));
+}
+
+// ---------------------------------------------------------------- pass 1: log-sum-exp of every row
+// mapQ: Qt {d, rows, Hkv}, box 64 x 128 x 1; mapK: keys {d, Hkv, T}, box 64 x 1 x 256.
+__global__ void __launch_bounds__(kThreads, 1)
+k_attn_lse(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK, AttnArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  __shared__ Sync sy;
+  __shared__ float2 s_mrg[2][2][kM];  // [segment parity][A tile][row]: column half 1's (max, sum)
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int d = a.d;
+  unsigned char* sA = smem;  // A tile t at sA + t * a_bytes(d)
+  unsigned char* sB[2] = {smem + 2 * a_bytes(d), smem + 2 * a_bytes(d) + b_bytes(d)};
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t atomA = kM * 128, atomB = kN * 128;  // bytes per 64-element atom column
+
+  pdl_wait();
+  pdl_trigger();
+  if (!a.st->layout_ok) return;
+  const int NB = a.blk_cu[a.R];
+  const int F1 = a.meta[0], C1 = a.meta[1];
+  const int64_t total = static_cast<int64_t>(a.Hkv) * F1;
+  const int64_t f_begin = static_cast<int64_t>(blockIdx.x) * C1;
+  if (f_begin >= total) return;
+  const int n_steps = static_cast<int>(min(f_begin + C1, total) - f_begin);
+
+  setup_sync(sy, warp);
   const uint32_t tmem = sy.tmem;
   volatile int* abort_flag = &sy.abort;
-
-  // B steps of an item (0: nothing to compute)
-  auto item_steps = [&](int id, int& a_y, int& a_z, int64_t& b0) {
-    if (PASS == 1) {
-      const P1Item it = p1_item(a, n_per_group, id);
-      a_y = static_cast<int>(it.row0);
-      a_z = it.g;
-      b0 = it.key0;
-      return (it.key_end - it.key0 + kN - 1) / kN;
-    }
-    const P2Item it = p2_item(a, n_per_group, id);
-    a_y = it.g;
-    a_z = it.kp0;
-    b0 = it.row_begin;
-    return it.row_end > it.row_begin ? static_cast<int>((it.row_end - it.row_begin + kN - 1) / kN) : 0;
-  };
+  FlatCursor cur;
+  cur.init(f_begin, F1, a.p1s_cu, NB);
 
   if (warp == kTmaWarp) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      tc::tma_prefetch_map(&mapA);
-      tc::tma_prefetch_map(&mapB);
-      uint32_t na = 0, nb = 0;  // A loads and B loads issued so far
-      for (int id = blockIdx.x; id < n_items && !*abort_flag; id += gridDim.x) {
-        int a_y, a_z;
-        int64_t b0;
-        const int steps = item_steps(id, a_y, a_z, b0);
-        if (steps <= 0) continue;
-        const int sa = na & 1;
-        if (na >= 2 && !tc::mbar_wait(&sy.a_empty[sa], ((na >> 1) - 1) & 1)) { *abort_flag = 1; break; }
-        tc::mbar_arrive_expect_tx(&sy.a_full[sa], static_cast<uint32_t>(a_bytes(d)));
-        for (int ac = 0; ac < d / 64; ++ac) tc::tma_load_3d(sA[sa] + ac * atomA, &mapA, ac * 64, a_y, a_z, &sy.a_full[sa]);
-        ++na;
-        for (int st = 0; st < steps; ++st, ++nb) {
-          const int s = nb & 1;
-          if (nb >= 2 && !tc::mbar_wait(&sy.b_empty[s], ((nb >> 1) - 1) & 1)) { *abort_flag = 1; break; }
-          tc::mbar_arrive_expect_tx(&sy.b_full[s], static_cast<uint32_t>(b_bytes(d)));
-          const int y = static_cast<int>(b0 + static_cast<int64_t>(st) * kN);
-          for (int ac = 0; ac < d / 64; ++ac) {
-            if (PASS == 1) tc::tma_load_3d(sB[s] + ac * atomB, &mapB, ac * 64, a_z, y, &sy.b_full[s]);  // {d, Hkv, T}
-            else tc::tma_load_3d(sB[s] + ac * atomB, &mapB, ac * 64, y, a_y, &sy.b_full[s]);            // {d, rows, Hkv}
-          }
+      tc::tma_prefetch_map(&mapQ);
+      tc::tma_prefetch_map(&mapK);
+      uint32_t na = 0, nb = 0;  // A (block) loads and B (key tile) loads issued so far
+      int key_base = 0;
+      bool new_seg = true;
+      for (int st = 0; st < n_steps && !*abort_flag; ++st) {
+        if (new_seg) {
+          if (na >= 1 && !tc::mbar_wait(&sy.a_empty[0], (na - 1) & 1)) { *abort_flag = 1; break; }
+          const Seg s = seg_of(a, cur.g, cur.b);
+          tc::mbar_arrive_expect_tx(&sy.a_full[0], static_cast<uint32_t>(2 * a_bytes(d)));
+          for (int t = 0; t < 2; ++t)
+            for (int ac = 0; ac < d / 64; ++ac)
+              tc::tma_load_3d(sA + t * a_bytes(d) + ac * atomA, &mapQ, ac * 64, static_cast<int>(s.R0) + t * kM,
+                              cur.g, &sy.a_full[0]);
+          ++na;
+          key_base = a.cu[s.r];
         }
+        const int sb = nb & 1;
+        if (nb >= 2 && !tc::mbar_wait(&sy.b_empty[sb], ((nb >> 1) - 1) & 1)) { *abort_flag = 1; break; }
+        tc::mbar_arrive_expect_tx(&sy.b_full[sb], static_cast<uint32_t>(b_bytes(d)));
+        for (int ac = 0; ac < d / 64; ++ac)
+          tc::tma_load_3d(sB[sb] + ac * atomB, &mapK, ac * 64, cur.g, key_base + cur.j * kN, &sy.b_full[sb]);
+        ++nb;
+        new_seg = st + 1 < n_steps && cur.next(a.p1s_cu, NB);
       }
       // let the copies in flight land before the CTA may exit
-      for (uint32_t k = (na >= 2 ? na - 2 : 0); k < na; ++k) tc::mbar_wait(&sy.a_full[k & 1], (k >> 1) & 1);
+      if (na >= 1) tc::mbar_wait(&sy.a_full[0], (na - 1) & 1);
       for (uint32_t k = (nb >= 2 ? nb - 2 : 0); k < nb; ++k) tc::mbar_wait(&sy.b_full[k & 1], (k >> 1) & 1);
     }
   } else if (warp == kMmaWarp) {
@@ -236,24 +369,27 @@ k_attn_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUte
     if (lane == 0) {
       const uint32_t idesc = tc::idesc_bf16(kM, kN);
       uint32_t na = 0, nb = 0;
-      for (int id = blockIdx.x; id < n_items && !*abort_flag; id += gridDim.x) {
-        int a_y, a_z;
-        int64_t b0;
-        const int steps = item_steps(id, a_y, a_z, b0);
-        if (steps <= 0) continue;
-        const int sa = na & 1;
-        if (!tc::mbar_wait(&sy.a_full[sa], (na >> 1) & 1)) { *abort_flag = 1; break; }
-        for (int st = 0; st < steps; ++st, ++nb) {
-          const int s = nb & 1;
-          if (!tc::mbar_wait(&sy.b_full[s], (nb >> 1) & 1)) { *abort_flag = 1; break; }
-          if (nb >= 2 && !tc::mbar_wait(&sy.acc_empty[s], ((nb >> 1) - 1) & 1)) { *abort_flag = 1; break; }
-          tc::fence_after_sync();
-          tc::mma_rows(tmem + s * kN, tc::smem_u32(sA[sa]), atomA, tc::smem_u32(sB[s]), atomB, d, idesc);
-          tc::mma_commit(&sy.b_empty[s]);
-          tc::mma_commit(&sy.acc_full[s]);
+      bool new_seg = true, stop = false;
+      for (int st = 0; st < n_steps && !stop && !*abort_flag; ++st) {
+        if (new_seg) {
+          if (!tc::mbar_wait(&sy.a_full[0], na & 1)) { *abort_flag = 1; break; }
+          ++na;
         }
-        tc::mma_commit(&sy.a_empty[sa]);
-        ++na;
+        const int sb = nb & 1;
+        if (!tc::mbar_wait(&sy.b_full[sb], (nb >> 1) & 1)) { *abort_flag = 1; break; }
+        for (int t = 0; t < 2; ++t) {
+          // accumulator t: its previous use (step nb - 1) must have been read out
+          if (nb >= 1 && !tc::mbar_wait(&sy.acc_empty[t], (nb - 1) & 1)) { *abort_flag = 1; stop = true; break; }
+          tc::fence_after_sync();
+          tc::mma_rows(tmem + t * kN, tc::smem_u32(sA + t * a_bytes(d)), atomA, tc::smem_u32(sB[sb]), atomB, d, idesc);
+          tc::mma_commit(&sy.acc_full[t]);
+        }
+        if (stop) break;
+        tc::mma_commit(&sy.b_empty[sb]);
+        ++nb;
+        const bool more = st + 1 < n_steps;
+        if (!more || cur.last_of_block()) tc::mma_commit(&sy.a_empty[0]);
+        new_seg = more && cur.next(a.p1s_cu, NB);
       }
       // every MMA issued has completed once this arrives
       tc::mma_commit(&sy.drain);
@@ -261,205 +397,307 @@ k_attn_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUte
     }
   } else {
     // ------------------------------------------------------------ epilogue (8 warps)
-    const int etid = threadIdx.x;               // 0 .. 255
+    // Warp w reads TMEM lanes 32(w%4)..+31 (its rows of both A tiles) and columns
+    // 128(w/4)..+127 of both accumulators; the two column halves of a row meet in
+    // shared memory when the row's partial is written.
     const int quad = warp & 3, half = warp >> 2;
-    const int lrow = quad * 32 + lane;          // TMEM lane: row (pass 1) or key (pass 2) of the tile
-    const uint32_t taddr = tmem + (static_cast<uint32_t>(quad * 32) << 16) + half * (kN / 2);
+    const int lrow = quad * 32 + lane;  // row of each A tile = TMEM lane
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16) + half * (kN / 2);
     const float c2 = a.c2;
-    // After a timeout (abort_flag) the epilogue keeps walking the same items and steps,
-    // skipping every wait and TMEM read, so that its named barriers still line up.
-    uint32_t nb = 0;
-    int it_count = 0;
-    for (int id = blockIdx.x; id < n_items; id += gridDim.x, ++it_count) {
-      const int slot = it_count & 1;
-      if (PASS == 1) {
-        const P1Item it = p1_item(a, n_per_group, id);
-        const int steps = (it.key_end - it.key0 + kN - 1) / kN;
-        const int64_t row = it.row0 + lrow;
-        const bool valid = row < it.row_end;
-        const int qpos = valid ? a.text_idx[row / a.G] : -1;
-        // keys up to min(qpos, key_end - 1) are visible to this row
-        const int last = min(qpos, it.key_end - 1);
-        float m = -INFINITY, l = 0.f;  // running max and sum, scaled (log2) domain
-        for (int st = 0; st < steps; ++st, ++nb) {
-          const int s = nb & 1;
-          bool ok = !__any_sync(0xffffffffu, *abort_flag != 0);
-          if (ok && !tc::mbar_wait_warp(&sy.acc_full[s], (nb >> 1) & 1)) {
-            if (lane == 0) *abort_flag = 1;
-            ok = false;
-          }
-          tc::fence_after_sync();
-          const int k0 = it.key0 + st * kN + half * (kN / 2);  // key of this thread's first column
-          const int lim = last - k0;                            // columns 0..lim are visible
-          const bool all_visible = __all_sync(0xffffffffu, lim >= kN / 2 - 1);
-          const bool any_visible = __any_sync(0xffffffffu, lim >= 0);
-          if (ok && any_visible) {
+    // After a timeout (abort_flag) the epilogue keeps walking the same steps, skipping
+    // every wait and TMEM read, so that its named barriers still line up.
+    int key_base = 0, qpos0 = -1, qpos1 = -1, par = 0;
+    bool new_seg = true;
+    float2* dst0 = nullptr;          // this row's partial (A tile 0, 1) of the current block
+    float2* dst1 = nullptr;
+    float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;  // running max and sum, log2 domain
+    for (int st = 0; st < n_steps; ++st) {
+      if (new_seg) {
+        const Seg s = seg_of(a, cur.g, cur.b);
+        key_base = a.cu[s.r];
+        const int64_t F0 = static_cast<int64_t>(cur.g) * F1 + a.p1s_cu[cur.b];
+        const int slot = static_cast<int>(blockIdx.x - F0 / C1);
+        const int64_t row0 = s.R0 + lrow, row1 = s.R0 + kM + lrow;
+        float2* base = a.p1_part + (static_cast<int64_t>(cur.g * NB + cur.b) * kBlk + lrow) * kAttnMaxChunks + slot;
+        qpos0 = row0 < s.R1 ? a.text_idx[row0 / a.G] : -1;
+        qpos1 = row1 < s.R1 ? a.text_idx[row1 / a.G] : -1;
+        dst0 = row0 < s.R1 ? base : nullptr;
+        dst1 = row1 < s.R1 ? base + static_cast<int64_t>(kM) * kAttnMaxChunks : nullptr;
+        m0 = m1 = -INFINITY;
+        l0 = l1 = 0.f;
+      }
 #pragma unroll 1
-            for (int p = 0; p < kN / 2 / 64; ++p) {
-              float v[64];
-              tc::tmem_ld64(taddr + s * kN + p * 64, v);
-              if (!all_visible) {
-#pragma unroll
-                for (int q = 0; q < 64; ++q) v[q] = (p * 64 + q <= lim) ? v[q] : -INFINITY;
-              }
-              float mx0 = v[0], mx1 = v[1], mx2 = v[2], mx3 = v[3];
-#pragma unroll
-              for (int q = 4; q < 64; q += 4) {
-                mx0 = fmaxf(mx0, v[q]);
-                mx1 = fmaxf(mx1, v[q + 1]);
-                mx2 = fmaxf(mx2, v[q + 2]);
-                mx3 = fmaxf(mx3, v[q + 3]);
-              }
-              const float mn = fmaxf(m, fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * c2);
-              if (mn != -INFINITY) {
-                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-                for (int q = 0; q < 64; q += 4) {
-                  s0 += tc::ex2(fmaf(v[q], c2, -mn));
-                  s1 += tc::ex2(fmaf(v[q + 1], c2, -mn));
-                  s2 += tc::ex2(fmaf(v[q + 2], c2, -mn));
-                  s3 += tc::ex2(fmaf(v[q + 3], c2, -mn));
-                }
-                l = l * tc::ex2(m - mn) + ((s0 + s1) + (s2 + s3));
-                m = mn;
-              }
-            }
-          }
-          tc::fence_before_sync();
-          __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&sy.acc_empty[s]);
+      for (int t = 0; t < 2; ++t) {
+        bool ok = !__any_sync(0xffffffffu, *abort_flag != 0);
+        if (ok && !tc::mbar_wait_warp(&sy.acc_full[t], st & 1)) {
+          if (lane == 0) *abort_flag = 1;
+          ok = false;
         }
-        // the two column halves of a row meet here; this chunk's (max, sum) per row goes
-        // to [row tile][row][chunk] for k_attn_merge
-        if (half == 1) s_mrg[slot][lrow] = make_float2(m, l);
+        tc::fence_after_sync();
+        // columns 0..lim of this warp's half are visible to the row
+        const int lim = (t ? qpos1 : qpos0) - (key_base + cur.j * kN + half * (kN / 2));
+        const int lim_max = __reduce_max_sync(0xffffffffu, lim);
+        if (ok && lim_max >= 0) {
+          const uint32_t taddr = tbase + t * kN;
+          float mt = t ? m1 : m0, lt = t ? l1 : l0;
+          if (__all_sync(0xffffffffu, lim >= kHalf - 1)) {
+            p1_slice<false>(taddr, kChunks, lim, c2, mt, lt);
+          } else {
+            // 32-column chunks 0 .. pe-1 hold a visible column for some lane
+            p1_slice<true>(taddr, min(kChunks, (lim_max >> 5) + 1), lim, c2, mt, lt);
+          }
+          if (t) { m1 = mt; l1 = lt; } else { m0 = mt; l0 = lt; }
+        }
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&sy.acc_empty[t]);
+      }
+      const bool more = st + 1 < n_steps;
+      if (!more || cur.last_of_block()) {
+        // the block ends here for this CTA: merge the column halves and write the partial
+        par ^= 1;
+        if (half == 1) {
+          s_mrg[par][0][lrow] = make_float2(m0, l0);
+          s_mrg[par][1][lrow] = make_float2(m1, l1);
+        }
         bar_epi();
         if (half == 0) {
-          const float2 o = s_mrg[slot][lrow];
-          const float M = fmaxf(m, o.x);
-          const float L = (M == -INFINITY) ? 0.f : l * tc::ex2(m - M) + o.y * tc::ex2(o.x - M);
-          const int64_t tile = static_cast<int64_t>(it.g) * a.qtile_cu[a.R] + it.qt;
-          a.p1_part[(tile * kM + lrow) * kAttnMaxChunks + it.chunk] = make_float2(M, L);
+          auto merge = [&](float m, float l, float2 o, float2* dst) {
+            const float M = fmaxf(m, o.x);
+            const float L = (M == -INFINITY) ? 0.f : l * tc::ex2(m - M) + o.y * tc::ex2(o.x - M);
+            *dst = make_float2(M, L);
+          };
+          if (dst0 != nullptr) merge(m0, l0, s_mrg[par][0][lrow], dst0);
+          if (dst1 != nullptr) merge(m1, l1, s_mrg[par][1][lrow], dst1);
         }
-      } else {
-        const P2Item it = p2_item(a, n_per_group, id);
-        const int steps =
-            it.row_end > it.row_begin ? static_cast<int>((it.row_end - it.row_begin + kN - 1) / kN) : 0;
-        const float* lse_g = a.lse_rows + static_cast<int64_t>(it.g) * a.rows;
-        // the rows' lse2 (+inf past the last row, which zeroes their terms); the next
-        // step's value is loaded while this step is processed
-        auto lse_of = [&](int st) {
-          const int64_t r = it.row_begin + static_cast<int64_t>(st) * kN + etid;
-          return (st < steps && r < it.row_end) ? lse_g[r] : INFINITY;
-        };
-        float lse_next = lse_of(0);
-        float m0 = 0.f, m1 = 0.f, m2 = 0.f, m3 = 0.f;
-        for (int st = 0; st < steps; ++st, ++nb) {
-          const int s = nb & 1;
-          s_lse[s][etid] = lse_next;
-          bar_epi();
-          lse_next = lse_of(st + 1);
-          bool ok = !__any_sync(0xffffffffu, *abort_flag != 0);
-          if (ok && !tc::mbar_wait_warp(&sy.acc_full[s], (nb >> 1) & 1)) {
-            if (lane == 0) *abort_flag = 1;
-            ok = false;
-          }
-          tc::fence_after_sync();
-#pragma unroll 1
-          for (int p = 0; p < (ok ? kN / 2 / 64 : 0); ++p) {
-            float v[64];
-            tc::tmem_ld64(taddr + s * kN + p * 64, v);
-            const float4* l4 = reinterpret_cast<const float4*>(&s_lse[s][half * (kN / 2) + p * 64]);
-#pragma unroll
-            for (int q4 = 0; q4 < 16; ++q4) {
-              const float4 lv = l4[q4];
-              m0 += tc::ex2(fmaf(v[4 * q4 + 0], c2, -lv.x));
-              m1 += tc::ex2(fmaf(v[4 * q4 + 1], c2, -lv.y));
-              m2 += tc::ex2(fmaf(v[4 * q4 + 2], c2, -lv.z));
-              m3 += tc::ex2(fmaf(v[4 * q4 + 3], c2, -lv.w));
-            }
-          }
-          tc::fence_before_sync();
-          __syncwarp();
-          if (lane == 0) tc::mbar_arrive(&sy.acc_empty[s]);
-        }
-        const float mass = (m0 + m1) + (m2 + m3);
-        if (half == 1) s_mrg[slot][lrow].x = mass;
-        bar_epi();
-        if (half == 0 && lrow < it.nk)
-          a.partial[static_cast<int64_t>(it.g) * a.T + it.kp0 + lrow] = mass + s_mrg[slot][lrow].x;
       }
+      new_seg = more && cur.next(a.p1s_cu, NB);
     }
   }
-
-  tc::fence_before_sync();
-  __syncthreads();
-  if (warp == kMmaWarp) {
-    tc::fence_after_sync();
-    tc::tmem_dealloc(tmem, kTmemCols);
-  }
-  if (threadIdx.x == 0 && sy.abort) record_error(a.st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));
+  teardown(sy, warp, tmem, a.st);
 }
 
-// ---------------------------------------------------------------- pass-1 chunk merge
-// lse2 of every row: the log2-sum-exp2 merge of its chunks' (max, sum). One thread per
-// (KV group, row); a row's chunks are contiguous.
-__global__ void __launch_bounds__(256)
-k_attn_merge(AttnArgs a) {
+// ---------------------------------------------------------------- pass 2: probability mass of every visual key
+// mapK: keys {d, Hkv, T}, box 64 x 1 x 128; mapQ: Qt {d, rows, Hkv}, box 64 x 256 x 1.
+__global__ void __launch_bounds__(kThreads, 1)
+k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapQ, AttnArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  __shared__ Sync sy;
+  __shared__ __align__(16) float s_lse[2][kBlk];  // [block parity][row of the block]
+  // key masses of the last steps, per column half, flushed to the accumulator every
+  // kMassWindow steps (global atomics inside the step loop would be waited for by the
+  // next step's TMEM fence)
+  __shared__ float s_mass[kMassWindow][2][kM];
+  __shared__ int s_tile[kMassWindow], s_nk[kMassWindow];
+  unsigned char* smem =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int d = a.d;
+  unsigned char* sB = smem;  // the block's rows
+  unsigned char* sA0 = smem + b_bytes(d);  // key tile s at sA0 + s * a_bytes(d)
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t atomA = kM * 128, atomB = kN * 128;
+
   pdl_wait();
   pdl_trigger();
   if (!a.st->layout_ok) return;
-  const int nq = a.qtile_cu[a.R];
-  const int64_t total = static_cast<int64_t>(a.Hkv) * nq * kM;
-  for (int64_t u = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; u < total;
-       u += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int lr = static_cast<int>(u % kM);
-    const int64_t tile = u / kM;
-    const int g = static_cast<int>(tile / nq), qt = static_cast<int>(tile - static_cast<int64_t>(g) * nq);
-    const int r = upper_index(a.qtile_cu, a.R, qt);
-    const int64_t row = static_cast<int64_t>(a.text_cu[r]) * a.G + static_cast<int64_t>(qt - a.qtile_cu[r]) * kM + lr;
-    if (row >= static_cast<int64_t>(a.text_cu[r + 1]) * a.G) continue;
-    const int nc = a.p1_cu[qt + 1] - a.p1_cu[qt];
-    const float4* src = reinterpret_cast<const float4*>(a.p1_part + u * kAttnMaxChunks);
-    float M = -INFINITY, L = 0.f;
-    auto merge = [&](float mc, float lc) {
-      const float Mn = fmaxf(M, mc);
-      if (Mn != -INFINITY) {
-        L = L * tc::ex2(M - Mn) + lc * tc::ex2(mc - Mn);
-        M = Mn;
+  const int NB = a.blk_cu[a.R];
+  const int F1 = a.meta[0], C1 = a.meta[1], F2 = a.meta[2], C2 = a.meta[3];
+  const int64_t total = static_cast<int64_t>(a.Hkv) * F2;
+  const int64_t f_begin = static_cast<int64_t>(blockIdx.x) * C2;
+  if (f_begin >= total) return;
+  const int n_steps = static_cast<int>(min(f_begin + C2, total) - f_begin);
+
+  setup_sync(sy, warp);
+  const uint32_t tmem = sy.tmem;
+  volatile int* abort_flag = &sy.abort;
+  FlatCursor cur;
+  cur.init(f_begin, F2, a.p2t_cu, NB);
+
+  if (warp == kTmaWarp) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      tc::tma_prefetch_map(&mapQ);
+      tc::tma_prefetch_map(&mapK);
+      uint32_t na = 0, nbl = 0;  // key tile loads and block loads issued so far
+      bool new_seg = true;
+      Seg s{};
+      TileCursor tile{};
+      for (int st = 0; st < n_steps && !*abort_flag; ++st) {
+        if (new_seg) {
+          if (nbl >= 1 && !tc::mbar_wait(&sy.b_empty[0], (nbl - 1) & 1)) { *abort_flag = 1; break; }
+          s = seg_of(a, cur.g, cur.b);
+          tc::mbar_arrive_expect_tx(&sy.b_full[0], static_cast<uint32_t>(b_bytes(d)));
+          for (int ac = 0; ac < d / 64; ++ac)
+            tc::tma_load_3d(sB + ac * atomB, &mapQ, ac * 64, static_cast<int>(s.R0), cur.g, &sy.b_full[0]);
+          ++nbl;
+          tile.init(a, s, cur.j);
+        } else {
+          tile.next(a, s);
+        }
+        const int sa = na % kP2Stages;
+        if (na >= kP2Stages && !tc::mbar_wait(&sy.a_empty[sa], ((na / kP2Stages) - 1) & 1)) { *abort_flag = 1; break; }
+        tc::mbar_arrive_expect_tx(&sy.a_full[sa], static_cast<uint32_t>(a_bytes(d)));
+        for (int ac = 0; ac < d / 64; ++ac)
+          tc::tma_load_3d(sA0 + sa * a_bytes(d) + ac * atomA, &mapK, ac * 64, cur.g, tile.kp0, &sy.a_full[sa]);
+        ++na;
+        new_seg = st + 1 < n_steps && cur.next(a.p2t_cu, NB);
       }
-    };
-    const int n4 = (nc + 1) >> 1;  // a float4 holds two chunks
-    for (int c4 = 0; c4 < n4; c4 += 8) {
-      float4 buf[8];
-#pragma unroll
-      for (int w = 0; w < 8; ++w)
-        buf[w] = (c4 + w < n4) ? __ldg(src + c4 + w) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
-#pragma unroll
-      for (int w = 0; w < 8; ++w) {
-        merge(buf[w].x, buf[w].y);
-        if (2 * (c4 + w) + 1 < nc) merge(buf[w].z, buf[w].w);
-      }
+      if (nbl >= 1) tc::mbar_wait(&sy.b_full[0], (nbl - 1) & 1);
+      for (uint32_t k = (na >= kP2Stages ? na - kP2Stages : 0); k < na; ++k)
+        tc::mbar_wait(&sy.a_full[k % kP2Stages], (k / kP2Stages) & 1);
     }
-    a.lse_rows[static_cast<int64_t>(g) * a.rows + row] = M + __log2f(L);
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = tc::idesc_bf16(kM, kN);
+      uint32_t na = 0, nbl = 0;
+      bool new_seg = true;
+      for (int st = 0; st < n_steps && !*abort_flag; ++st) {
+        if (new_seg) {
+          if (!tc::mbar_wait(&sy.b_full[0], nbl & 1)) { *abort_flag = 1; break; }
+          ++nbl;
+        }
+        const int sa = na % kP2Stages;
+        if (!tc::mbar_wait(&sy.a_full[sa], (na / kP2Stages) & 1)) { *abort_flag = 1; break; }
+        const int t = na & 1;  // accumulator of this step
+        if (na >= 2 && !tc::mbar_wait(&sy.acc_empty[t], ((na >> 1) - 1) & 1)) { *abort_flag = 1; break; }
+        tc::fence_after_sync();
+        tc::mma_rows(tmem + t * kN, tc::smem_u32(sA0 + sa * a_bytes(d)), atomA, tc::smem_u32(sB), atomB, d, idesc);
+        tc::mma_commit(&sy.a_empty[sa]);
+        tc::mma_commit(&sy.acc_full[t]);
+        ++na;
+        const bool more = st + 1 < n_steps;
+        if (!more || cur.last_of_block()) tc::mma_commit(&sy.b_empty[0]);
+        new_seg = more && cur.next(a.p2t_cu, NB);
+      }
+      tc::mma_commit(&sy.drain);
+      tc::mbar_wait(&sy.drain, 0);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (8 warps)
+    // Warp w reads TMEM lanes 32(w%4)..+31 (its keys) and columns 128(w/4)..+127 (rows
+    // of the block) of the step's accumulator; each column half adds its own share of a
+    // key's mass to the fixed-point accumulator.
+    const int quad = warp & 3, half = warp >> 2;
+    const int klane = quad * 32 + lane;  // key of the tile = TMEM lane
+    const int etid = threadIdx.x;        // 0 .. 255
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(quad * 32) << 16) + half * (kBlk / 2);
+    const float c2 = a.c2;
+    int par = 0, c1 = 0, img = -1;
+    float lse_own = INFINITY;  // lse2 of this thread's row of the block (row etid)
+    bool new_seg = true;
+    Seg s{};
+    TileCursor tile{};
+    for (int st = 0; st < n_steps; ++st) {
+      if (new_seg) {
+        s = seg_of(a, cur.g, cur.b);
+        c1 = static_cast<int>(s.R1 - s.R0);  // rows of the block that belong to the request
+        const int g = cur.g, b = cur.b;
+        const int64_t row = s.R0 + etid;
+        lse_own = INFINITY;
+        if (row < s.R1) {
+          if (a.lse_rows != nullptr) {
+            lse_own = a.lse_rows[static_cast<int64_t>(g) * a.rows + row];
+          } else {
+            // merge the row's pass-1 partials, eight loads in flight at a time
+            const int64_t F0 = static_cast<int64_t>(g) * F1 + a.p1s_cu[b];
+            const int steps = a.p1s_cu[b + 1] - a.p1s_cu[b];
+            const int n = static_cast<int>((F0 + steps - 1) / C1 - F0 / C1) + 1;
+            const float2* src = a.p1_part + (static_cast<int64_t>(g * NB + b) * kBlk + etid) * kAttnMaxChunks;
+            float M = -INFINITY, L = 0.f;
+            for (int k0 = 0; k0 < n; k0 += 8) {
+              float2 pk[8];
+#pragma unroll
+              for (int k = 0; k < 8; ++k) pk[k] = (k0 + k < n) ? src[k0 + k] : make_float2(-INFINITY, 0.f);
+#pragma unroll
+              for (int k = 0; k < 8; ++k) {
+                const float Mn = fmaxf(M, pk[k].x);
+                if (Mn != -INFINITY) {
+                  L = L * tc::ex2(M - Mn) + pk[k].y * tc::ex2(pk[k].x - Mn);
+                  M = Mn;
+                }
+              }
+            }
+            lse_own = M + __log2f(L);
+          }
+        }
+        tile.init(a, s, cur.j);
+        img = -1;
+      } else {
+        tile.next(a, s);
+      }
+      if (tile.i != img) {
+        // the lse2 vector of this (block, image): +inf on rows whose query precedes the
+        // image, so that their terms vanish; double-buffered by parity
+        img = tile.i;
+        par ^= 1;
+        s_lse[par][etid] = (etid >= tile.c0) ? lse_own : INFINITY;
+        bar_epi();
+      }
+      const int t = st & 1;                                  // accumulator of this step
+      const uint32_t use = static_cast<uint32_t>(st) >> 1;  // its use count
+      bool ok = !__any_sync(0xffffffffu, *abort_flag != 0);
+      if (ok && !tc::mbar_wait_warp(&sy.acc_full[t], use & 1)) {
+        if (lane == 0) *abort_flag = 1;
+        ok = false;
+      }
+      tc::fence_after_sync();
+      // does this warp's column half hold a visible row? (CTA-uniform)
+      const bool any = tile.c0 < (half + 1) * kHalf && c1 > half * kHalf;
+      float mass = 0.f;
+      if (ok && any) mass = p2_slice(tbase + t * kN, &s_lse[par][half * kHalf], c2);
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive(&sy.acc_empty[t]);
+      const int w = st % kMassWindow;
+      s_mass[w][half][klane] = mass;
+      if (etid == 0) {
+        s_tile[w] = tile.tile;
+        s_nk[w] = tile.nk;
+      }
+      if (w == kMassWindow - 1 || st + 1 == n_steps) {
+        // flush: one fixed-point integer add per (step, key), both column halves summed
+        // in fp32 first (integer adds: the result does not depend on their order)
+        bar_epi();
+        for (int e = etid; e < (w + 1) * kM; e += kEpiWarps * 32) {
+          const int ws = e / kM, k = e % kM;
+          if (k < s_nk[ws]) {
+            const float m = s_mass[ws][0][k] + s_mass[ws][1][k];
+            unsigned long long* dst = a.mass + static_cast<int64_t>(s_tile[ws]) * kM + k;
+            if (m <= 512.f) {  // at most one per row of the block
+              atomicAdd(dst, static_cast<unsigned long long>(__float2ll_rn(m * static_cast<float>(1ull << kAttnMassFracBits))));
+            } else {
+              atomicOr(dst, kMassNotFinite);  // NaN or inf inputs: the key scores NaN (bit 63; finite adds never reach it)
+            }
+          }
+        }
+        bar_epi();
+      }
+      new_seg = st + 1 < n_steps && cur.next(a.p2t_cu, NB);
+    }
   }
+  teardown(sy, warp, tmem, a.st);
 }
 
 // ---------------------------------------------------------------- repacking of the text queries
 // Qt[g][o*G + j][:] = q[text_idx[o], g*G + j, :]; with a supplied LSE also
 // lse_rows[g][o*G + j] = lse[g*G + j][text_idx[o]] * log2(e). One thread per 16 bytes.
+// Also clears the per-key mass accumulator of pass 2.
 __global__ void __launch_bounds__(256)
 k_attn_pack(const __nv_bfloat16* __restrict__ q, int64_t q_stride, int Hq, int G, int d,
             const int32_t* __restrict__ text_idx, const int32_t* __restrict__ text_cu, int R, int64_t rows,
             __nv_bfloat16* __restrict__ qt, const float* __restrict__ lse, int64_t lse_stride,
-            float* __restrict__ lse_rows, const DevStatus* st) {
+            float* __restrict__ lse_rows, unsigned long long* __restrict__ mass, int64_t n_mass, const DevStatus* st) {
   pdl_wait();
   pdl_trigger();
   if (!st->layout_ok) return;
   const int64_t n_text = text_cu[R];
   const int vec = d / 8;
   const int64_t total = n_text * Hq * vec;
-  for (int64_t u = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; u < total;
-       u += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const int64_t tid0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  for (int64_t u = tid0; u < n_mass; u += stride) mass[u] = 0ull;
+  for (int64_t u = tid0; u < total; u += stride) {
     const int c = static_cast<int>(u % vec);
     const int64_t oh = u / vec;
     const int h = static_cast<int>(oh % Hq);
@@ -474,8 +712,10 @@ k_attn_pack(const __nv_bfloat16* __restrict__ q, int64_t q_stride, int Hq, int G
 }
 
 // ---------------------------------------------------------------- finalize
+// s_t = mass_t * 2^-40 / (Hq * |Q_r|) for every visual token, and the fixed-point image sums.
 __global__ void __launch_bounds__(256)
-k_attn_finalize(const float* __restrict__ partial, int Hq, int Hkv, int64_t T, const int32_t* __restrict__ cu,
+k_attn_finalize(const unsigned long long* __restrict__ mass, const int32_t* __restrict__ ktile_cu, int Hq,
+                const int32_t* __restrict__ cu,
                 const int32_t* __restrict__ img_start, const int32_t* __restrict__ vis_cu,
                 const int32_t* __restrict__ img_req, const int32_t* __restrict__ text_cu, int NI,
                 float* __restrict__ scores, int64_t* __restrict__ img_sums, const DevStatus* st) {
@@ -487,12 +727,18 @@ k_attn_finalize(const float* __restrict__ partial, int Hq, int Hkv, int64_t T, c
        v += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int i = upper_index(vis_cu, NI, v);
     const int r = img_req[i];
-    const int64_t t = static_cast<int64_t>(cu[r]) + img_start[i] + (v - vis_cu[i]);
+    const int o = static_cast<int>(v - vis_cu[i]);  // key within the image
+    const int64_t t = static_cast<int64_t>(cu[r]) + img_start[i] + o;
     const int nq = text_cu[r + 1] - text_cu[r];
     float s = 0.f;
     if (nq > 0) {
-      for (int g = 0; g < Hkv; ++g) s += partial[static_cast<int64_t>(g) * T + t];
-      s = s / static_cast<float>(static_cast<int64_t>(Hq) * nq);
+      const unsigned long long m = mass[static_cast<int64_t>(ktile_cu[i] + o / kM) * kM + o % kM];
+      if (m & kMassNotFinite) {
+        s = __int_as_float(0x7fc00000);
+      } else {
+        s = __ll2float_rn(static_cast<long long>(m)) * (1.0f / static_cast<float>(1ull << kAttnMassFracBits));
+        s = s / static_cast<float>(static_cast<int64_t>(Hq) * nq);
+      }
     }
     scores[t] = s;
     atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + i), static_cast<unsigned long long>(fixed_point_score(s)));
@@ -533,17 +779,15 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   if (L.n_images == 0 || L.n_tokens == 0) return cudaSuccess;
   const int d = sa.head_dim, Hq = sa.n_q_heads, Hkv = sa.n_kv_heads;
   const AttnPlan plan = attn_plan(L, sa);
-  static bool attr_set[2] = {false, false};
-  const size_t smem = tc_smem_bytes(d);
-  const int di = d == 128 ? 1 : 0;
-  if (!attr_set[di]) {
-    cudaError_t e = cudaFuncSetAttribute(k_attn_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(tc_smem_bytes(128)));
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_attn_lse, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(lse_smem_bytes(128)));
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(k_attn_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(tc_smem_bytes(128)));
+    e = cudaFuncSetAttribute(k_attn_mass, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(mass_smem_bytes(128)));
     if (e != cudaSuccess) return e;
-    attr_set[0] = attr_set[1] = true;
+    attr_set = true;
   }
   DevStatus* st = ws_at<DevStatus>(ws, p.status);
   AttnArgs a{};
@@ -555,21 +799,21 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   a.NI = L.n_images;
   a.T = L.n_tokens;
   a.vis_cu = ws_at<int32_t>(ws, p.vis_cu);
-  a.img_req = ws_at<int32_t>(ws, p.img_req);
   a.text_idx = ws_at<int32_t>(ws, p.text_idx);
   a.text_cu = ws_at<int32_t>(ws, p.text_cu);
-  a.qtile_cu = ws_at<int32_t>(ws, p.qtile_cu);
-  a.p1_cu = ws_at<int32_t>(ws, p.p1_cu);
+  a.blk_cu = ws_at<int32_t>(ws, p.blk_cu);
+  a.p1s_cu = ws_at<int32_t>(ws, p.p1s_cu);
+  a.p2t_cu = ws_at<int32_t>(ws, p.p2t_cu);
   a.ktile_cu = ws_at<int32_t>(ws, p.ktile_cu);
-  a.lse_rows = ws_at<float>(ws, p.lse_rows);
+  a.meta = ws_at<int32_t>(ws, p.meta);
+  float* lse_rows = sa.lse != nullptr ? ws_at<float>(ws, p.lse_rows) : nullptr;
+  a.lse_rows = lse_rows;
   a.p1_part = sa.lse == nullptr ? ws_at<float2>(ws, p.p1_part) : nullptr;
-  a.partial = ws_at<float>(ws, p.partial);
+  a.mass = ws_at<unsigned long long>(ws, p.mass);
   a.rows = plan.rows;
-  a.p1_items_max = plan.p1_items_max;
   a.G = plan.G;
   a.Hkv = Hkv;
   a.d = d;
-  a.chunk_keys = plan.chunk_keys;
   a.c2 = sa.softmax_scale * kLog2e;
   a.st = st;
   __nv_bfloat16* qt = ws_at<__nv_bfloat16>(ws, p.qt);
@@ -580,37 +824,34 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   if (!make_map(&mk128, sa.k, d, Hkv, L.n_tokens, static_cast<uint64_t>(d) * 2, ks, 1, kM) ||
       !make_map(&mk256, sa.k, d, Hkv, L.n_tokens, static_cast<uint64_t>(d) * 2, ks, 1, kN) ||
       !make_map(&mq128, qt, d, plan.rows, Hkv, static_cast<uint64_t>(d) * 2, qs, kM, 1) ||
-      !make_map(&mq256, qt, d, plan.rows, Hkv, static_cast<uint64_t>(d) * 2, qs, kN, 1))
+      !make_map(&mq256, qt, d, plan.rows, Hkv, static_cast<uint64_t>(d) * 2, qs, kBlk, 1))
     return cudaErrorInvalidValue;
 
-  const int sms = device_sm_count();
+  const int sms = plan.grid;
   {
     const int64_t want = (plan.max_text * Hq * (d / 8) + 255) / 256;
     const int64_t cap = static_cast<int64_t>(sms) * 8;
     const int grid = static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
     cudaError_t e = launch_kernel(k_attn_pack, dim3(grid), dim3(256), 0, s, /*pdl=*/true,
                                   static_cast<const __nv_bfloat16*>(sa.q), sa.q_stride, Hq, plan.G, d, a.text_idx,
-                                  a.text_cu, L.n_requests, plan.rows, qt, sa.lse, sa.lse_stride, a.lse_rows,
-                                  static_cast<const DevStatus*>(st));
+                                  a.text_cu, L.n_requests, plan.rows, qt, sa.lse, sa.lse_stride, lse_rows, a.mass,
+                                  plan.n_ktiles_max * kM, static_cast<const DevStatus*>(st));
     if (e != cudaSuccess) return e;
   }
   if (sa.lse == nullptr) {
-    cudaError_t e = launch_kernel(k_attn_tc<1>, dim3(sms), dim3(kThreads), smem, s, /*pdl=*/true, mq128, mk256, a);
-    if (e != cudaSuccess) return e;
-    const int64_t rows_max = static_cast<int64_t>(Hkv) * plan.n_qtiles_max * kM;
-    const int64_t cap = static_cast<int64_t>(sms) * 4;
-    const int64_t want = (rows_max + 255) / 256;
-    e = launch_kernel(k_attn_merge, dim3(static_cast<unsigned>(want < cap ? want : cap)), dim3(256), 0, s,
-                      /*pdl=*/true, a);
+    cudaError_t e = launch_kernel(k_attn_lse, dim3(sms), dim3(kThreads), lse_smem_bytes(d), s, /*pdl=*/true, mq128,
+                                  mk256, a);
     if (e != cudaSuccess) return e;
   }
-  cudaError_t e = launch_kernel(k_attn_tc<2>, dim3(sms), dim3(kThreads), smem, s, /*pdl=*/true, mk128, mq256, a);
+  cudaError_t e =
+      launch_kernel(k_attn_mass, dim3(sms), dim3(kThreads), mass_smem_bytes(d), s, /*pdl=*/true, mk128, mq256, a);
   if (e != cudaSuccess) return e;
   const int64_t want = (L.n_tokens + 255) / 256;
   const int64_t cap = static_cast<int64_t>(sms) * 8;
   const int grid3 = static_cast<int>(want < cap ? want : cap);
-  return launch_kernel(k_attn_finalize, dim3(grid3), dim3(256), 0, s, /*pdl=*/true, a.partial, Hq, Hkv, L.n_tokens,
-                       L.cu_seqlens, L.img_start, a.vis_cu, a.img_req, a.text_cu, L.n_images, scores, img_sums,
+  return launch_kernel(k_attn_finalize, dim3(grid3), dim3(256), 0, s, /*pdl=*/true,
+                       static_cast<const unsigned long long*>(a.mass), a.ktile_cu, Hq, L.cu_seqlens, L.img_start, a.vis_cu,
+                       ws_at<int32_t>(ws, p.img_req), a.text_cu, L.n_images, scores, img_sums,
                        static_cast<const DevStatus*>(st));
 }
 
