@@ -191,7 +191,7 @@ def stage_roofline(acct, ms_step, hbm_gbs, bf16_tflops, peak_kind):
     return out
 
 
-def stage_accounting(wl, criterion, n_kept):
+def stage_accounting(wl, criterion, n_kept, lse=False):
     lay = wl.layout
     n_vis = int(lay.n_visual_per_request().sum())
     n_txt = lay.n_tokens - n_vis
@@ -205,7 +205,10 @@ def stage_accounting(wl, criterion, n_kept):
         flops = 0
     else:
         Hq, Hkv, d = wl.n_q_heads, wl.n_kv_heads, wl.head_dim
-        score_bytes = lay.n_tokens * Hkv * d * 2 + n_txt * Hq * d * 2
+        if lse:  # supplied LSE: visual keys, text queries and the text rows' LSE only
+            score_bytes = n_vis * Hkv * d * 2 + n_txt * Hq * d * 2 + n_txt * Hq * 4
+        else:
+            score_bytes = lay.n_tokens * Hkv * d * 2 + n_txt * Hq * d * 2
         stage_bytes = score_bytes + n_txt * D * 2 + n_kept * D * 2 + n_kept * pos_bytes * 2
         flops = 0
         vis = lay.visual_mask()
@@ -215,7 +218,8 @@ def stage_accounting(wl, criterion, n_kept):
             text_pos = np.nonzero(~v)[0]
             vis_prefix = np.concatenate([[0], np.cumsum(v)])
             for p in text_pos:
-                flops += 2 * Hq * d * (p + 1)              # pass 1: every visible key
+                if not lse:
+                    flops += 2 * Hq * d * (p + 1)          # pass 1: every visible key
                 flops += 2 * Hq * d * int(vis_prefix[p + 1])  # pass 2: visible visual keys
     return {"n_vis": n_vis, "n_txt": n_txt, "score_bytes": int(score_bytes), "stage_bytes": int(stage_bytes),
             "gather_bytes": int(gather), "flops": int(flops)}
@@ -294,9 +298,13 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     # the other scoring criterion (text-to-visual attention), timed the same way on the
     # same workload, for a secondary object of the line
-    sec = None
+    sec = sec_lse = None
     if second is not None:
         sec = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev)
+        lse = fa_lse(wl, bf16(wl.q), bf16(wl.k), torch)
+        torch.cuda.synchronize()
+        sec_lse = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev, lse=lse)
+        del lse
     clocks = sampler.stop() if sampler else None
     barrier(world)
     step_ms = [a.elapsed_time(b) for a, b in outer]
@@ -345,35 +353,65 @@ def run_ours(args, world, rank, local):
         "stage_roofline": stage_roofline(acct, ms_step, hbm, bf16_tf, peak_kind),
         "roofline": roof,
         "e2e": e2e,
-        "gpu_launches": K * (4 if crit == "hidden_variation" else 8),
+        "gpu_launches": K * (4 if crit == "hidden_variation" else 7),
         "clocks": clocks,
     }
-    if sec is not None:
-        hbm_s, bf16_s, _ = measured_peaks()
-        ms2 = sec["ms_per_step"]
-        line["text_attention"] = {
-            "criterion": "text_attention", "value": round(sec["acct"]["n_vis"] / (ms2 * 1e-3), 1), "unit": UNIT,
-            "ms_per_step": round(ms2, 5), "steps": sec["steps"], "latency_us": sec["latency_us"],
-            "steps_us": sec["steps_us"],
-            "stage_roofline": stage_roofline(sec["acct"], ms2, hbm_s, bf16_s, peak_kind),
-            "score_roofline": {"bound": "tensor", "kernel": "score (pack + lse + merge + mass + finalize)",
-                               "achieved": round(sec["acct"]["flops"] / (sec["steps_us"]["score"] * 1e-6) / 1e12, 2),
+    hbm_s, bf16_s, _ = measured_peaks()
+    for key, res, label in (("text_attention", sec, "score (pack + lse + mass + finalize)"),
+                            ("text_attention_lse", sec_lse, "score with a supplied LSE (pack + mass + finalize)")):
+        if res is None:
+            continue
+        ms2 = res["ms_per_step"]
+        score_us = res["steps_us"]["score"]
+        line[key] = {
+            "criterion": "text_attention", "lse": "supplied" if key.endswith("lse") else "computed",
+            "value": round(res["acct"]["n_vis"] / (ms2 * 1e-3), 1), "unit": UNIT,
+            "ms_per_step": round(ms2, 5), "steps": res["steps"], "latency_us": res["latency_us"],
+            "steps_us": res["steps_us"],
+            "stage_roofline": stage_roofline(res["acct"], ms2, hbm_s, bf16_s, peak_kind),
+            "score_roofline": {"bound": "tensor", "kernel": label,
+                               "achieved": round(res["acct"]["flops"] / (score_us * 1e-6) / 1e12, 2),
                                "peak": bf16_s, "unit": "TFLOP/s",
-                               "frac": round(sec["acct"]["flops"] / (sec["steps_us"]["score"] * 1e-6) / 1e12 / bf16_s, 4),
-                               "algorithmic_flops_per_launch": sec["acct"]["flops"]},
-            "gpu_launches": sec["launches"]}
-        line["gpu_launches"] += sec["launches"]
+                               "frac": round(res["acct"]["flops"] / (score_us * 1e-6) / 1e12 / bf16_s, 4),
+                               "algorithmic_flops_per_launch": res["acct"]["flops"]},
+            "gpu_launches": res["launches"]}
+        line["gpu_launches"] += res["launches"]
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, crit, args.cpu_seconds)
     return line
 
 
-def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev):
+def fa_lse(wl, q, k, torch):
+    """Natural-log LSE of every (head, text query) over its causally visible keys, [Hq, T] fp32.
+
+    This stands in for the normaliser a FlashAttention forward of the pruning layer
+    keeps; it is an input of the stage in that mode, computed here once with plain
+    torch before any timing."""
+    lay = wl.layout
+    Hq, Hkv = wl.n_q_heads, wl.n_kv_heads
+    G = Hq // Hkv
+    out = torch.zeros(Hq, lay.n_tokens, dtype=torch.float32, device=q.device)
+    vis = lay.visual_mask()
+    for r in range(lay.n_requests):
+        a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+        tp = torch.from_numpy(np.nonzero(~vis[a:b])[0]).to(q.device)
+        if tp.numel() == 0:
+            continue
+        keys = torch.arange(b - a, device=q.device)
+        mask = keys[None, :] > tp[:, None]
+        for h in range(Hq):
+            z = (q[a + tp, h].float() @ k[a:b, h // G].float().T) * wl.softmax_scale
+            out[h, a + tp] = torch.logsumexp(z.masked_fill(mask, float("-inf")), dim=1)
+    return out
+
+
+def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev, lse=None):
     """The attention criterion on the same workload: whole-call latency and per-step times."""
     crit = "text_attention"
+    extra = {} if lse is None else {"lse": lse}
     call = avtp.PruneCall(L, crit, keep_ratio=kr, keep_ratio_host=wl.keep_ratio, rows={"hidden": h_cur},
-                          planes={"pos": pos}, q=bf16(wl.q), k=bf16(wl.k), softmax_scale=wl.softmax_scale)
-    acct = stage_accounting(wl, crit, call.buffers.n_kept)
+                          planes={"pos": pos}, q=bf16(wl.q), k=bf16(wl.k), softmax_scale=wl.softmax_scale, **extra)
+    acct = stage_accounting(wl, crit, call.buffers.n_kept, lse=lse is not None)
     K = max(10, min(args.steps, 300))
     n_ev = avtp.N_STEP_EVENTS
     outer = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
@@ -408,7 +446,7 @@ def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp
             "latency_us": {"p50": round(step_ms[len(step_ms) // 2] * 1e3, 2),
                            "p90": round(step_ms[int(len(step_ms) * 0.9)] * 1e3, 2)},
             "steps_us": {k: round(v * 1e3, 2) for k, v in per_step.items()},
-            "launches": K * (8 if call._sa.lse is None else 6)}
+            "launches": K * (7 if lse is None else 6)}
 
 
 def run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp):
