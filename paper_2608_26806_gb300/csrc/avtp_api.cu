@@ -128,6 +128,7 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
     p.p1s_cu = take((static_cast<size_t>(a.n_blocks_max) + 1) * 4);
     p.p2t_cu = take((static_cast<size_t>(a.n_blocks_max) + 1) * 4);
     p.ktile_cu = take((NI + 1) * 4);
+    p.ktile_img = take(static_cast<size_t>(a.n_ktiles_max) * 4);
     p.meta = take(8 * 4);
     p.qt = take(Hkv * rows * static_cast<size_t>(sa->head_dim) * 2 + 16);
     p.lse_rows = (sa->lse != nullptr) ? take(Hkv * rows * 4 + 4) : 0;

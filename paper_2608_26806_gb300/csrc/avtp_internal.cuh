@@ -61,6 +61,7 @@ struct WsPlan {
   size_t p1s_cu;      // int32 [n_blocks_max + 1]: pass-1 key steps per row block
   size_t p2t_cu;      // int32 [n_blocks_max + 1]: pass-2 key tiles per row block
   size_t ktile_cu;    // int32 [n_img + 1]: key tiles per image
+  size_t ktile_img;   // int32 [n_ktiles_max]: image of every key tile
   size_t meta;        // int32 [8]: F1, C1, F2, C2 (flat pass lengths per KV group, steps per CTA)
   size_t qt;          // bf16 [Hkv, rows, d]: the text queries, packed by KV group
   size_t lse_rows;    // float [Hkv, rows]: log2-domain LSE of every row (supplied LSE only)

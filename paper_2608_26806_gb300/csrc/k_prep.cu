@@ -57,7 +57,8 @@ constexpr int kStageInts = 2560;
 
 __global__ void __launch_bounds__(kPrepThreads)
 k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t* req_budget, int32_t* text_idx,
-       int32_t* text_cu, int32_t* blk_cu, int32_t* p1s_cu, int32_t* p2t_cu, int32_t* ktile_cu, int32_t* meta) {
+       int32_t* text_cu, int32_t* blk_cu, int32_t* p1s_cu, int32_t* p2t_cu, int32_t* ktile_cu, int32_t* ktile_img,
+       int32_t* meta) {
   __shared__ int s_err, s_detail, s_max_steps;
   __shared__ int32_t s_warp[32];
   __shared__ int32_t s_stage[kStageInts];
@@ -198,6 +199,8 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
       // Key tiles of kAttnTileM visual keys per image.
       block_exclusive_scan<int32_t>(
           NI, [&](int i) { return (iln[i] + kAttnTileM - 1) / kAttnTileM; }, ktile_cu, s_warp);
+      for (int i = tid; i < NI; i += blockDim.x)
+        for (int t = ktile_cu[i]; t < ktile_cu[i + 1]; ++t) ktile_img[t] = i;
       // Pass 2 of block b: the key tiles of every image that at least one of the block's
       // queries follows. Images are sorted and the text ordinal of the first token after
       // image i, o_first(i), does not decrease with i, so those images are a prefix.
@@ -275,6 +278,7 @@ cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream
                                     b ? ws_at<int32_t>(ws, p.p1s_cu) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.p2t_cu) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr,
+                                    b ? ws_at<int32_t>(ws, p.ktile_img) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.meta) : nullptr);
   return cudaGetLastError();
 }

@@ -712,36 +712,48 @@ k_attn_pack(const __nv_bfloat16* __restrict__ q, int64_t q_stride, int Hq, int G
 }
 
 // ---------------------------------------------------------------- finalize
-// s_t = mass_t * 2^-40 / (Hq * |Q_r|) for every visual token, and the fixed-point image sums.
-__global__ void __launch_bounds__(256)
-k_attn_finalize(const unsigned long long* __restrict__ mass, const int32_t* __restrict__ ktile_cu, int Hq,
-                const int32_t* __restrict__ cu,
-                const int32_t* __restrict__ img_start, const int32_t* __restrict__ vis_cu,
+// One CTA per key tile (128 keys of one image): s_t = mass_t * 2^-40 / (Hq * |Q_r|), and
+// the tile's fixed-point score sum added to its image's sum with one atomic.
+__global__ void __launch_bounds__(kM)
+k_attn_finalize(const unsigned long long* __restrict__ mass, const int32_t* __restrict__ ktile_cu,
+                const int32_t* __restrict__ ktile_img, int Hq, const int32_t* __restrict__ cu,
+                const int32_t* __restrict__ img_start, const int32_t* __restrict__ img_len,
                 const int32_t* __restrict__ img_req, const int32_t* __restrict__ text_cu, int NI,
                 float* __restrict__ scores, int64_t* __restrict__ img_sums, const DevStatus* st) {
+  __shared__ long long s_part[kM / 32];
   pdl_wait();
   pdl_trigger();
   if (!st->layout_ok) return;
-  const int n_vis = vis_cu[NI];
-  for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < n_vis;
-       v += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int i = upper_index(vis_cu, NI, v);
+  for (int tile = blockIdx.x; tile < ktile_cu[NI]; tile += gridDim.x) {
+    const int i = ktile_img[tile];
     const int r = img_req[i];
-    const int o = static_cast<int>(v - vis_cu[i]);  // key within the image
-    const int64_t t = static_cast<int64_t>(cu[r]) + img_start[i] + o;
+    const int o = (tile - ktile_cu[i]) * kM + static_cast<int>(threadIdx.x);  // key within the image
     const int nq = text_cu[r + 1] - text_cu[r];
-    float s = 0.f;
-    if (nq > 0) {
-      const unsigned long long m = mass[static_cast<int64_t>(ktile_cu[i] + o / kM) * kM + o % kM];
-      if (m & kMassNotFinite) {
-        s = __int_as_float(0x7fc00000);
-      } else {
-        s = __ll2float_rn(static_cast<long long>(m)) * (1.0f / static_cast<float>(1ull << kAttnMassFracBits));
-        s = s / static_cast<float>(static_cast<int64_t>(Hq) * nq);
+    const unsigned long long m = mass[static_cast<int64_t>(tile) * kM + threadIdx.x];
+    long long fx = 0;
+    if (o < img_len[i]) {
+      float s = 0.f;
+      if (nq > 0) {
+        if (m & kMassNotFinite) {
+          s = __int_as_float(0x7fc00000);
+        } else {
+          s = __ll2float_rn(static_cast<long long>(m)) * (1.0f / static_cast<float>(1ull << kAttnMassFracBits));
+          s = s / static_cast<float>(static_cast<int64_t>(Hq) * nq);
+        }
       }
+      scores[static_cast<int64_t>(cu[r]) + img_start[i] + o] = s;
+      fx = fixed_point_score(s);
     }
-    scores[t] = s;
-    atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + i), static_cast<unsigned long long>(fixed_point_score(s)));
+    fx = warp_sum(fx);
+    if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = fx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      long long sum = 0;
+#pragma unroll
+      for (int w = 0; w < kM / 32; ++w) sum += s_part[w];
+      atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + i), static_cast<unsigned long long>(sum));
+    }
+    __syncthreads();
   }
 }
 
@@ -846,13 +858,13 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   cudaError_t e =
       launch_kernel(k_attn_mass, dim3(sms), dim3(kThreads), mass_smem_bytes(d), s, /*pdl=*/true, mk128, mq256, a);
   if (e != cudaSuccess) return e;
-  const int64_t want = (L.n_tokens + 255) / 256;
   const int64_t cap = static_cast<int64_t>(sms) * 8;
-  const int grid3 = static_cast<int>(want < cap ? want : cap);
-  return launch_kernel(k_attn_finalize, dim3(grid3), dim3(256), 0, s, /*pdl=*/true,
-                       static_cast<const unsigned long long*>(a.mass), a.ktile_cu, Hq, L.cu_seqlens, L.img_start, a.vis_cu,
-                       ws_at<int32_t>(ws, p.img_req), a.text_cu, L.n_images, scores, img_sums,
-                       static_cast<const DevStatus*>(st));
+  const int grid3 = static_cast<int>(plan.n_ktiles_max < cap ? plan.n_ktiles_max : cap);
+  return launch_kernel(k_attn_finalize, dim3(grid3), dim3(kM), 0, s, /*pdl=*/true,
+                       static_cast<const unsigned long long*>(a.mass), a.ktile_cu,
+                       static_cast<const int32_t*>(ws_at<int32_t>(ws, p.ktile_img)), Hq, L.cu_seqlens, L.img_start,
+                       L.img_len, static_cast<const int32_t*>(ws_at<int32_t>(ws, p.img_req)), a.text_cu, L.n_images,
+                       scores, img_sums, static_cast<const DevStatus*>(st));
 }
 
 }  // namespace avtp
