@@ -10,25 +10,24 @@
 //
 // Pass 1, k_attn_lse (skipped when the caller supplies FlashAttention's LSE): a block
 // is held as two 128-row A tiles and every key tile of 256 keys, from the request's
-// first token to the block's last query, feeds two MMAs (128 x 256 x d each, one per
-// A tile, fp32 accumulators in TMEM). Each A tile has its own accumulator and its own
-// four epilogue warps, so one tile's epilogue overlaps the other tile's MMA and every
-// key byte brought to the SM serves 256 rows. The epilogue keeps an online (max, sum)
-// per row and leaves one partial per (row, CTA) behind.
+// first token to the block's last query, feeds two MMAs (128 x 256 x d, one per A
+// tile, fp32 accumulators in TMEM), so every key byte brought to the SM serves 256
+// rows. The epilogue reads accumulator 0 while the MMA of tile 1 runs and keeps an
+// online (max, sum) per row; it leaves one partial per (row, CTA) behind.
 // Pass 2, k_attn_mass: a block is held as the MMA B operand (N = 256 rows) and the
 // tiles of 128 visual keys of every image that one of its queries follows stream
-// through it as A (M = 128 keys); the two accumulators alternate between the two
-// epilogue groups. A thread owns one key and sums exp2(z2 - lse2) over the block's
-// rows that see the key; lse2 comes from the pass-1 partials of the block (merged on
-// load) or from the supplied LSE. The per-key sums of all blocks and KV groups meet in
-// a 64-bit fixed-point accumulator (integer atomics: the result does not depend on
-// their order).
+// through it as A (M = 128 keys), into two accumulators used in turn. A thread owns
+// one key and sums exp2(z2 - lse2) over the rows of its column half; lse2 comes from
+// the pass-1 partials of the block (merged on load) or from the supplied LSE, and is
+// +inf on rows whose query precedes the key's image. The per-key sums of all blocks
+// and KV groups meet in a 64-bit fixed-point accumulator (integer atomics: the result
+// does not depend on their order).
 // k_attn_finalize turns the accumulator into scores and the fixed-point image sums.
 //
 // Both passes are persistent: the flat list of (KV group, block, key step) is split
-// into equal contiguous runs, one per CTA (one CTA per SM). Warps 0-3 and 4-7 are the
-// two epilogue groups (warp w reads TMEM lanes 32(w%4)..+31 of accumulator w/4), warp 8
-// issues the TMA loads, warp 9 owns TMEM and issues the MMAs. TMEM holds the two
+// into equal contiguous runs, one per CTA (one CTA per SM). Warps 0-7 are the epilogue
+// (warp w reads TMEM lanes 32(w%4)..+31 and column half w/4 of every accumulator),
+// warp 8 issues the TMA loads, warp 9 owns TMEM and issues the MMAs. TMEM holds two
 // 256-column accumulators.
 #include <cudaTypedefs.h>
 
