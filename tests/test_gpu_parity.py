@@ -70,6 +70,42 @@ def test_score_attention_with_supplied_lse(name):
     assert_scores_close(scores.cpu().numpy(), ref, wl.layout.visual_mask())
 
 
+# Layouts that stress the text-attention bookkeeping: row blocks of 256 (query, head)
+# rows that end mid-request or hold one row, requests without text or without images,
+# text only before the images, adjacent images, images of 1 and of 129 tokens, and
+# several blocks and key steps per request.
+_ATTN_EDGE_LAYOUTS = [
+    [[("i", 40), ("t", 3), ("i", 300), ("t", 100)], [("t", 5)], [("i", 17)],
+     [("t", 70), ("i", 129), ("i", 1), ("t", 1)]],
+    [[("t", 1), ("i", 256), ("t", 1)], [("i", 5), ("t", 200), ("i", 300), ("t", 9)]],
+    [[("t", 65), ("i", 10), ("t", 64), ("i", 7), ("t", 1)], [("t", 30), ("i", 600)]],
+    [[("t", 300), ("i", 513), ("t", 2), ("i", 700), ("t", 140)]],
+]
+
+
+@pytest.mark.parametrize("layout_id", range(len(_ATTN_EDGE_LAYOUTS)))
+@pytest.mark.parametrize("heads", [(4, 4, 64), (6, 2, 64), (12, 4, 128), (7, 1, 128)])
+@pytest.mark.parametrize("supplied_lse", [False, True])
+def test_score_attention_edge_layouts(layout_id, heads, supplied_lse):
+    Hq, Hkv, d = heads
+    wl = synth.make_custom(_ATTN_EDGE_LAYOUTS[layout_id], n_q_heads=Hq, n_kv_heads=Hkv, head_dim=d, hidden=64,
+                           seed=11 + layout_id, parts=("B",))
+    dw = DevWorkload(wl)
+    kw = {}
+    ref_lse = None
+    if supplied_lse:
+        lse = O.text_lse(wl.layout, wl.q, wl.k, Hq, Hkv, wl.softmax_scale)
+        kw["lse"] = torch.from_numpy(lse.astype(np.float32)).cuda()
+        ref_lse = lse.astype(np.float32).astype(np.float64)
+    scores, sums = avtp.score(dw.L, "text_attention", **kw, **dw.score_tensors("text_attention"))
+    torch.cuda.synchronize()
+    got = scores.cpu().numpy()
+    ref = O.score_text_attention(wl.layout, wl.q, wl.k, Hq, Hkv, wl.softmax_scale, lse=ref_lse)
+    vis = wl.layout.visual_mask()
+    assert_scores_close(got, ref, vis)
+    assert np.array_equal(sums.cpu().numpy(), O.image_sums(wl.layout, got))
+
+
 # ---------------------------------------------------------------- step 2
 @pytest.mark.parametrize("name", CONFIGS)
 @pytest.mark.parametrize("relative", [False, True])
