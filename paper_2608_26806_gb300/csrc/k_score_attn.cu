@@ -145,21 +145,31 @@ struct FlatCursor {
 };
 
 // Pass-2 key tiles of a block in order: tile j is tile jj of image i, the images of the
-// block's request in order. Image data is read when the walk enters a new image.
+// block's request in order. The request's fields are read when the walk enters a block;
+// the next image's fields are loaded as soon as the walk enters an image, so that their
+// latency is hidden behind the steps of the current image.
 struct TileCursor {
   int i, jj;           // image, tile within the image
   int kp0, nk, c0;     // first packed key, keys in the tile, first row of the block that sees it
   int tile;            // key tile over all images (row of the mass accumulator)
   int base, len, t0;   // packed position of the image's first key, its length, its first key tile
   int64_t c0_img;      // o_first(i) * G - R0
-  __device__ __forceinline__ void load_image(const AttnArgs& a, const Seg& s) {
-    const int r = s.r;
-    base = a.cu[r] + a.ist[i];
-    len = a.iln[i];
-    t0 = a.ktile_cu[i];
-    const int64_t o_first =
-        static_cast<int64_t>(a.text_cu[r]) + a.ist[i] + len - (a.vis_cu[i + 1] - a.vis_cu[a.icu[r]]);
-    c0_img = o_first * a.G - s.R0;
+  int cu_r, text_r, vis_r0, img_end;  // the request's first token, first text ordinal, first visual ordinal, image end
+  int n_ist, n_iln, n_t0, n_vis;      // image i + 1: start, length, first key tile, visual prefix after it
+  __device__ __forceinline__ void prefetch(const AttnArgs& a) {
+    if (i + 1 < img_end) {
+      n_ist = a.ist[i + 1];
+      n_iln = a.iln[i + 1];
+      n_t0 = a.ktile_cu[i + 1];
+      n_vis = a.vis_cu[i + 2];
+    }
+  }
+  __device__ __forceinline__ void apply(const Seg& s, int g, int ist, int iln, int tk0, int vis1) {
+    base = cu_r + ist;
+    len = iln;
+    t0 = tk0;
+    const int64_t o_first = static_cast<int64_t>(text_r) + ist + iln - (vis1 - vis_r0);
+    c0_img = o_first * g - s.R0;
   }
   __device__ __forceinline__ void fill() {
     kp0 = base + jj * kM;
@@ -168,17 +178,24 @@ struct TileCursor {
     c0 = c0_img > 0 ? static_cast<int>(c0_img) : 0;
   }
   __device__ __forceinline__ void init(const AttnArgs& a, const Seg& s, int j) {
-    const int tile = a.ktile_cu[a.icu[s.r]] + j;
-    i = upper_index(a.ktile_cu, a.NI, tile);
-    jj = tile - a.ktile_cu[i];
-    load_image(a, s);
+    const int r = s.r;
+    cu_r = a.cu[r];
+    text_r = a.text_cu[r];
+    vis_r0 = a.vis_cu[a.icu[r]];
+    img_end = a.icu[r + 1];
+    const int t = a.ktile_cu[a.icu[r]] + j;
+    i = upper_index(a.ktile_cu, a.NI, t);
+    jj = t - a.ktile_cu[i];
+    apply(s, a.G, a.ist[i], a.iln[i], a.ktile_cu[i], a.vis_cu[i + 1]);
+    prefetch(a);
     fill();
   }
   __device__ __forceinline__ void next(const AttnArgs& a, const Seg& s) {
     if ((++jj) * kM >= len) {
       ++i;
       jj = 0;
-      load_image(a, s);
+      apply(s, a.G, n_ist, n_iln, n_t0, n_vis);
+      prefetch(a);
     }
     fill();
   }
