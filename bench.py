@@ -298,13 +298,14 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     # the other scoring criterion (text-to-visual attention), timed the same way on the
     # same workload, for a secondary object of the line
-    sec = sec_lse = None
+    sec = sec_lse = prog = None
     if second is not None:
         sec = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev)
         lse = fa_lse(wl, bf16(wl.q), bf16(wl.k), torch)
         torch.cuda.synchronize()
         sec_lse = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev, lse=lse)
         del lse
+        prog = time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avtp, world, dev)
     clocks = sampler.stop() if sampler else None
     barrier(world)
     step_ms = [a.elapsed_time(b) for a, b in outer]
@@ -376,6 +377,9 @@ def run_ours(args, world, rank, local):
                                "algorithmic_flops_per_launch": res["acct"]["flops"]},
             "gpu_launches": res["launches"]}
         line["gpu_launches"] += res["launches"]
+    if prog is not None:
+        line["progressive"] = prog
+        line["gpu_launches"] += prog["gpu_launches"]
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, crit, args.cpu_seconds)
     return line
@@ -447,6 +451,78 @@ def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp
                            "p90": round(step_ms[int(len(step_ms) * 0.9)] * 1e3, 2)},
             "steps_us": {k: round(v * 1e3, 2) for k, v in per_step.items()},
             "launches": K * (7 if lse is None else 6)}
+
+
+def time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avtp, world, dev, stages=3):
+    """Progressive pruning (paper §3.3.2): the stage three times on a shrinking batch.
+
+    Each step prunes with criterion A at a per-stage keep ratio of 0.5^(1/3) (half of the
+    visual tokens survive the three stages). After each stage the next layout is built
+    on the device (avtp_pruned_layout) and the compacted h_cur becomes the next h_prior;
+    the next layer's hidden states are fixed synthetic inputs of the shrunk size."""
+    ratio = np.full(wl.layout.n_requests, np.float32(0.5 ** (1.0 / 3.0)), dtype=np.float32)
+    kr = torch.from_numpy(ratio).to(dev)
+    calls, layouts, bytes_total = [], [], 0
+    cur_L, cur_cur, cur_prior, cur_pos = L, h_cur, h_prior, pos
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(7)
+    for s_i in range(stages):
+        call = avtp.PruneCall(cur_L, "hidden_variation", keep_ratio=kr, keep_ratio_host=ratio, h_cur=cur_cur,
+                              h_prior=cur_prior, rows={"hidden": cur_cur}, planes={"pos": cur_pos})
+        n_vis = int(cur_L.n_vis_per_request.astype(np.int64).sum())
+        n_txt = cur_L.n_tokens - n_vis
+        D = cur_cur.shape[1]
+        bytes_total += 2 * n_vis * D * 2 + n_txt * D * 2 + call.buffers.n_kept * (D * 2 + cur_pos.shape[0] * 4 * 2)
+        calls.append(call)
+        call.run(stream)
+        if s_i + 1 < stages:
+            ws = avtp.new_workspace(avtp.workspace_size(cur_L), dev)
+            nxt = avtp.pruned_layout(cur_L, ratio, call.buffers.budgets, call.buffers.out_cu_seqlens, workspace=ws,
+                                     stream=stream)
+            layouts.append((cur_L, call, nxt, ws))
+            cur_prior = call.buffers.outputs["hidden"]
+            cur_cur = (cur_prior.float() + 0.5 * torch.randn(cur_prior.shape, generator=gen, device=dev)).to(torch.bfloat16)
+            cur_pos = call.buffers.outputs["pos"]
+            cur_L = nxt
+    torch.cuda.synchronize()
+
+    def step():
+        for s_i, call in enumerate(calls):
+            call.run(stream)
+            if s_i + 1 < stages:
+                prev_L, prev_call, nxt, ws = layouts[s_i]
+                avtp.pruned_layout(prev_L, ratio, prev_call.buffers.budgets, prev_call.buffers.out_cu_seqlens,
+                                   workspace=ws, stream=stream, into=nxt)
+
+    K = max(10, min(args.steps, 300))
+    for _ in range(max(3, args.warmup)):
+        flush()
+        step()
+    torch.cuda.synchronize()
+    for c in calls:
+        st = avtp.read_device_status(c.buffers.workspace)
+        if st != avtp.OK:
+            raise RuntimeError(f"device status after warm-up (progressive): {avtp.status_string(st)}")
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    barrier(world)
+    torch.cuda.synchronize()
+    for i in range(K):
+        flush()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    ms = sorted(a.elapsed_time(b) for a, b in ev)
+    p50 = ms[len(ms) // 2]
+    hbm, _, peak_kind = measured_peaks()
+    bound_us = bytes_total / (hbm * 1e9) * 1e6
+    return {"stages": stages, "keep_ratio_per_stage": round(float(ratio[0]), 6), "criterion": "hidden_variation",
+            "visual_tokens": [int(c.layout.n_vis_per_request.astype(np.int64).sum()) for c in calls],
+            "tokens": [int(c.layout.n_tokens) for c in calls], "steps": K,
+            "latency_us": {"p50": round(p50 * 1e3, 2), "p90": round(ms[int(len(ms) * 0.9)] * 1e3, 2)},
+            "stage_roofline": {"bound": "hbm", "algorithmic_bytes": int(bytes_total), "bound_us": round(bound_us, 2),
+                               "frac": round(bound_us / (p50 * 1e3), 4), "peak_gbs": hbm, "peak_kind": peak_kind},
+            "gpu_launches": K * (4 * stages + 2 * (stages - 1))}
 
 
 def run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp):

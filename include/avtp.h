@@ -241,6 +241,32 @@ AVTP_API avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_
 AVTP_API int64_t avtp_kept_count_host(const int32_t* cu_seqlens, const int32_t* img_cu, const int32_t* img_len,
                              const float* keep_ratio, int32_t n_requests);
 
+/* The layout of the batch avtp_prune produced, for running the stage again at a later
+ * layer (the progressive schedule of paper §3.3.2, where the compacted hidden states of
+ * this pruning point are the next one's h_prior, §3.3.1). Requests and their images
+ * stay; image i of request r starts at img_start[i] - sum_{j<i in r} (img_len[j] -
+ * budgets[j]) and holds budgets[i] tokens. Writes out_img_start and out_img_len
+ * (device int32 [n_images]); the pruned layout is then {n_requests, n_images,
+ * n_tokens = n_kept, cu_seqlens = out_cu_seqlens of avtp_prune, the same img_cu,
+ * out_img_start, out_img_len}, all on the device, with no host round trip.
+ * budgets: device int32 [n_images] as written by avtp_prune or avtp_allocate; a
+ * budget outside [0, img_len] is recorded as AVTP_ERR_DEVICE_INPUT and its image gets
+ * an empty span. An image that kept no token gets an empty span, which the next
+ * stage's validation rejects (with the default clamps every image of 20 or more
+ * tokens keeps at least one). Asynchronous on `stream`. */
+AVTP_API avtp_status_t avtp_pruned_layout(const avtp_layout_t* layout, const int32_t* budgets, int32_t* out_img_start,
+                                          int32_t* out_img_len, void* workspace, size_t workspace_bytes,
+                                          avtp_stream_t stream);
+
+/* avtp_kept_count_host from per-request visual token counts (host int32 [R]), for a
+ * layout whose image lengths live on the device only, such as one from
+ * avtp_pruned_layout. Returns sum_r floor(keep_ratio[r]*n_vis[r] + 0.5) + N_txt,r, or -1
+ * for invalid arguments. Optionally (NULL to skip) writes the pruned batch's host
+ * offsets out_cu_seqlens [R+1] and its visual counts out_n_vis [R], which are the
+ * inputs of the same call for the next stage. */
+AVTP_API int64_t avtp_kept_count_vis_host(const int32_t* cu_seqlens, const int32_t* n_vis, const float* keep_ratio,
+                                          int32_t n_requests, int32_t* out_cu_seqlens, int32_t* out_n_vis);
+
 /* Waits for `stream`, then reads the workspace's device status word into *out
  * (an avtp_status_t value; AVTP_OK if no device-side error was recorded since the
  * last entry point reset it). */

@@ -24,6 +24,9 @@ Language Models", AVTP):
 3.  Per image, keep the ``k_i`` most important visual tokens; text is kept (§3.1,
     §3.3.3); the result is an order-preserving subsequence (§3.1).
 4.  Compaction: a row gather of the kept tokens (§3.1, ``E_pruned = p(E_v)``).
+5.  The layout of the pruned batch, on which the stage runs again at a later layer in
+    a progressive schedule (§3.3.2), with the compacted hidden states of this pruning
+    point as that layer's h_prior (§3.3.1).
 
 Readings of points the paper leaves open (each is also listed with its reason in
 the design notes of the repository):
@@ -436,6 +439,34 @@ def compact(kept_idx: np.ndarray, rows: np.ndarray) -> np.ndarray:
 def compact_planes(kept_idx: np.ndarray, planes: np.ndarray) -> np.ndarray:
     """Gather along the token axis of a [P, T] array (e.g. M-RoPE position ids)."""
     return np.asarray(planes)[:, np.asarray(kept_idx, dtype=np.int64)]
+
+
+# ----------------------------------------------------------------------------
+# Layout of the pruned batch (progressive pruning, paper §3.3.2: the stage runs again
+# at later layers on the shortened sequence, with the previous pruning point's hidden
+# states as h_prior, §3.3.1)
+# ----------------------------------------------------------------------------
+def pruned_layout(layout, kept_idx: np.ndarray, out_cu_seqlens: np.ndarray) -> Dict[str, np.ndarray]:
+    """Image spans of the pruned batch, read off the kept tokens.
+
+    In request r of the pruned batch, image i starts at the number of kept tokens of the
+    request that lie before the image's span, and holds the kept tokens inside the span
+    (its budget). Requests and their image lists are unchanged. Returns cu_seqlens,
+    img_cu, img_start and img_len (int32) of the pruned batch.
+    """
+    kept = np.asarray(kept_idx, dtype=np.int64)
+    cu2 = np.asarray(out_cu_seqlens, dtype=np.int64)
+    starts, lens = [], []
+    for r in range(len(layout.cu_seqlens) - 1):
+        a = int(layout.cu_seqlens[r])
+        local = kept[cu2[r]:cu2[r + 1]] - a  # request-local positions of the kept tokens
+        for i in range(int(layout.img_cu[r]), int(layout.img_cu[r + 1])):
+            s0 = int(layout.img_start[i])
+            s1 = s0 + int(layout.img_len[i])
+            starts.append(int(np.count_nonzero(local < s0)))
+            lens.append(int(np.count_nonzero((local >= s0) & (local < s1))))
+    return {"cu_seqlens": cu2.astype(np.int32), "img_cu": np.asarray(layout.img_cu, dtype=np.int32).copy(),
+            "img_start": np.asarray(starts, dtype=np.int32), "img_len": np.asarray(lens, dtype=np.int32)}
 
 
 # ----------------------------------------------------------------------------

@@ -87,6 +87,8 @@ SIGNATURES = {
     "avtp_select_noalloc": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_void_p,
                                     c_void_p]),
     "avtp_kept_count_host": (c_int64, [c_void_p, c_void_p, c_void_p, c_void_p, c_int32]),
+    "avtp_pruned_layout": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "avtp_kept_count_vis_host": (c_int64, [c_void_p, c_void_p, c_void_p, c_int32, c_void_p, c_void_p]),
     "avtp_read_device_status": (c_int, [c_void_p, c_void_p, POINTER(c_int32)]),
     "avtp_status_string": (ctypes.c_char_p, [c_int32]),
     "avtp_version": (c_int32, []),
@@ -139,7 +141,11 @@ def _stream(stream) -> int:
 # ---------------------------------------------------------------- layout
 @dataclass
 class Layout:
-    """A varlen-packed multi-image layout on the device (int32 tensors) plus host copies."""
+    """A varlen-packed multi-image layout on the device (int32 tensors) plus host copies.
+
+    A layout made by ``pruned_layout`` keeps its image spans on the device only: its
+    host copy holds cu_seqlens, img_cu and the visual tokens per request (``n_vis``).
+    """
     cu_seqlens: torch.Tensor
     img_cu: torch.Tensor
     img_start: torch.Tensor
@@ -159,15 +165,22 @@ class Layout:
 
     @property
     def n_images(self) -> int:
-        return int(self.host["img_len"].shape[0])
+        return int(self.host["img_cu"][-1])
 
     @property
     def n_tokens(self) -> int:
         return int(self.host["cu_seqlens"][-1])
 
     @property
+    def n_vis_per_request(self) -> np.ndarray:
+        if "n_vis" in self.host:
+            return self.host["n_vis"]
+        csum = np.concatenate([[0], np.cumsum(self.host["img_len"].astype(np.int64))])
+        return (csum[self.host["img_cu"][1:]] - csum[self.host["img_cu"][:-1]]).astype(np.int32)
+
+    @property
     def n_text(self) -> int:
-        return self.n_tokens - int(self.host["img_len"].astype(np.int64).sum())
+        return self.n_tokens - int(self.n_vis_per_request.astype(np.int64).sum())
 
     def c(self) -> _Layout:
         return _Layout(self.n_requests, self.n_images, self.n_tokens, _ptr(self.cu_seqlens), _ptr(self.img_cu),
@@ -312,8 +325,53 @@ def compact(kept_idx: torch.Tensor, n_tokens: int, rows: Sequence[Tuple[torch.Te
                                workspace.numel(), _stream(stream)), "avtp_compact")
 
 
+def kept_count_vis_host(cu_seqlens: np.ndarray, n_vis: np.ndarray, keep_ratio: np.ndarray):
+    """avtp_kept_count_vis_host: the pruned batch's size, host offsets and visual tokens per request."""
+    cu = np.ascontiguousarray(np.asarray(cu_seqlens, dtype=np.int32))
+    nv = np.ascontiguousarray(np.asarray(n_vis, dtype=np.int32))
+    kr = np.ascontiguousarray(np.asarray(keep_ratio, dtype=np.float32))
+    R = int(cu.shape[0] - 1)
+    out_cu = np.zeros(R + 1, dtype=np.int32)
+    out_nv = np.zeros(R, dtype=np.int32)
+    n = load().avtp_kept_count_vis_host(cu.ctypes.data, nv.ctypes.data, kr.ctypes.data, R, out_cu.ctypes.data,
+                                        out_nv.ctypes.data)
+    if n < 0:
+        raise AVTPError(ERR_INVALID_ARG, "avtp_kept_count_vis_host")
+    return int(n), out_cu, out_nv
+
+
+def pruned_layout(layout: Layout, keep_ratio_host: np.ndarray, budgets: torch.Tensor, out_cu_seqlens: torch.Tensor,
+                  workspace=None, stream=None, into: Optional[Layout] = None) -> Layout:
+    """avtp_pruned_layout: the layout of the batch that avtp_prune produced (device arrays).
+
+    ``budgets`` and ``out_cu_seqlens`` are the prune call's device outputs; they are
+    read on the device, so the pruned layout is usable in the same stream at once.
+    ``into``: a layout returned by an earlier call whose device arrays are rewritten.
+    """
+    dev = layout.cu_seqlens.device
+    NI = layout.n_images
+    if into is not None:
+        img_start, img_len = into.img_start, into.img_len
+    else:
+        img_start = torch.empty(max(NI, 1), dtype=torch.int32, device=dev)
+        img_len = torch.empty(max(NI, 1), dtype=torch.int32, device=dev)
+    if workspace is None:
+        workspace = new_workspace(workspace_size(layout), dev)
+    lay = layout.c()
+    _check(load().avtp_pruned_layout(ctypes.byref(lay), _ptr(budgets), _ptr(img_start), _ptr(img_len),
+                                     _ptr(workspace), workspace.numel(), _stream(stream)), "avtp_pruned_layout")
+    if into is not None:
+        return into
+    _, cu_host, nv_host = kept_count_vis_host(layout.host["cu_seqlens"], layout.n_vis_per_request, keep_ratio_host)
+    host = {"cu_seqlens": cu_host, "img_cu": layout.host["img_cu"].copy(), "n_vis": nv_host}
+    return Layout(cu_seqlens=out_cu_seqlens[:layout.n_requests + 1], img_cu=layout.img_cu, img_start=img_start[:NI],
+                  img_len=img_len[:NI], host=host)
+
+
 def kept_count_host(layout_host: Dict[str, np.ndarray], keep_ratio: np.ndarray) -> int:
     """avtp_kept_count_host: sum_r floor(r_base*N_vis + 0.5) + N_txt over requests."""
+    if "n_vis" in layout_host:  # a pruned layout: image lengths on the device only
+        return kept_count_vis_host(layout_host["cu_seqlens"], layout_host["n_vis"], keep_ratio)[0]
     h = {k: np.ascontiguousarray(np.asarray(layout_host[k], dtype=np.int32))
          for k in ("cu_seqlens", "img_cu", "img_len")}
     kr = np.ascontiguousarray(np.asarray(keep_ratio, dtype=np.float32))

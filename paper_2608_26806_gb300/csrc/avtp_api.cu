@@ -119,6 +119,7 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
   p.req_budget = take(R * 4);
   p.img_sums = take(NI * 8 + 8);
   p.scores = take(T * 4 + 4);
+  p.scratch = take((NI + 1) * 4);
   if (sa != nullptr && sa->criterion == AVTP_CRIT_TEXT_ATTENTION) {
     const AttnPlan a = attn_plan(L, *sa);
     const size_t Hkv = static_cast<size_t>(sa->n_kv_heads), rows = static_cast<size_t>(a.rows);
@@ -329,6 +330,43 @@ int64_t avtp_kept_count_host(const int32_t* cu_seqlens, const int32_t* img_cu, c
     volatile double prod = static_cast<double>(kr) * static_cast<double>(nvis);
     const double x = prod + 0.5;
     total += static_cast<int64_t>(floor(x)) + (static_cast<int64_t>(cu_seqlens[r + 1]) - cu_seqlens[r] - nvis);
+  }
+  return total;
+}
+
+avtp_status_t avtp_pruned_layout(const avtp_layout_t* layout, const int32_t* budgets, int32_t* out_img_start,
+                                 int32_t* out_img_len, void* workspace, size_t workspace_bytes, avtp_stream_t stream) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if (layout->n_images > 0 && (budgets == nullptr || out_img_start == nullptr || out_img_len == nullptr))
+    return AVTP_ERR_INVALID_ARG;
+  const WsPlan p = plan_workspace(*layout, nullptr);
+  if ((st = check_ws(workspace, workspace_bytes, p)) != AVTP_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PrepArgs pa{};
+  pa.L = *layout;
+  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
+  return from_cuda(launch_pruned_layout(*layout, budgets, out_img_start, out_img_len, workspace, p, s));
+}
+
+int64_t avtp_kept_count_vis_host(const int32_t* cu_seqlens, const int32_t* n_vis, const float* keep_ratio,
+                                 int32_t n_requests, int32_t* out_cu_seqlens, int32_t* out_n_vis) {
+  if (cu_seqlens == nullptr || n_vis == nullptr || keep_ratio == nullptr || n_requests < 1) return -1;
+  int64_t total = 0;
+  if (out_cu_seqlens != nullptr) out_cu_seqlens[0] = 0;
+  for (int r = 0; r < n_requests; ++r) {
+    const int64_t Tr = static_cast<int64_t>(cu_seqlens[r + 1]) - cu_seqlens[r];
+    if (Tr < 0 || n_vis[r] < 0 || n_vis[r] > Tr) return -1;
+    const float kr = keep_ratio[r];
+    if (!(kr >= 0.f && kr <= 1.f)) return -1;
+    // floor(kr * N + 0.5) with each operation rounded once (built with FMA contraction off)
+    volatile double prod = static_cast<double>(kr) * static_cast<double>(n_vis[r]);
+    const double x = prod + 0.5;
+    const int64_t kept_vis = static_cast<int64_t>(floor(x));
+    total += kept_vis + (Tr - n_vis[r]);
+    if (total > 0x7fffffffLL) return -1;
+    if (out_cu_seqlens != nullptr) out_cu_seqlens[r + 1] = static_cast<int32_t>(total);
+    if (out_n_vis != nullptr) out_n_vis[r] = static_cast<int32_t>(kept_vis);
   }
   return total;
 }

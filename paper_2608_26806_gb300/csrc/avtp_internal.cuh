@@ -54,6 +54,7 @@ struct WsPlan {
   size_t req_budget;  // int32 [R]: B_r
   size_t img_sums;    // int64 [n_img]: used by avtp_prune when the caller passes NULL
   size_t scores;      // float [T]: used by avtp_prune when the caller passes NULL
+  size_t scratch;     // int32 [n_img + 1]: per-call scratch of the pruned-layout kernel
   // criterion B (text attention); "rows" = rows per KV group = max_text * G
   size_t text_idx;    // int32 [T]: packed position of each text ordinal
   size_t text_cu;     // int32 [R + 1]: text ordinals per request
@@ -213,6 +214,9 @@ constexpr int kMaxWarmCtas = 96;
 int alloc_select_ctas_per_sm();  // from the occupancy calculator (about 4: 256 threads, 64 registers)
 int prune_reserve_sms(const avtp_layout_t& L);
 int prune_warm_ctas(const avtp_layout_t& L);
+
+cudaError_t launch_pruned_layout(const avtp_layout_t& L, const int32_t* budgets, int32_t* out_start, int32_t* out_len,
+                                 void* ws, const WsPlan& p, cudaStream_t s);
 
 cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
                            int n_sets, void* ws, const WsPlan& p, cudaStream_t s);

@@ -266,7 +266,45 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
   }
 }
 
+// The image spans of the pruned batch: image i of request r moves left by the tokens
+// pruned from the request's earlier images and keeps budgets[i] tokens. One CTA: an
+// exclusive scan of the pruned counts over all images, less the request's first entry.
+__global__ void __launch_bounds__(kPrepThreads)
+k_pruned_layout(avtp_layout_t L, const int32_t* __restrict__ budgets, const int32_t* __restrict__ img_req,
+                int32_t* __restrict__ out_start, int32_t* __restrict__ out_len, int32_t* __restrict__ scratch,
+                DevStatus* st) {
+  __shared__ int32_t s_warp[32];
+  if (!st->layout_ok) return;
+  const int NI = L.n_images;
+  // dropped[i] = img_len - budget (0 for a budget outside [0, img_len], which is recorded)
+  auto dropped = [&](int i) {
+    const int32_t k = budgets[i], n = L.img_len[i];
+    return (k >= 0 && k <= n) ? n - k : 0;
+  };
+  block_exclusive_scan<int32_t>(NI, dropped, scratch, s_warp);
+  for (int i = threadIdx.x; i < NI; i += blockDim.x) {
+    const int32_t k = budgets[i], n = L.img_len[i];
+    if (k < 0 || k > n) {
+      record_error(st, AVTP_ERR_DEVICE_INPUT, i);
+      out_start[i] = 0;
+      out_len[i] = 0;
+      continue;
+    }
+    const int first = L.img_cu[img_req[i]];  // the request's first image
+    out_start[i] = L.img_start[i] - (scratch[i] - scratch[first]);
+    out_len[i] = k;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_pruned_layout(const avtp_layout_t& L, const int32_t* budgets, int32_t* out_start, int32_t* out_len,
+                                 void* ws, const WsPlan& p, cudaStream_t s) {
+  if (L.n_images == 0) return cudaSuccess;
+  k_pruned_layout<<<1, kPrepThreads, 0, s>>>(L, budgets, ws_at<int32_t>(ws, p.img_req), out_start, out_len,
+                                             ws_at<int32_t>(ws, p.scratch), ws_at<DevStatus>(ws, p.status));
+  return cudaGetLastError();
+}
 
 cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s) {
   const bool b = a.build_text_tiles != 0;

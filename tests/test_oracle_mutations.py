@@ -46,6 +46,10 @@ MUTATIONS = {
                      "keep = np.zeros(b - a, dtype=bool)"),
     "fixed point truncates": ("return np.rint(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)",
                               "return np.trunc(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)"),
+    "pruned image starts after its first kept token": ("starts.append(int(np.count_nonzero(local < s0)))",
+                                                       "starts.append(int(np.count_nonzero(local <= s0)))"),
+    "pruned image span keeps its old length": ("lens.append(int(np.count_nonzero((local >= s0) & (local < s1))))",
+                                               "lens.append(s1 - s0)"),
 }
 
 PIN_TESTS = [name for name, fn in inspect.getmembers(pins, inspect.isfunction) if name.startswith("test_")]

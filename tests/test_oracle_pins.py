@@ -421,3 +421,61 @@ def test_compact_is_row_gather():
         assert out[j].tobytes() == rows[t].tobytes()
         for p in range(3):
             assert outp[p, j] == planes[p, t]
+
+
+# ---------------------------------------------------------------- the pruned layout (progressive pruning)
+def test_pruned_layout_golden():
+    g = _load("pruned_layout.json")
+    lay = synth.Layout(**{k: np.asarray(v, dtype=np.int32) for k, v in g["layout"].items()})
+    got = O.pruned_layout(lay, np.asarray(g["kept_idx"]), np.asarray(g["out_cu_seqlens"]))
+    for k, v in g["expected"].items():
+        assert got[k].tolist() == v, k
+
+
+def _pruned_case(seed):
+    rng = np.random.default_rng(seed)
+    reqs = []
+    for _ in range(rng.integers(1, 4)):
+        segs = []
+        for _ in range(rng.integers(1, 6)):
+            if rng.random() < 0.6:
+                segs.append(("i", int(rng.integers(1, 40))))
+            else:
+                segs.append(("t", int(rng.integers(1, 9))))
+        reqs.append(segs)
+    lay = synth.Layout.from_segments(reqs)
+    scores = rng.standard_normal(lay.n_tokens).astype(np.float32)
+    budgets = np.array([rng.integers(0, n + 1) for n in lay.img_len], dtype=np.int32)
+    kept = O.select(lay, scores, budgets)
+    vis = lay.visual_mask()
+    cu2 = [0]
+    for r in range(lay.n_requests):
+        a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+        n_txt = int((~vis[a:b]).sum())
+        cu2.append(cu2[-1] + n_txt + int(budgets[int(lay.img_cu[r]):int(lay.img_cu[r + 1])].sum()))
+    return lay, budgets, kept, np.asarray(cu2, dtype=np.int32)
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_pruned_layout_closed_form(seed):
+    # in request r, image i moves left by the tokens pruned from the request's earlier
+    # images, and keeps its budget
+    lay, budgets, kept, cu2 = _pruned_case(seed)
+    got = O.pruned_layout(lay, kept, cu2)
+    for r in range(lay.n_requests):
+        dropped = 0
+        for i in range(int(lay.img_cu[r]), int(lay.img_cu[r + 1])):
+            assert got["img_start"][i] == lay.img_start[i] - dropped
+            assert got["img_len"][i] == budgets[i]
+            dropped += int(lay.img_len[i]) - int(budgets[i])
+    assert got["cu_seqlens"].tolist() == cu2.tolist()
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_pruned_layout_marks_exactly_the_kept_visual_tokens(seed):
+    lay, budgets, kept, cu2 = _pruned_case(seed)
+    got = O.pruned_layout(lay, kept, cu2)
+    lay2 = synth.Layout(cu_seqlens=got["cu_seqlens"], img_cu=got["img_cu"], img_start=got["img_start"],
+                        img_len=got["img_len"])
+    # the visual mask of the pruned batch is the gathered visual mask of the original
+    assert np.array_equal(lay2.visual_mask(), lay.visual_mask()[kept])
