@@ -38,7 +38,7 @@ FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 STEP_NAMES = ("validate", "score", "allocate_select", "compact")
 SCORE_KERNELS = {"hidden_variation": ["k_score_hvar"],
-                 "text_attention": ["k_attn_tc", "k_attn_pack", "k_attn_merge", "k_attn_finalize"]}
+                 "text_attention": ["k_attn_lse", "k_attn_mass", "k_attn_pack", "k_attn_finalize"]}
 
 
 # ---------------------------------------------------------------- helpers
@@ -68,6 +68,15 @@ def reduce_max(value: float, world: int, device=None) -> float:
     t = torch.tensor([value], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_rate(units_per_step: int, steps: int, total_ms: float, world: int, device=None):
+    """Every rank's units over the slowest rank's time: (units/s, ms per step of the slowest rank).
+
+    Each rank runs its own replica of the workload (weak scaling), so the job's units
+    are world x units_per_step x steps."""
+    total_ms_max = reduce_max(total_ms, world, device)
+    return units_per_step * steps * world / (total_ms_max * 1e-3), total_ms_max / steps
 
 
 def barrier(world: int):
@@ -313,7 +322,7 @@ def run_ours(args, world, rank, local):
                 for j, name in enumerate(STEP_NAMES)}
     serial_ms = [inner[i][0].elapsed_time(inner[i][n_ev - 1]) for i in range(K)]
     total_ms = sum(step_ms)
-    total_ms_max = reduce_max(total_ms, world, dev)
+    value, ms_step = whole_job_rate(acct["n_vis"], K, total_ms, world, dev)
 
     # end to end through the public API: pinned host inputs -> device -> prune -> host outputs
     e2e = run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp)
@@ -336,8 +345,6 @@ def run_ours(args, world, rank, local):
                 "peak": bf16_tf, "unit": "TFLOP/s", "frac": round(achieved / bf16_tf, 4), "peak_kind": peak_kind,
                 "algorithmic_flops_per_launch": acct["flops"], "avg_launch_us": round(score_ms * 1e3, 2),
                 "traffic": None}
-    ms_step = total_ms_max / K
-    value = acct["n_vis"] * K * world / (total_ms_max * 1e-3)
     srt = sorted(step_ms)
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
