@@ -60,7 +60,7 @@ typedef enum {
   AVTP_ERR_UNSUPPORTED = 2,   /* head_dim not 64/128, misaligned rows, Hq % Hkv != 0 */
   AVTP_ERR_RANGE = 3,         /* a size above the documented limits                  */
   AVTP_ERR_CUDA = 4,          /* a CUDA runtime call failed (launch, copy)           */
-  AVTP_ERR_TIMEOUT = 5,       /* a bounded device wait gave up (reserved)            */
+  AVTP_ERR_TIMEOUT = 5,       /* a bounded device wait gave up (about one second)    */
   AVTP_ERR_DEVICE_INPUT = 6,  /* device-side data failed validation                  */
   AVTP_ERR_WORKSPACE = 7      /* workspace null, misaligned or too small             */
 } avtp_status_t;
@@ -266,6 +266,22 @@ AVTP_API avtp_status_t avtp_pruned_layout(const avtp_layout_t* layout, const int
  * inputs of the same call for the next stage. */
 AVTP_API int64_t avtp_kept_count_vis_host(const int32_t* cu_seqlens, const int32_t* n_vis, const float* keep_ratio,
                                           int32_t n_requests, int32_t* out_cu_seqlens, int32_t* out_n_vis);
+
+/* Check of the failure path every pipeline kernel takes when a wait on an mbarrier (a
+ * TMA copy, a tensor-core commit, a hand-off between warps) does not complete: one CTA
+ * of 64 threads waits on a fresh count-1 mbarrier with the library's bounded waits,
+ * thread 0 with the single-thread form and warp 1 with the warp-wide form.
+ *   arrive != 0: thread 0 arrives first, both waits complete, the status word stays
+ *                AVTP_OK.
+ *   arrive == 0: nothing arrives; each wait gives up after limit_ns nanoseconds of the
+ *                GPU's global timer and the kernel records AVTP_ERR_TIMEOUT in the
+ *                status word (detail = 0 or 1, the waiter that recorded first) and
+ *                returns. Nothing traps or faults; the context stays usable.
+ * The pipeline kernels use a limit of one second. limit_ns in [1000, 10^10];
+ * workspace: device, 256-byte aligned, at least 16 bytes (its status word is reset
+ * first). Asynchronous on `stream`; read the outcome with avtp_read_device_status(). */
+AVTP_API avtp_status_t avtp_wait_selftest(int64_t limit_ns, int32_t arrive, void* workspace, size_t workspace_bytes,
+                                          avtp_stream_t stream);
 
 /* Waits for `stream`, then reads the workspace's device status word into *out
  * (an avtp_status_t value; AVTP_OK if no device-side error was recorded since the

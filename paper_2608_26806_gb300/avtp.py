@@ -89,6 +89,7 @@ SIGNATURES = {
     "avtp_kept_count_host": (c_int64, [c_void_p, c_void_p, c_void_p, c_void_p, c_int32]),
     "avtp_pruned_layout": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "avtp_kept_count_vis_host": (c_int64, [c_void_p, c_void_p, c_void_p, c_int32, c_void_p, c_void_p]),
+    "avtp_wait_selftest": (c_int, [c_int64, c_int32, c_void_p, c_size_t, c_void_p]),
     "avtp_read_device_status": (c_int, [c_void_p, c_void_p, POINTER(c_int32)]),
     "avtp_status_string": (ctypes.c_char_p, [c_int32]),
     "avtp_version": (c_int32, []),
@@ -381,6 +382,14 @@ def kept_count_host(layout_host: Dict[str, np.ndarray], keep_ratio: np.ndarray) 
     if n < 0:
         raise AVTPError(ERR_INVALID_ARG, "avtp_kept_count_host")
     return int(n)
+
+
+def wait_selftest(limit_ns: int, arrive: bool, workspace: torch.Tensor, stream=None) -> None:
+    """Runs the bounded-wait check kernel (``avtp_wait_selftest``); read the outcome
+    with :func:`read_device_status` (``ERR_TIMEOUT`` when ``arrive`` is false)."""
+    _check(load().avtp_wait_selftest(int(limit_ns), 1 if arrive else 0, _ptr(workspace),
+                                     workspace.numel() * workspace.element_size(), _stream(stream)),
+           "avtp_wait_selftest")
 
 
 def read_device_status(workspace: torch.Tensor, stream=None) -> int:

@@ -371,6 +371,18 @@ int64_t avtp_kept_count_vis_host(const int32_t* cu_seqlens, const int32_t* n_vis
   return total;
 }
 
+avtp_status_t avtp_wait_selftest(int64_t limit_ns, int32_t arrive, void* workspace, size_t workspace_bytes,
+                                 avtp_stream_t stream) {
+  if (limit_ns < 1000 || limit_ns > 10000000000LL) return AVTP_ERR_INVALID_ARG;
+  if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1)) != 0 ||
+      workspace_bytes < sizeof(DevStatus))
+    return AVTP_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  avtp_status_t st = from_cuda(cudaMemsetAsync(workspace, 0, sizeof(DevStatus), s));
+  if (st != AVTP_OK) return st;
+  return from_cuda(launch_wait_selftest(static_cast<uint64_t>(limit_ns), arrive != 0, workspace, s));
+}
+
 avtp_status_t avtp_read_device_status(const void* workspace, avtp_stream_t stream, int32_t* out) {
   if (workspace == nullptr || out == nullptr) return AVTP_ERR_INVALID_ARG;
   DevStatus h{};

@@ -46,6 +46,31 @@ __device__ __forceinline__ void record_error(DevStatus* st, int32_t code, int32_
   if (atomicCAS(&st->code, 0, code) == 0) st->detail = detail;
 }
 
+// ---------------------------------------------------------------- bounded waits
+// Every wait on an mbarrier gives up after about kWaitLimitNs of the global timer
+// without the phase completing (or after kWaitSpinCap polls, should the timer not
+// advance); the kernel then records AVTP_ERR_TIMEOUT and returns instead of hanging.
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // one second
+constexpr uint32_t kWaitSpinCap = 1u << 28;
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Called after each failed poll (polls counts them from 1): true once the wait has run
+// past limit_ns. The timer is read every 64 polls only, and started at the first such
+// read, so that the short waits of a running pipeline never touch it.
+__device__ __forceinline__ bool wait_expired(uint32_t polls, uint64_t& t0, uint64_t limit_ns) {
+  if ((polls & 63u) != 0) return false;
+  const uint64_t now = global_ns();
+  if (polls == 64) {
+    t0 = now;
+    return false;
+  }
+  return now - t0 > limit_ns || polls >= kWaitSpinCap;
+}
+
 // ---------------------------------------------------------------- workspace
 struct WsPlan {
   size_t status;      // DevStatus
@@ -220,6 +245,8 @@ cudaError_t launch_pruned_layout(const avtp_layout_t& L, const int32_t* budgets,
 
 cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
                            int n_sets, void* ws, const WsPlan& p, cudaStream_t s);
+
+cudaError_t launch_wait_selftest(uint64_t limit_ns, int arrive, void* ws, cudaStream_t s);
 
 int device_sm_count();
 

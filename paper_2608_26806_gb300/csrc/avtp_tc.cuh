@@ -17,8 +17,6 @@
 namespace avtp {
 namespace tc {
 
-constexpr uint32_t kSpinLimit = 1u << 24;  // bounded mbarrier waits (each try may suspend briefly)
-
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -46,17 +44,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// One thread waits for the phase with the given parity to complete; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i)
+// One thread waits for the phase with the given parity to complete; false once the
+// wait has run past limit_ns without it.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns = kWaitLimitNs) {
+  uint64_t t0 = 0;
+  for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-  return false;
+    if (wait_expired(i, t0, limit_ns)) return false;
+  }
 }
-// The whole warp waits (warp-uniform result); false on timeout.
-__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i)
+// The whole warp waits (warp-uniform result); false once the wait has run past limit_ns.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, uint64_t limit_ns = kWaitLimitNs) {
+  uint64_t t0 = 0;
+  for (uint32_t i = 1;; ++i) {
     if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
-  return false;
+    if (__any_sync(0xffffffffu, wait_expired(i, t0, limit_ns))) return false;
+  }
 }
 
 // ---------------------------------------------------------------- TMA

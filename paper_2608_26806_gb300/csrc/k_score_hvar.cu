@@ -35,7 +35,6 @@ constexpr int kChunkElems = 1024;         // bf16 per tensor per slot (2 KiB)
 constexpr int kChunkBytes = kChunkElems * 2;
 constexpr int kSlotBytes = 2 * kChunkBytes;
 constexpr size_t kSmemBytes = static_cast<size_t>(kWarps) * kSlots * kSlotBytes;  // 192 KiB
-constexpr uint32_t kMaxSpins = 1u << 22;  // bounded mbarrier wait
 // Layouts up to this many images / requests are staged in shared memory. Kept small
 // (about 10 KiB with the barriers) so that a CTA of the selection kernel, launched
 // while this kernel still runs, fits on the same SM next to the 192-KiB pipeline.
@@ -260,9 +259,9 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   while (in_flight > 0) {
     const uint32_t parity = (phase_bits >> slot_take) & 1u;
     // warp-uniform bounded wait: a completed phase stays visible, so every lane gets there
-    uint32_t spins = 0;
-    while (!__all_sync(0xffffffffu, mbar_try_wait(&wbar[slot_take], parity))) {
-      if (++spins >= kMaxSpins) { timed_out = true; break; }
+    uint64_t t0 = 0;
+    for (uint32_t polls = 1; !__all_sync(0xffffffffu, mbar_try_wait(&wbar[slot_take], parity)); ++polls) {
+      if (__any_sync(0xffffffffu, wait_expired(polls, t0, kWaitLimitNs))) { timed_out = true; break; }
     }
     if (timed_out) break;
     phase_bits ^= 1u << slot_take;
@@ -317,12 +316,14 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   }
   if (!timed_out && run_img >= 0) flush_run();
   if (timed_out) {
-    // drain: give the copies still in flight a bounded chance to land before the CTA exits
-    for (int k = 0; k < kSlots; ++k) {
-      const uint32_t parity = (phase_bits >> k) & 1u;
-      for (uint32_t spins = 0; spins < kMaxSpins && !__all_sync(0xffffffffu, mbar_try_wait(&wbar[k], parity));
-           ++spins) {
-      }
+    // drain: give the copies still in flight (slot_take and the in_flight - 1 slots after
+    // it) a bounded chance to land before the CTA exits
+    for (int k = 0; k < in_flight; ++k) {
+      const int slot = (slot_take + k) % kSlots;
+      const uint32_t parity = (phase_bits >> slot) & 1u;
+      uint64_t t0 = 0;
+      for (uint32_t polls = 1; !__all_sync(0xffffffffu, mbar_try_wait(&wbar[slot], parity)); ++polls)
+        if (__any_sync(0xffffffffu, wait_expired(polls, t0, kWaitLimitNs))) break;
     }
     pdl_wait();  // the validation kernel resets the status word: record after it
     if (lane == 0) record_error(st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));

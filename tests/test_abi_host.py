@@ -156,3 +156,11 @@ def test_workspace_size_grows_with_attention_bookkeeping(lib):
     assert lib.avtp_workspace_size(ctypes.byref(lay), ctypes.byref(_attn_args()), ctypes.byref(b)) == avtp.OK
     assert b.value > a.value >= 10000 * 4
     assert a.value % 256 == 0 and b.value % 256 == 0
+
+
+def test_host_validation_of_wait_selftest_arguments(lib):
+    for bad in (-1, 0, 999, 10_000_000_001):
+        assert lib.avtp_wait_selftest(bad, 0, FAKE, 256, None) == avtp.ERR_INVALID_ARG
+    assert lib.avtp_wait_selftest(1_000_000, 0, None, 256, None) == avtp.ERR_WORKSPACE
+    assert lib.avtp_wait_selftest(1_000_000, 0, FAKE + 8, 256, None) == avtp.ERR_WORKSPACE
+    assert lib.avtp_wait_selftest(1_000_000, 0, FAKE, 8, None) == avtp.ERR_WORKSPACE
