@@ -315,6 +315,7 @@ def run_ours(args, world, rank, local):
         sec_lse = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev, lse=lse)
         del lse
         prog = time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avtp, world, dev)
+    variants = time_variants(args, call, stream, flush, torch, avtp, 4 if crit == "hidden_variation" else 7)
     clocks = sampler.stop() if sampler else None
     barrier(world)
     step_ms = [a.elapsed_time(b) for a, b in outer]
@@ -345,7 +346,6 @@ def run_ours(args, world, rank, local):
                 "peak": bf16_tf, "unit": "TFLOP/s", "frac": round(achieved / bf16_tf, 4), "peak_kind": peak_kind,
                 "algorithmic_flops_per_launch": acct["flops"], "avg_launch_us": round(score_ms * 1e3, 2),
                 "traffic": None}
-    srt = sorted(step_ms)
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": round(ms_step, 5), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -354,14 +354,15 @@ def run_ours(args, world, rank, local):
                    "seq_len": lay.n_tokens, "visual_tokens": acct["n_vis"], "kept_tokens": n_kept,
                    "hidden": wl.hidden, "images": lay.n_images, "keep_ratio": float(wl.keep_ratio[0]),
                    "parallelism": f"replicas{world}", "l2": "flushed before every timed step: 256 MiB write, then 256 MiB read (clean), outside the step's events"},
-        "latency_us": {"p50": round(srt[len(srt) // 2] * 1e3, 2), "p90": round(srt[int(len(srt) * 0.9)] * 1e3, 2),
-                       "mean": round(statistics.mean(step_ms) * 1e3, 2)},
+        "latency_us": _latency(step_ms),
+        "warm_l2": variants["warm_l2"],
+        "graph": variants["graph"],
         "steps_us": {k: round(statistics.mean(v) * 1e3, 2) for k, v in per_step.items()},
         "serialized_step_us": round(statistics.mean(serial_ms) * 1e3, 2),
         "stage_roofline": stage_roofline(acct, ms_step, hbm, bf16_tf, peak_kind),
         "roofline": roof,
         "e2e": e2e,
-        "gpu_launches": K * (4 if crit == "hidden_variation" else 7),
+        "gpu_launches": K * (4 if crit == "hidden_variation" else 7) + variants["launches"],
         "clocks": clocks,
     }
     hbm_s, bf16_s, _ = measured_peaks()
@@ -390,6 +391,57 @@ def run_ours(args, world, rank, local):
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, crit, args.cpu_seconds)
     return line
+
+
+def _latency(ms):
+    srt = sorted(ms)
+    return {"p50": round(srt[len(srt) // 2] * 1e3, 2), "p90": round(srt[int(len(srt) * 0.9)] * 1e3, 2),
+            "mean": round(statistics.mean(ms) * 1e3, 2)}
+
+
+def time_variants(args, call, stream, flush, torch, avtp, per_step):
+    """The headline step two more ways: with L2 left warm between steps (stream
+    launches, back to back), and replayed from a CUDA graph (L2 flushed, then warm)."""
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+
+    def loop(launch, flushed):
+        for i in range(K):
+            if flushed:
+                flush()
+            ev[i][0].record(stream)
+            launch()
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        return _latency([a.elapsed_time(b) for a, b in ev])
+
+    for _ in range(3):
+        call.run(stream)
+    torch.cuda.synchronize()
+    out = {"warm_l2": {"latency_us": loop(lambda: call.run(stream), False), "steps": K, "launch": "stream"},
+           "launches": K * per_step}
+    try:
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=side):
+            call.run(side)
+        torch.cuda.synchronize()
+        for _ in range(3):
+            flush()
+            graph.replay()
+        torch.cuda.synchronize()
+        cold = loop(graph.replay, True)
+        warm = loop(graph.replay, False)
+        st = avtp.read_device_status(call.buffers.workspace)
+        if st != avtp.OK:
+            raise RuntimeError(f"device status after graph replays: {avtp.status_string(st)}")
+        out["graph"] = {"latency_us": cold, "warm_l2_latency_us": warm, "steps": K,
+                        "l2": "flushed before every replay (cold), then back to back (warm)"}
+        out["launches"] += 2 * K * per_step
+    except Exception as e:  # a capture the runtime refuses: report it, keep the stream numbers
+        out["graph"] = {"unavailable": f"{type(e).__name__}: {str(e)[:200]}"}
+    return out
 
 
 def fa_lse(wl, q, k, torch):

@@ -223,21 +223,27 @@ __device__ __forceinline__ void p1_slice(uint32_t taddr, int pe, int lim, float 
 #pragma unroll
       for (int q = 0; q < 32; ++q) v[q] = (p * 32 + q <= lim) ? v[q] : -INFINITY;
     }
-    float mx0 = fmaxf(v[0], v[1]), mx1 = fmaxf(v[2], v[3]);
+    // max as a tree (depth 5); exact in any order
+    float t16[16];
 #pragma unroll
-    for (int q = 4; q < 32; q += 4) {
-      mx0 = fmaxf(mx0, fmaxf(v[q], v[q + 1]));
-      mx1 = fmaxf(mx1, fmaxf(v[q + 2], v[q + 3]));
+    for (int q = 0; q < 16; ++q) t16[q] = fmaxf(v[2 * q], v[2 * q + 1]);
+#pragma unroll
+    for (int w = 8; w >= 1; w >>= 1) {
+#pragma unroll
+      for (int q = 0; q < w; ++q) t16[q] = fmaxf(t16[q], t16[q + w]);
     }
-    const float mn = fmaxf(m, fmaxf(mx0, mx1) * c2);
-    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    const float mn = fmaxf(m, t16[0] * c2);
+    // four partial sums (columns q mod 4), two per packed register
+    const float2 cc = make_float2(c2, c2), nm = make_float2(-mn, -mn);
+    float2 s01 = make_float2(0.f, 0.f), s23 = s01;
 #pragma unroll
     for (int q = 0; q < 32; q += 4) {
-      s0 += tc::ex2(fmaf(v[q], c2, -mn));
-      s1 += tc::ex2(fmaf(v[q + 1], c2, -mn));
-      s2 += tc::ex2(fmaf(v[q + 2], c2, -mn));
-      s3 += tc::ex2(fmaf(v[q + 3], c2, -mn));
+      const float2 a01 = tc::ffma2(make_float2(v[q], v[q + 1]), cc, nm);
+      const float2 a23 = tc::ffma2(make_float2(v[q + 2], v[q + 3]), cc, nm);
+      s01 = tc::add2(s01, make_float2(tc::ex2(a01.x), tc::ex2(a01.y)));
+      s23 = tc::add2(s23, make_float2(tc::ex2(a23.x), tc::ex2(a23.y)));
     }
+    const float s0 = s01.x, s1 = s01.y, s2 = s23.x, s3 = s23.y;
     // a row with nothing visible yet keeps (-inf, 0); exp2(-inf - -inf) would be NaN
     if (mn != -INFINITY) {
       l = l * tc::ex2(m - mn) + ((s0 + s1) + (s2 + s3));
@@ -254,21 +260,27 @@ __device__ __forceinline__ void p1_slice(uint32_t taddr, int pe, int lim, float 
   }
 }
 
-// Pass 2: sum of exp2(c2 * z - lse2[c]) over the columns c of a key; a column that does
-// not see the key carries lse2 = +inf, which makes its term 0.
-__device__ __forceinline__ float p2_slice(uint32_t taddr, const float* lse, float c2) {
+// Pass 2: sum of exp2(c2 * z - lse2[c]) over the columns c of a key. `nlse` holds
+// -lse2; a column that does not see the key carries -inf, which makes its term 0.
+__device__ __forceinline__ float p2_slice(uint32_t taddr, const float* nlse, float c2) {
   uint32_t ra[32], rb[32];
-  float m0 = 0.f, m1 = 0.f, m2 = 0.f, m3 = 0.f;
+  // four partial sums (columns q mod 4), two per packed register
+  float2 m01 = make_float2(0.f, 0.f), m23 = m01;
+  const float2 cc = make_float2(c2, c2);
   auto chunk = [&](uint32_t(&r)[32], uint32_t(&nx)[32], int p) {
     if (p + 1 < kChunks) tc::tmem_ld32_async(taddr + (p + 1) * 32, nx);
-    const float4* l4 = reinterpret_cast<const float4*>(lse + p * 32);
+    const float4* l4 = reinterpret_cast<const float4*>(nlse + p * 32);
 #pragma unroll
     for (int q4 = 0; q4 < 8; ++q4) {
       const float4 lv = l4[q4];
-      m0 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 0]), c2, -lv.x));
-      m1 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 1]), c2, -lv.y));
-      m2 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 2]), c2, -lv.z));
-      m3 += tc::ex2(fmaf(__uint_as_float(r[4 * q4 + 3]), c2, -lv.w));
+      const float2 a01 =
+          tc::ffma2(make_float2(__uint_as_float(r[4 * q4 + 0]), __uint_as_float(r[4 * q4 + 1])), cc,
+                    make_float2(lv.x, lv.y));
+      const float2 a23 =
+          tc::ffma2(make_float2(__uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3])), cc,
+                    make_float2(lv.z, lv.w));
+      m01 = tc::add2(m01, make_float2(tc::ex2(a01.x), tc::ex2(a01.y)));
+      m23 = tc::add2(m23, make_float2(tc::ex2(a23.x), tc::ex2(a23.y)));
     }
     if (p + 1 < kChunks) tc::tmem_wait(nx);
   };
@@ -279,7 +291,7 @@ __device__ __forceinline__ float p2_slice(uint32_t taddr, const float* lse, floa
     chunk(ra, rb, p);
     chunk(rb, ra, p + 1);
   }
-  return (m0 + m1) + (m2 + m3);
+  return (m01.x + m01.y) + (m23.x + m23.y);
 }
 
 __device__ __forceinline__ void setup_sync(Sync& sy, int warp) {
@@ -499,7 +511,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapQ, AttnArgs a) {
   extern __shared__ unsigned char smem_raw[];
   __shared__ Sync sy;
-  __shared__ __align__(16) float s_lse[2][kBlk];  // [block parity][row of the block]
+  __shared__ __align__(16) float s_lse[2][kBlk];  // -lse2, [block parity][row of the block]
   // key masses of the last steps, per column half, flushed to the accumulator every
   // kMassWindow steps (global atomics inside the step loop would be waited for by the
   // next step's TMEM fence)
@@ -643,11 +655,11 @@ k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CU
         tile.next(a, s);
       }
       if (tile.i != img) {
-        // the lse2 vector of this (block, image): +inf on rows whose query precedes the
+        // the -lse2 vector of this (block, image): -inf on rows whose query precedes the
         // image, so that their terms vanish; double-buffered by parity
         img = tile.i;
         par ^= 1;
-        s_lse[par][etid] = (etid >= tile.c0) ? lse_own : INFINITY;
+        s_lse[par][etid] = (etid >= tile.c0) ? -lse_own : -INFINITY;
         bar_epi();
       }
       const int t = st & 1;                                  // accumulator of this step

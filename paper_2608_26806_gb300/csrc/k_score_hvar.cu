@@ -36,7 +36,7 @@ constexpr int kChunkBytes = kChunkElems * 2;
 constexpr int kSlotBytes = 2 * kChunkBytes;
 constexpr size_t kSmemBytes = static_cast<size_t>(kWarps) * kSlots * kSlotBytes;  // 192 KiB
 // Layouts up to this many images / requests are staged in shared memory. Kept small
-// (about 10 KiB with the barriers) so that a CTA of the selection kernel, launched
+// (about 11 KiB with the barriers) so that a CTA of the selection kernel, launched
 // while this kernel still runs, fits on the same SM next to the 192-KiB pipeline.
 constexpr int kStageImages = 1024;
 constexpr int kStageRequests = 256;
@@ -153,6 +153,7 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   __shared__ int32_t s_vcu[kStageImages + 1];
   __shared__ int32_t s_gstart[kStageImages];
   __shared__ int32_t s_icu[kStageRequests + 1];
+  __shared__ int32_t s_cu[kStageRequests + 1];
   __shared__ int32_t s_warp[kWarps];
   pdl_trigger();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -170,14 +171,19 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   map.NI = NI;
   const bool staged = NI <= kStageImages && R <= kStageRequests;
   if (staged) {
-    for (int j = threadIdx.x; j <= R; j += kThreads) s_icu[j] = min(max(icu[j], 0), NI);
-    for (int j = threadIdx.x; j < NI; j += kThreads) s_vcu[j] = max(iln[j], 0);
+    // all four layout arrays in one round of loads, so that one DRAM latency (not two)
+    // precedes the first bulk copy
+    for (int j = threadIdx.x; j <= R; j += kThreads) {
+      s_icu[j] = min(max(icu[j], 0), NI);
+      s_cu[j] = cu[j];
+    }
+    for (int j = threadIdx.x; j < NI; j += kThreads) {
+      s_vcu[j] = max(iln[j], 0);
+      s_gstart[j] = ist[j];
+    }
     __syncthreads();
     block_scan_inplace(s_vcu, NI, s_warp);
-    for (int j = threadIdx.x; j < NI; j += kThreads) {
-      const int r = upper_index(s_icu, R, j);  // request of image j
-      s_gstart[j] = cu[r] + ist[j];
-    }
+    for (int j = threadIdx.x; j < NI; j += kThreads) s_gstart[j] += s_cu[upper_index(s_icu, R, j)];  // request of j
     __syncthreads();
     map.vcu = s_vcu;
     map.gstart = s_gstart;
