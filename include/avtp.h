@@ -133,7 +133,9 @@ typedef struct {
 
 /* One set of rows to gather: out[j] = in[kept_idx[j]] for j in [0, n_kept).
  * Device pointers; sizes and strides in bytes. Any row size works; rows whose
- * size, strides and pointers are 16-byte multiples take the vectorised path. */
+ * size, strides and pointers are 16-byte multiples take the vectorised path.
+ * When n_kept is 0 nothing is read or written, and the pointers may be NULL
+ * (an empty output tensor). */
 typedef struct {
   const void* in;
   void* out;

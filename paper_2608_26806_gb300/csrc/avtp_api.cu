@@ -64,12 +64,13 @@ avtp_status_t check_alloc_args(const avtp_alloc_args_t* a) {
   return AVTP_OK;
 }
 
-avtp_status_t check_sets(const avtp_rows_t* sets, int32_t n_sets) {
+// With n_kept = 0 no row is touched, so the pointers of a set may be NULL.
+avtp_status_t check_sets(const avtp_rows_t* sets, int32_t n_sets, int64_t n_kept) {
   if (n_sets < 0 || n_sets > AVTP_MAX_ROW_SETS) return AVTP_ERR_INVALID_ARG;
   if (n_sets > 0 && sets == nullptr) return AVTP_ERR_INVALID_ARG;
   for (int i = 0; i < n_sets; ++i) {
     const avtp_rows_t& s = sets[i];
-    if (s.in == nullptr || s.out == nullptr) return AVTP_ERR_INVALID_ARG;
+    if (n_kept > 0 && (s.in == nullptr || s.out == nullptr)) return AVTP_ERR_INVALID_ARG;
     if (s.row_bytes < 1 || s.in_stride < s.row_bytes || s.out_stride < s.row_bytes) return AVTP_ERR_INVALID_ARG;
   }
   return AVTP_OK;
@@ -257,7 +258,7 @@ avtp_status_t avtp_select(const avtp_layout_t* layout, const float* scores, cons
 
 avtp_status_t avtp_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
                            int32_t n_sets, void* workspace, size_t workspace_bytes, avtp_stream_t stream) {
-  avtp_status_t st = check_sets(sets, n_sets);
+  avtp_status_t st = check_sets(sets, n_sets, n_kept);
   if (st != AVTP_OK) return st;
   if (n_kept < 0 || n_tokens < 0 || (n_kept > 0 && kept_idx == nullptr)) return AVTP_ERR_INVALID_ARG;
   if (workspace == nullptr || (reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1)) != 0 ||
@@ -279,7 +280,7 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   if (st != AVTP_OK) return st;
   if ((st = check_score_args(layout, score_args)) != AVTP_OK) return st;
   if ((st = check_alloc_args(alloc_args)) != AVTP_OK) return st;
-  if ((st = check_sets(sets, n_sets)) != AVTP_OK) return st;
+  if ((st = check_sets(sets, n_sets, n_kept)) != AVTP_OK) return st;
   if (out_cu_seqlens == nullptr || n_kept < 0 || (n_kept > 0 && kept_idx == nullptr)) return AVTP_ERR_INVALID_ARG;
   if (layout->n_images > 0 && budgets == nullptr) return AVTP_ERR_INVALID_ARG;
   const WsPlan p = plan_workspace(*layout, score_args);

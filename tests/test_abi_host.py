@@ -146,6 +146,10 @@ def test_host_validation_of_alloc_and_compact_arguments(lib):
     rows[0] = avtp._Rows(FAKE, FAKE, 16, 16, 16)
     assert lib.avtp_compact(FAKE, 10, 100, rows, 1, None, 1 << 20, None) == avtp.ERR_WORKSPACE
     assert lib.avtp_compact(FAKE, -1, 100, rows, 1, FAKE, 1 << 20, None) == avtp.ERR_INVALID_ARG
+    rows[0] = avtp._Rows(None, FAKE, 16, 16, 16)  # a NULL row pointer with rows to gather
+    assert lib.avtp_compact(FAKE, 10, 100, rows, 1, FAKE, 1 << 20, None) == avtp.ERR_INVALID_ARG
+    rows[0] = avtp._Rows(FAKE, None, 16, 16, 16)
+    assert lib.avtp_compact(FAKE, 10, 100, rows, 1, FAKE, 1 << 20, None) == avtp.ERR_INVALID_ARG
 
 
 def test_workspace_size_grows_with_attention_bookkeeping(lib):

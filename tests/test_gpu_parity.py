@@ -223,6 +223,40 @@ def test_prune_fused_budget_rule_across_alphas(alpha, relative):
     assert np.array_equal(out.kept_idx.cpu().numpy(), ref["kept_idx"])
 
 
+# batches at the edge of the layout rules: no image at all, nothing visual kept (an
+# empty output), a one-token image, and a mix of them
+_DEGENERATE = {
+    "text_only": ([[("t", 7)], [("t", 3)]], 0.5),
+    "keep_no_visual": ([[("i", 5)], [("i", 3)]], 0.05),
+    "single_token": ([[("i", 1)]], 0.95),
+    "mixed": ([[("t", 4)], [("i", 1), ("t", 2)], [("i", 6)]], 0.05),
+}
+
+
+@pytest.mark.parametrize("case", sorted(_DEGENERATE))
+@pytest.mark.parametrize("criterion", ["hidden_variation", "text_attention"])
+def test_prune_degenerate_batches(case, criterion):
+    segs, kr = _DEGENERATE[case]
+    wl = synth.make_custom(segs, keep_ratio=kr, parts=("A", "B", "pos"))
+    dw = DevWorkload(wl)
+    relative = criterion == "text_attention"
+    out = avtp.prune(dw.L, criterion, keep_ratio=dw.keep_ratio, keep_ratio_host=wl.keep_ratio,
+                     rows={"hidden": dw.t["h_cur"]}, planes={"pos": dw.t["pos"]}, **dw.score_tensors(criterion))
+    torch.cuda.synchronize()
+    assert avtp.read_device_status(out.workspace) == avtp.OK
+    lay = wl.layout
+    got = out.scores.cpu().numpy()
+    assert_scores_close(got, oracle_scores(wl, criterion), lay.visual_mask())
+    ref = O.prune(lay, keep_ratio=wl.keep_ratio, scores_f32=got, relative=relative,
+                  rows={"hidden": wl.h_cur}, planes={"pos": wl.pos})
+    assert out.n_kept == len(ref["kept_idx"])
+    assert np.array_equal(out.budgets[:lay.n_images].cpu().numpy(), ref["budgets"])
+    assert np.array_equal(out.out_cu_seqlens.cpu().numpy(), ref["out_cu_seqlens"])
+    assert np.array_equal(out.kept_idx[:out.n_kept].cpu().numpy(), ref["kept_idx"])
+    assert np.array_equal(bits_of(out.outputs["hidden"]), ref["hidden"])
+    assert np.array_equal(out.outputs["pos"].cpu().numpy(), ref["pos"])
+
+
 # ---------------------------------------------------------------- step 3
 def _select_case(lay, scores_f32, budgets):
     L = dev_layout(lay)
