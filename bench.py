@@ -327,6 +327,7 @@ def run_ours(args, world, rank, local):
 
     # end to end through the public API: pinned host inputs -> device -> prune -> host outputs
     e2e = run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp)
+    e2e_pipe = run_e2e_pipelined(args, wl, crit, L, call, dev, torch, avtp)
 
     if rank != 0:
         return None
@@ -362,6 +363,7 @@ def run_ours(args, world, rank, local):
         "stage_roofline": stage_roofline(acct, ms_step, hbm, bf16_tf, peak_kind),
         "roofline": roof,
         "e2e": e2e,
+        "e2e_pipelined": e2e_pipe,
         "gpu_launches": K * (4 if crit == "hidden_variation" else 7) + variants["launches"],
         "clocks": clocks,
     }
@@ -634,6 +636,116 @@ def run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp):
     n_vis = int(wl.layout.n_visual_per_request().sum())
     return {"value": round(n_vis / (ms * 1e-3), 1), "unit": UNIT, "ms_per_step": round(ms, 4),
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps}
+
+
+def run_e2e_pipelined(args, wl, crit, L, call, dev, torch, avtp):
+    """The same end-to-end metric with consecutive steps overlapped, as a serving loop
+    would run them: step i + 1's inputs are copied in while step i computes and copies
+    its outputs out. Each step still copies all its inputs in and all its outputs out.
+    Two prepared calls with their own device inputs and outputs alternate, and three
+    streams (copy in, compute, copy out) are ordered by events."""
+    from paper_2608_26806_gb300 import avtp as A
+
+    calls = [call]
+    # a second call on its own copies of every device input
+    L2 = A.Layout.from_host(L.host["cu_seqlens"], L.host["img_cu"], L.host["img_start"], L.host["img_len"],
+                            device=dev)
+    st0 = call._keep_alive[3]
+    kr2 = call._keep_alive[0].clone()
+    h_cur2 = call._keep_alive[1]["hidden"].clone()
+    pos2 = call._keep_alive[2]["pos"].clone()
+    if crit == "hidden_variation":
+        st2 = dict(h_cur=h_cur2, h_prior=st0["h_prior"].clone())
+    else:
+        st2 = dict(q=st0["q"].clone(), k=st0["k"].clone(), softmax_scale=st0["softmax_scale"])
+    calls.append(A.PruneCall(L2, crit, keep_ratio=kr2, keep_ratio_host=wl.keep_ratio, rows={"hidden": h_cur2},
+                             planes={"pos": pos2}, **st2))
+    layouts = [L, L2]
+
+    host_in = {"h_cur": torch.from_numpy(np.ascontiguousarray(wl.h_cur).view(np.int16)).pin_memory(),
+               "pos": torch.from_numpy(wl.pos).pin_memory()}
+    if crit == "hidden_variation":
+        host_in["h_prior"] = torch.from_numpy(np.ascontiguousarray(wl.h_prior).view(np.int16)).pin_memory()
+    else:
+        host_in["q"] = torch.from_numpy(np.ascontiguousarray(wl.q).view(np.int16)).pin_memory()
+        host_in["k"] = torch.from_numpy(np.ascontiguousarray(wl.k).view(np.int16)).pin_memory()
+    for name in ("cu_seqlens", "img_cu", "img_start", "img_len"):
+        host_in["lay_" + name] = torch.from_numpy(L.host[name].copy()).pin_memory()
+    host_in["keep_ratio"] = torch.from_numpy(wl.keep_ratio.copy()).pin_memory()
+
+    def dests(c, lay):
+        d = {"h_cur": c._keep_alive[1]["hidden"], "pos": c._keep_alive[2]["pos"], "lay_cu_seqlens": lay.cu_seqlens,
+             "lay_img_cu": lay.img_cu, "lay_img_start": lay.img_start, "lay_img_len": lay.img_len,
+             "keep_ratio": c._keep_alive[0]}
+        sc = c._keep_alive[3]
+        if crit == "hidden_variation":
+            d["h_prior"] = sc["h_prior"]
+        else:
+            d["q"], d["k"] = sc["q"], sc["k"]
+        return d
+
+    dst = [dests(c, lay) for c, lay in zip(calls, layouts)]
+    outs = []
+    for c in calls:
+        b = c.buffers
+        outs.append([b.kept_idx[:b.n_kept], b.budgets, b.out_cu_seqlens] + list(b.outputs.values()))
+    host_out = [[torch.empty(o.shape, dtype=o.dtype).pin_memory() for o in outs[j]] for j in range(2)]
+    s_in, s_comp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    in_done = [torch.cuda.Event() for _ in range(2)]
+    comp_done = [torch.cuda.Event() for _ in range(2)]
+    out_done = [torch.cuda.Event() for _ in range(2)]
+    for j in range(2):  # every buffer starts free
+        comp_done[j].record(s_comp)
+        out_done[j].record(s_out)
+
+    def step(i):
+        j = i & 1
+        s_in.wait_event(comp_done[j])  # step i - 2 has read these inputs
+        with torch.cuda.stream(s_in):
+            for k, h in host_in.items():
+                d = dst[j][k]
+                d.view(torch.int16 if d.dtype == torch.bfloat16 else d.dtype).copy_(
+                    h.view(torch.int16) if d.dtype == torch.bfloat16 else h, non_blocking=True)
+        in_done[j].record(s_in)
+        s_comp.wait_event(in_done[j])
+        s_comp.wait_event(out_done[j])  # step i - 2's outputs have been copied out
+        calls[j].run(s_comp)
+        comp_done[j].record(s_comp)
+        s_out.wait_event(comp_done[j])
+        with torch.cuda.stream(s_out):
+            for o, h in zip(outs[j], host_out[j]):
+                h.copy_(o, non_blocking=True)
+        out_done[j].record(s_out)
+
+    steps = max(4, min(50, args.e2e_steps))
+    for i in range(4):
+        step(i)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(s_in)
+    s_comp.wait_stream(s_in)
+    s_out.wait_stream(s_in)
+    for i in range(steps):
+        step(i)
+    s_out.wait_stream(s_comp)
+    s_out.wait_stream(s_in)
+    ev1.record(s_out)
+    torch.cuda.synchronize()
+    for c in calls:
+        st = A.read_device_status(c.buffers.workspace)
+        if st != A.OK:
+            raise RuntimeError(f"device status after the pipelined steps: {A.status_string(st)}")
+    # the last step's outputs equal those of the serial path
+    for o, h in zip(outs[(steps - 1) & 1], host_out[(steps - 1) & 1]):
+        if not torch.equal(o.cpu(), h):
+            raise RuntimeError("pipelined end-to-end outputs differ from the device outputs")
+    ms = ev0.elapsed_time(ev1) / steps
+    n_vis = int(wl.layout.n_visual_per_request().sum())
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+    d2h = sum(o.numel() * o.element_size() for o in outs[0])
+    return {"value": round(n_vis / (ms * 1e-3), 1), "unit": UNIT, "ms_per_step": round(ms, 4),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": steps,
+            "launch": "two prepared calls alternating; copy-in, compute and copy-out streams overlap consecutive steps"}
 
 
 # ---------------------------------------------------------------- CPU oracle (baseline / reference arm)
