@@ -163,11 +163,19 @@ int device_sm_count() {
   return cached[dev];
 }
 
+// SMs the scoring kernel leaves to the selection kernel, at most.
+constexpr int kMaxReserveSms = 32;
+
 int prune_reserve_sms(const avtp_layout_t& L) {
   if (L.n_tokens > 32768 || L.n_images < 1) return 0;
   const int64_t ctas = prune_warm_ctas(L);
+  // one SM per selection CTA: CTAs packed on one SM slow each other's budget rule
+  // (measured: the stage 1.5-2 us longer on the Qwen3-VL-8B-shaped request with four
+  // per SM). Past kMaxReserveSms they share SMs, as many as the occupancy allows.
+  if (ctas <= kMaxReserveSms) return static_cast<int>(ctas);
   const int per_sm = alloc_select_ctas_per_sm();
-  return static_cast<int>((ctas + per_sm - 1) / per_sm);
+  const int64_t packed = (ctas + per_sm - 1) / per_sm;
+  return static_cast<int>(packed > kMaxReserveSms ? packed : kMaxReserveSms);
 }
 
 int prune_warm_ctas(const avtp_layout_t& L) {
