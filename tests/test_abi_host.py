@@ -73,6 +73,35 @@ def test_kept_count_matches_oracle_budget_rule(lib):
         assert avtp.kept_count_host(host, kr) == expect
 
 
+def test_kept_count_from_visual_counts_matches_the_layout_form(lib):
+    # avtp_kept_count_vis_host sizes a later progressive stage from per-request visual
+    # counts; its total, offsets and kept visual counts follow the oracle's budget rule
+    rng = np.random.default_rng(23)
+    for _ in range(50):
+        R = int(rng.integers(1, 6))
+        reqs = []
+        for _ in range(R):
+            segs = [("t", int(rng.integers(0, 40)))]
+            for _ in range(int(rng.integers(0, 8))):
+                segs += [("i", int(rng.integers(1, 1500))), ("t", int(rng.integers(0, 4)))]
+            reqs.append(segs)
+        lay = synth.Layout.from_segments(reqs)
+        kr = rng.choice(np.array([0.0, 0.05, 0.25, 0.33, 0.5, 0.79, 1.0], dtype=np.float32), size=R)
+        vis = lay.n_visual_per_request().astype(np.int32)
+        n, out_cu, out_nv = avtp.kept_count_vis_host(lay.cu_seqlens, vis, kr)
+        host = dict(cu_seqlens=lay.cu_seqlens, img_cu=lay.img_cu, img_len=lay.img_len)
+        assert n == avtp.kept_count_host(host, kr)
+        assert out_cu[0] == 0 and out_cu[-1] == n
+        for r in range(R):
+            kept_vis = O.global_budget(kr[r], int(vis[r]))
+            assert out_nv[r] == kept_vis
+            T_r = int(lay.cu_seqlens[r + 1] - lay.cu_seqlens[r])
+            assert out_cu[r + 1] - out_cu[r] == kept_vis + T_r - int(vis[r])
+    with pytest.raises(avtp.AVTPError):  # more visual tokens than the request holds
+        avtp.kept_count_vis_host(np.array([0, 4], dtype=np.int32), np.array([5], dtype=np.int32),
+                                 np.array([0.5], dtype=np.float32))
+
+
 def test_kept_count_rejects_bad_ratio(lib):
     host = dict(cu_seqlens=np.array([0, 10]), img_cu=np.array([0, 1]), img_len=np.array([5]))
     with pytest.raises(avtp.AVTPError):
