@@ -40,6 +40,7 @@ _CRITERIA = {"hidden_variation": CRIT_HIDDEN_VARIATION, "text_attention": CRIT_T
 
 
 class AVTPError(RuntimeError):
+    """A non-OK status from the library: ``code`` (an avtp_status_t value) and the call it came from."""
     def __init__(self, code: int, where: str):
         self.code = int(code)
         super().__init__(f"{where}: {status_string(code)} (status {code})")
@@ -97,6 +98,7 @@ SIGNATURES = {
 
 
 def library_path() -> str:
+    """Path of the in-tree libavtp.so that ``load()`` opens."""
     return _build.LIB_PATH
 
 
@@ -121,6 +123,7 @@ def load() -> ctypes.CDLL:
 
 
 def status_string(code: int) -> str:
+    """avtp_status_string: static English text for a status code."""
     return load().avtp_status_string(int(code)).decode()
 
 
@@ -155,6 +158,7 @@ class Layout:
 
     @staticmethod
     def from_host(cu_seqlens, img_cu, img_start, img_len, device="cuda") -> "Layout":
+        """Copies host layout arrays (int32) to ``device`` and keeps the host copies."""
         host = {k: np.ascontiguousarray(np.asarray(v, dtype=np.int32))
                 for k, v in dict(cu_seqlens=cu_seqlens, img_cu=img_cu, img_start=img_start, img_len=img_len).items()}
         dev = {k: torch.from_numpy(v.copy()).to(device) for k, v in host.items()}
@@ -162,18 +166,22 @@ class Layout:
 
     @property
     def n_requests(self) -> int:
+        """R, the number of varlen-packed requests."""
         return int(self.host["cu_seqlens"].shape[0] - 1)
 
     @property
     def n_images(self) -> int:
+        """Images over all requests."""
         return int(self.host["img_cu"][-1])
 
     @property
     def n_tokens(self) -> int:
+        """T, the packed tokens over all requests."""
         return int(self.host["cu_seqlens"][-1])
 
     @property
     def n_vis_per_request(self) -> np.ndarray:
+        """Visual tokens of each request (int32 [R])."""
         if "n_vis" in self.host:
             return self.host["n_vis"]
         csum = np.concatenate([[0], np.cumsum(self.host["img_len"].astype(np.int64))])
@@ -181,9 +189,11 @@ class Layout:
 
     @property
     def n_text(self) -> int:
+        """Text tokens over all requests."""
         return self.n_tokens - int(self.n_vis_per_request.astype(np.int64).sum())
 
     def c(self) -> _Layout:
+        """The avtp_layout_t the C calls take (pointers into the device tensors)."""
         return _Layout(self.n_requests, self.n_images, self.n_tokens, _ptr(self.cu_seqlens), _ptr(self.img_cu),
                        _ptr(self.img_start) if self.n_images else None, _ptr(self.img_len) if self.n_images else None)
 
@@ -236,6 +246,7 @@ def _row_sets(rows: Sequence[Tuple[torch.Tensor, torch.Tensor]]) -> Tuple[ctypes
 
 
 def workspace_size(layout: Layout, criterion=None, **score_tensors) -> int:
+    """avtp_workspace_size: bytes of workspace a call needs for this layout and scoring setup."""
     lay = layout.c()
     sa = _score_args(criterion, max_text_tokens=layout.n_text, **score_tensors) if criterion is not None else None
     out = c_size_t()
@@ -393,6 +404,7 @@ def wait_selftest(limit_ns: int, arrive: bool, workspace: torch.Tensor, stream=N
 
 
 def read_device_status(workspace: torch.Tensor, stream=None) -> int:
+    """avtp_read_device_status: waits for ``stream`` and returns the workspace's status word."""
     out = c_int32()
     _check(load().avtp_read_device_status(_ptr(workspace), _stream(stream), ctypes.byref(out)),
            "avtp_read_device_status")
@@ -414,6 +426,7 @@ class PruneBuffers:
 
 def prune_buffers(layout: Layout, keep_ratio_host: np.ndarray, criterion, score_tensors: Dict[str, torch.Tensor],
                   rows: Dict[str, torch.Tensor], planes: Dict[str, torch.Tensor]) -> PruneBuffers:
+    """Every output buffer and the workspace of an avtp_prune call, sized on the host (no device read)."""
     dev = layout.cu_seqlens.device
     n_kept = kept_count_host(layout.host, keep_ratio_host)
     outputs = {}
@@ -463,6 +476,7 @@ class PruneCall:
         self._keep_alive = (keep_ratio, rows, planes, score_tensors)
 
     def run(self, stream=None, step_events: Optional[Sequence] = None) -> PruneBuffers:
+        """Launches the prepared avtp_prune call on ``stream``; ``step_events`` (5 CUDA events) times its steps."""
         b = self.buffers
         ev = None
         if step_events is not None:  # 5 events: start, after validation, scoring, allocation+selection, compaction
