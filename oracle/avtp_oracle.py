@@ -80,7 +80,10 @@ SUM_MAGNITUDE_BITS = 42  # |S_i| <= n_i * 2^42: scores clamped to +-2^10, 32 fra
 # helpers
 # ----------------------------------------------------------------------------
 def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
-    """Decode bf16 bit patterns (uint16) to fp64 (exact widening)."""
+    """Decode bf16 bit patterns (uint16) to fp64 (exact widening).
+
+    Input decoding only, not a step of the paper's method.
+    """
     u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
     return u.view(np.float32).astype(np.float64)
 
@@ -128,6 +131,7 @@ def score_hidden_variation(layout, h_cur: np.ndarray, h_prior: np.ndarray) -> np
 # ----------------------------------------------------------------------------
 def attention_logits(layout, q, k, r: int, h: int, n_q_heads: int, n_kv_heads: int, scale: float):
     """Scaled logits of request r, head h: text queries (rows) x all request keys.
+    Follows paper §3.3.2, the attention of text queries to visual tokens; grouped-query heads.
 
     Returns ``(z, text_local)``; ``z`` is fp64 [|Q_r|, T_r] with ``-inf`` where the key
     lies after the query (causal mask).
@@ -147,13 +151,17 @@ def attention_logits(layout, q, k, r: int, h: int, n_q_heads: int, n_kv_heads: i
 
 
 def logsumexp_rows(z: np.ndarray) -> np.ndarray:
-    """Natural-log sum of exp over each row, with max subtraction."""
+    """Natural-log sum of exp over each row, with max subtraction.
+
+    Follows paper §3.3.2, the softmax normaliser.
+    """
     m = np.max(z, axis=1)
     return m + np.log(np.sum(np.exp(z - m[:, None]), axis=1))
 
 
 def text_lse(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float) -> np.ndarray:
     """Per (head, text query) natural-log LSE of the scaled causal logits: fp64 [Hq, T].
+    Follows paper §3.3.2; the normaliser a FlashAttention forward also returns (§3.2).
 
     This is the normaliser a FlashAttention-style forward pass keeps per query row;
     visual rows are left 0.
@@ -172,6 +180,7 @@ def text_lse(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float) -> np.
 def score_text_attention(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float,
                          lse: Optional[np.ndarray] = None) -> np.ndarray:
     """Mean over heads and text queries of the causal softmax probability of each visual key.
+    Follows paper §3.3.2, the attention quantity kept per visual token.
 
     ``q``: bf16 bits [T, Hq, d]; ``k``: bf16 bits [T, Hkv, d]; ``lse`` (optional) [Hq, T]
     natural-log normalisers for the text rows; when given they replace the
@@ -203,12 +212,18 @@ def score_text_attention(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: f
 # Step 2: per-image sums, adaptive ratios and integer budgets (paper §3.3.3, App. A.2)
 # ----------------------------------------------------------------------------
 def to_fp32(scores: np.ndarray) -> np.ndarray:
-    """The interface type of scores is fp32 (round to nearest)."""
+    """The interface type of scores is fp32 (round to nearest).
+
+    The paper fixes no precision; fp32 is the scores' type at the library boundary.
+    """
     return np.asarray(scores, dtype=np.float64).astype(np.float32)
 
 
 def fixed_point(scores_f32: np.ndarray) -> np.ndarray:
-    """``rint(fx(s) * 2^32)`` as int64; fx: NaN -> 0, clamp to [-2^10, 2^10]."""
+    """``rint(fx(s) * 2^32)`` as int64; fx: NaN -> 0, clamp to [-2^10, 2^10].
+
+    Follows paper §3.3.3, the terms of the per-image sums.
+    """
     s = np.asarray(scores_f32, dtype=np.float32).astype(np.float64)
     s = np.where(np.isnan(s), 0.0, s)
     s = np.clip(s, -FX_SCORE_LIMIT, FX_SCORE_LIMIT)
@@ -216,7 +231,10 @@ def fixed_point(scores_f32: np.ndarray) -> np.ndarray:
 
 
 def image_sums(layout, scores_f32: np.ndarray) -> np.ndarray:
-    """Fixed-point per-image sums ``S_i`` (int64 [n_img]) of the fp32 scores."""
+    """Fixed-point per-image sums ``S_i`` (int64 [n_img]) of the fp32 scores.
+
+    Follows paper §3.3.3, the sums behind the mean importance Ibar_i.
+    """
     fx = fixed_point(scores_f32)
     n_img = len(layout.img_len)
     out = np.zeros(n_img, dtype=np.int64)
@@ -227,7 +245,10 @@ def image_sums(layout, scores_f32: np.ndarray) -> np.ndarray:
 
 
 def global_budget(keep_ratio_f32: float, n_vis: int) -> int:
-    """``B_r = floor(keep_ratio * N_vis + 0.5)`` with the fp32 ratio widened to fp64."""
+    """``B_r = floor(keep_ratio * N_vis + 0.5)`` with the fp32 ratio widened to fp64.
+
+    Follows paper §3.3.3 and §4.1, the request's keep ratio.
+    """
     kr = float(np.float32(keep_ratio_f32))
     return int(math.floor(kr * float(n_vis) + 0.5))
 
@@ -237,19 +258,28 @@ def _clamp(x, lo, hi):
 
 
 def reciprocal(n: int) -> int:
-    """``floor(2^62 / n)``: the fixed-point reciprocal the per-image means are taken with."""
+    """``floor(2^62 / n)``: the fixed-point reciprocal the per-image means are taken with.
+
+    Follows paper §3.3.3, exact integer form of the means.
+    """
     return (1 << RECIP_BITS) // int(n)
 
 
 def round_shift(x: int, s: int) -> int:
-    """``x / 2^s`` rounded to nearest with ties upward (``floor(x / 2^s + 1/2)``); s <= 0 shifts left."""
+    """``x / 2^s`` rounded to nearest with ties upward (``floor(x / 2^s + 1/2)``); s <= 0 shifts left.
+
+    Follows paper §3.3.3, exact integer form of the ratios.
+    """
     if s <= 0:
         return x << (-s)
     return (x + (1 << (s - 1))) >> s
 
 
 def fp32_parts(v) -> Tuple[int, int]:
-    """Exact decomposition of an fp32 value as ``M * 2^E`` with an integer ``|M| < 2^24``."""
+    """Exact decomposition of an fp32 value as ``M * 2^E`` with an integer ``|M| < 2^24``.
+
+    Follows paper §3.3.3, exact integer form of alpha and r_base.
+    """
     f = float(np.float32(v))
     if f == 0.0:
         return 0, 0
@@ -300,19 +330,26 @@ def adaptive_ratio_grid(S: Sequence[int], n: Sequence[int], r_base_f32, alpha_f3
 
 
 def ratio_to_grid(r: float) -> int:
-    """A ratio on the 2^-40 grid: ``rint(clamp(r, -2^20, 2^20) * 2^40)`` (exact integer)."""
+    """A ratio on the 2^-40 grid: ``rint(clamp(r, -2^20, 2^20) * 2^40)`` (exact integer).
+
+    Follows paper §3.3.3 and App. A.2, ratios and clamps on one grid.
+    """
     r = _clamp(r, -RATIO_LIMIT, RATIO_LIMIT)
     return int(np.rint(r * float(2 ** RATIO_FRAC_BITS)))
 
 
 def kept_mass(R: Sequence[int], n: Sequence[int], lam: int, R_min: int, R_max: int) -> int:
-    """``G(lambda) = sum_i n_i * clamp(R_i + lambda, R_min, R_max)`` in 2^-40 token units (exact)."""
+    """``G(lambda) = sum_i n_i * clamp(R_i + lambda, R_min, R_max)`` in 2^-40 token units (exact).
+
+    Follows paper App. A.2, the clamped total.
+    """
     return sum(int(n[i]) * _clamp(int(R[i]) + lam, R_min, R_max) for i in range(len(n)))
 
 
 def water_fill(R: Sequence[int], n: Sequence[int], B: int, R_min: int, R_max: int) -> int:
     """The smallest grid shift lambda with ``G(lambda) >= B * 2^40``, searched in
     ``[R_min - max R, R_max - min R]`` (the ends when no point inside qualifies).
+    Follows paper App. A.2, clamps with the total restored.
 
     G is non-decreasing in lambda, so integer bisection finds it exactly.
     """
@@ -334,7 +371,10 @@ def water_fill(R: Sequence[int], n: Sequence[int], B: int, R_min: int, R_max: in
 
 def integer_budgets(R: Sequence[int], n: Sequence[int], B: int, lam: int,
                     R_min: int, R_max: int) -> List[int]:
-    """Largest-remainder rounding of ``x_i = n_i * clamp(R_i + lambda)`` to a total of B."""
+    """Largest-remainder rounding of ``x_i = n_i * clamp(R_i + lambda)`` to a total of B.
+
+    Follows paper §3.3.3, integer budgets summing to the global budget.
+    """
     m = len(n)
     one = 1 << RATIO_FRAC_BITS
     x = [int(n[i]) * _clamp(int(R[i]) + lam, R_min, R_max) for i in range(m)]
@@ -358,6 +398,7 @@ def integer_budgets(R: Sequence[int], n: Sequence[int], B: int, lam: int,
 def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
              r_min: float = 0.05, r_max: float = 0.95, relative: bool = False) -> Dict[str, np.ndarray]:
     """Per-image budgets ``k_i`` and the packed output offsets ``out_cu_seqlens``.
+    Follows paper §3.3.3 with the clamps of App. A.2.
 
     fp32 parameters (``keep_ratio``, ``alpha``, ``r_min``, ``r_max``) enter exactly.
     The sums must satisfy ``|S_i| <= n_i * 2^42`` (every fixed-point score is within
@@ -405,14 +446,20 @@ def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
 # Step 3: per-image top-k, text kept, ascending order (paper §3.1, §3.3.3)
 # ----------------------------------------------------------------------------
 def rank_key(score: float, pos: int):
-    """Sort key: score descending, position ascending; NaN below every number."""
+    """Sort key: score descending, position ascending; NaN below every number.
+
+    Follows paper §3.3.3, the most important tokens first.
+    """
     if math.isnan(score):
         return (1, 0.0, pos)
     return (0, -score, pos)
 
 
 def select(layout, scores_f32: np.ndarray, budgets: np.ndarray) -> np.ndarray:
-    """Packed global indices of the kept tokens (int32), ascending within each request."""
+    """Packed global indices of the kept tokens (int32), ascending within each request.
+
+    Follows paper §3.1, an order-preserving subsequence; §3.3.3, k_i tokens per image.
+    """
     sc = np.asarray(scores_f32, dtype=np.float32)
     kept: List[int] = []
     for r in range(len(layout.cu_seqlens) - 1):
@@ -432,12 +479,18 @@ def select(layout, scores_f32: np.ndarray, budgets: np.ndarray) -> np.ndarray:
 # Step 4: compaction (paper §3.1)
 # ----------------------------------------------------------------------------
 def compact(kept_idx: np.ndarray, rows: np.ndarray) -> np.ndarray:
-    """``out[j] = rows[kept_idx[j]]`` along axis 0 (any dtype, bit-exact)."""
+    """``out[j] = rows[kept_idx[j]]`` along axis 0 (any dtype, bit-exact).
+
+    Follows paper §3.1, E_pruned = p(E_v).
+    """
     return np.asarray(rows)[np.asarray(kept_idx, dtype=np.int64)]
 
 
 def compact_planes(kept_idx: np.ndarray, planes: np.ndarray) -> np.ndarray:
-    """Gather along the token axis of a [P, T] array (e.g. M-RoPE position ids)."""
+    """Gather along the token axis of a [P, T] array (e.g. M-RoPE position ids).
+
+    Follows paper §3.1, the position ids of the kept tokens.
+    """
     return np.asarray(planes)[:, np.asarray(kept_idx, dtype=np.int64)]
 
 
@@ -448,6 +501,7 @@ def compact_planes(kept_idx: np.ndarray, planes: np.ndarray) -> np.ndarray:
 # ----------------------------------------------------------------------------
 def pruned_layout(layout, kept_idx: np.ndarray, out_cu_seqlens: np.ndarray) -> Dict[str, np.ndarray]:
     """Image spans of the pruned batch, read off the kept tokens.
+    Follows paper §3.3.2, the progressive schedule; §3.3.1, h_prior.
 
     In request r of the pruned batch, image i starts at the number of kept tokens of the
     request that lie before the image's span, and holds the kept tokens inside the span
@@ -478,6 +532,7 @@ def prune(layout, *, criterion: str = "hidden_variation", keep_ratio, alpha: flo
           scale=None, lse=None, scores_f32=None, rows: Optional[Dict[str, np.ndarray]] = None,
           planes: Optional[Dict[str, np.ndarray]] = None) -> Dict[str, np.ndarray]:
     """score -> per-image sums -> budgets -> selection -> compaction.
+    Follows paper §3.1-§3.3, the whole stage.
 
     ``scores_f32`` (optional) replaces step 1, to run steps 2-4 on given scores.
     ``rows``: name -> [T, ...] arrays gathered along axis 0; ``planes``: name ->
