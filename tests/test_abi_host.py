@@ -45,6 +45,30 @@ def test_library_exports_every_declared_symbol(lib):
         assert name in avtp.SIGNATURES  # the binding wraps each one
 
 
+def _c_type_matches(c_type: str, ct) -> bool:
+    c_type = " ".join(c_type.replace("const", " ").split())
+    if "*" in c_type or c_type == "avtp_stream_t":
+        return ct in (ctypes.c_void_p, ctypes.c_char_p) or (isinstance(ct, type) and issubclass(ct, ctypes._Pointer))
+    return {"int64_t": ctypes.c_int64, "int32_t": ctypes.c_int32, "size_t": ctypes.c_size_t,
+            "avtp_status_t": ctypes.c_int, "int": ctypes.c_int}.get(c_type.split()[0]) is ct
+
+
+def test_binding_signatures_match_the_header():
+    # every argument of every declared call: same count, and pointer / integer width alike
+    text = open(HEADER).read()
+    decls = re.findall(r"AVTP_API\s+([\w\s\*]+?)\b(avtp_\w+)\s*\(([^;]*?)\)\s*;", text, re.S)
+    assert len(decls) == len(declared_functions())
+    for ret, name, params in decls:
+        res, args = avtp.SIGNATURES[name]
+        plist = [] if params.strip() in ("", "void") else [p.strip() for p in params.split(",")]
+        assert len(plist) == len(args), name
+        for p, ct in zip(plist, args):
+            c_type = re.sub(r"\b\w+$", "", p).strip() if "*" not in p.split()[-1] else p
+            c_type = p[:p.rfind("*") + 1] if "*" in p else c_type
+            assert _c_type_matches(c_type, ct), (name, p, ct)
+        assert _c_type_matches(ret.strip(), res), (name, ret, res)
+
+
 def test_status_strings(lib):
     assert avtp.status_string(avtp.OK) == "ok"
     assert "workspace" in avtp.status_string(avtp.ERR_WORKSPACE)
