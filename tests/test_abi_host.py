@@ -6,6 +6,7 @@ every invalid-argument path returns before the first CUDA call.
 import ctypes
 import os
 import re
+import shutil
 import subprocess
 
 import numpy as np
@@ -221,3 +222,37 @@ def test_host_validation_of_wait_selftest_arguments(lib):
     assert lib.avtp_wait_selftest(1_000_000, 0, None, 256, None) == avtp.ERR_WORKSPACE
     assert lib.avtp_wait_selftest(1_000_000, 0, FAKE + 8, 256, None) == avtp.ERR_WORKSPACE
     assert lib.avtp_wait_selftest(1_000_000, 0, FAKE, 8, None) == avtp.ERR_WORKSPACE
+
+
+def test_binding_structs_match_the_c_layout(tmp_path):
+    if shutil.which("gcc") is None:
+        pytest.skip("needs a host C compiler")
+    # sizeof and every field offset of the ABI structs, from the header compiled by the
+    # host C compiler, against the ctypes mirrors of the binding
+    structs = {"avtp_layout_t": avtp._Layout, "avtp_score_args_t": avtp._ScoreArgs,
+               "avtp_alloc_args_t": avtp._AllocArgs, "avtp_rows_t": avtp._Rows}
+    renamed = {"in_": "in"}  # a Python keyword in the mirror
+    lines = ["#include <stdio.h>", "#include <stddef.h>", '#include "avtp.h"', "int main(void) {"]
+    for c_name, py in structs.items():
+        lines.append(f'  printf("{c_name} size %zu\\n", sizeof({c_name}));')
+        for f, _ in py._fields_:
+            cf = renamed.get(f, f)
+            lines.append(f'  printf("{c_name} {f} %zu\\n", offsetof({c_name}, {cf}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "abi.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "abi"
+    cc = subprocess.run(["gcc", "-std=c11", "-I", os.path.dirname(HEADER), str(src), "-o", str(exe)],
+                        capture_output=True, text=True)
+    assert cc.returncode == 0, cc.stderr
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    got = {}
+    for ln in out:
+        if ln:
+            c_name, field, value = ln.split()
+            got[(c_name, field)] = int(value)
+    for c_name, py in structs.items():
+        assert got[(c_name, "size")] == ctypes.sizeof(py), c_name
+        for f, _ in py._fields_:
+            assert got[(c_name, f)] == getattr(py, f).offset, (c_name, f)
+
