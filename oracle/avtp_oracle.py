@@ -35,44 +35,33 @@ the design notes of the repository):
   fp32-rounded score, with ``fx`` mapping NaN to 0 and clamping to +-2^10, so that
   every summation order gives the same integer.
 * ``Ibar_avg`` is the token-weighted mean ``sum_i S_i / 2^32 / N_vis``.
-* The adaptive ratios are computed in exact integer arithmetic on a 2^-40 grid:
-  means through fixed-point reciprocals ``floor(2^62 / n)``, fp32 alpha and
-  r_base decomposed exactly, one rounding (nearest, ties upward) per product
-  (see ``adaptive_ratio_grid``).
-* The global budget is ``B_r = floor(keep_ratio_r * N_vis_r + 0.5)``.
+* The budget rule is computed in exact rational arithmetic (``fractions.Fraction``):
+  the means, the ratios, the shift and the kept masses are the plain formulas, and the
+  fp32 parameters (keep ratio, alpha, clamps) enter as the exact values they hold.
+* The global budget is ``B_r = floor(keep_ratio_r * N_vis_r + 1/2)``.
 * ``relative=1`` replaces the additive rule by ``r_i = r_base*(1 + alpha*(Ibar_i/Ibar_avg - 1))``
   (``r_base`` when ``Ibar_avg == 0``); criterion 1B's raw values are of order
   1/N, where the additive rule would leave every ratio at ``r_base``.
-* The clamps go on the same grid: ``R_min = rint(r_min * 2^40)``, ``R_max`` likewise.
-* A shift lambda (water-fill) restores the clamped total: lambda is the smallest
-  grid value with ``G(lambda) = sum_i n_i * clamp(R_i + lambda, R_min, R_max) >= B_r * 2^40``
-  on ``[R_min - max R, R_max - min R]`` (an end of that range if none inside
-  qualifies). G is exact integer arithmetic, so lambda is a definition, not the
-  output of one particular search.
-* Integer budgets: ``x_i = n_i * clamp(R_i + lambda)`` (2^-40 token units),
-  ``k_i = min(floor(x_i), n_i)``, then largest remainder (ties to the lower image
-  index) until ``sum k_i = B_r``; a surplus is removed from the smallest
-  remainders (ties to the higher index).
+* A shift lambda (water-fill) restores the clamped total:
+  ``sum_i n_i * clamp(r_i + lambda, r_min, r_max) = B_r``; when B_r lies outside
+  ``[N r_min, N r_max]`` every image takes the nearer clamp.
+* Integer budgets: ``x_i = n_i * clamp(r_i + lambda)``, ``k_i = min(floor(x_i), n_i)``,
+  then largest remainder (ties to the lower image index) until ``sum k_i = B_r``; a
+  surplus is removed from the smallest remainders (ties to the higher index).
 * Top-k order: score descending, position ascending; NaN ranks below -inf;
   -0 equals +0.
-
-Apart from the fp64 global budget (``kr * N + 0.5``, exact for fp32 ratios and
-N < 2^29) the budget rule is exact integer arithmetic, so a device implementation
-of the same integer steps reproduces every budget exactly.
 """
 from __future__ import annotations
 
 import math
-from typing import Dict, List, Optional, Sequence, Tuple
+from fractions import Fraction
+from typing import Dict, List, Optional, Sequence
 
 import numpy as np
 
 FX_FRAC_BITS = 32
 FX_SCORE_LIMIT = 1024.0  # |score| is clamped to 2^10 before the fixed-point conversion
 NORM_EPS = 1e-8
-RATIO_FRAC_BITS = 40     # ratios, shifts and kept masses live on a 2^-40 integer grid
-RATIO_LIMIT = 2.0 ** 20  # ratios are saturated to +-2^20 before going on the grid
-RECIP_BITS = 62          # per-image means are taken with floor(2^62 / n) reciprocals
 SUM_MAGNITUDE_BITS = 42  # |S_i| <= n_i * 2^42: scores clamped to +-2^10, 32 fraction bits
 
 
@@ -245,141 +234,94 @@ def image_sums(layout, scores_f32: np.ndarray) -> np.ndarray:
 
 
 def global_budget(keep_ratio_f32: float, n_vis: int) -> int:
-    """``B_r = floor(keep_ratio * N_vis + 0.5)`` with the fp32 ratio widened to fp64.
+    """``B_r = floor(keep_ratio * N_vis + 1/2)``, the fp32 ratio taken exactly.
 
     Follows paper §3.3.3 and §4.1, the request's keep ratio.
     """
-    kr = float(np.float32(keep_ratio_f32))
-    return int(math.floor(kr * float(n_vis) + 0.5))
+    return math.floor(Fraction(float(np.float32(keep_ratio_f32))) * int(n_vis) + Fraction(1, 2))
 
 
 def _clamp(x, lo, hi):
     return min(max(x, lo), hi)
 
 
-def reciprocal(n: int) -> int:
-    """``floor(2^62 / n)``: the fixed-point reciprocal the per-image means are taken with.
+def image_means(S: Sequence[int], n: Sequence[int]) -> List[Fraction]:
+    """``Ibar_i = S_i / (2^32 n_i)``: the mean importance of each image, exactly.
 
-    Follows paper §3.3.3, exact integer form of the means.
+    Follows paper §3.3.3, the mean importance of an image.
     """
-    return (1 << RECIP_BITS) // int(n)
+    return [Fraction(int(S[i]), (1 << FX_FRAC_BITS) * int(n[i])) for i in range(len(n))]
 
 
-def round_shift(x: int, s: int) -> int:
-    """``x / 2^s`` rounded to nearest with ties upward (``floor(x / 2^s + 1/2)``); s <= 0 shifts left.
+def average_importance(S: Sequence[int], n: Sequence[int]) -> Fraction:
+    """``Ibar_avg = sum_i S_i / (2^32 N_vis)``, the token-weighted mean over the request's images.
 
-    Follows paper §3.3.3, exact integer form of the ratios.
+    Follows paper §3.3.3, the average importance across images (token-weighted reading).
     """
-    if s <= 0:
-        return x << (-s)
-    return (x + (1 << (s - 1))) >> s
+    return Fraction(sum(int(v) for v in S), (1 << FX_FRAC_BITS) * sum(int(v) for v in n))
 
 
-def fp32_parts(v) -> Tuple[int, int]:
-    """Exact decomposition of an fp32 value as ``M * 2^E`` with an integer ``|M| < 2^24``.
+def adaptive_ratios(S: Sequence[int], n: Sequence[int], r_base_f32, alpha_f32, relative: bool) -> List[Fraction]:
+    """The adaptive keep ratio of every image, before the clamps, as exact rationals.
 
-    Follows paper §3.3.3, exact integer form of alpha and r_base.
+    Follows paper §3.3.3: ``r_i = r_base + alpha * (Ibar_i - Ibar_avg)``; with ``relative``,
+    ``r_i = r_base * (1 + alpha * (Ibar_i / Ibar_avg - 1))`` (``r_base`` when ``Ibar_avg == 0``).
+    The fp32 parameters enter as the exact values they hold.
     """
-    f = float(np.float32(v))
-    if f == 0.0:
-        return 0, 0
-    m, e = math.frexp(f)  # f = m * 2^e with 0.5 <= |m| < 1
-    return int(m * (1 << 24)), e - 24
+    r_base = Fraction(float(np.float32(r_base_f32)))
+    alpha = Fraction(float(np.float32(alpha_f32)))
+    ibar = image_means(S, n)
+    avg = average_importance(S, n)
+    if not relative:
+        return [r_base + alpha * (ib - avg) for ib in ibar]
+    if avg == 0:
+        return [r_base for _ in ibar]
+    return [r_base * (1 + alpha * (ib / avg - 1)) for ib in ibar]
 
 
-def _sat(x: int, lim: int) -> int:
-    return min(max(x, -lim), lim)
+def clamped_total(r: Sequence[Fraction], n: Sequence[int], lam: Fraction, r_min: Fraction, r_max: Fraction) -> Fraction:
+    """``G(lambda) = sum_i n_i * clamp(r_i + lambda, r_min, r_max)``: the kept total after a shift.
 
-
-def adaptive_ratio_grid(S: Sequence[int], n: Sequence[int], r_base_f32, alpha_f32,
-                        relative: bool) -> List[int]:
-    """The adaptive keep ratios of paper §3.3.3 on the 2^-40 grid, in exact integers.
-
-    Means of the fixed-point sums (units of 2^-32), through reciprocals:
-      ``Ibar_i = round(S_i * floor(2^62 / n_i) / 2^62)``, ``Ibar_avg = round(sum S * floor(2^62 / N) / 2^62)``.
-    Additive rule: ``r_i = r_base + alpha * (Ibar_i - Ibar_avg)``, i.e.
-      ``R_i = R_base + round(alpha * (Ibar_i - Ibar_avg) * 2^8)``.
-    Relative rule: ``r_i = r_base * (1 + alpha * (Ibar_i / Ibar_avg - 1))``, i.e.
-      ``R_i = R_base + round(r_base * alpha * q_i)`` with the ratio on the 2^-40 grid
-      ``q_i = sgn(Ibar_avg) * round((Ibar_i - Ibar_avg) * floor(2^62 / |Ibar_avg|) / 2^22)``
-      saturated to +-2^60, and ``R_i = R_base`` when ``Ibar_avg == 0``.
-    ``R_base = rint(r_base * 2^40)``; fp32 alpha and r_base enter as exact ``M * 2^E``;
-    every product is exact and rounded once; ``R_i`` saturates to +-2^60.
+    Follows paper App. A.2, the ratios clamped to [r_min, r_max].
     """
-    N = sum(int(x) for x in n)
-    total = sum(int(x) for x in S)
-    ibar = [round_shift(int(S[i]) * reciprocal(int(n[i])), RECIP_BITS) for i in range(len(n))]
-    avg = round_shift(total * reciprocal(N), RECIP_BITS)
-    Rb = ratio_to_grid(float(np.float32(r_base_f32)))
-    A, E = fp32_parts(alpha_f32)
-    Bm, Be = fp32_parts(r_base_f32)
-    lim = 1 << 60
-    R = []
-    for i in range(len(n)):
-        d = ibar[i] - avg
-        if not relative:
-            delta = round_shift(A * d, -(E + 8))
-        elif avg == 0:
-            delta = 0
-        else:
-            sgn = 1 if avg > 0 else -1
-            q = _sat(sgn * round_shift(d * ((1 << RECIP_BITS) // abs(avg)), RECIP_BITS - RATIO_FRAC_BITS), lim)
-            delta = round_shift(Bm * A * q, -(Be + E))
-        R.append(_sat(Rb + delta, lim))
-    return R
+    return sum((int(n[i]) * _clamp(r[i] + lam, r_min, r_max) for i in range(len(n))), Fraction(0))
 
 
-def ratio_to_grid(r: float) -> int:
-    """A ratio on the 2^-40 grid: ``rint(clamp(r, -2^20, 2^20) * 2^40)`` (exact integer).
+def water_fill(r: Sequence[Fraction], n: Sequence[int], B: int, r_min: Fraction, r_max: Fraction) -> Fraction:
+    """The shift lambda that restores the request's budget after the clamps: ``G(lambda) = B``.
+    Follows paper App. A.2, clamped ratios with the global total kept.
 
-    Follows paper §3.3.3 and App. A.2, ratios and clamps on one grid.
+    G is continuous, non-decreasing and linear between the breakpoints ``r_min - r_i`` and
+    ``r_max - r_i``. Below the lowest breakpoint every image sits at ``r_min`` and above the
+    highest at ``r_max``; when B lies outside ``[N r_min, N r_max]`` the nearer end is
+    returned (every image at that clamp). Otherwise lambda is the point where the linear
+    piece between the two breakpoints that bracket B reaches B; where G is flat at B
+    (every image clamped) any such point gives the same clamped ratios.
     """
-    r = _clamp(r, -RATIO_LIMIT, RATIO_LIMIT)
-    return int(np.rint(r * float(2 ** RATIO_FRAC_BITS)))
+    pts = sorted(set([r_min - v for v in r] + [r_max - v for v in r]))
+    G = [clamped_total(r, n, p, r_min, r_max) for p in pts]
+    if B <= G[0]:
+        return pts[0]
+    if B >= G[-1]:
+        return pts[-1]
+    for k in range(len(pts) - 1):
+        if G[k] < B <= G[k + 1]:
+            return pts[k] + (B - G[k]) * (pts[k + 1] - pts[k]) / (G[k + 1] - G[k])
+    raise AssertionError("unreachable: G is non-decreasing and B lies within its range")
 
 
-def kept_mass(R: Sequence[int], n: Sequence[int], lam: int, R_min: int, R_max: int) -> int:
-    """``G(lambda) = sum_i n_i * clamp(R_i + lambda, R_min, R_max)`` in 2^-40 token units (exact).
+def integer_budgets(x: Sequence[Fraction], n: Sequence[int], B: int) -> List[int]:
+    """Largest-remainder rounding of the kept masses ``x_i`` to integers summing to B.
+    Follows paper §3.3.3, integer budgets whose total is the global budget.
 
-    Follows paper App. A.2, the clamped total.
-    """
-    return sum(int(n[i]) * _clamp(int(R[i]) + lam, R_min, R_max) for i in range(len(n)))
-
-
-def water_fill(R: Sequence[int], n: Sequence[int], B: int, R_min: int, R_max: int) -> int:
-    """The smallest grid shift lambda with ``G(lambda) >= B * 2^40``, searched in
-    ``[R_min - max R, R_max - min R]`` (the ends when no point inside qualifies).
-    Follows paper App. A.2, clamps with the total restored.
-
-    G is non-decreasing in lambda, so integer bisection finds it exactly.
-    """
-    target = int(B) << RATIO_FRAC_BITS
-    lo = R_min - max(R)
-    hi = R_max - min(R)
-    if kept_mass(R, n, lo, R_min, R_max) >= target:
-        return lo
-    if kept_mass(R, n, hi, R_min, R_max) < target:
-        return hi
-    while hi - lo > 1:  # invariant: G(lo) < target <= G(hi)
-        mid = (lo + hi) // 2
-        if kept_mass(R, n, mid, R_min, R_max) >= target:
-            hi = mid
-        else:
-            lo = mid
-    return hi
-
-
-def integer_budgets(R: Sequence[int], n: Sequence[int], B: int, lam: int,
-                    R_min: int, R_max: int) -> List[int]:
-    """Largest-remainder rounding of ``x_i = n_i * clamp(R_i + lambda)`` to a total of B.
-
-    Follows paper §3.3.3, integer budgets summing to the global budget.
+    ``k_i = floor(x_i)``; while the total is short, one more token goes to each of the
+    images still below ``n_i`` with the largest ``x_i - floor(x_i)`` (ties to the lower
+    index); while it is over, one token is taken from the images above 0 with the
+    smallest remainders (ties to the higher index).
     """
     m = len(n)
-    one = 1 << RATIO_FRAC_BITS
-    x = [int(n[i]) * _clamp(int(R[i]) + lam, R_min, R_max) for i in range(m)]
-    frac = [v % one for v in x]
-    k = [min(v // one, int(n[i])) for i, v in enumerate(x)]
+    k = [min(math.floor(v), int(n[i])) for i, v in enumerate(x)]
+    frac = [v - math.floor(v) for v in x]
     while sum(k) < B:
         need = B - sum(k)
         elig = [i for i in range(m) if k[i] < int(n[i])]
@@ -398,19 +340,19 @@ def integer_budgets(R: Sequence[int], n: Sequence[int], B: int, lam: int,
 def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
              r_min: float = 0.05, r_max: float = 0.95, relative: bool = False) -> Dict[str, np.ndarray]:
     """Per-image budgets ``k_i`` and the packed output offsets ``out_cu_seqlens``.
-    Follows paper §3.3.3 with the clamps of App. A.2.
+    Follows paper §3.3.3 with the clamps of App. A.2, in exact rational arithmetic.
 
-    fp32 parameters (``keep_ratio``, ``alpha``, ``r_min``, ``r_max``) enter exactly.
-    The sums must satisfy ``|S_i| <= n_i * 2^42`` (every fixed-point score is within
-    +-2^42), and every keep ratio must lie within the clamps ``[r_min, r_max]`` (else
-    no ratio shift meets both the clamps and the global budget); otherwise ValueError. Returns a dict with ``budgets`` int32
-    [n_img], ``out_cu_seqlens`` int32 [R+1] and, for inspection, ``ratios`` (on the
-    grid, before the clamps) and ``lam`` per request.
+    Per request: ``B = floor(r_base N_vis + 1/2)``; the ratios of ``adaptive_ratios``;
+    the shift of ``water_fill``; ``x_i = n_i clamp(r_i + lambda, r_min, r_max)``; the
+    integers of ``integer_budgets``. The sums must satisfy ``|S_i| <= n_i * 2^42`` (every
+    fixed-point score is within +-2^42), and every keep ratio must lie within the clamps
+    ``[r_min, r_max]`` (else no ratio shift meets both the clamps and the global budget);
+    otherwise ValueError. Returns ``budgets`` int32 [n_img], ``out_cu_seqlens`` int32 [R+1]
+    and, for inspection, ``ratios`` (before the clamps) and ``lam`` per request, as floats.
     """
     R = len(layout.cu_seqlens) - 1
-    alpha = float(np.float32(alpha))
-    r_min = float(np.float32(r_min))
-    r_max = float(np.float32(r_max))
+    fr_min = Fraction(float(np.float32(r_min)))
+    fr_max = Fraction(float(np.float32(r_max)))
     budgets = np.zeros(len(layout.img_len), dtype=np.int32)
     out_cu = np.zeros(R + 1, dtype=np.int32)
     ratios = np.zeros(len(layout.img_len), dtype=np.float64)
@@ -421,23 +363,21 @@ def allocate(layout, S: np.ndarray, keep_ratio: np.ndarray, alpha: float = 1.0,
         n_vis = sum(n)
         T_r = int(layout.cu_seqlens[rq + 1]) - int(layout.cu_seqlens[rq])
         n_txt = T_r - n_vis
-        r_base = float(np.float32(keep_ratio[rq]))
-        if not (r_min <= r_base <= r_max):
-            raise ValueError(f"request {rq}: keep ratio {r_base} outside the clamps [{r_min}, {r_max}]")
+        r_base = Fraction(float(np.float32(keep_ratio[rq])))
+        if not (fr_min <= r_base <= fr_max):
+            raise ValueError(f"request {rq}: keep ratio {float(r_base)} outside the clamps [{r_min}, {r_max}]")
         B = global_budget(keep_ratio[rq], n_vis)
         if i1 > i0:
             Sr = [int(v) for v in S[i0:i1]]
             for j in range(len(n)):
                 if abs(Sr[j]) > n[j] << SUM_MAGNITUDE_BITS:
                     raise ValueError(f"image {i0 + j}: |S_i| exceeds n_i * 2^{SUM_MAGNITUDE_BITS}")
-            Rg = adaptive_ratio_grid(Sr, n, r_base, alpha, relative)
-            r = [v / float(1 << RATIO_FRAC_BITS) for v in Rg]
-            R_min, R_max = ratio_to_grid(r_min), ratio_to_grid(r_max)
-            lam = water_fill(Rg, n, B, R_min, R_max)
-            k = integer_budgets(Rg, n, B, lam, R_min, R_max)
-            budgets[i0:i1] = k
-            ratios[i0:i1] = r
-            lams[rq] = lam / float(2 ** RATIO_FRAC_BITS)
+            r = adaptive_ratios(Sr, n, keep_ratio[rq], alpha, relative)
+            lam = water_fill(r, n, B, fr_min, fr_max)
+            x = [n[i] * _clamp(r[i] + lam, fr_min, fr_max) for i in range(len(n))]
+            budgets[i0:i1] = integer_budgets(x, n, B)
+            ratios[i0:i1] = [float(v) for v in r]
+            lams[rq] = float(lam)
         out_cu[rq + 1] = out_cu[rq] + B + n_txt
     return {"budgets": budgets, "out_cu_seqlens": out_cu, "ratios": ratios, "lam": lams}
 

@@ -19,12 +19,16 @@ from oracle import avtp_oracle
 SRC_PATH = inspect.getsourcefile(avtp_oracle)
 
 MUTATIONS = {
-    "ratio sign flipped": ("delta = round_shift(A * d, -(E + 8))", "delta = round_shift(-A * d, -(E + 8))"),
-    "ratio off by a factor of two": ("delta = round_shift(A * d, -(E + 8))", "delta = round_shift(A * d, -(E + 9))"),
-    "image-weighted mean": ("avg = round_shift(total * reciprocal(N), RECIP_BITS)", "avg = sum(ibar) // len(ibar)"),
-    "relative rule ignores the sign of the mean": ("sgn = 1 if avg > 0 else -1", "sgn = 1"),
-    "relative rule drops r_base": ("delta = round_shift(Bm * A * q, -(Be + E))",
-                                   "delta = round_shift(A * q, -E)"),
+    "ratio sign flipped": ("return [r_base + alpha * (ib - avg) for ib in ibar]",
+                           "return [r_base - alpha * (ib - avg) for ib in ibar]"),
+    "ratio off by a factor of two": ("return [Fraction(int(S[i]), (1 << FX_FRAC_BITS) * int(n[i])) for i in range(len(n))]",
+                                     "return [Fraction(int(S[i]), (1 << (FX_FRAC_BITS - 1)) * int(n[i])) for i in range(len(n))]"),
+    "image-weighted mean": ("return Fraction(sum(int(v) for v in S), (1 << FX_FRAC_BITS) * sum(int(v) for v in n))",
+                            "return sum(image_means(S, n), Fraction(0)) / len(n)"),
+    "relative rule drops r_base": ("return [r_base * (1 + alpha * (ib / avg - 1)) for ib in ibar]",
+                                   "return [(1 + alpha * (ib / avg - 1)) for ib in ibar]"),
+    "relative rule ignores alpha": ("return [r_base * (1 + alpha * (ib / avg - 1)) for ib in ibar]",
+                                    "return [r_base * (ib / avg) for ib in ibar]"),
     "GQA head mapping": ("g = h // (n_q_heads // n_kv_heads)", "g = h % n_kv_heads"),
     "causal mask off by one": ("visible = keys[None, :] <= text_local[:, None]",
                                "visible = keys[None, :] < text_local[:, None]"),
@@ -36,10 +40,11 @@ MUTATIONS = {
     "remainder tie to higher index": ("order = sorted(elig, key=lambda i: (-frac[i], i))",
                                       "order = sorted(elig, key=lambda i: (-frac[i], -i))"),
     "no clamp": ("return min(max(x, lo), hi)", "return x"),
-    "water-fill takes the last short shift": ("    return hi\n\n\ndef integer_budgets", "    return lo\n\n\ndef integer_budgets"),
-    "remainder from the wrong end": ("frac = [v % one for v in x]", "frac = [one - 1 - v % one for v in x]"),
-    "budget rounding floor": ("return int(math.floor(kr * float(n_vis) + 0.5))",
-                              "return int(math.floor(kr * float(n_vis)))"),
+    "water-fill takes the last short breakpoint": ("return pts[k] + (B - G[k]) * (pts[k + 1] - pts[k]) / (G[k + 1] - G[k])",
+                                                   "return pts[k]"),
+    "remainder from the wrong end": ("frac = [v - math.floor(v) for v in x]", "frac = [1 - (v - math.floor(v)) for v in x]"),
+    "budget rounding floor": ("return math.floor(Fraction(float(np.float32(keep_ratio_f32))) * int(n_vis) + Fraction(1, 2))",
+                              "return math.floor(Fraction(float(np.float32(keep_ratio_f32))) * int(n_vis))"),
     "ties by higher position": ("return (0, -score, pos)", "return (0, -score, -pos)"),
     "NaN ranked high": ("return (1, 0.0, pos)", "return (-1, 0.0, pos)"),
     "text dropped": ("keep = ~_request_visual_local(layout, r)  # text always kept",

@@ -326,32 +326,105 @@ def test_relative_rule_is_proportional_to_image_mass():
     assert np.all(np.abs(res["budgets"] - x) < 1.0)
 
 
-@pytest.mark.parametrize("relative", [False, True])
-def test_ratios_match_the_real_formula(relative):
-    # Section 3.3.3 in exact rationals: Ibar_i = S_i / (2^32 n_i), Ibar_avg = sum S / (2^32 N),
-    # r_i = r_base + alpha (Ibar_i - Ibar_avg)  or  r_base (1 + alpha (Ibar_i / Ibar_avg - 1)).
-    # The integer grid must agree to well below one token; means of either sign.
-    from fractions import Fraction as F
+def test_relative_rule_is_scale_invariant():
+    # Ibar_i / Ibar_avg does not change when every score is multiplied by the same
+    # positive factor, so neither do the relative rule's budgets; means of ~1e-7 included
     rng = np.random.default_rng(15)
-    for trial in range(80):
-        m = int(rng.integers(1, 12))
-        n = rng.integers(1, 5000, size=m)
-        sign = -1 if trial % 3 == 0 else 1
-        mean = rng.uniform(0.1, 2.0, size=m)
-        S = (sign * np.rint(mean * 2.0 ** 32) * n).astype(np.int64) + rng.integers(-n, n + 1)
-        alpha = float(np.float32(rng.choice([0.0, 0.3, 1.0, 2.0, 5.0])))
-        kr = np.float32(rng.choice([0.05, 0.125, 0.33, 0.5, 0.9]))
+    for trial in range(40):
+        m = int(rng.integers(1, 9))
+        n = rng.integers(1, 400, size=m)
         lay = synth.Layout.from_segments([[("t", 1)] + [("i", int(v)) for v in n]])
-        res = O.allocate(lay, S, np.array([kr], dtype=np.float32), alpha, 0.0, 1.0, relative)
-        N = int(n.sum())
-        avg = F(int(S.sum()), 2 ** 32 * N)
-        for i in range(m):
-            ib = F(int(S[i]), 2 ** 32 * int(n[i]))
-            if relative:
-                exact = F(float(kr)) * (1 + F(alpha) * (ib / avg - 1))
-            else:
-                exact = F(float(kr)) + F(alpha) * (ib - avg)
-            assert abs(float(F(res["ratios"][i]) - exact)) < 2.0 ** -24, (trial, i, relative)
+        S = rng.integers(1, 2 ** 12, size=m).astype(np.int64) * n + rng.integers(0, n)
+        kr = np.array([rng.choice([0.125, 0.33, 0.5])], dtype=np.float32)
+        alpha = float(rng.choice([0.5, 1.0, 3.0]))
+        k1 = O.allocate(lay, S, kr, alpha, 0.05, 0.95, True)["budgets"]
+        for c in (3, 2 ** 20 + 7):
+            k2 = O.allocate(lay, S * c, kr, alpha, 0.05, 0.95, True)["budgets"]
+            assert k2.tolist() == k1.tolist(), (trial, c)
+
+
+def test_additive_rule_ignores_a_common_shift_of_the_means():
+    # adding the same c to every image's mean moves every r_i by alpha*c - alpha*c = 0
+    rng = np.random.default_rng(16)
+    for trial in range(40):
+        m = int(rng.integers(1, 9))
+        n = rng.integers(1, 400, size=m)
+        lay = synth.Layout.from_segments([[("i", int(v)) for v in n] + [("t", 2)]])
+        S = rng.integers(0, 2 ** 33, size=m).astype(np.int64) * n + rng.integers(0, n)
+        kr = np.array([rng.choice([0.125, 0.33, 0.5, 0.9])], dtype=np.float32)
+        alpha = float(rng.choice([0.5, 1.0, 5.0]))
+        k1 = O.allocate(lay, S, kr, alpha)["budgets"]
+        c = int(rng.integers(-2 ** 31, 2 ** 31))
+        k2 = O.allocate(lay, S + c * n, kr, alpha)["budgets"]
+        assert k2.tolist() == k1.tolist(), trial
+
+
+def _bisect_shift(r, n, B, lo_r, hi_r, iters=200):
+    # an independent route to the shift: bisection on the clamped total in exact
+    # rationals, keeping G(lo) < B <= G(hi)
+    from fractions import Fraction as F
+
+    def G(lam):
+        return sum(int(n[i]) * min(max(r[i] + lam, lo_r), hi_r) for i in range(len(n)))
+
+    lo, hi = lo_r - max(r) - 1, hi_r - min(r) + 1  # G(lo) = N r_min, G(hi) = N r_max
+    for _ in range(iters):
+        mid = (lo + hi) / 2
+        if G(mid) >= B:
+            hi = mid
+        else:
+            lo = mid
+    return lo, hi, G
+
+
+@pytest.mark.parametrize("relative", [False, True])
+def test_shift_restores_the_budget_and_matches_bisection(relative):
+    from fractions import Fraction as F
+    rng = np.random.default_rng(17)
+    r_min, r_max = F(float(np.float32(0.05))), F(float(np.float32(0.95)))
+    for trial in range(40):
+        m = int(rng.integers(1, 7))
+        n = [int(v) for v in rng.integers(1, 300, size=m)]
+        S = [int(v) * n[i] + int(rng.integers(0, n[i])) for i, v in enumerate(rng.integers(1, 2 ** 33, size=m))]
+        kr = np.float32(rng.choice([0.05, 0.125, 0.33, 0.5, 0.9]))
+        alpha = float(rng.choice([1.0, 4.0, 20.0]))  # large alpha: clamps bind
+        r = O.adaptive_ratios(S, n, kr, alpha, relative)
+        B = O.global_budget(kr, sum(n))
+        lam = O.water_fill(r, n, B, r_min, r_max)
+        lo, hi, G = _bisect_shift(r, n, B, r_min, r_max)
+        N = sum(n)
+        if N * r_min < B < N * r_max:
+            assert G(lam) == B, trial
+            assert lo <= lam <= hi, trial
+        x = [n[i] * min(max(r[i] + lam, r_min), r_max) for i in range(m)]
+        assert all(n[i] * r_min <= x[i] <= n[i] * r_max for i in range(m))
+
+
+def test_largest_remainder_is_the_closest_integer_vector():
+    # Rounding to integers with a fixed total: the largest-remainder vector minimises
+    # sum (k_i - x_i)^2 over every integer vector with sum B and 0 <= k_i <= n_i; among
+    # several minimisers (equal remainders) the rule favours the lower index, i.e. the
+    # lexicographically largest one. Checked by enumeration.
+    from fractions import Fraction as F
+    rng = np.random.default_rng(18)
+    for trial in range(150):
+        m = int(rng.integers(1, 5))
+        n = [int(v) for v in rng.integers(1, 6, size=m)]
+        den = int(rng.choice([1, 2, 3, 4, 7, 10]))
+        # kept masses with sum B (the water-fill's output) or just above it (every image at r_min)
+        x = [F(int(rng.integers(0, n[i] * den + 1)), den) for i in range(m)]
+        B = math.floor(sum(x))
+        if trial % 5 == 0 and B > 0:
+            B -= 1
+        got = O.integer_budgets(x, n, B)
+        best = None
+        for k in itertools.product(*[range(v + 1) for v in n]):
+            if sum(k) != B:
+                continue
+            key = (sum((k[i] - x[i]) ** 2 for i in range(m)), tuple(-v for v in k))
+            if best is None or key < best[0]:
+                best = (key, list(k))
+        assert got == best[1], (trial, x, B)
 
 
 # ---------------------------------------------------------------- step 3
