@@ -27,6 +27,10 @@ Language Models", AVTP):
 5.  The layout of the pruned batch, on which the stage runs again at a later layer in
     a progressive schedule (§3.3.2), with the compacted hidden states of this pruning
     point as that layer's h_prior (§3.3.1).
+6.  Pruning-layer selection (§3.3.2): per sample and layer the attention mass on the
+    visual tokens, the per-sample ranking of the layers, the mean rank, the top-k layers.
+    The attention of step 1B may also take the request's last token as its only query
+    (§4.1, the output token's attention that FAST-V ranks by).
 
 Readings of points the paper leaves open (each is also listed with its reason in
 the design notes of the repository):
@@ -118,25 +122,43 @@ def score_hidden_variation(layout, h_cur: np.ndarray, h_prior: np.ndarray) -> np
 # ----------------------------------------------------------------------------
 # Step 1B: text-to-visual attention (attention quantity of paper §3.3.2)
 # ----------------------------------------------------------------------------
-def attention_logits(layout, q, k, r: int, h: int, n_q_heads: int, n_kv_heads: int, scale: float):
-    """Scaled logits of request r, head h: text queries (rows) x all request keys.
+QUERY_SETS = ("text", "last")
+
+
+def query_positions(layout, r: int, query_set: str = "text") -> np.ndarray:
+    """Request-local positions of the queries whose attention scores the visual keys.
+
+    ``"text"``: every text token of the request (the attention of §3.3.2 kept per token).
+    ``"last"``: the request's last token alone, the token whose output predicts the first
+    generated token (the attention FAST-V ranks visual tokens by, §4.1).
+    """
+    T_r = int(layout.cu_seqlens[r + 1]) - int(layout.cu_seqlens[r])
+    if query_set == "text":
+        return np.nonzero(~_request_visual_local(layout, r))[0]
+    if query_set == "last":
+        return np.arange(T_r - 1, T_r) if T_r > 0 else np.zeros(0, dtype=np.int64)
+    raise ValueError(query_set)
+
+
+def attention_logits(layout, q, k, r: int, h: int, n_q_heads: int, n_kv_heads: int, scale: float,
+                     query_set: str = "text"):
+    """Scaled logits of request r, head h: the query set's rows x all request keys.
     Follows paper §3.3.2, the attention of text queries to visual tokens; grouped-query heads.
 
-    Returns ``(z, text_local)``; ``z`` is fp64 [|Q_r|, T_r] with ``-inf`` where the key
-    lies after the query (causal mask).
+    Returns ``(z, qpos)``; ``z`` is fp64 [|Q_r|, T_r] with ``-inf`` where the key
+    lies after the query (causal mask); ``qpos`` the queries' request-local positions.
     """
     a = int(layout.cu_seqlens[r])
     b = int(layout.cu_seqlens[r + 1])
-    vis = _request_visual_local(layout, r)
-    text_local = np.nonzero(~vis)[0]
+    qpos = query_positions(layout, r, query_set)
     g = h // (n_q_heads // n_kv_heads)
-    Qh = bf16_to_f64(q[a + text_local, h, :])        # [nq, d]
+    Qh = bf16_to_f64(q[a + qpos, h, :])              # [nq, d]
     Kg = bf16_to_f64(k[a:b, g, :])                   # [T_r, d]
     z = float(scale) * (Qh @ Kg.T)                   # [nq, T_r]
     keys = np.arange(b - a)
-    visible = keys[None, :] <= text_local[:, None]
+    visible = keys[None, :] <= qpos[:, None]
     z = np.where(visible, z, -np.inf)
-    return z, text_local
+    return z, qpos
 
 
 def logsumexp_rows(z: np.ndarray) -> np.ndarray:
@@ -148,32 +170,33 @@ def logsumexp_rows(z: np.ndarray) -> np.ndarray:
     return m + np.log(np.sum(np.exp(z - m[:, None]), axis=1))
 
 
-def text_lse(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float) -> np.ndarray:
-    """Per (head, text query) natural-log LSE of the scaled causal logits: fp64 [Hq, T].
+def text_lse(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float, query_set: str = "text") -> np.ndarray:
+    """Per (head, query) natural-log LSE of the scaled causal logits: fp64 [Hq, T].
     Follows paper §3.3.2; the normaliser a FlashAttention forward also returns (§3.2).
 
     This is the normaliser a FlashAttention-style forward pass keeps per query row;
-    visual rows are left 0.
+    the entries of tokens outside the query set are left 0.
     """
     T = int(layout.cu_seqlens[-1])
     out = np.zeros((n_q_heads, T), dtype=np.float64)
     for r in range(len(layout.cu_seqlens) - 1):
         a = int(layout.cu_seqlens[r])
         for h in range(n_q_heads):
-            z, text_local = attention_logits(layout, q, k, r, h, n_q_heads, n_kv_heads, scale)
-            if text_local.size:
-                out[h, a + text_local] = logsumexp_rows(z)
+            z, qpos = attention_logits(layout, q, k, r, h, n_q_heads, n_kv_heads, scale, query_set)
+            if qpos.size:
+                out[h, a + qpos] = logsumexp_rows(z)
     return out
 
 
 def score_text_attention(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: float,
-                         lse: Optional[np.ndarray] = None) -> np.ndarray:
-    """Mean over heads and text queries of the causal softmax probability of each visual key.
-    Follows paper §3.3.2, the attention quantity kept per visual token.
+                         lse: Optional[np.ndarray] = None, query_set: str = "text") -> np.ndarray:
+    """Mean over heads and queries of the causal softmax probability of each visual key.
+    Follows paper §3.3.2, the attention quantity kept per visual token; with
+    ``query_set="last"``, §4.1's attention of the output token.
 
     ``q``: bf16 bits [T, Hq, d]; ``k``: bf16 bits [T, Hkv, d]; ``lse`` (optional) [Hq, T]
-    natural-log normalisers for the text rows; when given they replace the
-    oracle's own. Returns fp64 [T] (text entries 0).
+    natural-log normalisers for the query rows; when given they replace the
+    oracle's own. Returns fp64 [T] (non-visual entries 0).
     """
     T = int(layout.cu_seqlens[-1])
     out = np.zeros(T, dtype=np.float64)
@@ -181,16 +204,16 @@ def score_text_attention(layout, q, k, n_q_heads: int, n_kv_heads: int, scale: f
         a = int(layout.cu_seqlens[r])
         b = int(layout.cu_seqlens[r + 1])
         vis = _request_visual_local(layout, r)
-        nq = int((~vis).sum())
+        nq = len(query_positions(layout, r, query_set))
         if nq == 0:
             continue
         acc = np.zeros(b - a, dtype=np.float64)
         for h in range(n_q_heads):
-            z, text_local = attention_logits(layout, q, k, r, h, n_q_heads, n_kv_heads, scale)
+            z, qpos = attention_logits(layout, q, k, r, h, n_q_heads, n_kv_heads, scale, query_set)
             if lse is None:
                 norm = logsumexp_rows(z)
             else:
-                norm = np.asarray(lse, dtype=np.float64)[h, a + text_local]
+                norm = np.asarray(lse, dtype=np.float64)[h, a + qpos]
             P = np.exp(z - norm[:, None])  # exp(-inf) = 0 on masked keys
             acc += np.sum(P, axis=0)
         out[a:b][vis] = acc[vis] / (n_q_heads * nq)
@@ -461,6 +484,64 @@ def pruned_layout(layout, kept_idx: np.ndarray, out_cu_seqlens: np.ndarray) -> D
             lens.append(int(np.count_nonzero((local >= s0) & (local < s1))))
     return {"cu_seqlens": cu2.astype(np.int32), "img_cu": np.asarray(layout.img_cu, dtype=np.int32).copy(),
             "img_start": np.asarray(starts, dtype=np.int32), "img_len": np.asarray(lens, dtype=np.int32)}
+
+
+# ----------------------------------------------------------------------------
+# Pruning-layer selection (paper §3.3.2): the layers whose attention to visual tokens
+# ranks highest across sample requests
+# ----------------------------------------------------------------------------
+def layer_attention(layout, img_sums: np.ndarray) -> np.ndarray:
+    """``A_l^(i) = sum_j Attention(l, v_j)`` of one layer for every request (sample) i.
+    Follows paper §3.3.2, the cumulative attention a layer assigns to the visual tokens.
+
+    ``Attention(l, v_j)`` is read as the text-attention score of token ``v_j`` at layer l
+    (``score_text_attention``), so ``A`` is the sum of the request's fixed-point per-image
+    sums of that criterion: int64 [R], units of 2^-32.
+    """
+    R = len(layout.cu_seqlens) - 1
+    out = np.zeros(R, dtype=np.int64)
+    for r in range(R):
+        out[r] = sum(int(v) for v in img_sums[int(layout.img_cu[r]):int(layout.img_cu[r + 1])])
+    return out
+
+
+def layer_ranks(A: np.ndarray) -> np.ndarray:
+    """``Rank(A_l^(i))``: per sample, the rank of each of the L layers, 1 for the most attention.
+    Follows paper §3.3.2, the per-sample ranking of the layers.
+
+    ``A``: int [N, L]. Equal values rank by the lower layer index, so each sample's ranks
+    are a permutation of 1..L. Returns int64 [N, L].
+    """
+    A = np.asarray(A)
+    N, L = A.shape
+    ranks = np.zeros((N, L), dtype=np.int64)
+    for i in range(N):
+        order = sorted(range(L), key=lambda l: (-int(A[i, l]), l))
+        for p, l in enumerate(order):
+            ranks[i, l] = p + 1
+    return ranks
+
+
+def mean_ranks(A: np.ndarray):
+    """``R_l = (1/N) sum_i Rank(A_l^(i))``, with the exact integer sum of ranks beside it.
+    Follows paper §3.3.2, the average ranking across the samples.
+
+    Returns ``(rank_sum int64 [L], R fp64 [L])``.
+    """
+    ranks = layer_ranks(A)
+    rank_sum = ranks.sum(axis=0).astype(np.int64)
+    return rank_sum, rank_sum / float(ranks.shape[0])
+
+
+def select_layers(A: np.ndarray, k: int) -> np.ndarray:
+    """The k pruning layers: the best (lowest) average ranks, ties to the lower layer index.
+    Follows paper §3.3.2, the top-k layers chosen as pruning layers.
+
+    Returns int32 [k], best first.
+    """
+    rank_sum, _ = mean_ranks(A)
+    order = sorted(range(len(rank_sum)), key=lambda l: (int(rank_sum[l]), l))
+    return np.asarray(order[:k], dtype=np.int32)
 
 
 # ----------------------------------------------------------------------------

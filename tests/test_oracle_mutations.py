@@ -30,8 +30,8 @@ MUTATIONS = {
     "relative rule ignores alpha": ("return [r_base * (1 + alpha * (ib / avg - 1)) for ib in ibar]",
                                     "return [r_base * (ib / avg) for ib in ibar]"),
     "GQA head mapping": ("g = h // (n_q_heads // n_kv_heads)", "g = h % n_kv_heads"),
-    "causal mask off by one": ("visible = keys[None, :] <= text_local[:, None]",
-                               "visible = keys[None, :] < text_local[:, None]"),
+    "causal mask off by one": ("visible = keys[None, :] <= qpos[:, None]",
+                               "visible = keys[None, :] < qpos[:, None]"),
     "logits transposed": ("z = float(scale) * (Qh @ Kg.T)",
                           "z = float(scale) * (Kg @ Qh.T).T[:, ::-1]"),
     "norm of wrong row": ("nb = np.sqrt(np.sum(b * b, axis=1))", "nb = np.sqrt(np.sum(a * a, axis=1))"),
@@ -51,6 +51,16 @@ MUTATIONS = {
                      "keep = np.zeros(b - a, dtype=bool)"),
     "fixed point truncates": ("return np.rint(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)",
                               "return np.trunc(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)"),
+    "last query set takes the first token": ("return np.arange(T_r - 1, T_r) if T_r > 0 else np.zeros(0, dtype=np.int64)",
+                                             "return np.arange(0, 1) if T_r > 0 else np.zeros(0, dtype=np.int64)"),
+    "layers ranked in ascending attention": ("order = sorted(range(L), key=lambda l: (-int(A[i, l]), l))",
+                                             "order = sorted(range(L), key=lambda l: (int(A[i, l]), l))"),
+    "layer ties to the higher index": ("order = sorted(range(L), key=lambda l: (-int(A[i, l]), l))",
+                                       "order = sorted(range(L), key=lambda l: (-int(A[i, l]), -l))"),
+    "layers chosen by the worst mean rank": ("order = sorted(range(len(rank_sum)), key=lambda l: (int(rank_sum[l]), l))",
+                                             "order = sorted(range(len(rank_sum)), key=lambda l: (-int(rank_sum[l]), l))"),
+    "layer mass misses the last image": ("out[r] = sum(int(v) for v in img_sums[int(layout.img_cu[r]):int(layout.img_cu[r + 1])])",
+                                         "out[r] = sum(int(v) for v in img_sums[int(layout.img_cu[r]):int(layout.img_cu[r + 1]) - 1])"),
     "pruned image starts after its first kept token": ("starts.append(int(np.count_nonzero(local < s0)))",
                                                        "starts.append(int(np.count_nonzero(local <= s0)))"),
     "pruned image span keeps its old length": ("lens.append(int(np.count_nonzero((local >= s0) & (local < s1))))",

@@ -80,7 +80,7 @@ def test_text_attention_golden():
     assert np.allclose(s, g["expected_scores"], rtol=1e-14, atol=1e-16), g["derivation"]
 
 
-def _brute_force_scores(lay, q, k, Hq, Hkv, scale):
+def _brute_force_scores(lay, q, k, Hq, Hkv, scale, query_set="text"):
     """Full square causal attention per request via scipy softmax; GQA by np.repeat."""
     out = np.zeros(lay.n_tokens)
     vis_all = lay.visual_mask()
@@ -93,11 +93,15 @@ def _brute_force_scores(lay, q, k, Hq, Hkv, scale):
         mask = np.tril(np.ones((b - a, b - a), dtype=bool))            # key <= query
         logits = np.where(mask[None], logits, -np.inf)
         P = ssp.softmax(logits, axis=-1)
-        text = ~vis_all[a:b]
-        nq = text.sum()
+        if query_set == "text":
+            rows = ~vis_all[a:b]
+        else:  # the request's last token alone
+            rows = np.zeros(b - a, dtype=bool)
+            rows[-1] = b > a
+        nq = rows.sum()
         if nq == 0:
             continue
-        s = P[:, text, :].sum(axis=(0, 1)) / (Hq * nq)
+        s = P[:, rows, :].sum(axis=(0, 1)) / (Hq * nq)
         out[a:b][vis_all[a:b]] = s[vis_all[a:b]]
     return out
 
@@ -110,6 +114,45 @@ def test_text_attention_matches_full_square_attention(Hq, Hkv):
     s = O.score_text_attention(wl.layout, wl.q, wl.k, Hq, Hkv, scale)
     ref = _brute_force_scores(wl.layout, wl.q, wl.k, Hq, Hkv, scale)
     assert np.allclose(s, ref, rtol=1e-12, atol=1e-15)
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(4, 2), (6, 6)])
+def test_last_token_attention_matches_full_square_attention(Hq, Hkv):
+    for segs in ([[("t", 5), ("i", 12), ("t", 3), ("i", 7), ("t", 4)], [("i", 9), ("t", 6)]],
+                 [[("t", 2), ("i", 11)], [("i", 4)]]):  # requests ending in an image
+        wl = synth.make_custom(segs, hidden=32, n_q_heads=Hq, n_kv_heads=Hkv, head_dim=16, seed=4, parts=("B",))
+        s = O.score_text_attention(wl.layout, wl.q, wl.k, Hq, Hkv, wl.softmax_scale, query_set="last")
+        ref = _brute_force_scores(wl.layout, wl.q, wl.k, Hq, Hkv, wl.softmax_scale, query_set="last")
+        assert np.allclose(s, ref, rtol=1e-12, atol=1e-15)
+
+
+def test_last_token_attention_golden():
+    g = _load("text_attention_last.json")
+    for case in g["cases"]:
+        lay = synth.Layout.from_segments([[(k, n) for k, n in case["layout"]]])
+        q = _bits(case["q"]).reshape(-1, 1, 1)
+        k = _bits(case["k"]).reshape(-1, 1, 1)
+        last = O.score_text_attention(lay, q, k, 1, 1, case["scale"], query_set="last")
+        text = O.score_text_attention(lay, q, k, 1, 1, case["scale"], query_set="text")
+        assert np.allclose(last, case["expected_last"], rtol=1e-14, atol=1e-16), case["name"]
+        assert np.allclose(text, case["expected_text"], rtol=1e-14, atol=1e-16), case["name"]
+
+
+def test_last_token_mass_is_its_softmax_row():
+    # the last token's softmax row sums to one over the request's keys, so the visual
+    # scores plus the text keys' probabilities make one, for every head
+    wl = synth.make_custom([[("t", 3), ("i", 10), ("t", 2), ("i", 6), ("t", 1)]], n_q_heads=2, n_kv_heads=1,
+                           head_dim=16, seed=8, parts=("B",))
+    vis = wl.layout.visual_mask()
+    total = 0.0
+    for h in range(2):
+        z, qpos = O.attention_logits(wl.layout, wl.q, wl.k, 0, h, 2, 1, wl.softmax_scale, "last")
+        assert qpos.tolist() == [wl.layout.n_tokens - 1]
+        P = np.exp(z - O.logsumexp_rows(z)[:, None])[0]
+        assert P.sum() == pytest.approx(1.0, abs=1e-13)
+        total += P[~vis].sum()
+    s = O.score_text_attention(wl.layout, wl.q, wl.k, 2, 1, wl.softmax_scale, query_set="last")
+    assert s[vis].sum() + total / 2 == pytest.approx(1.0, abs=1e-13)
 
 
 def test_tiny_config_matches_full_square_attention():
@@ -425,6 +468,66 @@ def test_largest_remainder_is_the_closest_integer_vector():
             if best is None or key < best[0]:
                 best = (key, list(k))
         assert got == best[1], (trial, x, B)
+
+
+# ---------------------------------------------------------------- pruning-layer selection
+def test_layer_selection_golden():
+    g = _load("layer_selection.json")
+    A = np.asarray(g["A"], dtype=np.int64)
+    assert O.layer_ranks(A).tolist() == g["expected_ranks"], g["derivation"]
+    rank_sum, R = O.mean_ranks(A)
+    assert rank_sum.tolist() == g["expected_rank_sum"]
+    assert np.allclose(R, np.asarray(g["expected_rank_sum"]) / 3.0, rtol=0, atol=1e-15)
+    for k, top in g["expected_top"].items():
+        assert O.select_layers(A, int(k)).tolist() == top, k
+
+
+def test_layer_ranks_match_scipy_ordinal_ranks():
+    # scipy's ordinal ranking of -A breaks ties by position: the lower layer first
+    import scipy.stats as sst
+    rng = np.random.default_rng(41)
+    for trial in range(30):
+        N, L = int(rng.integers(1, 6)), int(rng.integers(1, 40))
+        A = rng.integers(-5, 6, size=(N, L)).astype(np.int64) * int(rng.integers(1, 2 ** 40))
+        ranks = O.layer_ranks(A)
+        for i in range(N):
+            assert ranks[i].tolist() == sst.rankdata(-A[i], method="ordinal").astype(int).tolist()
+
+
+def test_layer_selection_invariances():
+    rng = np.random.default_rng(42)
+    for trial in range(30):
+        N, L = int(rng.integers(1, 8)), int(rng.integers(2, 30))
+        A = rng.permutation(N * L).reshape(N, L).astype(np.int64) * 7 + 3  # distinct values
+        rank_sum, _ = O.mean_ranks(A)
+        # the order of the samples does not matter
+        assert O.mean_ranks(A[rng.permutation(N)])[0].tolist() == rank_sum.tolist()
+        # relabelling the layers relabels the result
+        perm = rng.permutation(L)
+        assert O.mean_ranks(A[:, perm])[0].tolist() == rank_sum[perm].tolist()
+        # scaling one sample's attention by a positive factor changes none of its ranks
+        B = A.copy()
+        B[int(rng.integers(0, N))] *= 5
+        assert O.layer_ranks(B).tolist() == O.layer_ranks(A).tolist()
+        # the selected layers have the best mean ranks
+        k = int(rng.integers(1, L + 1))
+        top = O.select_layers(A, k)
+        worst_in = max(rank_sum[top])
+        rest = np.setdiff1d(np.arange(L), top)
+        assert len(rest) == 0 or worst_in <= min(rank_sum[rest])
+
+
+def test_layer_attention_sums_the_visual_fixed_point_scores():
+    wl = synth.make_custom([[("t", 3), ("i", 10), ("t", 2), ("i", 6)], [("i", 4), ("t", 5)], [("t", 2)]],
+                           seed=12, parts=("B",))
+    s = O.to_fp32(O.score_text_attention(wl.layout, wl.q, wl.k, 4, 2, wl.softmax_scale))
+    A = O.layer_attention(wl.layout, O.image_sums(wl.layout, s))
+    fx = O.fixed_point(s)
+    vis = wl.layout.visual_mask()
+    for r in range(wl.layout.n_requests):
+        a, b = int(wl.layout.cu_seqlens[r]), int(wl.layout.cu_seqlens[r + 1])
+        assert int(A[r]) == int(fx[a:b][vis[a:b]].sum())
+    assert int(A[2]) == 0  # a request without images has no visual attention
 
 
 # ---------------------------------------------------------------- step 3
