@@ -122,10 +122,14 @@ typedef struct {
 typedef struct {
   const float* keep_ratio;  /* device [R]: base keep ratio r_base of each request, within
                              * [r_min, r_max] (else AVTP_ERR_DEVICE_INPUT: no shift of the
-                             * ratios could meet both the clamps and the request's budget) */
+                             * ratios could meet both the clamps and the request's budget)
+                             * and a multiple of 2^-32 (else AVTP_ERR_DEVICE_INPUT) */
   float alpha;              /* variance control alpha of paper §3.3.3, in [0, 1024]; paper uses 1.0 */
   float r_min;              /* ratio clamps of App. A.2: 0 <= r_min <= r_max <= 1; paper uses 0.05 */
-  float r_max;              /*                                                        and 0.95 */
+  float r_max;              /*                                                        and 0.95.
+                             * alpha, r_min and r_max must be multiples of 2^-32 (every fp32
+                             * value of at least 2^-9 is one), else AVTP_ERR_RANGE: the rule is
+                             * computed exactly, and this bounds its integers */
   int32_t relative;         /* 0: r_i = r_base + alpha*(Ibar_i - Ibar_avg) (paper §3.3.3)
                              * 1: r_i = r_base*(1 + alpha*(Ibar_i/Ibar_avg - 1)), for scores of
                              *    order 1/N such as the text-attention criterion */
@@ -162,18 +166,19 @@ AVTP_API avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_
 
 /* Step 2 (paper §3.3.3, App. A.2). From img_sums (device int64 [n_images]) writes
  * budgets (device int32 [n_images]) and out_cu_seqlens (device int32 [R+1]),
- * the packed offsets of the pruned batch. Per request: B_r = floor(r_base*N_vis+0.5);
- * the ratios r_i of the rule above are taken in exact integers on a 2^-40 grid:
- * Ibar_i = round(S_i*floor(2^62/n_i)/2^62) and Ibar_avg likewise with sum S and
- * N_vis (units of 2^-32); R_i = rint(r_base*2^40) + round(alpha*(Ibar_i-Ibar_avg)*2^8),
- * or for the relative rule + round(r_base*alpha*q_i) with
- * q_i = sgn(Ibar_avg)*round((Ibar_i-Ibar_avg)*floor(2^62/|Ibar_avg|)/2^22);
- * fp32 alpha, r_base exact, one rounding (nearest, ties up) per product, R_i
- * saturated to +-2^60;
- * lambda = smallest integer with sum n_i*clamp(R_i+lambda, R_min, R_max) >= B_r*2^40;
- * k_i = min(floor(x_i/2^40), n_i) with x_i = n_i*clamp(R_i+lambda), then
- * largest remainder (ties to the lower index) until sum k_i = B_r.
- * Every |img_sums[i]| must be at most img_len[i]*2^42 (avtp_score's sums are);
+ * the packed offsets of the pruned batch. Per request, in exact rational arithmetic:
+ *   B_r = floor(r_base*N_vis + 1/2);  Ibar_i = S_i / (2^32 n_i);  Ibar_avg = sum S / (2^32 N_vis);
+ *   r_i = r_base + alpha*(Ibar_i - Ibar_avg), or with `relative`
+ *   r_i = r_base*(1 + alpha*(Ibar_i/Ibar_avg - 1)) (r_base when sum S = 0);
+ *   lambda with sum_i n_i*clamp(r_i + lambda, r_min, r_max) = B_r (every image at the
+ *   nearer clamp when B_r lies outside [N_vis*r_min, N_vis*r_max]);
+ *   x_i = n_i*clamp(r_i + lambda, r_min, r_max), k_i = floor(x_i), then largest
+ *   remainder: one more token for the images with the largest x_i - floor(x_i) (ties
+ *   to the lower index) until sum k_i = B_r (a surplus is taken from the smallest
+ *   remainders, ties to the higher index).
+ * No step rounds: the budgets are those of the exact rule.
+ * Every |img_sums[i]| must be at most img_len[i]*2^42 (avtp_score's sums are), and
+ * each keep ratio a multiple of 2^-32 (every fp32 value of at least 2^-9 is);
  * otherwise the request's budgets are not written and the call reports
  * AVTP_ERR_DEVICE_INPUT. */
 AVTP_API avtp_status_t avtp_allocate(const avtp_layout_t* layout, const int64_t* img_sums, const avtp_alloc_args_t* args,
@@ -202,9 +207,10 @@ AVTP_API avtp_status_t avtp_select(const avtp_layout_t* layout, const float* sco
  * the library until the process exits. Limits: at most
  * AVTP_NOALLOC_MAX_IMAGES images and AVTP_NOALLOC_MAX_REQUESTS requests;
  * larger layouts return AVTP_ERR_RANGE before anything is launched.
- * The first call on each device looks up the array's device address
- * (cudaGetSymbolAddress, which may load the library's GPU module); make that
- * first call before any stream capture. All calls share the one array, so calls
+ * Every call looks up the array's device address on the current device
+ * (cudaGetSymbolAddress, which allocates nothing); the first call on a device may
+ * load the library's GPU module, so make that first call before any stream
+ * capture. All calls share the one array, so calls
  * that overlap on the GPU race and must not be issued; calls ordered on one
  * stream are fine, since each call rewrites the scratch it reads.
  * device_status (optional device int32, NULL to skip) receives the device-side

@@ -1,33 +1,32 @@
-// Per-request budget rule (paper §3.3.3 adaptive keep ratio, App. A.2 clamps),
-// computed by ONE WARP, in exact integer arithmetic on a 2^-40 ratio grid.
-//
-// Ratios (S_i in units of 2^-32, each product exact, rounded once to nearest, ties up):
-//   Ibar_i   = round(S_i * floor(2^62 / n_i) / 2^62)
-//   Ibar_avg = round(sum_i S_i * floor(2^62 / N_vis) / 2^62)
-//   R_i = R_base + round(alpha * (Ibar_i - Ibar_avg) * 2^8)                       (relative = 0)
-//   R_i = R_base + round(r_base * alpha * q_i),                                    (relative = 1)
-//         q_i = sgn(Ibar_avg) * round((Ibar_i - Ibar_avg) * floor(2^62 / |Ibar_avg|) / 2^22),
-//         saturated to +-2^60 (R_i = R_base when Ibar_avg == 0)
-//   with R_base = rint(r_base * 2^40), fp32 alpha and r_base taken as exact M * 2^E,
-//   and R_i saturated to +-2^60. R_min, R_max = rint(r_min * 2^40), rint(r_max * 2^40).
-// Water-fill and rounding:
-//   G(l) = sum_i n_i * clamp(R_i + l, R_min, R_max),
-//   lambda = min { l in [R_min - max R, R_max - min R] : G(l) >= B * 2^40 } (an end of the range if none),
-//   x_i = n_i * clamp(R_i + lambda), k_i = min(x_i >> 40, n_i), then largest remainder.
+// Per-request budget rule (paper §3.3.3 adaptive keep ratio, App. A.2 clamps), run by
+// ONE WARP. Two stages:
+//  1. An integer approximation on a 2^-40 ratio grid proposes the water-fill shift:
+//       Ibar_i   ~ round(S_i * floor(2^62 / n_i) / 2^62)            (units of 2^-32)
+//       Ibar_avg ~ round(sum_i S_i * floor(2^62 / N_vis) / 2^62)
+//       R_i = R_base + round(alpha * (Ibar_i - Ibar_avg) * 2^8)                 (additive)
+//       R_i = R_base + round(r_base * alpha * q_i),                              (relative)
+//         q_i = sgn(Ibar_avg) * round((Ibar_i - Ibar_avg) * floor(2^62 / |Ibar_avg|) / 2^22)
+//       lambda = min { l : sum_i n_i * clamp(R_i + l, R_min, R_max) >= B * 2^40 }.
+//     Multiplies and shifts only, with the reciprocals taken before the sums arrive.
+//  2. The exact stage of avtp_exact.cuh takes the partition of the images into
+//     clamped-low, free and clamped-high that this shift implies, checks it in exact
+//     rational arithmetic (searching the breakpoints exactly when it does not hold),
+//     and computes the kept masses x_i, their floors and the largest-remainder
+//     rounding exactly. The budgets are therefore those of the plain rule, whatever
+//     the grid's rounding.
 //
 // G is continuous, non-decreasing and linear between the breakpoints
-// R_min - R_i and R_max - R_i, so for up to kBreakpointImages images lambda is
-// found exactly: evaluate G at every breakpoint, take the two that bracket the
-// target and solve the linear piece between them with one integer division.
+// R_min - R_i and R_max - R_i, so for up to kBreakpointImages images the grid's lambda
+// is found at the breakpoints: evaluate G at every breakpoint, take the two that bracket
+// the target and solve the linear piece between them with one integer division.
 // Beyond that a 32-way multisection gives the same lambda.
 //
 // Everything is warp-synchronous (shuffles and __syncwarp only): on this part a
-// block-wide barrier or a dependent fp64 operation or division costs far more
-// than the arithmetic, so the reciprocals are taken before the sums are known
-// and the rest is integer multiplies and shifts.
+// block-wide barrier or a dependent fp64 operation or division costs far more than
+// the arithmetic.
 #pragma once
 
-#include "avtp_internal.cuh"
+#include "avtp_exact.cuh"
 
 namespace avtp {
 
@@ -51,27 +50,6 @@ __device__ __forceinline__ int64_t warp_min64(int64_t v) {
     v = u < v ? u : v;
   }
   return v;
-}
-
-// Per-warp scratch, m_cap entries each.
-struct WarpAllocSmem {
-  int64_t* R;  // ratio grid values
-  int64_t* X;  // on entry: S_i (fixed-point sums); on exit: remainders
-  int32_t* n;  // on entry: image sizes
-  int32_t* K;  // on exit: budgets
-};
-
-__host__ __device__ constexpr size_t warp_alloc_smem_bytes(int m_cap) {
-  return static_cast<size_t>(m_cap) * (8 + 8 + 4 + 4);
-}
-
-__device__ __forceinline__ WarpAllocSmem carve_warp_alloc(unsigned char* base, int m_cap) {
-  WarpAllocSmem s;
-  s.R = reinterpret_cast<int64_t*>(base);
-  s.X = s.R + m_cap;
-  s.n = reinterpret_cast<int32_t*>(s.X + m_cap);
-  s.K = s.n + m_cap;
-  return s;
 }
 
 // The grid values of the clamps, rint(r * 2^40) (exact for fp32 inputs >= 2^-17).
@@ -105,6 +83,7 @@ __device__ __forceinline__ void fp32_parts(float v, int64_t* M, int* E) {
 // The parts of the ratio rule that do not depend on the sums. alpha in [0, 1024]
 // and r_base in [0, 1] (validated before any launch) keep `shift` >= 5.
 struct RatioRule {
+  float r_base_f;  // the request's keep ratio
   int64_t Rb;    // rint(r_base * 2^40)
   int64_t coef;  // alpha (additive) or r_base * alpha (relative) is coef * 2^-shift on the grid
   int shift;
@@ -113,6 +92,7 @@ struct RatioRule {
 
 __device__ __forceinline__ RatioRule make_ratio_rule(float r_base, float alpha, int relative) {
   RatioRule q;
+  q.r_base_f = r_base;
   q.Rb = ratio_grid(r_base);
   int64_t A, Bm;
   int E, Be;
@@ -162,27 +142,40 @@ __device__ __forceinline__ int64_t grid_ratio(const RatioRule& q, int64_t ibar, 
   return clamp64(q.Rb + delta, -kGridSat, kGridSat);
 }
 
-// All 32 lanes call with identical scalars. sm.X[j] = S_j and sm.n[j] = n_j for j < m on entry.
-// Returns AVTP_OK, AVTP_ERR_DEVICE_INPUT for a sum beyond n_j * 2^42, or AVTP_ERR_RANGE
-// if the rounding loop did not converge (never expected).
-static __device__ __noinline__ int warp_allocate(const WarpAllocSmem& sm, int m, int64_t B, int32_t N, float r_base_f, float alpha_f,
-                              int64_t Rmin, int64_t Rmax, int relative) {
+// The exact stage for a request whose images sit in sm (S, n, R on the grid) and whose
+// grid shift is lam: the width that holds the rule's products, see avtp_exact.cuh.
+__device__ __forceinline__ int exact_stage(const WarpAllocSmem& sm, int m, int64_t B, int32_t N, int64_t T,
+                                           float r_base_f, float alpha_f, float r_min_f, float r_max_f, int relative,
+                                           int64_t lam, int64_t Rmin, int64_t Rmax) {
+  const ExactRule q = make_exact_rule(B, N, T, r_base_f, alpha_f, r_min_f, r_max_f, relative);
+  if (relative && q.mode == kExactGeneral) return exact_budgets<I256>(sm, m, q, lam, Rmin, Rmax);
+  return exact_budgets<i128>(sm, m, q, lam, Rmin, Rmax);
+}
+
+// All 32 lanes call with identical scalars. sm.S[j] = S_j and sm.n[j] = n_j for j < m on
+// entry; the budgets are left in sm.K. Returns AVTP_OK, AVTP_ERR_DEVICE_INPUT for a sum
+// beyond n_j * 2^42, or AVTP_ERR_RANGE if the rounding loop did not converge (never
+// expected).
+static __device__ __noinline__ int warp_allocate(const WarpAllocSmem& sm, int m, int64_t B, int32_t N, float r_base_f,
+                                                 float alpha_f, float r_min_f, float r_max_f, int relative) {
   const int lane = threadIdx.x & 31;
+  const int64_t Rmin = ratio_grid(r_min_f), Rmax = ratio_grid(r_max_f);
   // ---- ratios on the grid
   int64_t part = 0;
   bool bad = false;
   for (int j = lane; j < m; j += 32) {
-    const int64_t S = sm.X[j], lim = static_cast<int64_t>(sm.n[j]) << kSumMagnitudeBits;
+    const int64_t S = sm.S[j], lim = static_cast<int64_t>(sm.n[j]) << kSumMagnitudeBits;
     bad |= S > lim || S < -lim;
     part += S;
   }
   if (__any_sync(0xffffffffu, bad)) return AVTP_ERR_DEVICE_INPUT;
-  const int64_t avg = grid_mean(warp_sum(part), recip62(N));
+  const int64_t T = warp_sum(part);
+  const int64_t avg = grid_mean(T, recip62(N));
   const int64_t inv_avg = (relative && avg != 0) ? recip62(avg > 0 ? avg : -avg) : 0;
   const RatioRule rule = make_ratio_rule(r_base_f, alpha_f, relative);
   int64_t mx = INT64_MIN, mn = INT64_MAX;
   for (int j = lane; j < m; j += 32) {
-    const int64_t g = grid_ratio(rule, grid_mean(sm.X[j], recip62(sm.n[j])), avg, inv_avg);
+    const int64_t g = grid_ratio(rule, grid_mean(sm.S[j], recip62(sm.n[j])), avg, inv_avg);
     sm.R[j] = g;
     mx = g > mx ? g : mx;
     mn = g < mn ? g : mn;
@@ -191,7 +184,7 @@ static __device__ __noinline__ int warp_allocate(const WarpAllocSmem& sm, int m,
   mn = warp_min64(mn);
   __syncwarp();
 
-  // ---- exact water-fill
+  // ---- the grid's water-fill shift
   const int64_t target = B << kRatioFracBits;
   auto G = [&](int64_t lam) {
     int64_t acc = 0;
@@ -256,60 +249,7 @@ static __device__ __noinline__ int warp_allocate(const WarpAllocSmem& sm, int m,
     }
   }
 
-  // ---- integer budgets and largest remainder
-  const int64_t kFracMask = (int64_t(1) << kRatioFracBits) - 1;
-  for (int j = lane; j < m; j += 32) {
-    const int64_t x = static_cast<int64_t>(sm.n[j]) * clamp64(sm.R[j] + lam, Rmin, Rmax);
-    const int64_t fl = x >> kRatioFracBits;
-    sm.K[j] = static_cast<int32_t>(fl < sm.n[j] ? fl : sm.n[j]);
-    sm.X[j] = x & kFracMask;
-  }
-  __syncwarp();
-  for (int round = 0; round < 64; ++round) {
-    int64_t ks = 0;
-    for (int j = lane; j < m; j += 32) ks += sm.K[j];
-    const int64_t D = B - warp_sum(ks);
-    if (D == 0) return AVTP_OK;
-    // decide every image from the same snapshot of K (sm.R is free by now), then apply
-    for (int j = lane; j < m; j += 32) {
-      int dec = 0;
-      if (D > 0 && sm.K[j] < sm.n[j]) {
-        int64_t rank = 0;  // eligible images ahead of j: larger remainder, or equal and lower index
-        for (int l = 0; l < m; ++l)
-          rank += (sm.K[l] < sm.n[l]) && (sm.X[l] > sm.X[j] || (sm.X[l] == sm.X[j] && l < j));
-        dec = rank < D ? 1 : 0;
-      } else if (D < 0 && sm.K[j] > 0) {
-        int64_t rank = 0;  // eligible images ahead of j: smaller remainder, or equal and higher index
-        for (int l = 0; l < m; ++l)
-          rank += (sm.K[l] > 0) && (sm.X[l] < sm.X[j] || (sm.X[l] == sm.X[j] && l > j));
-        dec = rank < -D ? -1 : 0;
-      }
-      sm.R[j] = dec;
-    }
-    __syncwarp();
-    for (int j = lane; j < m; j += 32) sm.K[j] += static_cast<int32_t>(sm.R[j]);
-    __syncwarp();
-  }
-  return AVTP_ERR_RANGE;
-}
-
-// The k-th largest (1 <= k <= 32) of the 32 lanes' values: a bitonic sort across the
-// warp (15 compare-exchange stages by shuffle), then one broadcast. Out of line and
-// rolled: it is fetched once per call from a cold instruction cache.
-static __device__ __noinline__ uint64_t warp_kth_largest(uint64_t v, int k) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll 1
-  for (int size = 2; size <= 32; size <<= 1) {
-#pragma unroll 1
-    for (int j = size >> 1; j > 0; j >>= 1) {
-      const uint64_t p = __shfl_xor_sync(0xffffffffu, v, j);
-      // descending overall: the lower lane of a pair keeps the larger value in blocks
-      // whose `size` bit is clear, the smaller one otherwise
-      const bool keep_max = ((lane & j) == 0) == ((lane & size) == 0);
-      v = keep_max ? (p > v ? p : v) : (p < v ? p : v);
-    }
-  }
-  return __shfl_sync(0xffffffffu, v, k - 1);
+  return exact_stage(sm, m, B, N, T, r_base_f, alpha_f, r_min_f, r_max_f, relative, lam, Rmin, Rmax);
 }
 
 // lambda from the breakpoints, for warp_allocate32 when a clamp binds near the
@@ -358,25 +298,181 @@ static __device__ __noinline__ int64_t breakpoint_lambda32(int m, int64_t R, int
   return lam;
 }
 
-// The same rule for requests of at most 32 images, held in registers: lane j owns
-// image j (S_j, n_j in; its budget out). Identical results and status to warp_allocate.
+// ---------------------------------------------------------------- the register path's exact stage
+// For requests of at most 32 images, lane j owning image j: the arithmetic of
+// exact_budgets (avtp_exact.cuh) held in registers, with no shared memory and no call on
+// the common path. Every kept mass is written as x_i = X_i / (2^64 Q) with integers
+// X_i >= 0 and Q >= 1 common to the request:
+//   every image at r_min:   X_i = n_i m 2^32,  Q = 1
+//   every image at r_max:   X_i = n_i M 2^32,  Q = 1
+//   one common ratio:       X_i = n_i B 2^64,  Q = N
+//   general:                X_i of avtp_exact.cuh (its E is 2^64 Q), Q = N_F for the
+//                           additive rule and |sum S| N_F for the relative one,
+// so k_i = floor((X_i >> 64) / Q), and the remainders order as the pairs
+// ((X_i >> 64) mod Q, X_i mod 2^64). Returns kExactFallback when the grid's partition
+// does not verify or the rounding would give an image more than one token; the caller
+// then runs the general stage.
+constexpr int kExactFallback = -1;
+
+__device__ __forceinline__ unsigned bit_length_u128(u128 v) {
+  const uint64_t hi = static_cast<uint64_t>(v >> 64), lo = static_cast<uint64_t>(v);
+  return hi ? 128u - __clzll(static_cast<long long>(hi)) : (lo ? 64u - __clzll(static_cast<long long>(lo)) : 0u);
+}
+
+__device__ __forceinline__ float u128_to_float(u128 v) {
+  return __ull2float_rn(static_cast<uint64_t>(v >> 64)) * 18446744073709551616.f +
+         __ull2float_rn(static_cast<uint64_t>(v));
+}
+
+// Descending bitonic sort across the warp: lane i ends with the i-th largest of the 32
+// values. Out of line and rolled: it is fetched once per call from a cold cache.
+static __device__ __noinline__ uint64_t warp_sort_desc(uint64_t v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll 1
+  for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll 1
+    for (int j = size >> 1; j > 0; j >>= 1) {
+      const uint64_t p = __shfl_xor_sync(0xffffffffu, v, j);
+      // descending overall: the lower lane of a pair keeps the larger value in blocks
+      // whose `size` bit is clear, the smaller one otherwise
+      const bool keep_max = ((lane & j) == 0) == ((lane & size) == 0);
+      v = keep_max ? (p > v ? p : v) : (p < v ? p : v);
+    }
+  }
+  return v;
+}
+
+template <bool kRel>
+__device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int64_t R, int64_t lam, int64_t Rmin,
+                                       int64_t Rmax, int64_t B, int64_t N, int64_t T, int64_t Rb, int64_t Aa,
+                                       int64_t mq, int64_t Mq, int32_t* k_out) {
+  const int lane = threadIdx.x & 31;
+  if (!has) { S = 0; n = 0; }
+  u128 Xh = 0, Q = 1;  // X_i >> 64, and the request's Q
+  uint64_t Xl = 0;     // X_i mod 2^64
+  if ((B << 32) <= N * mq || (B << 32) >= N * Mq) {
+    const u128 X = static_cast<u128>(n * ((B << 32) <= N * mq ? mq : Mq)) << 32;
+    Xh = X >> 64;
+    Xl = static_cast<uint64_t>(X);
+  } else if (Aa == 0 || (kRel && (T == 0 || Rb == 0))) {
+    Xh = static_cast<u128>(n * B);
+    Q = static_cast<u128>(N);
+  } else {
+    // ---- the partition the grid's shift implies, checked exactly
+    const int64_t g = R + lam;
+    const int cls = !has ? kClsFree : (g <= Rmin ? kClsLow : (g >= Rmax ? kClsHigh : kClsFree));
+    const int64_t sgn = (kRel && T < 0) ? -1 : 1;
+    const int64_t y = sgn * S;
+    const int64_t NL = warp_sum(cls == kClsLow ? n : int64_t(0));
+    const int64_t NH = warp_sum(cls == kClsHigh ? n : int64_t(0));
+    const int64_t NF = warp_sum(cls == kClsFree ? n : int64_t(0));
+    const int64_t YF = warp_sum(cls == kClsFree ? y : int64_t(0));
+    if (NF == 0) return kExactFallback;
+    const int64_t W = (B << 32) - mq * NL - Mq * NH;
+    const i128 Dd = static_cast<i128>(y) * NF - static_cast<i128>(n) * YF;
+    const i128 nlo = static_cast<i128>(n) * mq * NF, nhi = static_cast<i128>(n) * Mq * NF;
+    bool ok;
+    if (!kRel) {
+      // Kn = alpha 2^32, Kd = 2^32: every product below 2^127
+      const i128 v = static_cast<i128>(Aa) * Dd + (static_cast<i128>(n) * W << 32);
+      const i128 lo = nlo << 32, hi = nhi << 32;
+      ok = cls == kClsLow ? v <= lo : (cls == kClsHigh ? v >= hi : (v >= lo && v <= hi));
+      const u128 X = static_cast<u128>(cls == kClsLow ? lo : (cls == kClsHigh ? hi : v));
+      Xh = X >> 64;
+      Xl = static_cast<uint64_t>(X);
+      Q = static_cast<u128>(NF);
+    } else {
+      // Kn = (r_base 2^32)(alpha 2^32) N, Kd = |sum S| 2^32: 256-bit products
+      const i128 Kn = static_cast<i128>(Rb) * Aa * N;
+      const i128 Kd = static_cast<i128>(T < 0 ? -T : T) << 32;
+      const I256 v = i256_add(i256_mul(Kn, Dd), i256_mul(Kd, static_cast<i128>(n) * W));
+      const I256 lo = i256_mul(Kd, nlo), hi = i256_mul(Kd, nhi);
+      ok = cls == kClsLow ? i256_cmp(v, lo) <= 0
+                          : (cls == kClsHigh ? i256_cmp(v, hi) >= 0 : (i256_cmp(v, lo) >= 0 && i256_cmp(v, hi) <= 0));
+      const I256& X = cls == kClsLow ? lo : (cls == kClsHigh ? hi : v);
+      Xh = (static_cast<u128>(X.w[2]) << 64) | X.w[1];  // X < 2^192: the top word is 0
+      Xl = X.w[0];
+      Q = static_cast<u128>(T < 0 ? -T : T) * static_cast<u128>(NF);
+    }
+    if (!__all_sync(0xffffffffu, !has || ok)) return kExactFallback;
+  }
+  // ---- floor and remainder: a float quotient, then an exact correction
+  uint32_t q = 0;
+  if (Xh != 0) {
+    const float qf = u128_to_float(Xh) / u128_to_float(Q);
+    q = qf < 4194304.f ? static_cast<uint32_t>(qf) : 4194304u;
+  }
+  i128 r = static_cast<i128>(Xh) - static_cast<i128>(Q) * q;
+#pragma unroll 1
+  for (int it = 0; it < 4 && r < 0; ++it) { --q; r += static_cast<i128>(Q); }
+#pragma unroll 1
+  for (int it = 0; it < 4 && r >= static_cast<i128>(Q); ++it) { ++q; r -= static_cast<i128>(Q); }
+  const u128 rem_hi = static_cast<u128>(r);
+  int32_t K = has ? static_cast<int32_t>(q < static_cast<uint32_t>(n) ? q : static_cast<uint32_t>(n)) : 0;
+  // ---- largest remainder: one token for each of the |D| images served first
+  const int64_t D = B - warp_sum(static_cast<int64_t>(K));
+  if (D != 0) {
+    const bool up = D > 0;
+    const int need = static_cast<int>(up ? D : -D);
+    const bool elig = has && (up ? K < n : K > 0);
+    if (__popc(__ballot_sync(0xffffffffu, elig)) < need) return kExactFallback;
+    // 59-bit prefix of the remainder (rem_hi 2^64 + Xl < 2^(bq + 64)), then the index
+    const unsigned s = bit_length_u128(Q) + 5u;
+    const uint64_t prefix = s >= 64 ? static_cast<uint64_t>(rem_hi >> (s - 64))
+                                    : static_cast<uint64_t>((rem_hi << (64 - s)) | (Xl >> s));
+    const uint64_t kPrefixMask = (uint64_t(1) << 59) - 1;
+    const uint64_t key = !elig ? 0ull
+                         : (up ? (prefix << 5) | static_cast<uint64_t>(31 - lane)
+                               : ((kPrefixMask - prefix) << 5) | static_cast<uint64_t>(lane));
+    const uint64_t sorted = warp_sort_desc(key);
+    const uint64_t thr = __shfl_sync(0xffffffffu, sorted, need - 1);
+    const uint64_t nxt = __shfl_sync(0xffffffffu, sorted, need < 32 ? need : 31);
+    bool served = elig && key >= thr;
+    if (need < 32 && nxt != 0 && (nxt >> 5) == (thr >> 5)) {
+      // the cut falls among remainders with the same prefix: order those exactly
+      const bool in_group = elig && (key >> 5) == (thr >> 5);
+      const unsigned group = __ballot_sync(0xffffffffu, in_group);
+      const int quota = need - __popc(__ballot_sync(0xffffffffu, elig && (key >> 5) > (thr >> 5)));
+      const uint64_t rh1 = static_cast<uint64_t>(rem_hi >> 64), rh0 = static_cast<uint64_t>(rem_hi);
+      int rank = 0;
+      for (unsigned g = group; g != 0; g &= g - 1) {
+        const int l = __ffs(g) - 1;
+        const uint64_t a1 = __shfl_sync(0xffffffffu, rh1, l), a0 = __shfl_sync(0xffffffffu, rh0, l);
+        const uint64_t al = __shfl_sync(0xffffffffu, Xl, l);
+        int c = a1 != rh1 ? (a1 > rh1 ? 1 : -1) : (a0 != rh0 ? (a0 > rh0 ? 1 : -1) : (al != Xl ? (al > Xl ? 1 : -1) : 0));
+        if (!up) c = -c;  // removing: the smaller remainder first
+        rank += (l != lane && (c > 0 || (c == 0 && (up ? l < lane : l > lane)))) ? 1 : 0;
+      }
+      if (in_group) served = rank < quota;
+    }
+    if (served) K += up ? 1 : -1;
+  }
+  *k_out = K;
+  return AVTP_OK;
+}
+
+// The same rule for requests of at most 32 images, with the grid stage held in
+// registers: lane j owns image j (S_j, n_j in; its budget out). The exact stage then
+// runs on sm (32 entries). Identical results and status to warp_allocate.
 // Out of line so that a warm-up call and the real one share the same code.
 // inv_n = floor(2^62 / n_j) and inv_N = floor(2^62 / N) come from the caller, which
 // can take them before the sums are ready; after that no division is left on the
 // common path.
-// Fast path for lambda: without clamps G is linear with slope N, so the smallest
-// solution is lambda0 = ceil((B * 2^40 - sum n_i R_i) / N); when no clamp binds
-// at lambda0 - 1 or lambda0, G is that line on [lambda0 - 1, lambda0] and
-// lambda0 is exact. Otherwise the breakpoints decide.
-static __device__ __noinline__ int warp_allocate32(int m, int64_t S, int32_t n, int64_t inv_n, int64_t B, int32_t N,
-                                                   int64_t inv_N, const RatioRule& rule, int64_t Rmin, int64_t Rmax,
-                                                   int32_t* k_out) {
+// Fast path for the grid's lambda: without clamps G is linear with slope N, so the
+// smallest solution is lambda0 = ceil((B * 2^40 - sum n_i R_i) / N); when no clamp binds
+// at lambda0 - 1 or lambda0, G is that line on [lambda0 - 1, lambda0] and lambda0 is
+// exact. Otherwise the breakpoints decide.
+static __device__ __noinline__ int warp_allocate32(const WarpAllocSmem& sm, int m, int64_t S, int32_t n, int64_t inv_n,
+                                                   int64_t B, int32_t N, int64_t inv_N, const RatioRule& rule,
+                                                   float alpha_f, float r_min_f, float r_max_f, int32_t* k_out) {
   const int lane = threadIdx.x & 31;
   const bool has = lane < m;
+  const int64_t Rmin = ratio_grid(r_min_f), Rmax = ratio_grid(r_max_f);
   // ---- ratios on the grid
   const int64_t lim = static_cast<int64_t>(n) << kSumMagnitudeBits;
   if (__any_sync(0xffffffffu, has && (S > lim || S < -lim))) return AVTP_ERR_DEVICE_INPUT;
-  const int64_t avg = grid_mean(warp_sum(has ? S : int64_t(0)), inv_N);
+  const int64_t T = warp_sum(has ? S : int64_t(0));
+  const int64_t avg = grid_mean(T, inv_N);
   const int64_t inv_avg = (rule.relative && avg != 0) ? recip62(avg > 0 ? avg : -avg) : 0;
   const int64_t R = has ? grid_ratio(rule, grid_mean(S, inv_n), avg, inv_avg) : 0;
   const int64_t mx = warp_max64(has ? R : INT64_MIN);
@@ -384,7 +480,7 @@ static __device__ __noinline__ int warp_allocate32(int m, int64_t S, int32_t n, 
   const int64_t target = B << kRatioFracBits;
   const int64_t nl = has ? n : 0;
 
-  // ---- exact water-fill
+  // ---- the grid's water-fill shift
   int64_t lam;
   bool found = false;
   const int64_t kSafe = int64_t(1) << 42;  // keeps n * R and the sums inside int64
@@ -400,32 +496,24 @@ static __device__ __noinline__ int warp_allocate32(int m, int64_t S, int32_t n, 
   }
   if (!found) lam = breakpoint_lambda32(m, R, nl, has, target, Rmin, Rmax, mx, mn);
 
-  // ---- integer budgets and largest remainder
-  const int64_t x = nl * clamp64(R + lam, Rmin, Rmax);
-  const int64_t fl = x >> kRatioFracBits;
-  int32_t K = has ? static_cast<int32_t>(fl < nl ? fl : nl) : 0;
-  const int64_t X = x & ((int64_t(1) << kRatioFracBits) - 1);
-  for (int round = 0; round < 64; ++round) {
-    const int64_t D = B - warp_sum(static_cast<int64_t>(K));
-    if (D == 0) {
-      *k_out = K;
-      return AVTP_OK;
+  // ---- the exact stage, in registers; the general one when that cannot settle it
+  const int64_t Rb = units32(rule.r_base_f), Aa = units32(alpha_f), mq = units32(r_min_f), Mq = units32(r_max_f);
+  int32_t K = 0;
+  int err = rule.relative ? exact32<true>(has, S, n, R, lam, Rmin, Rmax, B, N, T, Rb, Aa, mq, Mq, &K)
+                          : exact32<false>(has, S, n, R, lam, Rmin, Rmax, B, N, T, Rb, Aa, mq, Mq, &K);
+  if (err == kExactFallback) {
+    if (has) {
+      sm.S[lane] = S;
+      sm.n[lane] = n;
+      sm.R[lane] = R;
     }
-    const bool elig = has && (D > 0 ? K < n : K > 0);
-    // One unique key per eligible lane, larger = served first: adding, larger
-    // remainder then lower index; removing, smaller remainder then higher index.
-    // Remainders are below 2^40, so a key fits in 45 bits; ineligible lanes get 0.
-    const uint64_t rem = static_cast<uint64_t>(X);
-    const uint64_t key = !elig ? 0ull
-                         : (D > 0 ? (rem << 5) | static_cast<uint64_t>(31 - lane)
-                                  : (((uint64_t(1) << kRatioFracBits) - 1 - rem) << 5) | static_cast<uint64_t>(lane));
-    // the |D|-th largest key (0 when fewer lanes are eligible): every eligible lane at
-    // or above it moves by one
-    const uint64_t thr = warp_kth_largest(key, static_cast<int>(D > 0 ? (D < 32 ? D : 32) : (-D < 32 ? -D : 32)));
-    if (elig && key >= thr) K += D > 0 ? 1 : -1;
+    __syncwarp();
+    err = exact_stage(sm, m, B, N, T, rule.r_base_f, alpha_f, r_min_f, r_max_f, rule.relative, lam, Rmin, Rmax);
+    K = has ? sm.K[lane] : 0;
+    __syncwarp();
   }
   *k_out = K;
-  return AVTP_ERR_RANGE;
+  return err;
 }
 
 }  // namespace avtp

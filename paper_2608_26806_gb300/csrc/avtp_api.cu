@@ -61,6 +61,8 @@ avtp_status_t check_alloc_args(const avtp_alloc_args_t* a) {
   if (!(a->alpha >= 0.f && a->alpha <= 1024.f)) return AVTP_ERR_INVALID_ARG;
   if (!(a->r_min >= 0.f && a->r_min <= a->r_max && a->r_max <= 1.f)) return AVTP_ERR_INVALID_ARG;
   if (a->relative != 0 && a->relative != 1) return AVTP_ERR_INVALID_ARG;
+  if (!multiple_of_2m32(a->alpha) || !multiple_of_2m32(a->r_min) || !multiple_of_2m32(a->r_max))
+    return AVTP_ERR_RANGE;
   return AVTP_OK;
 }
 
@@ -152,15 +154,12 @@ bool pdl_enabled() {
 }
 
 int device_sm_count() {
-  static int cached[64] = {0};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (cached[dev] == 0) {
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
-    cached[dev] = n;
-  }
-  return cached[dev];
+  static PerDevice sms;
+  int n = 0;
+  const cudaError_t e = once_per_device(sms, [](int dev, int* v) {
+    return cudaDeviceGetAttribute(v, cudaDevAttrMultiProcessorCount, dev);
+  }, &n);
+  return (e == cudaSuccess && n > 0) ? n : 148;
 }
 
 // SMs the scoring kernel leaves to the selection kernel, at most.

@@ -5,7 +5,9 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <string.h>
 
+#include <mutex>
 #include <utility>
 
 #include "avtp.h"
@@ -115,6 +117,21 @@ __host__ __device__ __forceinline__ T* ws_at(void* ws, size_t off) {
   return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
 }
 
+// ---------------------------------------------------------------- parameter domain
+// True when v * 2^32 is an integer: the budget rule takes alpha, the clamps and the keep
+// ratios as exact multiples of 2^-32 (every fp32 value of at least 2^-9 is one).
+__host__ __device__ __forceinline__ bool multiple_of_2m32(float v) {
+  uint32_t b;
+  memcpy(&b, &v, sizeof b);
+  const int e8 = static_cast<int>((b >> 23) & 0xffu);
+  const uint32_t mant = b & 0x7fffffu;
+  if (e8 == 0) return mant == 0;  // zero; a subnormal is below 2^-126
+  const int sh = e8 - 150 + 32;   // v * 2^32 = (mant + 2^23) * 2^sh
+  if (sh >= 0) return true;
+  if (sh <= -24) return false;
+  return ((mant | 0x800000u) & ((1u << -sh) - 1u)) == 0;
+}
+
 // ---------------------------------------------------------------- small device helpers
 __device__ __forceinline__ int64_t fixed_point_score(float s) {
   // rint(fx(s) * 2^32) with fx: NaN -> 0, clamp to [-2^10, 2^10], rounding half to
@@ -193,6 +210,40 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
   cfg.attrs = use ? attr : nullptr;
   cfg.numAttrs = use ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// ---------------------------------------------------------------- per-device set-up
+// CUDA keeps function attributes (shared-memory size, carveout) per device, so a process
+// that runs the library on several devices must set them on each. PerDevice records, per
+// device ordinal, that a set-up succeeded (and an int it computed), under a lock.
+constexpr int kMaxDevices = 64;
+struct PerDevice {
+  std::mutex mu;
+  bool done[kMaxDevices] = {};
+  int value[kMaxDevices] = {};
+};
+
+// Runs fn(dev, &value) for the current device unless it already succeeded there; returns
+// its error. *out (optional) receives the value it stored.
+template <class F>
+cudaError_t once_per_device(PerDevice& pd, F&& fn, int* out = nullptr) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) {
+    int v = 0;
+    e = fn(dev, &v);
+    if (out != nullptr) *out = v;
+    return e;
+  }
+  std::lock_guard<std::mutex> lock(pd.mu);
+  if (!pd.done[dev]) {
+    e = fn(dev, &pd.value[dev]);
+    if (e != cudaSuccess) return e;
+    pd.done[dev] = true;
+  }
+  if (out != nullptr) *out = pd.value[dev];
+  return cudaSuccess;
 }
 
 // ---------------------------------------------------------------- launchers (one per kernel)

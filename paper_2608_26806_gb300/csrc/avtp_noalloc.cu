@@ -16,8 +16,6 @@
 // request map) at the start of each call, so nothing stale is read. Two calls
 // that overlap on the GPU (different streams, no ordering between them) race
 // on the array and must not be issued.
-#include <mutex>
-
 #include "avtp_internal.cuh"
 
 namespace avtp {
@@ -35,23 +33,15 @@ constexpr size_t kScratchBytes = kOffReqBudget + align256(4 * static_cast<size_t
 // array: its device address comes from cudaGetSymbolAddress below.
 static __device__ __align__(256) unsigned char g_select_scratch[kScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of the scratch on the current device, looked up once per device.
+// Device address of the scratch on the current device. It is looked up on every call:
+// the lookup allocates nothing, and an address cached across calls would go stale if
+// the device's context were reset and the library's module reloaded elsewhere. The
+// first lookup on a device may load the library's GPU module.
 avtp_status_t scratch_for_current_device(void** out) {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess) return AVTP_ERR_CUDA;
-  if (dev < 0 || dev >= kMaxDevices) return AVTP_ERR_RANGE;
-  std::lock_guard<std::mutex> lock(g_mutex);
-  if (g_scratch_ptr[dev] == nullptr) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_select_scratch);
-    if (e != cudaSuccess || p == nullptr) return AVTP_ERR_CUDA;
-    g_scratch_ptr[dev] = p;
-  }
-  *out = g_scratch_ptr[dev];
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_select_scratch);
+  if (e != cudaSuccess || p == nullptr) return AVTP_ERR_CUDA;
+  *out = p;
   return AVTP_OK;
 }
 

@@ -26,13 +26,12 @@ k_allocate(const int32_t* __restrict__ img_cu, const int32_t* __restrict__ img_l
   if (m == 0) return;
   const WarpAllocSmem sm = carve_warp_alloc(smem + static_cast<size_t>(warp) * warp_alloc_smem_bytes(m_cap), m_cap);
   for (int j = lane; j < m; j += 32) {
-    sm.X[j] = img_sums[i0 + j];
+    sm.S[j] = img_sums[i0 + j];
     sm.n[j] = img_len[i0 + j];
   }
   __syncwarp();
   const int32_t N = vis_cu[i0 + m] - vis_cu[i0];
-  const int err = warp_allocate(sm, m, req_budget[r], N, keep_ratio[r], alpha, ratio_grid(r_min), ratio_grid(r_max),
-                                relative);
+  const int err = warp_allocate(sm, m, req_budget[r], N, keep_ratio[r], alpha, r_min, r_max, relative);
   if (err != AVTP_OK) {
     if (lane == 0) record_error(st, err, r);
     return;

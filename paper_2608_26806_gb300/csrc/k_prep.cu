@@ -143,7 +143,7 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
     for (int r = tid; r < R; r += blockDim.x) {
       const float kr = a.keep_ratio[r];
       const int32_t nvis = vis_cu[icu[r + 1]] - vis_cu[icu[r]];
-      if (!(kr >= a.r_min && kr <= a.r_max)) {
+      if (!(kr >= a.r_min && kr <= a.r_max) || !multiple_of_2m32(kr)) {
         fail(AVTP_ERR_DEVICE_INPUT, r);
         req_budget[r] = 0;
       } else {

@@ -819,16 +819,15 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   if (L.n_images == 0 || L.n_tokens == 0) return cudaSuccess;
   const int d = sa.head_dim, Hq = sa.n_q_heads, Hkv = sa.n_kv_heads;
   const AttnPlan plan = attn_plan(L, sa);
-  static bool attr_set = false;
-  if (!attr_set) {
+  static PerDevice attrs;
+  cudaError_t ae = once_per_device(attrs, [](int, int*) {
     cudaError_t e = cudaFuncSetAttribute(k_attn_lse, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(lse_smem_bytes(128)));
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(k_attn_mass, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(mass_smem_bytes(128)));
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+    return cudaFuncSetAttribute(k_attn_mass, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(mass_smem_bytes(128)));
+  });
+  if (ae != cudaSuccess) return ae;
   DevStatus* st = ws_at<DevStatus>(ws, p.status);
   AttnArgs a{};
   a.cu = L.cu_seqlens;

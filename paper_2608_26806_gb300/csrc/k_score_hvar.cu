@@ -342,13 +342,12 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
 cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
                               int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s, int reserve_sms) {
   if (L.n_images == 0 || L.n_tokens == 0) return cudaSuccess;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_score_hvar, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(kSmemBytes));
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  static PerDevice attrs;
+  cudaError_t ae = once_per_device(attrs, [](int, int*) {
+    return cudaFuncSetAttribute(k_score_hvar, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(kSmemBytes));
+  });
+  if (ae != cudaSuccess) return ae;
   const int64_t want = (L.n_tokens + kWarps - 1) / kWarps;
   // one 192 KiB CTA per SM, except the SMs left to the next kernel
   int64_t cap = static_cast<int64_t>(device_sm_count()) - reserve_sms;

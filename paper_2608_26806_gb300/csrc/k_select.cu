@@ -397,13 +397,15 @@ struct AllocParams {
   int warm_ctas;     // CTAs below this index warm their instruction cache before the wait
 };
 
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 3)
 k_alloc_select(SelectArgs a, AllocParams ap) {
   extern __shared__ __align__(16) unsigned char dsmem[];  // budget scratch for requests of > 32 images
+  __shared__ __align__(16) unsigned char rule32[warp_alloc_smem_bytes(32)];  // ... and of at most 32
   __shared__ SelShared sh;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = blockIdx.x;
   const WarpAllocSmem wsm = carve_warp_alloc(dsmem, ap.m_cap);
+  const WarpAllocSmem wsm32 = carve_warp_alloc(rule32, 32);
 
   // ---- set-up from the call's inputs only, overlapped with the scoring kernel.
   // The layout is not validated yet, so every index is clamped; nothing here is
@@ -427,7 +429,7 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
   }
   // warp 0: the request's sizes and the scalars of the budget rule
   int32_t N = 0, n_lane = 0, vis_before = 0;
-  int64_t B = 0, Rmin = 0, Rmax = 0, inv_n = 0, inv_N = 0;
+  int64_t B = 0, inv_n = 0, inv_N = 0;
   float kr = 0.f;
   RatioRule rule{};
   if (warp == 0 && b < a.NI) {
@@ -444,8 +446,6 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
     kr = ap.keep_ratio[r];
     // B_r = floor(r_base * N_vis + 0.5), each operation rounded once
     B = static_cast<int64_t>(floor(__dadd_rn(__dmul_rn(static_cast<double>(kr), static_cast<double>(N)), 0.5)));
-    Rmin = ratio_grid(ap.r_min);
-    Rmax = ratio_grid(ap.r_max);
     rule = make_ratio_rule(kr, ap.alpha, ap.relative);
     inv_N = recip62(N);
     inv_n = recip62(n_lane);
@@ -461,7 +461,7 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
     if (warp == 0) {
       const int64_t S = lane < m ? (static_cast<int64_t>(n_lane) << 30) : 0;
       int32_t K = 0;
-      const int err = warp_allocate32(m, S, n_lane, inv_n, B, N, inv_N, rule, Rmin, Rmax, &K);
+      const int err = warp_allocate32(wsm32, m, S, n_lane, inv_n, B, N, inv_N, rule, ap.alpha, ap.r_min, ap.r_max, &K);
       asm volatile("" ::"r"(K), "r"(err));
 #pragma unroll
       for (int q = 0; q < 8; ++q) sh.hist[0][lane * 8 + q] = 0;
@@ -498,14 +498,14 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
     if (m <= 32) {
       const int64_t S = lane < m ? ap.img_sums[i0 + lane] : 0;
       int32_t K;
-      err = warp_allocate32(m, S, n_lane, inv_n, B, N, inv_N, rule, Rmin, Rmax, &K);
+      err = warp_allocate32(wsm32, m, S, n_lane, inv_n, B, N, inv_N, rule, ap.alpha, ap.r_min, ap.r_max, &K);
       k = __shfl_sync(kFull, K, li);
       before = warp_sum(lane < li ? K : 0);
       total = warp_sum(lane < m ? K : 0);
     } else {
-      for (int j = lane; j < m; j += 32) wsm.X[j] = ap.img_sums[i0 + j];
+      for (int j = lane; j < m; j += 32) wsm.S[j] = ap.img_sums[i0 + j];
       __syncwarp();
-      err = warp_allocate(wsm, m, B, N, kr, ap.alpha, Rmin, Rmax, ap.relative);
+      err = warp_allocate(wsm, m, B, N, kr, ap.alpha, ap.r_min, ap.r_max, ap.relative);
       int bs = 0, ts = 0;
       for (int j = lane; j < m; j += 32) {
         ts += wsm.K[j];
@@ -619,13 +619,12 @@ cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int
 }
 
 int alloc_select_ctas_per_sm() {
-  static int cached = 0;
-  if (cached == 0) {
-    int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_alloc_select, kThreads, 0) != cudaSuccess || n < 1) n = 1;
-    cached = n;
-  }
-  return cached;
+  static PerDevice occ;
+  int n = 0;
+  const cudaError_t e = once_per_device(occ, [](int, int* v) {
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(v, k_alloc_select, kThreads, 0);
+  }, &n);
+  return (e == cudaSuccess && n >= 1) ? n : 1;
 }
 
 cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
@@ -646,15 +645,14 @@ cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums,
   if (ap.m_cap < 1) ap.m_cap = 1;
   // the budget scratch is only used for requests of more than 32 images
   const size_t smem = ap.m_cap > 32 ? warp_alloc_smem_bytes(ap.m_cap) : 0;
-  static bool carveout_set = false;
-  if (!carveout_set) {
-    // same shared-memory configuration as the scoring kernels, so that a CTA of this
-    // kernel can start on an SM where a scoring CTA still runs
-    cudaError_t e = cudaFuncSetAttribute(k_alloc_select, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                         cudaSharedmemCarveoutMaxShared);
-    if (e != cudaSuccess) return e;
-    carveout_set = true;
-  }
+  // same shared-memory configuration as the scoring kernels, so that a CTA of this
+  // kernel can start on an SM where a scoring CTA still runs
+  static PerDevice carveout;
+  const cudaError_t ce = once_per_device(carveout, [](int, int*) {
+    return cudaFuncSetAttribute(k_alloc_select, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                cudaSharedmemCarveoutMaxShared);
+  });
+  if (ce != cudaSuccess) return ce;
   if (smem > 16 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(k_alloc_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));

@@ -51,4 +51,7 @@ def assert_scores_close(got: np.ndarray, ref: np.ndarray, mask: np.ndarray):
 
 
 def near_tie(a: float, b: float) -> bool:
-    return abs(a - b) <= 2.0 * (ATOL + RTOL * max(abs(a), abs(b)))
+    """Oracle scores a and b are within the score tolerance of each other."""
+    if np.isnan(a) or np.isnan(b):
+        return np.isnan(a) and np.isnan(b)
+    return abs(a - b) <= ATOL + RTOL * max(abs(a), abs(b))

@@ -2,10 +2,11 @@
 
 4 requests x 64 images x 1024 visual tokens (+512 text tokens each), hidden 4096,
 32/8 heads of 128: 264,192 tokens, about 8 GB on the device. The requests are
-independent and identically shaped, so the oracle scores request 0 (criterion A:
-every visual row; criterion B: every visual key, from the full causal attention of
-that request) and checks steps 2-4 on the whole batch fed the GPU's own scores:
-budgets, kept indices and the gathered rows bit-exact.
+independent, so the oracle scores them one at a time: criterion A on every visual row
+of all four requests, criterion B on every visual key of requests 0 and 3 (the full
+causal attention of each). Request 3's rows of h_cur start past 2^31 bytes and its text
+queries too, where a 32-bit offset would show. Steps 2-4 are checked on the whole batch
+fed the GPU's own scores: budgets, kept indices and the gathered rows bit-exact.
 """
 import numpy as np
 import pytest
@@ -30,14 +31,14 @@ def long_workload():
     torch.cuda.empty_cache()
 
 
-def _request0(wl):
-    """Layout and tensors of request 0 alone (its tokens are the first T_0 packed rows)."""
+def _request(wl, r):
+    """Layout of request r alone and its packed token range [a, b)."""
     lay = wl.layout
-    T0 = int(lay.cu_seqlens[1])
-    n0 = int(lay.img_cu[1])
-    sub = synth.Layout(cu_seqlens=np.array([0, T0], dtype=np.int32), img_cu=np.array([0, n0], dtype=np.int32),
-                       img_start=lay.img_start[:n0].copy(), img_len=lay.img_len[:n0].copy())
-    return sub, T0
+    a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+    i0, i1 = int(lay.img_cu[r]), int(lay.img_cu[r + 1])
+    sub = synth.Layout(cu_seqlens=np.array([0, b - a], dtype=np.int32), img_cu=np.array([0, i1 - i0], dtype=np.int32),
+                       img_start=lay.img_start[i0:i1].copy(), img_len=lay.img_len[i0:i1].copy())
+    return sub, a, b
 
 
 @pytest.mark.parametrize("criterion", ["hidden_variation", "text_attention"])
@@ -51,14 +52,19 @@ def test_prune_long_workload(long_workload, criterion):
     assert avtp.read_device_status(out.workspace) == avtp.OK
     got = out.scores.cpu().numpy()
 
-    # step 1 on request 0 against the oracle
-    sub, T0 = _request0(wl)
-    if criterion == "hidden_variation":
-        ref = O.score_hidden_variation(sub, wl.h_cur[:T0], wl.h_prior[:T0])
-    else:
-        ref = O.score_text_attention(sub, wl.q[:T0], wl.k[:T0], wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
-    vis0 = sub.visual_mask()
-    np.testing.assert_allclose(got[:T0][vis0], ref[vis0], rtol=RTOL, atol=ATOL)
+    # step 1 against the oracle, request by request
+    row_bytes = wl.h_cur.shape[1] * 2
+    requests = range(lay.n_requests) if criterion == "hidden_variation" else (0, lay.n_requests - 1)
+    for r in requests:
+        sub, a, b = _request(wl, r)
+        if r == lay.n_requests - 1:
+            assert b * row_bytes > 2 ** 31  # the last request's rows end past 2^31 bytes
+        if criterion == "hidden_variation":
+            ref = O.score_hidden_variation(sub, wl.h_cur[a:b], wl.h_prior[a:b])
+        else:
+            ref = O.score_text_attention(sub, wl.q[a:b], wl.k[a:b], wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
+        vis = sub.visual_mask()
+        np.testing.assert_allclose(got[a:b][vis], ref[vis], rtol=RTOL, atol=ATOL, err_msg=f"request {r}")
 
     # steps 2-4 on the whole batch, fed the GPU's scores: bit-exact
     exp = O.prune(lay, keep_ratio=wl.keep_ratio, scores_f32=got, relative=relative, planes={"pos": wl.pos})

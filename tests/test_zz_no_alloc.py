@@ -8,15 +8,16 @@ keeps its scratch in a fixed device array inside the library, instead of in
 a caller workspace.
 
 These tests call it through the C ABI, twice in a row on one stream with
-different layouts. Each result must equal the workspace-based avtp_select
-exactly: kept indices are integers, so the tolerance is bit-exact, as for
-avtp_select itself. This file is named to be collected last; it also passes on
-its own in a fresh process.
+different layouts. Each result must equal the workspace-based avtp_select and
+the oracle's selection exactly: kept indices are integers, so the tolerance is
+bit-exact, as for avtp_select itself. This file is named to be collected last;
+it also passes on its own in a fresh process.
 """
 import numpy as np
 import pytest
 import torch
 
+from oracle import avtp_oracle as O
 from paper_2608_26806_gb300 import avtp, synth
 from tests.gpu_util import dev_layout, ensure_built
 
@@ -47,7 +48,8 @@ def _case(segments, seed):
         out_cu[r + 1] = out_cu[r] + k + int((~vis[a:b]).sum())
     L = dev_layout(lay)
     return dict(L=L, scores=torch.from_numpy(sc).cuda(), budgets=torch.from_numpy(budgets).cuda(),
-                out_cu=torch.from_numpy(out_cu).cuda(), n_kept=int(out_cu[-1]))
+                out_cu=torch.from_numpy(out_cu).cuda(), n_kept=int(out_cu[-1]),
+                expected=O.select(lay, sc, budgets))
 
 
 SEG_A = [[("t", 64)] + sum([[("t", 1), ("i", n), ("t", 1)] for n in (256, 1024, 640, 320, 900, 3000)], []) +
@@ -72,6 +74,7 @@ def test_noalloc_select_matches_workspace_select_twice_in_a_row():
         torch.cuda.synchronize()
         assert int(st.item()) == avtp.OK
         assert torch.equal(kept[:c["n_kept"]].cpu(), ref.cpu())
+        assert np.array_equal(kept[:c["n_kept"]].cpu().numpy(), c["expected"])
         assert torch.all(kept[c["n_kept"]:].cpu() == -7)  # nothing written past n_kept
 
 
