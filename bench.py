@@ -200,7 +200,7 @@ def stage_roofline(acct, ms_step, hbm_gbs, bf16_tflops, peak_kind):
     return out
 
 
-def stage_accounting(wl, criterion, n_kept, lse=False):
+def stage_accounting(wl, criterion, n_kept, lse=False, query_set="text"):
     lay = wl.layout
     n_vis = int(lay.n_visual_per_request().sum())
     n_txt = lay.n_tokens - n_vis
@@ -212,6 +212,19 @@ def stage_accounting(wl, criterion, n_kept, lse=False):
         # compulsory: both visual rows once, text rows once (kept), kept rows written, positions
         stage_bytes = score_bytes + n_txt * D * 2 + n_kept * D * 2 + n_kept * pos_bytes * 2
         flops = 0
+    elif query_set == "last":
+        # the request's last token as the only query (CUDA-core path): every key once, the
+        # last token's query rows; FMAs, not tensor-core work, so the stage is HBM-bound
+        Hq, Hkv, d = wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+        R = lay.n_requests
+        score_bytes = lay.n_tokens * Hkv * d * 2 + R * Hq * d * 2
+        stage_bytes = score_bytes + n_txt * D * 2 + n_kept * D * 2 + n_kept * pos_bytes * 2
+        fma_flops = 0
+        for r in range(R):
+            T_r = int(lay.cu_seqlens[r + 1]) - int(lay.cu_seqlens[r])
+            fma_flops += 2 * Hq * d * T_r + 2 * Hq * d * int(lay.n_visual_per_request()[r])
+        return {"n_vis": n_vis, "n_txt": n_txt, "score_bytes": int(score_bytes), "stage_bytes": int(stage_bytes),
+                "gather_bytes": int(gather), "flops": 0, "fma_flops": int(fma_flops)}
     else:
         Hq, Hkv, d = wl.n_q_heads, wl.n_kv_heads, wl.head_dim
         if lse:  # supplied LSE: visual keys, text queries and the text rows' LSE only
@@ -307,13 +320,15 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     # the other scoring criterion (text-to-visual attention), timed the same way on the
     # same workload, for a secondary object of the line
-    sec = sec_lse = prog = None
+    sec = sec_lse = sec_last = prog = None
     if second is not None:
         sec = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev)
         lse = fa_lse(wl, bf16(wl.q), bf16(wl.k), torch)
         torch.cuda.synchronize()
         sec_lse = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev, lse=lse)
         del lse
+        sec_last = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev,
+                                  query_set="last")
         prog = time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avtp, world, dev)
     variants = time_variants(args, call, stream, flush, torch, avtp, 4 if crit == "hidden_variation" else 7)
     clocks = sampler.stop() if sampler else None
@@ -325,9 +340,13 @@ def run_ours(args, world, rank, local):
     total_ms = sum(step_ms)
     value, ms_step = whole_job_rate(acct["n_vis"], K, total_ms, world, dev)
 
-    # end to end through the public API: pinned host inputs -> device -> prune -> host outputs
+    # end to end through the public API: pinned host inputs -> device -> prune -> host outputs,
+    # with the process (and so the pinned buffers it touches first) on the GPU's NUMA node
+    numa, prev_cpus = bind_to_gpu_numa_node(dev.index if dev.index is not None else 0)
     e2e = run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp)
     e2e_pipe = run_e2e_pipelined(args, wl, crit, L, call, dev, torch, avtp)
+    e2e["numa"] = numa
+    os.sched_setaffinity(0, prev_cpus)
 
     if rank != 0:
         return None
@@ -387,11 +406,33 @@ def run_ours(args, world, rank, local):
                                "algorithmic_flops_per_launch": res["acct"]["flops"]},
             "gpu_launches": res["launches"]}
         line["gpu_launches"] += res["launches"]
+    if sec_last is not None:
+        ms3 = sec_last["ms_per_step"]
+        score_us = sec_last["steps_us"]["score"]
+        a3 = sec_last["acct"]
+        line["text_attention_last"] = {
+            "criterion": "text_attention", "query_set": "last (the request's last token, §4.1)",
+            "path": "CUDA cores", "value": round(a3["n_vis"] / (ms3 * 1e-3), 1), "unit": UNIT,
+            "ms_per_step": round(ms3, 5), "steps": sec_last["steps"], "latency_us": sec_last["latency_us"],
+            "steps_us": sec_last["steps_us"],
+            "stage_roofline": stage_roofline(a3, ms3, hbm_s, bf16_s, peak_kind),
+            "score_roofline": {"bound": "hbm", "kernel": "score (lse + merge + mass + finalize)",
+                               "achieved": round(a3["score_bytes"] / (score_us * 1e-6) / 1e9, 1), "peak": hbm_s,
+                               "unit": "GB/s",
+                               "frac": round(a3["score_bytes"] / (score_us * 1e-6) / 1e9 / hbm_s, 4),
+                               "algorithmic_bytes_per_launch": a3["score_bytes"],
+                               "fma_flops_per_launch": a3["fma_flops"]},
+            "gpu_launches": sec_last["launches"]}
+        line["gpu_launches"] += sec_last["launches"]
     if prog is not None:
         line["progressive"] = prog
         line["gpu_launches"] += prog["gpu_launches"]
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, crit, args.cpu_seconds)
+        if not args.no_all_core_baseline:
+            n_img = int(wl.layout.img_cu[1])
+            line["cpu_baseline"]["all_cores"] = cpu_baseline_all_cores(args.config, crit, n_img,
+                                                                       min(10.0, args.cpu_seconds))
     return line
 
 
@@ -470,13 +511,15 @@ def fa_lse(wl, q, k, torch):
     return out
 
 
-def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev, lse=None):
+def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev, lse=None,
+                   query_set="text"):
     """The attention criterion on the same workload: whole-call latency and per-step times."""
     crit = "text_attention"
     extra = {} if lse is None else {"lse": lse}
     call = avtp.PruneCall(L, crit, keep_ratio=kr, keep_ratio_host=wl.keep_ratio, rows={"hidden": h_cur},
-                          planes={"pos": pos}, q=bf16(wl.q), k=bf16(wl.k), softmax_scale=wl.softmax_scale, **extra)
-    acct = stage_accounting(wl, crit, call.buffers.n_kept, lse=lse is not None)
+                          planes={"pos": pos}, q=bf16(wl.q), k=bf16(wl.k), softmax_scale=wl.softmax_scale,
+                          query_set=query_set, **extra)
+    acct = stage_accounting(wl, crit, call.buffers.n_kept, lse=lse is not None, query_set=query_set)
     K = max(10, min(args.steps, 300))
     n_ev = avtp.N_STEP_EVENTS
     outer = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
@@ -511,7 +554,7 @@ def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp
             "latency_us": {"p50": round(step_ms[len(step_ms) // 2] * 1e3, 2),
                            "p90": round(step_ms[int(len(step_ms) * 0.9)] * 1e3, 2)},
             "steps_us": {k: round(v * 1e3, 2) for k, v in per_step.items()},
-            "launches": K * (7 if lse is None else 6)}
+            "launches": K * ((7 if lse is None else 6) if query_set == "text" else 7)}
 
 
 def time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avtp, world, dev, stages=3):
@@ -807,6 +850,85 @@ def cpu_baseline(wl, crit, seconds):
                       f"{int(sub.img_len.sum())} visual tokens), criterion {crit}, {el:.1f} s"}
 
 
+def _oracle_worker(config, crit, n_img, seconds, start_at):
+    """One process of the all-core oracle baseline: the same bounded sample, run from a
+    common start time for `seconds`; returns (visual tokens done, seconds)."""
+    from oracle import avtp_oracle as O
+    from paper_2608_26806_gb300 import synth
+
+    parts = ("A", "pos") if crit == "hidden_variation" else ("A", "B", "pos")
+    wl = synth.make_workload(config, parts=parts)
+    sub, t = _sub_workload(wl, n_img)
+    while time.time() < start_at:
+        time.sleep(0.005)
+    t0 = time.perf_counter()
+    runs = 0
+    while True:
+        _oracle_step(O, sub, t, wl, crit)
+        runs += 1
+        if time.perf_counter() - t0 > seconds:
+            break
+    return runs * int(sub.img_len.sum()), time.perf_counter() - t0
+
+
+def cpu_baseline_all_cores(config, crit, n_img, seconds):
+    """The oracle on every host core: one process per core (spawned, one BLAS thread each),
+    all running the same bounded sample over a common window."""
+    import multiprocessing as mp
+
+    cores = len(os.sched_getaffinity(0))
+    saved = {k: os.environ.get(k) for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")}
+    for k in saved:
+        os.environ[k] = "1"
+    try:
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(cores) as pool:
+            start_at = time.time() + 25.0  # every worker has built its sample by then
+            res = pool.starmap(_oracle_worker, [(config, crit, n_img, seconds, start_at)] * cores)
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    tokens = sum(r[0] for r in res)
+    window = max(r[1] for r in res)
+    return {"value": round(tokens / window, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{cores} processes, each the oracle pipeline over the same request-0 sample "
+                      f"({n_img} images) for {seconds:.0f} s from a common start, criterion {crit}"}
+
+
+def bind_to_gpu_numa_node(dev_index):
+    """Pin this process to the CPUs of the GPU's NUMA node (when the platform reports one),
+    so that pinned host buffers allocated afterwards sit on that node (first touch).
+    Returns (what was done, the previous CPU set to restore)."""
+    prev = os.sched_getaffinity(0)
+    info = {"gpu_numa_node": None, "bound": False, "process_cpus": len(prev)}
+    try:
+        import subprocess
+
+        bus = subprocess.run(["nvidia-smi", "--query-gpu=pci.bus_id", "--format=csv,noheader", "-i",
+                              str(dev_index)], capture_output=True, text=True, timeout=20).stdout.strip()
+        dom, rest = bus.split(":", 1)
+        path = f"/sys/bus/pci/devices/{dom[-4:].lower()}:{rest.lower()}/numa_node"
+        node = int(open(path).read().strip())
+        info["gpu_numa_node"] = node
+        if node >= 0:
+            cpulist = open(f"/sys/devices/system/node/node{node}/cpulist").read().strip()
+            cpus = set()
+            for part in cpulist.split(","):
+                if part:
+                    a, _, b = part.partition("-")
+                    cpus.update(range(int(a), int(b or a) + 1))
+            cpus &= prev
+            if cpus:
+                os.sched_setaffinity(0, cpus)
+                info.update(bound=True, process_cpus=len(cpus), node_cpulist=cpulist)
+    except Exception as e:  # noqa: BLE001 - a platform without the information keeps the default placement
+        info["note"] = f"no NUMA binding: {type(e).__name__}"
+    return info, prev
+
+
 def run_reference(args, world, rank):
     if rank != 0:
         return None
@@ -858,6 +980,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-all-core-baseline", action="store_true",
+                    help="skip the oracle timed on every host core (about 35 s)")
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-secondary", action="store_true",
                     help="skip the attention-criterion object (timed after the headline criterion)")

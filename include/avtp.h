@@ -74,6 +74,21 @@ typedef enum {
   AVTP_CRIT_TEXT_ATTENTION = 1
 } avtp_criterion_t;
 
+/* Queries whose attention scores the visual keys under AVTP_CRIT_TEXT_ATTENTION. */
+typedef enum {
+  AVTP_QUERIES_TEXT = 0,  /* every text token of the request (paper §3.3.2)                     */
+  AVTP_QUERIES_LAST = 1   /* the request's last token alone, the token whose output predicts the
+                           * first generated token: the attention FAST-V ranks by (paper §4.1) */
+} avtp_query_set_t;
+
+/* Where AVTP_CRIT_TEXT_ATTENTION computes its logits. */
+typedef enum {
+  AVTP_PATH_AUTO = 0,    /* tensor cores when the rows of a request and KV group (queries x
+                          * heads of the group) fill their 128-row tiles, CUDA cores otherwise */
+  AVTP_PATH_TENSOR = 1,  /* tcgen05 tensor cores (AVTP_QUERIES_TEXT only)                   */
+  AVTP_PATH_CUDA = 2     /* CUDA-core FMA, a thread per key                                  */
+} avtp_attn_path_t;
+
 typedef struct {
   int32_t n_requests;         /* R >= 1 (host scalar)                         */
   int32_t n_images;           /* total images over all requests, >= 0 (host)  */
@@ -117,6 +132,12 @@ typedef struct {
    * queries repacked by KV group). 0: n_tokens. A batch with more text tokens
    * than this reports AVTP_ERR_RANGE. */
   int64_t max_text_tokens;
+  /* AVTP_CRIT_TEXT_ATTENTION: the query set (avtp_query_set_t) and the path
+   * (avtp_attn_path_t); 0 and 0 give every text token and the automatic choice.
+   * AVTP_PATH_TENSOR with AVTP_QUERIES_LAST returns AVTP_ERR_UNSUPPORTED. With
+   * AVTP_QUERIES_LAST a supplied lse holds the last token's row of each request. */
+  int32_t query_set;
+  int32_t path;
 } avtp_score_args_t;
 
 typedef struct {
@@ -274,6 +295,30 @@ AVTP_API avtp_status_t avtp_pruned_layout(const avtp_layout_t* layout, const int
  * inputs of the same call for the next stage. */
 AVTP_API int64_t avtp_kept_count_vis_host(const int32_t* cu_seqlens, const int32_t* n_vis, const float* keep_ratio,
                                           int32_t n_requests, int32_t* out_cu_seqlens, int32_t* out_n_vis);
+
+/* Pruning-layer selection (paper §3.3.2): the attention a layer assigns to the visual
+ * tokens of each sample, A_l^(i) = sum_j Attention(l, v_j), is the sum of the sample
+ * request's fixed-point image sums of AVTP_CRIT_TEXT_ATTENTION at that layer (run
+ * avtp_score with that layer's q and k). avtp_layer_attention writes that sum, for every
+ * request r of the layout, to A[r * n_layers + layer] (device int64 [R, n_layers], units
+ * of 2^-32); one call per layer fills one column. img_sums: device int64 [n_images] from
+ * avtp_score. The layout is validated as in the other calls (workspace of
+ * avtp_workspace_size(layout, NULL) bytes). Asynchronous on `stream`. */
+#define AVTP_MAX_LAYERS 1024
+AVTP_API avtp_status_t avtp_layer_attention(const avtp_layout_t* layout, const int64_t* img_sums, int64_t* A,
+                                            int32_t n_layers, int32_t layer, void* workspace, size_t workspace_bytes,
+                                            avtp_stream_t stream);
+
+/* The layer ranking of paper §3.3.2 over n_samples samples and n_layers layers (at most
+ * AVTP_MAX_LAYERS): per sample, Rank(A_l^(i)) = 1 for the layer with the most attention
+ * (equal values rank the lower layer first); rank_sum[l] = sum_i Rank(A_l^(i)), so the
+ * average rank is R_l = rank_sum[l] / n_samples (device int64 [n_layers]); top_layers
+ * (device int32 [k], 1 <= k <= n_layers) receives the k layers with the best average
+ * rank, best first, ties to the lower layer. A: device int64 [n_samples, n_layers],
+ * row-major, as avtp_layer_attention writes it. Exact integer arithmetic. Asynchronous
+ * on `stream`. */
+AVTP_API avtp_status_t avtp_layer_select(const int64_t* A, int32_t n_samples, int32_t n_layers, int32_t k,
+                                         int64_t* rank_sum, int32_t* top_layers, avtp_stream_t stream);
 
 /* Check of the failure path every pipeline kernel takes when a wait on an mbarrier (a
  * TMA copy, a tensor-core commit, a hand-off between warps) does not complete: one CTA

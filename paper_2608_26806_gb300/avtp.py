@@ -37,6 +37,11 @@ MAX_ROW_SETS = 8
 N_STEP_EVENTS = 5
 
 _CRITERIA = {"hidden_variation": CRIT_HIDDEN_VARIATION, "text_attention": CRIT_TEXT_ATTENTION}
+# avtp_query_set_t and avtp_attn_path_t
+QUERIES_TEXT, QUERIES_LAST = 0, 1
+PATH_AUTO, PATH_TENSOR, PATH_CUDA = 0, 1, 2
+_QUERY_SETS = {"text": QUERIES_TEXT, "last": QUERIES_LAST}
+_PATHS = {"auto": PATH_AUTO, "tensor": PATH_TENSOR, "cuda": PATH_CUDA}
 
 
 class AVTPError(RuntimeError):
@@ -57,7 +62,7 @@ class _ScoreArgs(ctypes.Structure):
                 ("h_cur_stride", c_int64), ("h_prior_stride", c_int64), ("q", c_void_p), ("k", c_void_p),
                 ("n_q_heads", c_int32), ("n_kv_heads", c_int32), ("head_dim", c_int32), ("q_stride", c_int64),
                 ("k_stride", c_int64), ("softmax_scale", c_float), ("lse", c_void_p), ("lse_stride", c_int64),
-                ("max_text_tokens", c_int64)]
+                ("max_text_tokens", c_int64), ("query_set", c_int32), ("path", c_int32)]
 
 
 class _AllocArgs(ctypes.Structure):
@@ -91,6 +96,9 @@ SIGNATURES = {
     "avtp_pruned_layout": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "avtp_kept_count_vis_host": (c_int64, [c_void_p, c_void_p, c_void_p, c_int32, c_void_p, c_void_p]),
     "avtp_wait_selftest": (c_int, [c_int64, c_int32, c_void_p, c_size_t, c_void_p]),
+    "avtp_layer_attention": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_int32, c_int32, c_void_p, c_size_t,
+                                     c_void_p]),
+    "avtp_layer_select": (c_int, [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p, c_void_p]),
     "avtp_read_device_status": (c_int, [c_void_p, c_void_p, POINTER(c_int32)]),
     "avtp_status_string": (ctypes.c_char_p, [c_int32]),
     "avtp_version": (c_int32, []),
@@ -98,8 +106,9 @@ SIGNATURES = {
 
 
 def library_path() -> str:
-    """Path of the in-tree libavtp.so that ``load()`` opens."""
-    return _build.LIB_PATH
+    """Path of the in-tree libavtp.so that ``load()`` opens: the diagnostic timeline build
+    when the environment sets AVTP_TIMELINE=1, the normal build otherwise."""
+    return _build.TIMELINE_LIB_PATH if os.environ.get("AVTP_TIMELINE") == "1" else _build.LIB_PATH
 
 
 def load() -> ctypes.CDLL:
@@ -110,7 +119,7 @@ def load() -> ctypes.CDLL:
     path = library_path()
     if not os.path.exists(path):
         if os.environ.get("AVTP_AUTOBUILD") == "1":
-            _build.build()
+            _build.build(timeline=path == _build.TIMELINE_LIB_PATH)
         else:
             raise RuntimeError(f"libavtp.so is not built ({path}); run __graft_entry__.build() first")
     lib = ctypes.CDLL(path)
@@ -120,6 +129,25 @@ def load() -> ctypes.CDLL:
         fn.argtypes = args
     _LIB = lib
     return lib
+
+
+TIMELINE_EVENTS = ("prep_begin", "prep_end", "score_begin", "score_end", "select_begin", "select_waited",
+                   "rule_end", "select_end", "compact_begin", "compact_waited", "compact_end")
+
+
+def timeline(workspace: torch.Tensor) -> Dict[str, Tuple[int, int]]:
+    """Phase stamps of the last avtp_prune on ``workspace`` (timeline build only): event ->
+    (earliest, latest) global-timer nanoseconds over the CTAs that reached it; events no CTA
+    reached are left out. Synchronises the device."""
+    torch.cuda.synchronize()
+    n = len(TIMELINE_EVENTS)
+    raw = workspace[16:16 + 16 * n].cpu().numpy().view(np.uint64)
+    out = {}
+    for i, name in enumerate(TIMELINE_EVENTS):
+        lo, hi = int(raw[i]), int(raw[n + i])
+        if lo != 2 ** 64 - 1:
+            out[name] = (lo, hi)
+    return out
 
 
 def status_string(code: int) -> str:
@@ -199,9 +227,11 @@ class Layout:
 
 
 def _score_args(criterion, h_cur=None, h_prior=None, q=None, k=None, softmax_scale=None, lse=None,
-                max_text_tokens=0) -> _ScoreArgs:
+                max_text_tokens=0, query_set="text", path="auto") -> _ScoreArgs:
     a = _ScoreArgs()
     a.max_text_tokens = int(max_text_tokens)
+    a.query_set = _QUERY_SETS[query_set] if isinstance(query_set, str) else int(query_set)
+    a.path = _PATHS[path] if isinstance(path, str) else int(path)
     a.criterion = _CRITERIA[criterion] if isinstance(criterion, str) else int(criterion)
     if a.criterion == CRIT_HIDDEN_VARIATION:
         for t in (h_cur, h_prior):
@@ -262,17 +292,22 @@ def new_workspace(nbytes: int, device="cuda") -> torch.Tensor:
 
 # ---------------------------------------------------------------- entry points
 def score(layout: Layout, criterion, *, h_cur=None, h_prior=None, q=None, k=None, softmax_scale=None, lse=None,
-          scores=None, img_sums=None, workspace=None, stream=None):
-    """avtp_score: per-token scores (fp32 [T], text entries untouched) and fixed-point per-image sums."""
+          query_set="text", path="auto", scores=None, img_sums=None, workspace=None, stream=None):
+    """avtp_score: per-token scores (fp32 [T], text entries untouched) and fixed-point per-image sums.
+
+    Text attention: ``query_set`` "text" (every text token) or "last" (the request's last
+    token); ``path`` "auto", "tensor" (tcgen05) or "cuda" (CUDA cores)."""
     dev = layout.cu_seqlens.device
-    sa = _score_args(criterion, h_cur, h_prior, q, k, softmax_scale, lse, max_text_tokens=layout.n_text)
+    sa = _score_args(criterion, h_cur, h_prior, q, k, softmax_scale, lse, max_text_tokens=layout.n_text,
+                     query_set=query_set, path=path)
     if scores is None:
         scores = torch.zeros(layout.n_tokens, dtype=torch.float32, device=dev)
     if img_sums is None:
         img_sums = torch.empty(max(layout.n_images, 1), dtype=torch.int64, device=dev)
     if workspace is None:
         workspace = new_workspace(workspace_size(layout, criterion, h_cur=h_cur, h_prior=h_prior, q=q, k=k,
-                                                 softmax_scale=softmax_scale, lse=lse), dev)
+                                                 softmax_scale=softmax_scale, lse=lse, query_set=query_set,
+                                                 path=path), dev)
     lay = layout.c()
     _check(load().avtp_score(ctypes.byref(lay), ctypes.byref(sa), _ptr(scores), _ptr(img_sums), _ptr(workspace),
                              workspace.numel(), _stream(stream)), "avtp_score")
@@ -401,6 +436,31 @@ def wait_selftest(limit_ns: int, arrive: bool, workspace: torch.Tensor, stream=N
     _check(load().avtp_wait_selftest(int(limit_ns), 1 if arrive else 0, _ptr(workspace),
                                      workspace.numel() * workspace.element_size(), _stream(stream)),
            "avtp_wait_selftest")
+
+
+def layer_attention(layout: Layout, img_sums: torch.Tensor, A: torch.Tensor, layer: int, workspace=None,
+                    stream=None) -> torch.Tensor:
+    """avtp_layer_attention: column ``layer`` of A (int64 [R, n_layers]) <- each request's
+    sum of text-attention image sums at that layer (pruning-layer selection, §3.3.2)."""
+    if A.dtype != torch.int64 or A.dim() != 2 or not A.is_contiguous() or A.shape[0] != layout.n_requests:
+        raise ValueError("A must be a contiguous int64 [R, n_layers] tensor")
+    if workspace is None:
+        workspace = new_workspace(workspace_size(layout), A.device)
+    lay = layout.c()
+    _check(load().avtp_layer_attention(ctypes.byref(lay), _ptr(img_sums), _ptr(A), A.shape[1], int(layer),
+                                       _ptr(workspace), workspace.numel(), _stream(stream)), "avtp_layer_attention")
+    return A
+
+
+def layer_select(A: torch.Tensor, k: int, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """avtp_layer_select: (rank_sum int64 [n_layers], top_layers int32 [k]) from A [N, n_layers]."""
+    if A.dtype != torch.int64 or A.dim() != 2 or not A.is_contiguous():
+        raise ValueError("A must be a contiguous int64 [n_samples, n_layers] tensor")
+    rank_sum = torch.empty(A.shape[1], dtype=torch.int64, device=A.device)
+    top = torch.empty(int(k), dtype=torch.int32, device=A.device)
+    _check(load().avtp_layer_select(_ptr(A), A.shape[0], A.shape[1], int(k), _ptr(rank_sum), _ptr(top),
+                                    _stream(stream)), "avtp_layer_select")
+    return rank_sum, top
 
 
 def read_device_status(workspace: torch.Tensor, stream=None) -> int:

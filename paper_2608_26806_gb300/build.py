@@ -20,6 +20,9 @@ CSRC = os.path.join(PKG_DIR, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG_DIR, "_build")
 LIB_PATH = os.path.join(BUILD_DIR, "libavtp.so")
+# diagnostic variant: the fused stage records phase stamps (-DAVTP_TIMELINE), built apart
+TIMELINE_BUILD_DIR = os.path.join(BUILD_DIR, "timeline")
+TIMELINE_LIB_PATH = os.path.join(TIMELINE_BUILD_DIR, "libavtp.so")
 
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH_FLAGS + [
@@ -48,16 +51,16 @@ def _deps() -> List[str]:
     return files
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB_PATH):
+def up_to_date(lib_path: str = LIB_PATH) -> bool:
+    if not os.path.exists(lib_path):
         return False
-    t = os.path.getmtime(LIB_PATH)
+    t = os.path.getmtime(lib_path)
     return all(os.path.getmtime(f) <= t for f in _deps())
 
 
-def _compile(src: str, verbose: bool, ptxas_info: bool) -> str:
-    obj = os.path.join(BUILD_DIR, os.path.basename(src)[:-3] + ".o")
-    cmd = [nvcc_path(), "-c", src, "-o", obj] + NVCC_FLAGS
+def _compile(src: str, verbose: bool, ptxas_info: bool, out_dir: str = BUILD_DIR, extra=()) -> str:
+    obj = os.path.join(out_dir, os.path.basename(src)[:-3] + ".o")
+    cmd = [nvcc_path(), "-c", src, "-o", obj] + NVCC_FLAGS + list(extra)
     if ptxas_info:
         cmd += ["-Xptxas", "-v"]
     res = subprocess.run(cmd, capture_output=True, text=True)
@@ -68,22 +71,27 @@ def _compile(src: str, verbose: bool, ptxas_info: bool) -> str:
     return obj
 
 
-def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
-    """Compile and link libavtp.so; return its path."""
-    if not force and up_to_date():
-        return LIB_PATH
-    os.makedirs(BUILD_DIR, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False, timeline: bool = False) -> str:
+    """Compile and link libavtp.so; return its path. ``timeline``: the diagnostic variant
+    whose fused stage records phase stamps, in its own folder."""
+    out_dir = TIMELINE_BUILD_DIR if timeline else BUILD_DIR
+    lib_path = TIMELINE_LIB_PATH if timeline else LIB_PATH
+    extra = ["-DAVTP_TIMELINE"] if timeline else []
+    if not force and up_to_date(lib_path):
+        return lib_path
+    os.makedirs(out_dir, exist_ok=True)
     srcs = sources()
     with cf.ThreadPoolExecutor(max_workers=min(len(srcs), os.cpu_count() or 4)) as ex:
-        objs = list(ex.map(lambda s: _compile(s, verbose, ptxas_info), srcs))
-    tmp = LIB_PATH + ".tmp"
+        objs = list(ex.map(lambda s: _compile(s, verbose, ptxas_info, out_dir, extra), srcs))
+    tmp = lib_path + ".tmp"
     cmd = [nvcc_path(), "-shared", "-o", tmp] + objs + ARCH_FLAGS + ["-Xcompiler", "-fvisibility=hidden"]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stderr}")
-    os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose=True, ptxas_info="--ptxas" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose=True, ptxas_info="--ptxas" in sys.argv,
+                timeline="--timeline" in sys.argv))

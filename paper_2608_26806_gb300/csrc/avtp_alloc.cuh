@@ -342,10 +342,11 @@ static __device__ __noinline__ uint64_t warp_sort_desc(uint64_t v) {
   return v;
 }
 
+// cls: this lane's image in the partition to check (kClsFree, kClsLow or kClsHigh);
+// all_free: every image is free, which needs no class sums.
 template <bool kRel>
-__device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int64_t R, int64_t lam, int64_t Rmin,
-                                       int64_t Rmax, int64_t B, int64_t N, int64_t T, int64_t Rb, int64_t Aa,
-                                       int64_t mq, int64_t Mq, int32_t* k_out) {
+__device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int cls, bool all_free, int64_t B, int64_t N,
+                                       int64_t T, int64_t Rb, int64_t Aa, int64_t mq, int64_t Mq, int32_t* k_out) {
   const int lane = threadIdx.x & 31;
   if (!has) { S = 0; n = 0; }
   u128 Xh = 0, Q = 1;  // X_i >> 64, and the request's Q
@@ -358,15 +359,17 @@ __device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int64_t R
     Xh = static_cast<u128>(n * B);
     Q = static_cast<u128>(N);
   } else {
-    // ---- the partition the grid's shift implies, checked exactly
-    const int64_t g = R + lam;
-    const int cls = !has ? kClsFree : (g <= Rmin ? kClsLow : (g >= Rmax ? kClsHigh : kClsFree));
+    // ---- the partition, checked exactly
+    if (!has) cls = kClsFree;
     const int64_t sgn = (kRel && T < 0) ? -1 : 1;
     const int64_t y = sgn * S;
-    const int64_t NL = warp_sum(cls == kClsLow ? n : int64_t(0));
-    const int64_t NH = warp_sum(cls == kClsHigh ? n : int64_t(0));
-    const int64_t NF = warp_sum(cls == kClsFree ? n : int64_t(0));
-    const int64_t YF = warp_sum(cls == kClsFree ? y : int64_t(0));
+    int64_t NL = 0, NH = 0, NF = N, YF = sgn * T;
+    if (!all_free) {
+      NL = warp_sum(cls == kClsLow ? n : int64_t(0));
+      NH = warp_sum(cls == kClsHigh ? n : int64_t(0));
+      NF = warp_sum(cls == kClsFree ? n : int64_t(0));
+      YF = warp_sum(cls == kClsFree ? y : int64_t(0));
+    }
     if (NF == 0) return kExactFallback;
     const int64_t W = (B << 32) - mq * NL - Mq * NH;
     const i128 Dd = static_cast<i128>(y) * NF - static_cast<i128>(n) * YF;
@@ -451,27 +454,21 @@ __device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int64_t R
   return AVTP_OK;
 }
 
-// The same rule for requests of at most 32 images, with the grid stage held in
-// registers: lane j owns image j (S_j, n_j in; its budget out). The exact stage then
-// runs on sm (32 entries). Identical results and status to warp_allocate.
-// Out of line so that a warm-up call and the real one share the same code.
-// inv_n = floor(2^62 / n_j) and inv_N = floor(2^62 / N) come from the caller, which
-// can take them before the sums are ready; after that no division is left on the
-// common path.
-// Fast path for the grid's lambda: without clamps G is linear with slope N, so the
-// smallest solution is lambda0 = ceil((B * 2^40 - sum n_i R_i) / N); when no clamp binds
-// at lambda0 - 1 or lambda0, G is that line on [lambda0 - 1, lambda0] and lambda0 is
-// exact. Otherwise the breakpoints decide.
-static __device__ __noinline__ int warp_allocate32(const WarpAllocSmem& sm, int m, int64_t S, int32_t n, int64_t inv_n,
-                                                   int64_t B, int32_t N, int64_t inv_N, const RatioRule& rule,
-                                                   float alpha_f, float r_min_f, float r_max_f, int32_t* k_out) {
+// A clamp binds: the grid's shift proposes the partition, checked exactly; the general
+// stage when that does not settle it. Out of line: fetched only when it runs.
+// The grid's shift: without clamps G is linear with slope N, so the smallest solution is
+// lambda0 = ceil((B * 2^40 - sum n_i R_i) / N); when no clamp binds at lambda0 - 1 or
+// lambda0, G is that line on [lambda0 - 1, lambda0] and lambda0 is exact. Otherwise the
+// breakpoints decide.
+static __device__ __noinline__ int warp_allocate32_clamped(const WarpAllocSmem& sm, int m, int64_t S, int32_t n,
+                                                           int64_t inv_n, int64_t B, int32_t N, int64_t inv_N,
+                                                           int64_t T, const RatioRule& rule, float alpha_f,
+                                                           float r_min_f, float r_max_f, int64_t Rb, int64_t Aa,
+                                                           int64_t mq, int64_t Mq, int32_t* k_out) {
   const int lane = threadIdx.x & 31;
   const bool has = lane < m;
   const int64_t Rmin = ratio_grid(r_min_f), Rmax = ratio_grid(r_max_f);
   // ---- ratios on the grid
-  const int64_t lim = static_cast<int64_t>(n) << kSumMagnitudeBits;
-  if (__any_sync(0xffffffffu, has && (S > lim || S < -lim))) return AVTP_ERR_DEVICE_INPUT;
-  const int64_t T = warp_sum(has ? S : int64_t(0));
   const int64_t avg = grid_mean(T, inv_N);
   const int64_t inv_avg = (rule.relative && avg != 0) ? recip62(avg > 0 ? avg : -avg) : 0;
   const int64_t R = has ? grid_ratio(rule, grid_mean(S, inv_n), avg, inv_avg) : 0;
@@ -496,11 +493,12 @@ static __device__ __noinline__ int warp_allocate32(const WarpAllocSmem& sm, int 
   }
   if (!found) lam = breakpoint_lambda32(m, R, nl, has, target, Rmin, Rmax, mx, mn);
 
-  // ---- the exact stage, in registers; the general one when that cannot settle it
-  const int64_t Rb = units32(rule.r_base_f), Aa = units32(alpha_f), mq = units32(r_min_f), Mq = units32(r_max_f);
+  // ---- the exact stage on the grid's partition, in registers
+  const int64_t g = R + lam;
+  const int cls = g <= Rmin ? kClsLow : (g >= Rmax ? kClsHigh : kClsFree);
   int32_t K = 0;
-  int err = rule.relative ? exact32<true>(has, S, n, R, lam, Rmin, Rmax, B, N, T, Rb, Aa, mq, Mq, &K)
-                          : exact32<false>(has, S, n, R, lam, Rmin, Rmax, B, N, T, Rb, Aa, mq, Mq, &K);
+  int err = rule.relative ? exact32<true>(has, S, n, cls, false, B, N, T, Rb, Aa, mq, Mq, &K)
+                          : exact32<false>(has, S, n, cls, false, B, N, T, Rb, Aa, mq, Mq, &K);
   if (err == kExactFallback) {
     if (has) {
       sm.S[lane] = S;
@@ -514,6 +512,35 @@ static __device__ __noinline__ int warp_allocate32(const WarpAllocSmem& sm, int 
   }
   *k_out = K;
   return err;
+}
+
+// The same rule for requests of at most 32 images, held in registers: lane j owns image
+// j (S_j, n_j in; its budget out). The partition with every image free (no clamp binds,
+// the common case) is checked exactly first; only when it fails does the grid search for
+// the shift (warp_allocate32_clamped), and only when that partition fails too does the
+// general stage run on sm (32 entries). Identical results and status to warp_allocate.
+// Out of line so that a warm-up call and the real one share the same code.
+// inv_n = floor(2^62 / n_j) and inv_N = floor(2^62 / N) come from the caller, which
+// can take them before the sums are ready.
+static __device__ __noinline__ int warp_allocate32(const WarpAllocSmem& sm, int m, int64_t S, int32_t n, int64_t inv_n,
+                                                   int64_t B, int32_t N, int64_t inv_N, const RatioRule& rule,
+                                                   float alpha_f, float r_min_f, float r_max_f, int32_t* k_out) {
+  const int lane = threadIdx.x & 31;
+  const bool has = lane < m;
+  const int64_t lim = static_cast<int64_t>(n) << kSumMagnitudeBits;
+  if (__any_sync(0xffffffffu, has && (S > lim || S < -lim))) return AVTP_ERR_DEVICE_INPUT;
+  const int64_t T = warp_sum(has ? S : int64_t(0));
+  const int64_t Rb = units32(rule.r_base_f), Aa = units32(alpha_f), mq = units32(r_min_f), Mq = units32(r_max_f);
+  int32_t K = 0;
+  // ---- first the partition of the common case, no clamp binding: no search needed
+  int err = rule.relative ? exact32<true>(has, S, n, kClsFree, true, B, N, T, Rb, Aa, mq, Mq, &K)
+                          : exact32<false>(has, S, n, kClsFree, true, B, N, T, Rb, Aa, mq, Mq, &K);
+  if (err != kExactFallback) {
+    *k_out = K;
+    return err;
+  }
+  return warp_allocate32_clamped(sm, m, S, n, inv_n, B, N, inv_N, T, rule, alpha_f, r_min_f, r_max_f, Rb, Aa, mq,
+                                 Mq, k_out);
 }
 
 }  // namespace avtp

@@ -51,6 +51,10 @@ avtp_status_t check_score_args(const avtp_layout_t* L, const avtp_score_args_t* 
     if (!aligned16(a->q) || !aligned16(a->k)) return AVTP_ERR_UNSUPPORTED;
     if (!(a->softmax_scale > 0.f) || !isfinite(a->softmax_scale)) return AVTP_ERR_INVALID_ARG;
     if (a->lse != nullptr && a->lse_stride < L->n_tokens) return AVTP_ERR_INVALID_ARG;
+    if (a->query_set != AVTP_QUERIES_TEXT && a->query_set != AVTP_QUERIES_LAST) return AVTP_ERR_INVALID_ARG;
+    if (a->path != AVTP_PATH_AUTO && a->path != AVTP_PATH_TENSOR && a->path != AVTP_PATH_CUDA)
+      return AVTP_ERR_INVALID_ARG;
+    if (a->path == AVTP_PATH_TENSOR && a->query_set == AVTP_QUERIES_LAST) return AVTP_ERR_UNSUPPORTED;
     return AVTP_OK;
   }
   return AVTP_ERR_INVALID_ARG;
@@ -106,6 +110,13 @@ AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa) {
   return a;
 }
 
+bool attn_uses_cuda_cores(const avtp_layout_t& L, const avtp_score_args_t& sa) {
+  if (sa.path == AVTP_PATH_CUDA || sa.query_set == AVTP_QUERIES_LAST) return true;
+  if (sa.path == AVTP_PATH_TENSOR) return false;
+  const AttnPlan a = attn_plan(L, sa);
+  return a.rows <= kNarrowAutoRows;
+}
+
 WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
   WsPlan p{};
   const size_t R = static_cast<size_t>(L.n_requests), NI = static_cast<size_t>(L.n_images);
@@ -134,11 +145,18 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
     p.ktile_cu = take((NI + 1) * 4);
     p.ktile_img = take(static_cast<size_t>(a.n_ktiles_max) * 4);
     p.meta = take(8 * 4);
-    p.qt = take(Hkv * rows * static_cast<size_t>(sa->head_dim) * 2 + 16);
-    p.lse_rows = (sa->lse != nullptr) ? take(Hkv * rows * 4 + 4) : 0;
-    p.p1_part = (sa->lse == nullptr)
-                    ? take(Hkv * static_cast<size_t>(a.n_blocks_max) * kAttnBlockRows * kAttnMaxChunks * 8)
-                    : 0;
+    if (attn_uses_cuda_cores(L, *sa)) {
+      const NarrowPlan np = narrow_plan(L, *sa, a.max_text);
+      const size_t nrows = static_cast<size_t>(np.rows);
+      p.lse_rows = take(Hkv * nrows * 4 + 4);
+      p.p1_part = (sa->lse == nullptr) ? take(Hkv * static_cast<size_t>(np.NS) * nrows * 8 + 8) : 0;
+    } else {
+      p.qt = take(Hkv * rows * static_cast<size_t>(sa->head_dim) * 2 + 16);
+      p.lse_rows = (sa->lse != nullptr) ? take(Hkv * rows * 4 + 4) : 0;
+      p.p1_part = (sa->lse == nullptr)
+                      ? take(Hkv * static_cast<size_t>(a.n_blocks_max) * kAttnBlockRows * kAttnMaxChunks * 8)
+                      : 0;
+    }
     p.mass = take(static_cast<size_t>(a.n_ktiles_max) * kAttnTileM * 8);
   }
   p.total = off;
@@ -203,6 +221,8 @@ static avtp_status_t score_impl(const avtp_layout_t* L, const avtp_score_args_t*
                                 int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s, int reserve_sms = 0) {
   if (a->criterion == AVTP_CRIT_HIDDEN_VARIATION)
     return from_cuda(launch_score_hvar(*L, *a, scores, img_sums, ws, p, s, reserve_sms));
+  if (attn_uses_cuda_cores(*L, *a))
+    return from_cuda(launch_score_narrow(*L, *a, scores, img_sums, ws, p, attn_plan(*L, *a), s));
   return from_cuda(launch_score_attn(*L, *a, scores, img_sums, ws, p, s));
 }
 
@@ -297,6 +317,13 @@ avtp_status_t avtp_prune(const avtp_layout_t* layout, const avtp_score_args_t* s
   int64_t* sums = img_sums != nullptr ? img_sums : ws_at<int64_t>(workspace, p.img_sums);
 
   if ((st = record(step_events, 0, s)) != AVTP_OK) return st;
+#ifdef AVTP_TIMELINE
+  // the timeline words: earliest stamps start at all ones, latest at zero
+  char* tl = static_cast<char*>(workspace) + p.status + kTimelineOffset;
+  if (cudaMemsetAsync(tl, 0xff, kTlEvents * sizeof(uint64_t), s) != cudaSuccess ||
+      cudaMemsetAsync(tl + kTlEvents * sizeof(uint64_t), 0, kTlEvents * sizeof(uint64_t), s) != cudaSuccess)
+    return AVTP_ERR_CUDA;
+#endif
   PrepArgs pa{};
   pa.L = *layout;
   pa.keep_ratio = alloc_args->keep_ratio;
@@ -389,6 +416,32 @@ avtp_status_t avtp_wait_selftest(int64_t limit_ns, int32_t arrive, void* workspa
   avtp_status_t st = from_cuda(cudaMemsetAsync(workspace, 0, sizeof(DevStatus), s));
   if (st != AVTP_OK) return st;
   return from_cuda(launch_wait_selftest(static_cast<uint64_t>(limit_ns), arrive != 0, workspace, s));
+}
+
+avtp_status_t avtp_layer_attention(const avtp_layout_t* layout, const int64_t* img_sums, int64_t* A,
+                                   int32_t n_layers, int32_t layer, void* workspace, size_t workspace_bytes,
+                                   avtp_stream_t stream) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if (A == nullptr || (layout->n_images > 0 && img_sums == nullptr)) return AVTP_ERR_INVALID_ARG;
+  if (n_layers < 1 || layer < 0 || layer >= n_layers) return AVTP_ERR_INVALID_ARG;
+  if (n_layers > AVTP_MAX_LAYERS) return AVTP_ERR_RANGE;
+  const WsPlan p = plan_workspace(*layout, nullptr);
+  if ((st = check_ws(workspace, workspace_bytes, p)) != AVTP_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PrepArgs pa{};
+  pa.L = *layout;
+  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
+  return from_cuda(launch_layer_attention(*layout, img_sums, A, n_layers, layer, workspace, p, s));
+}
+
+avtp_status_t avtp_layer_select(const int64_t* A, int32_t n_samples, int32_t n_layers, int32_t k, int64_t* rank_sum,
+                                int32_t* top_layers, avtp_stream_t stream) {
+  if (A == nullptr || rank_sum == nullptr || top_layers == nullptr) return AVTP_ERR_INVALID_ARG;
+  if (n_samples < 1 || n_layers < 1 || k < 1 || k > n_layers) return AVTP_ERR_INVALID_ARG;
+  if (n_layers > AVTP_MAX_LAYERS) return AVTP_ERR_RANGE;
+  return from_cuda(launch_layer_select(A, n_samples, n_layers, k, rank_sum, top_layers,
+                                       reinterpret_cast<cudaStream_t>(stream)));
 }
 
 avtp_status_t avtp_read_device_status(const void* workspace, avtp_stream_t stream, int32_t* out) {

@@ -73,6 +73,33 @@ __device__ __forceinline__ bool wait_expired(uint32_t polls, uint64_t& t0, uint6
   return now - t0 > limit_ns || polls >= kWaitSpinCap;
 }
 
+// ---------------------------------------------------------------- phase timeline (diagnostic build)
+// Built with -DAVTP_TIMELINE, the kernels of the fused stage record global-timer stamps of
+// their phases in the bytes between the workspace's status word and its first array
+// (every workspace slice is 256-byte aligned, so 240 bytes are free there): for every
+// event the earliest stamp over the CTAs that reach it (first kTlEvents words) and the
+// latest (next kTlEvents words). avtp_prune presets those words before its first kernel.
+// The normal build records nothing and never touches them.
+enum TimelineEvent {
+  kTlPrepBegin = 0, kTlPrepEnd, kTlScoreBegin, kTlScoreEnd, kTlSelBegin, kTlSelWaited, kTlRuleEnd, kTlSelEnd,
+  kTlCompactBegin, kTlCompactWaited, kTlCompactEnd, kTlEvents
+};
+constexpr size_t kTimelineOffset = 16;  // bytes after the start of the workspace
+static_assert(kTimelineOffset + 2 * kTlEvents * sizeof(uint64_t) <= 256, "timeline must fit before the first array");
+
+__device__ __forceinline__ void timeline_stamp(DevStatus* st, int ev) {
+#ifdef AVTP_TIMELINE
+  unsigned long long* tl = reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(st) + kTimelineOffset);
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  atomicMin(tl + ev, t);
+  atomicMax(tl + kTlEvents + ev, t);
+#else
+  (void)st;
+  (void)ev;
+#endif
+}
+
 // ---------------------------------------------------------------- workspace
 struct WsPlan {
   size_t status;      // DevStatus
@@ -109,6 +136,22 @@ struct AttnPlan {
   int grid;              // CTAs of the persistent tensor-core kernels (one per SM)
 };
 AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa);
+
+// The CUDA-core path of criterion B (k_score_narrow.cu): rows per KV group are the
+// batch's queries (at most) times G; pass 1 splits every (request, KV group) into NS key
+// ranges.
+constexpr int kNarrowMaxSplits = 64;
+// AVTP_PATH_AUTO takes the CUDA cores when every (request, KV group) has at most this
+// many rows, judged from the batch's text-token bound (AVTP_QUERIES_TEXT), and always
+// for AVTP_QUERIES_LAST.
+constexpr int64_t kNarrowAutoRows = 32;
+struct NarrowPlan {
+  int G;
+  int64_t rows;
+  int NS;
+};
+NarrowPlan narrow_plan(const avtp_layout_t& L, const avtp_score_args_t& sa, int64_t max_text);
+bool attn_uses_cuda_cores(const avtp_layout_t& L, const avtp_score_args_t& sa);
 
 WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa);
 
@@ -264,6 +307,11 @@ cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& s
 
 cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
                               int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s);
+cudaError_t launch_score_narrow(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores, int64_t* img_sums,
+                                void* ws, const WsPlan& p, const AttnPlan& plan, cudaStream_t s);
+// Scores and fixed-point image sums from the per-key mass of either criterion-B path.
+cudaError_t launch_attn_finalize(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
+                                 int64_t* img_sums, void* ws, const WsPlan& p, const AttnPlan& plan, cudaStream_t s);
 
 cudaError_t launch_allocate(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
                             int32_t* budgets, void* ws, const WsPlan& p, cudaStream_t s);
@@ -298,6 +346,11 @@ cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_to
                            int n_sets, void* ws, const WsPlan& p, cudaStream_t s);
 
 cudaError_t launch_wait_selftest(uint64_t limit_ns, int arrive, void* ws, cudaStream_t s);
+
+cudaError_t launch_layer_attention(const avtp_layout_t& L, const int64_t* img_sums, int64_t* A, int n_layers,
+                                   int layer, void* ws, const WsPlan& p, cudaStream_t s);
+cudaError_t launch_layer_select(const int64_t* A, int n_samples, int n_layers, int k, int64_t* rank_sum,
+                                int32_t* top_layers, cudaStream_t s);
 
 int device_sm_count();
 

@@ -3,10 +3,12 @@
 //
 // Large rows (hidden states, K/V rows): one warp per row, 16-byte vector loads and
 // stores; a lane issues all its loads of an 8-KiB piece of the row before its first
-// store, so that a row costs one memory round trip (the kept rows are usually still in
-// L2: the scoring kernel reads h_cur with an evict-last policy). Small rows (position ids, one element
-// per plane): one thread per row. All row sets go in one launch; the block index
-// range is split between the sets on the host.
+// store, so that a row costs one memory round trip (the scoring kernel reads h_cur with
+// an evict-last policy, so some kept rows are still in L2). Small rows (position ids, one
+// element per plane): one thread per row. All row sets go in one launch; the block index
+// range is split between the sets on the host. A single-thread bulk-copy ring per SM
+// (global -> shared -> global) was slower: the gather moves its bytes at about the HBM
+// rate already, and one issuing thread per SM kept fewer of them in flight.
 #include "avtp_internal.cuh"
 
 namespace avtp {
@@ -50,11 +52,8 @@ __device__ __forceinline__ void copy_row_thread(const char* src, char* dst, int6
   for (int64_t u = 0; u < bytes / U; ++u) d[u] = s[u];
 }
 
-__global__ void __launch_bounds__(kThreads)
-k_compact(CompactParams P, const int32_t* __restrict__ kept_idx, int64_t n_kept, int64_t n_tokens, DevStatus* st) {
-  pdl_wait();  // kept_idx comes from the selection kernel
-  pdl_trigger();
-  const int b = blockIdx.x;
+__device__ __forceinline__ void compact_block(const CompactParams& P, int b, const int32_t* __restrict__ kept_idx,
+                                              int64_t n_kept, int64_t n_tokens, DevStatus* st) {
   int si = 0;
   while (si + 1 < P.n_sets && b >= P.set[si + 1].block_begin) ++si;
   const RowSetDev S = P.set[si];
@@ -88,7 +87,7 @@ k_compact(CompactParams P, const int32_t* __restrict__ kept_idx, int64_t n_kept,
     }
   } else {
     const int64_t j = row0 + threadIdx.x;
-    if (threadIdx.x >= S.rows_per_block || j >= n_kept) return;
+    if (static_cast<int>(threadIdx.x) >= S.rows_per_block || j >= n_kept) return;
     const int64_t t = kept_idx[j];
     if (t < 0 || t >= n_tokens) {
       record_error(st, AVTP_ERR_DEVICE_INPUT, static_cast<int32_t>(j));
@@ -104,6 +103,29 @@ k_compact(CompactParams P, const int32_t* __restrict__ kept_idx, int64_t n_kept,
       default: copy_row_thread<1>(src, dst, S.row_bytes); break;
     }
   }
+}
+
+// Grid-stride over the blocks of work (a block = kWarps rows of a vector set, or kThreads
+// rows of a small set), with a grid the SMs hold at once: a second wave would start
+// only when the first ends.
+__global__ void __launch_bounds__(kThreads)
+k_compact(CompactParams P, int n_blocks, const int32_t* __restrict__ kept_idx, int64_t n_kept, int64_t n_tokens,
+          DevStatus* st) {
+  if (threadIdx.x == 0) timeline_stamp(st, kTlCompactBegin);
+  pdl_wait();  // kept_idx comes from the selection kernel
+  pdl_trigger();
+  if (threadIdx.x == 0) timeline_stamp(st, kTlCompactWaited);
+  for (int b = blockIdx.x; b < n_blocks; b += gridDim.x) compact_block(P, b, kept_idx, n_kept, n_tokens, st);
+  if ((threadIdx.x & 31) == 0) timeline_stamp(st, kTlCompactEnd);
+}
+
+int compact_ctas_per_sm() {
+  static PerDevice occ;
+  int n = 0;
+  const cudaError_t e = once_per_device(occ, [](int, int* v) {
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(v, k_compact, kThreads, 0);
+  }, &n);
+  return (e == cudaSuccess && n >= 1) ? n : 1;
 }
 
 int access_unit(const avtp_rows_t& s) {
@@ -137,8 +159,10 @@ cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_to
     blocks += (n_kept + d.rows_per_block - 1) / d.rows_per_block;
   }
   if (blocks > 0x7fffffff) return cudaErrorInvalidConfiguration;
-  return launch_kernel(k_compact, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0, s, /*pdl=*/true, P,
-                       kept_idx, n_kept, n_tokens, ws_at<DevStatus>(ws, p.status));
+  const int64_t wave = static_cast<int64_t>(compact_ctas_per_sm()) * device_sm_count();
+  const int64_t grid = blocks < wave ? blocks : wave;
+  return launch_kernel(k_compact, dim3(static_cast<unsigned>(grid)), dim3(kThreads), 0, s, /*pdl=*/true, P,
+                       static_cast<int>(blocks), kept_idx, n_kept, n_tokens, ws_at<DevStatus>(ws, p.status));
 }
 
 }  // namespace avtp

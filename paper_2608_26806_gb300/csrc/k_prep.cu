@@ -66,6 +66,7 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
   // stream has finished, so the next kernel may be scheduled at once.
   pdl_trigger();
   const int tid = threadIdx.x;
+  if (tid == 0) timeline_stamp(st, kTlPrepBegin);
   const int R = a.L.n_requests, NI = a.L.n_images;
   const int64_t T = a.L.n_tokens;
   const int32_t* cu = a.L.cu_seqlens;
@@ -263,6 +264,7 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
     st->code = s_err;
     st->detail = s_detail;
     st->layout_ok = (s_err == 0) ? 1 : 0;
+    timeline_stamp(st, kTlPrepEnd);
   }
 }
 

@@ -746,7 +746,7 @@ __global__ void __launch_bounds__(kM)
 k_attn_finalize(const unsigned long long* __restrict__ mass, const int32_t* __restrict__ ktile_cu,
                 const int32_t* __restrict__ ktile_img, int Hq, const int32_t* __restrict__ cu,
                 const int32_t* __restrict__ img_start, const int32_t* __restrict__ img_len,
-                const int32_t* __restrict__ img_req, const int32_t* __restrict__ text_cu, int NI,
+                const int32_t* __restrict__ img_req, const int32_t* __restrict__ text_cu, int NI, int last,
                 float* __restrict__ scores, int64_t* __restrict__ img_sums, const DevStatus* st) {
   __shared__ long long s_part[kM / 32];
   pdl_wait();
@@ -756,7 +756,8 @@ k_attn_finalize(const unsigned long long* __restrict__ mass, const int32_t* __re
     const int i = ktile_img[tile];
     const int r = img_req[i];
     const int o = (tile - ktile_cu[i]) * kM + static_cast<int>(threadIdx.x);  // key within the image
-    const int nq = text_cu[r + 1] - text_cu[r];
+    // the request's queries: its text tokens, or its last token alone
+    const int nq = last ? (cu[r + 1] > cu[r] ? 1 : 0) : text_cu[r + 1] - text_cu[r];
     const unsigned long long m = mass[static_cast<int64_t>(tile) * kM + threadIdx.x];
     long long fx = 0;
     if (o < img_len[i]) {
@@ -885,13 +886,21 @@ cudaError_t launch_score_attn(const avtp_layout_t& L, const avtp_score_args_t& s
   cudaError_t e =
       launch_kernel(k_attn_mass, dim3(sms), dim3(kThreads), mass_smem_bytes(d), s, /*pdl=*/true, mk128, mq256, a);
   if (e != cudaSuccess) return e;
-  const int64_t cap = static_cast<int64_t>(sms) * 8;
+  return launch_attn_finalize(L, sa, scores, img_sums, ws, p, plan, s);
+}
+
+cudaError_t launch_attn_finalize(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
+                                 int64_t* img_sums, void* ws, const WsPlan& p, const AttnPlan& plan, cudaStream_t s) {
+  const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
   const int grid3 = static_cast<int>(plan.n_ktiles_max < cap ? plan.n_ktiles_max : cap);
   return launch_kernel(k_attn_finalize, dim3(grid3), dim3(kM), 0, s, /*pdl=*/true,
-                       static_cast<const unsigned long long*>(a.mass), a.ktile_cu,
-                       static_cast<const int32_t*>(ws_at<int32_t>(ws, p.ktile_img)), Hq, L.cu_seqlens, L.img_start,
-                       L.img_len, static_cast<const int32_t*>(ws_at<int32_t>(ws, p.img_req)), a.text_cu, L.n_images,
-                       scores, img_sums, static_cast<const DevStatus*>(st));
+                       static_cast<const unsigned long long*>(ws_at<unsigned long long>(ws, p.mass)),
+                       static_cast<const int32_t*>(ws_at<int32_t>(ws, p.ktile_cu)),
+                       static_cast<const int32_t*>(ws_at<int32_t>(ws, p.ktile_img)), sa.n_q_heads, L.cu_seqlens,
+                       L.img_start, L.img_len, static_cast<const int32_t*>(ws_at<int32_t>(ws, p.img_req)),
+                       static_cast<const int32_t*>(ws_at<int32_t>(ws, p.text_cu)), L.n_images,
+                       sa.query_set == AVTP_QUERIES_LAST ? 1 : 0, scores, img_sums,
+                       static_cast<const DevStatus*>(ws_at<DevStatus>(ws, p.status)));
 }
 
 }  // namespace avtp

@@ -156,6 +156,7 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   __shared__ int32_t s_cu[kStageRequests + 1];
   __shared__ int32_t s_warp[kWarps];
   pdl_trigger();
+  if (threadIdx.x == 0) timeline_stamp(st, kTlScoreBegin);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   unsigned char* wbuf = smem + static_cast<size_t>(warp) * kSlots * kSlotBytes;
   uint64_t* wbar = bars[warp];
@@ -335,6 +336,7 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     if (lane == 0) record_error(st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));
   }
   pdl_wait();  // completion of this grid implies completion of the one before it
+  if (lane == 0) timeline_stamp(st, kTlScoreEnd);
 }
 
 }  // namespace

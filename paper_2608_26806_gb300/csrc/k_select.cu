@@ -397,13 +397,14 @@ struct AllocParams {
   int warm_ctas;     // CTAs below this index warm their instruction cache before the wait
 };
 
-__global__ void __launch_bounds__(kThreads, 3)
+__global__ void __launch_bounds__(kThreads, 2)
 k_alloc_select(SelectArgs a, AllocParams ap) {
   extern __shared__ __align__(16) unsigned char dsmem[];  // budget scratch for requests of > 32 images
   __shared__ __align__(16) unsigned char rule32[warp_alloc_smem_bytes(32)];  // ... and of at most 32
   __shared__ SelShared sh;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = blockIdx.x;
+  if (tid == 0) timeline_stamp(a.st, kTlSelBegin);
   const WarpAllocSmem wsm = carve_warp_alloc(dsmem, ap.m_cap);
   const WarpAllocSmem wsm32 = carve_warp_alloc(rule32, 32);
 
@@ -483,6 +484,7 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
   // ---- wait for the scores and per-image sums (and, through them, the validation)
   pdl_wait();
   pdl_trigger();
+  if (tid == 0) timeline_stamp(a.st, kTlSelWaited);
   if (!a.st->layout_ok) return;
   if (b >= a.NI) {
     leading_text(a, b - a.NI);
@@ -518,6 +520,7 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
 #pragma unroll
     for (int q = 0; q < 8; ++q) sh.hist[0][lane * 8 + q] = 0;  // warp 0 takes no part in the first pass
     if (lane == 0) {
+      timeline_stamp(a.st, kTlRuleEnd);
       sh.k = k;
       sh.before = before;
       sh.total = total;
@@ -587,6 +590,7 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
   if (!fast) block_select(sc, n, k, t0, base, a.kept_idx, sh, stage, kmin, kmax, kmin != kmax);
   const int e = s0 + n;
   for (int p = e + tid; p < nxt; p += kThreads) a.kept_idx[base + k + (p - e)] = a.cu[r] + p;
+  if (tid == 0) timeline_stamp(a.st, kTlSelEnd);
 }
 
 SelectArgs make_args(const avtp_layout_t& L, const float* scores, const int32_t* out_cu_seqlens, int32_t* kept_idx,

@@ -37,6 +37,17 @@ def test_hand_counted_example():
     assert bl["score_bytes"] == 3 * 1 * 4 * 2 + 3 * 2 * 4 * 2 + 3 * 2 * 4
 
 
+def test_last_token_accounting_by_hand():
+    # the request's last token as the only query: every key once, one query row per head;
+    # FMAs (not tensor-core FLOPs): the 6 keys it sees in pass 1, the 3 visual keys in pass 2
+    wl = _wl([[("t", 2), ("i", 3), ("t", 1)]])
+    c = bench.stage_accounting(wl, "text_attention", 4, query_set="last")
+    assert c["score_bytes"] == 6 * 1 * 4 * 2 + 1 * 2 * 4 * 2
+    assert c["stage_bytes"] == c["score_bytes"] + 3 * 8 * 2 + 4 * 8 * 2 + 4 * 4 * 2
+    assert c["flops"] == 0
+    assert c["fma_flops"] == 2 * 2 * 4 * 6 + 2 * 2 * 4 * 3
+
+
 def test_flops_equal_brute_force_mask_counts():
     rng = np.random.default_rng(4)
     for _ in range(40):

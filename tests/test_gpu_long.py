@@ -41,6 +41,19 @@ def _request(wl, r):
     return sub, a, b
 
 
+def test_score_long_workload_last_token(long_workload):
+    # the last-token query set on the CUDA-core path: every visual key of all four requests
+    wl, dw = long_workload
+    lay = wl.layout
+    scores, sums = avtp.score(dw.L, "text_attention", query_set="last", **dw.score_tensors("text_attention"))
+    torch.cuda.synchronize()
+    got = scores.cpu().numpy()
+    ref = O.score_text_attention(lay, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale, query_set="last")
+    vis = lay.visual_mask()
+    np.testing.assert_allclose(got[vis], ref[vis], rtol=RTOL, atol=ATOL)
+    assert np.array_equal(sums.cpu().numpy(), O.image_sums(lay, got))
+
+
 @pytest.mark.parametrize("criterion", ["hidden_variation", "text_attention"])
 def test_prune_long_workload(long_workload, criterion):
     wl, dw = long_workload

@@ -106,6 +106,86 @@ def test_score_attention_edge_layouts(layout_id, heads, supplied_lse):
     assert np.array_equal(sums.cpu().numpy(), O.image_sums(wl.layout, got))
 
 
+# ---------------------------------------------------------------- step 1B: query sets and paths
+@pytest.mark.parametrize("name", CONFIGS)
+def test_score_last_token_parity(name):
+    # the request's last token as the only query (the output token's attention, §4.1),
+    # on the CUDA-core path that query set always takes
+    wl, dw = workload(name)
+    scores, sums = avtp.score(dw.L, "text_attention", query_set="last", **dw.score_tensors("text_attention"))
+    torch.cuda.synchronize()
+    got = scores.cpu().numpy()
+    ref = O.score_text_attention(wl.layout, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale,
+                                 query_set="last")
+    assert_scores_close(got, ref, wl.layout.visual_mask())
+    assert np.array_equal(sums.cpu().numpy(), O.image_sums(wl.layout, got))
+
+
+@pytest.mark.parametrize("path", ["tensor", "cuda"])
+@pytest.mark.parametrize("supplied_lse", [False, True])
+def test_score_text_attention_both_paths_on_tiny(path, supplied_lse):
+    wl, dw = workload("tiny")
+    kw, ref_lse = {}, None
+    if supplied_lse:
+        lse = O.text_lse(wl.layout, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
+        kw["lse"] = torch.from_numpy(lse.astype(np.float32)).cuda()
+        ref_lse = lse.astype(np.float32).astype(np.float64)
+    scores, sums = avtp.score(dw.L, "text_attention", path=path, **kw, **dw.score_tensors("text_attention"))
+    torch.cuda.synchronize()
+    got = scores.cpu().numpy()
+    ref = O.score_text_attention(wl.layout, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale, lse=ref_lse)
+    assert_scores_close(got, ref, wl.layout.visual_mask())
+    assert np.array_equal(sums.cpu().numpy(), O.image_sums(wl.layout, got))
+
+
+@pytest.mark.parametrize("layout_id", range(len(_ATTN_EDGE_LAYOUTS)))
+@pytest.mark.parametrize("heads", [(4, 4, 64), (6, 2, 64), (12, 4, 128), (7, 1, 128)])
+@pytest.mark.parametrize("query_set", ["text", "last"])
+@pytest.mark.parametrize("supplied_lse", [False, True])
+def test_score_cuda_core_path_edge_layouts(layout_id, heads, query_set, supplied_lse):
+    Hq, Hkv, d = heads
+    wl = synth.make_custom(_ATTN_EDGE_LAYOUTS[layout_id], n_q_heads=Hq, n_kv_heads=Hkv, head_dim=d, hidden=64,
+                           seed=11 + layout_id, parts=("B",))
+    dw = DevWorkload(wl)
+    kw, ref_lse = {}, None
+    if supplied_lse:
+        lse = O.text_lse(wl.layout, wl.q, wl.k, Hq, Hkv, wl.softmax_scale, query_set=query_set)
+        kw["lse"] = torch.from_numpy(lse.astype(np.float32)).cuda()
+        ref_lse = lse.astype(np.float32).astype(np.float64)
+    scores, sums = avtp.score(dw.L, "text_attention", path="cuda", query_set=query_set, **kw,
+                              **dw.score_tensors("text_attention"))
+    torch.cuda.synchronize()
+    got = scores.cpu().numpy()
+    ref = O.score_text_attention(wl.layout, wl.q, wl.k, Hq, Hkv, wl.softmax_scale, lse=ref_lse, query_set=query_set)
+    assert_scores_close(got, ref, wl.layout.visual_mask())
+    assert np.array_equal(sums.cpu().numpy(), O.image_sums(wl.layout, got))
+
+
+def test_prune_last_token_end_to_end():
+    wl, dw = workload("qwen3_vl_8b")
+    out = avtp.prune(dw.L, "text_attention", keep_ratio=dw.keep_ratio, keep_ratio_host=wl.keep_ratio,
+                     rows={"hidden": dw.t["h_cur"]}, planes={"pos": dw.t["pos"]}, query_set="last",
+                     **dw.score_tensors("text_attention"))
+    torch.cuda.synchronize()
+    assert avtp.read_device_status(out.workspace) == avtp.OK
+    got = out.scores.cpu().numpy()
+    ref64 = O.score_text_attention(wl.layout, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale,
+                                   query_set="last")
+    assert_scores_close(got, ref64, wl.layout.visual_mask())
+    ref = O.prune(wl.layout, keep_ratio=wl.keep_ratio, scores_f32=got, relative=True, rows={"hidden": wl.h_cur},
+                  planes={"pos": wl.pos})
+    assert np.array_equal(out.budgets[:wl.layout.n_images].cpu().numpy(), ref["budgets"])
+    assert np.array_equal(out.kept_idx.cpu().numpy(), ref["kept_idx"])
+    assert np.array_equal(bits_of(out.outputs["hidden"]), ref["hidden"])
+
+
+def test_tensor_path_rejects_the_last_token_set():
+    wl, dw = workload("tiny")
+    with pytest.raises(avtp.AVTPError) as e:
+        avtp.score(dw.L, "text_attention", path="tensor", query_set="last", **dw.score_tensors("text_attention"))
+    assert e.value.code == avtp.ERR_UNSUPPORTED
+
+
 # ---------------------------------------------------------------- step 2
 @pytest.mark.parametrize("name", CONFIGS)
 @pytest.mark.parametrize("relative", [False, True])
