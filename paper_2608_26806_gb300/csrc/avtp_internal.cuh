@@ -141,10 +141,12 @@ AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa);
 // batch's queries (at most) times G; pass 1 splits every (request, KV group) into NS key
 // ranges.
 constexpr int kNarrowMaxSplits = 64;
-// AVTP_PATH_AUTO takes the CUDA cores when every (request, KV group) has at most this
-// many rows, judged from the batch's text-token bound (AVTP_QUERIES_TEXT), and always
-// for AVTP_QUERIES_LAST.
-constexpr int64_t kNarrowAutoRows = 32;
+// AVTP_PATH_AUTO takes the CUDA cores for AVTP_QUERIES_LAST, and for AVTP_QUERIES_TEXT
+// only when the batch has at most this many rows per KV group (judged from its text-token
+// bound). Measured on Qwen3-shaped heads the tensor-core path was faster from 4 rows per
+// group up (flat near 33 us to 512 rows, the CUDA cores growing with the rows), so the
+// text query set keeps to the tensor cores.
+constexpr int64_t kNarrowAutoRows = 0;
 struct NarrowPlan {
   int G;
   int64_t rows;

@@ -12,8 +12,8 @@
 // key at a time (its d elements read as 16-byte vectors; the request's rows, in blocks
 // of kRB, sit in shared memory as fp32) and keeps an online (max, sum) per row of the
 // block; the CTA leaves one partial per (row, split).
-// k_narrow_merge: merges the splits into lse2 per row (or converts a supplied natural-log
-// LSE) and clears the per-key mass accumulator.
+// k_narrow_merge: merges the splits into lse2 per row (a warp per row), or converts a
+// supplied natural-log LSE, and clears the per-key mass accumulator.
 // k_narrow_mass (pass 2): one CTA per (key tile of an image, KV group), a thread per key:
 // the key's probability under every row whose query follows it, summed and added to the
 // 64-bit fixed-point accumulator that k_attn_finalize turns into scores.
@@ -74,6 +74,14 @@ __device__ __forceinline__ int64_t query_pos(const NarrowArgs& a, int r, int64_t
   return a.last ? static_cast<int64_t>(a.cu[r + 1]) - 1 : static_cast<int64_t>(a.text_idx[o]);
 }
 
+// (m, s) <- the online merge of (m, s) and (m2, s2), with -inf for "no key yet".
+__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2) {
+  const float M = fmaxf(m, m2);
+  if (M == -INFINITY) return;
+  s = (m == -INFINITY ? 0.f : s * exp2f(m - M)) + (m2 == -INFINITY ? 0.f : s2 * exp2f(m2 - M));
+  m = M;
+}
+
 // A block of up to kRB rows of request r, group g, starting at row rb: the queries as
 // fp32 in shared memory, their positions, and (pass 2) their lse2.
 struct RowBlock {
@@ -118,16 +126,21 @@ __device__ void load_rows(const NarrowArgs& a, int r, int g, int64_t o0, int n_r
   }
 }
 
-// z[rr] = c2 * q_rr . k for the kRB rows of the block and key t of group g.
+// z[rr] = c2 * q_rr . k for the kRB rows of the block and key t of group g. All of the
+// key's D/8 16-byte loads are issued before the first FMA: a key costs one memory round
+// trip, not D/8 of them.
+template <int D>
 __device__ __forceinline__ void block_logits(const NarrowArgs& a, int64_t t, int g, const float* qs, float* z) {
-  const uint4* kp = reinterpret_cast<const uint4*>(a.k + t * a.k_stride + static_cast<int64_t>(g) * a.d);
+  const uint4* kp = reinterpret_cast<const uint4*>(a.k + t * a.k_stride + static_cast<int64_t>(g) * D);
+  uint4 kv[D / 8];
+#pragma unroll
+  for (int c = 0; c < D / 8; ++c) kv[c] = __ldg(kp + c);
   float acc[kRB];
 #pragma unroll
   for (int rr = 0; rr < kRB; ++rr) acc[rr] = 0.f;
-  const int nc = a.d / 8;
-  for (int c = 0; c < nc; ++c) {
-    const uint4 v = __ldg(kp + c);
-    const uint32_t* w = reinterpret_cast<const uint32_t*>(&v);
+#pragma unroll
+  for (int c = 0; c < D / 8; ++c) {
+    const uint32_t* w = reinterpret_cast<const uint32_t*>(&kv[c]);
     float kf[8];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -136,8 +149,8 @@ __device__ __forceinline__ void block_logits(const NarrowArgs& a, int64_t t, int
     }
 #pragma unroll
     for (int rr = 0; rr < kRB; ++rr) {
-      const float4 q0 = *reinterpret_cast<const float4*>(qs + rr * a.d + c * 8);
-      const float4 q1 = *reinterpret_cast<const float4*>(qs + rr * a.d + c * 8 + 4);
+      const float4 q0 = *reinterpret_cast<const float4*>(qs + rr * D + c * 8);
+      const float4 q1 = *reinterpret_cast<const float4*>(qs + rr * D + c * 8 + 4);
       float s = acc[rr];
       s = fmaf(kf[0], q0.x, s);
       s = fmaf(kf[1], q0.y, s);
@@ -154,15 +167,8 @@ __device__ __forceinline__ void block_logits(const NarrowArgs& a, int64_t t, int
   for (int rr = 0; rr < kRB; ++rr) z[rr] = acc[rr] * a.c2;
 }
 
-// (m, s) <- the online merge of (m, s) and (m2, s2), with -inf for "no key yet".
-__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2) {
-  const float M = fmaxf(m, m2);
-  if (M == -INFINITY) return;
-  s = (m == -INFINITY ? 0.f : s * exp2f(m - M)) + (m2 == -INFINITY ? 0.f : s2 * exp2f(m2 - M));
-  m = M;
-}
-
 // ---------------------------------------------------------------- pass 1
+template <int D>
 __global__ void __launch_bounds__(kNT)
 k_narrow_lse(NarrowArgs a) {
   extern __shared__ __align__(16) float nsm[];
@@ -194,7 +200,7 @@ k_narrow_lse(NarrowArgs a) {
       for (int rr = 0; rr < kRB; ++rr) { m[rr] = -INFINITY; s[rr] = 0.f; }
       for (int64_t t = ks + threadIdx.x; t < ke; t += kNT) {
         float z[kRB];
-        block_logits(a, t, g, nsm, z);
+        block_logits<D>(a, t, g, nsm, z);
 #pragma unroll
         for (int rr = 0; rr < kRB; ++rr) {
           if (t > s_qpos[rr]) continue;  // after the query (or a row past the request's)
@@ -244,36 +250,40 @@ k_narrow_merge(NarrowArgs a, int64_t n_rows_used) {
   for (int64_t u = tid0; u < a.n_mass; u += stride) a.mass[u] = 0ull;
   // rows in use: R * G (last-token set) or (text tokens of the batch) * G
   const int64_t n_text = a.last ? 0 : a.text_cu[a.R];
-  for (int64_t u = tid0; u < static_cast<int64_t>(a.Hkv) * n_rows_used; u += stride) {
+  // a warp per row: the lanes merge the splits, then a shuffle tree
+  const int lane = threadIdx.x & 31;
+  const int64_t wstride = stride >> 5;
+  for (int64_t u = tid0 >> 5; u < static_cast<int64_t>(a.Hkv) * n_rows_used; u += wstride) {
     const int g = static_cast<int>(u / n_rows_used);
     const int64_t ro = u % n_rows_used;
-    if (!a.last && ro / a.G >= n_text) continue;  // no such text token in this batch
+    const int64_t o = ro / a.G;
+    if (!a.last && o >= n_text) continue;                        // no such text token in this batch
+    if (a.last && a.cu[o + 1] == a.cu[o]) continue;              // a request without tokens has no query
     float l2;
     if (a.lse != nullptr) {
-      const int64_t o = ro / a.G;
       const int h = g * a.G + static_cast<int>(ro % a.G);
-      int r;
-      if (a.last) r = static_cast<int>(o);
-      else r = upper_index(a.text_cu, a.R, o);
-      if (a.last && a.cu[r + 1] == a.cu[r]) continue;  // a request without tokens has no query
+      const int r = a.last ? static_cast<int>(o) : upper_index(a.text_cu, a.R, o);
       l2 = a.lse[static_cast<int64_t>(h) * a.lse_stride + query_pos(a, r, o)] * kLog2e;
     } else {
-      if (a.last) {
-        const int r = static_cast<int>(ro / a.G);
-        if (a.cu[r + 1] == a.cu[r]) continue;
-      }
       float M = -INFINITY, Sm = 0.f;
-      for (int sp = 0; sp < a.NS; ++sp) {
+      for (int sp = lane; sp < a.NS; sp += 32) {
         const float2 p = a.part[(static_cast<int64_t>(g) * a.NS + sp) * a.rows + ro];
         merge_ms(M, Sm, p.x, p.y);
       }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, M, off);
+        const float s2 = __shfl_xor_sync(0xffffffffu, Sm, off);
+        merge_ms(M, Sm, m2, s2);
+      }
       l2 = M + log2f(Sm);
     }
-    a.lse2[static_cast<int64_t>(g) * a.rows + ro] = l2;
+    if (lane == 0) a.lse2[static_cast<int64_t>(g) * a.rows + ro] = l2;
   }
 }
 
 // ---------------------------------------------------------------- pass 2
+template <int D>
 __global__ void __launch_bounds__(kNT)
 k_narrow_mass(NarrowArgs a) {
   extern __shared__ __align__(16) float nsm[];
@@ -304,7 +314,7 @@ k_narrow_mass(NarrowArgs a) {
       __syncthreads();
       if (!has) continue;
       float z[kRB];
-      block_logits(a, t, g, nsm, z);
+      block_logits<D>(a, t, g, nsm, z);
 #pragma unroll
       for (int rr = 0; rr < kRB; ++rr)
         if (t <= s_qpos[rr]) mass += exp2f(z[rr] - s_l2[rr]);
@@ -376,11 +386,12 @@ cudaError_t launch_score_narrow(const avtp_layout_t& L, const avtp_score_args_t&
   if (sa.lse == nullptr) {
     const int64_t units = static_cast<int64_t>(L.n_requests) * a.Hkv * a.NS;
     const int grid = static_cast<int>(units < cap ? units : cap);
-    cudaError_t e = launch_kernel(k_narrow_lse, dim3(grid), dim3(kNT), qsm, s, /*pdl=*/true, a);
+    cudaError_t e = sa.head_dim == 64 ? launch_kernel(k_narrow_lse<64>, dim3(grid), dim3(kNT), qsm, s, true, a)
+                                      : launch_kernel(k_narrow_lse<128>, dim3(grid), dim3(kNT), qsm, s, true, a);
     if (e != cudaSuccess) return e;
   }
   {
-    const int64_t work = (a.n_mass > a.Hkv * a.rows ? a.n_mass : a.Hkv * a.rows);
+    const int64_t work = (a.n_mass > 32 * a.Hkv * a.rows ? a.n_mass : 32 * a.Hkv * a.rows);
     const int64_t want = (work + 255) / 256;
     const int grid = static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
     cudaError_t e = launch_kernel(k_narrow_merge, dim3(grid), dim3(256), 0, s, /*pdl=*/true, a, a.rows);
@@ -388,7 +399,8 @@ cudaError_t launch_score_narrow(const avtp_layout_t& L, const avtp_score_args_t&
   }
   const int64_t units2 = plan.n_ktiles_max * a.Hkv;
   const int grid2 = static_cast<int>(units2 < 1 ? 1 : (units2 < cap ? units2 : cap));
-  cudaError_t e = launch_kernel(k_narrow_mass, dim3(grid2), dim3(kNT), qsm, s, /*pdl=*/true, a);
+  cudaError_t e = sa.head_dim == 64 ? launch_kernel(k_narrow_mass<64>, dim3(grid2), dim3(kNT), qsm, s, true, a)
+                                    : launch_kernel(k_narrow_mass<128>, dim3(grid2), dim3(kNT), qsm, s, true, a);
   if (e != cudaSuccess) return e;
   return launch_attn_finalize(L, sa, scores, img_sums, ws, p, plan, s);
 }
