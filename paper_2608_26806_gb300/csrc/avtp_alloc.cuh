@@ -324,24 +324,6 @@ __device__ __forceinline__ float u128_to_float(u128 v) {
          __ull2float_rn(static_cast<uint64_t>(v));
 }
 
-// Descending bitonic sort across the warp: lane i ends with the i-th largest of the 32
-// values. Out of line and rolled: it is fetched once per call from a cold cache.
-static __device__ __noinline__ uint64_t warp_sort_desc(uint64_t v) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll 1
-  for (int size = 2; size <= 32; size <<= 1) {
-#pragma unroll 1
-    for (int j = size >> 1; j > 0; j >>= 1) {
-      const uint64_t p = __shfl_xor_sync(0xffffffffu, v, j);
-      // descending overall: the lower lane of a pair keeps the larger value in blocks
-      // whose `size` bit is clear, the smaller one otherwise
-      const bool keep_max = ((lane & j) == 0) == ((lane & size) == 0);
-      v = keep_max ? (p > v ? p : v) : (p < v ? p : v);
-    }
-  }
-  return v;
-}
-
 // cls: this lane's image in the partition to check (kClsFree, kClsLow or kClsHigh);
 // all_free: every image is free, which needs no class sums.
 template <bool kRel>
@@ -402,7 +384,8 @@ __device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int cls, 
   // ---- floor and remainder: a float quotient, then an exact correction
   uint32_t q = 0;
   if (Xh != 0) {
-    const float qf = u128_to_float(Xh) / u128_to_float(Q);
+    // within a few units of the true quotient (below 2^22 + 1), which the loops correct
+    const float qf = __fdividef(u128_to_float(Xh), u128_to_float(Q));
     q = qf < 4194304.f ? static_cast<uint32_t>(qf) : 4194304u;
   }
   i128 r = static_cast<i128>(Xh) - static_cast<i128>(Q) * q;
@@ -413,32 +396,48 @@ __device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int cls, 
   const u128 rem_hi = static_cast<u128>(r);
   int32_t K = has ? static_cast<int32_t>(q < static_cast<uint32_t>(n) ? q : static_cast<uint32_t>(n)) : 0;
   // ---- largest remainder: one token for each of the |D| images served first
-  const int64_t D = B - warp_sum(static_cast<int64_t>(K));
+  // (0 <= K and the sum of the K below 2^31, so one 32-bit warp reduction gives it)
+  const int64_t D = B - static_cast<int64_t>(__reduce_add_sync(0xffffffffu, static_cast<uint32_t>(K)));
   if (D != 0) {
     const bool up = D > 0;
     const int need = static_cast<int>(up ? D : -D);
     const bool elig = has && (up ? K < n : K > 0);
-    if (__popc(__ballot_sync(0xffffffffu, elig)) < need) return kExactFallback;
-    // 59-bit prefix of the remainder (rem_hi 2^64 + Xl < 2^(bq + 64)), then the index
+    unsigned cand = __ballot_sync(0xffffffffu, elig);
+    if (__popc(cand) < need) return kExactFallback;
+    // 59-bit prefix of the remainder (rem_hi 2^64 + Xl < 2^(bq + 64)); its order is the
+    // order of the remainders, up to ties among equal prefixes
     const unsigned s = bit_length_u128(Q) + 5u;
     const uint64_t prefix = s >= 64 ? static_cast<uint64_t>(rem_hi >> (s - 64))
                                     : static_cast<uint64_t>((rem_hi << (64 - s)) | (Xl >> s));
     const uint64_t kPrefixMask = (uint64_t(1) << 59) - 1;
-    const uint64_t key = !elig ? 0ull
-                         : (up ? (prefix << 5) | static_cast<uint64_t>(31 - lane)
-                               : ((kPrefixMask - prefix) << 5) | static_cast<uint64_t>(lane));
-    const uint64_t sorted = warp_sort_desc(key);
-    const uint64_t thr = __shfl_sync(0xffffffffu, sorted, need - 1);
-    const uint64_t nxt = __shfl_sync(0xffffffffu, sorted, need < 32 ? need : 31);
-    bool served = elig && key >= thr;
-    if (need < 32 && nxt != 0 && (nxt >> 5) == (thr >> 5)) {
-      // the cut falls among remainders with the same prefix: order those exactly
-      const bool in_group = elig && (key >> 5) == (thr >> 5);
-      const unsigned group = __ballot_sync(0xffffffffu, in_group);
-      const int quota = need - __popc(__ballot_sync(0xffffffffu, elig && (key >> 5) > (thr >> 5)));
+    // adding: the largest remainders first; removing: the smallest
+    const uint64_t pkey = !elig ? 0ull : (up ? prefix : kPrefixMask - prefix);
+    // the `need` largest keys by a bitwise radix select with ballots, from the highest bit
+    // any candidate sets: a bit splits the candidates into ones (served first) and zeros
+    int left = need;
+    unsigned served = 0;
+    const unsigned hi_or = __reduce_or_sync(0xffffffffu, static_cast<uint32_t>(pkey >> 32));
+    const unsigned lo_or = __reduce_or_sync(0xffffffffu, static_cast<uint32_t>(pkey));
+    int bit = hi_or ? 63 - __clz(hi_or) : (lo_or ? 31 - __clz(lo_or) : -1);
+#pragma unroll 1
+    for (; bit >= 0 && __popc(cand) > left; --bit) {
+      const unsigned ones = __ballot_sync(0xffffffffu, (pkey >> bit) & 1ull) & cand;
+      const int c = __popc(ones);
+      if (c >= left) {
+        cand = ones;
+      } else {
+        served |= ones;
+        left -= c;
+        cand &= ~ones;
+      }
+    }
+    if (__popc(cand) > left) {
+      // the cut falls among candidates with equal prefixes: order those exactly, ties to the
+      // lower image when adding and to the higher one when removing
+      const bool in_group = (cand >> lane) & 1u;
       const uint64_t rh1 = static_cast<uint64_t>(rem_hi >> 64), rh0 = static_cast<uint64_t>(rem_hi);
       int rank = 0;
-      for (unsigned g = group; g != 0; g &= g - 1) {
+      for (unsigned g = cand; g != 0; g &= g - 1) {
         const int l = __ffs(g) - 1;
         const uint64_t a1 = __shfl_sync(0xffffffffu, rh1, l), a0 = __shfl_sync(0xffffffffu, rh0, l);
         const uint64_t al = __shfl_sync(0xffffffffu, Xl, l);
@@ -446,9 +445,11 @@ __device__ __forceinline__ int exact32(bool has, int64_t S, int64_t n, int cls, 
         if (!up) c = -c;  // removing: the smaller remainder first
         rank += (l != lane && (c > 0 || (c == 0 && (up ? l < lane : l > lane)))) ? 1 : 0;
       }
-      if (in_group) served = rank < quota;
+      served |= __ballot_sync(0xffffffffu, in_group && rank < left);
+    } else {
+      served |= cand;
     }
-    if (served) K += up ? 1 : -1;
+    if ((served >> lane) & 1u) K += up ? 1 : -1;
   }
   *k_out = K;
   return AVTP_OK;
@@ -519,10 +520,11 @@ static __device__ __noinline__ int warp_allocate32_clamped(const WarpAllocSmem& 
 // the common case) is checked exactly first; only when it fails does the grid search for
 // the shift (warp_allocate32_clamped), and only when that partition fails too does the
 // general stage run on sm (32 entries). Identical results and status to warp_allocate.
-// Out of line so that a warm-up call and the real one share the same code.
 // inv_n = floor(2^62 / n_j) and inv_N = floor(2^62 / N) come from the caller, which
-// can take them before the sums are ready.
-static __device__ __noinline__ int warp_allocate32(const WarpAllocSmem& sm, int m, int64_t S, int32_t n, int64_t inv_n,
+// can take them before the sums are ready. Inlined: the fused selection kernel calls it
+// from one place for both its warm-up run and its real run, and a call would put the
+// caller's state on the stack.
+__device__ __forceinline__ int warp_allocate32(const WarpAllocSmem& sm, int m, int64_t S, int32_t n, int64_t inv_n,
                                                    int64_t B, int32_t N, int64_t inv_N, const RatioRule& rule,
                                                    float alpha_f, float r_min_f, float r_max_f, int32_t* k_out) {
   const int lane = threadIdx.x & 31;

@@ -186,13 +186,11 @@ constexpr int kMaxReserveSms = 32;
 int prune_reserve_sms(const avtp_layout_t& L) {
   if (L.n_tokens > 32768 || L.n_images < 1) return 0;
   const int64_t ctas = prune_warm_ctas(L);
-  // one SM per selection CTA: CTAs packed on one SM slow each other's budget rule
-  // (measured: the stage 1.5-2 us longer on the Qwen3-VL-8B-shaped request with four
-  // per SM). Past kMaxReserveSms they share SMs, as many as the occupancy allows.
-  if (ctas <= kMaxReserveSms) return static_cast<int>(ctas);
-  const int per_sm = alloc_select_ctas_per_sm();
-  const int64_t packed = (ctas + per_sm - 1) / per_sm;
-  return static_cast<int>(packed > kMaxReserveSms ? packed : kMaxReserveSms);
+  // one SM per selection CTA (its registers fill most of an SM; two on one SM slowed each
+  // other's budget rule) and one for the validation kernel, which runs when the scoring
+  // kernel starts: at most kMaxReserveSms, the CTAs beyond start when the scoring
+  // kernel's CTAs end
+  return static_cast<int>(ctas + 1 < kMaxReserveSms ? ctas + 1 : kMaxReserveSms);
 }
 
 int prune_warm_ctas(const avtp_layout_t& L) {

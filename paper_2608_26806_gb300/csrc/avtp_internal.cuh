@@ -81,8 +81,8 @@ __device__ __forceinline__ bool wait_expired(uint32_t polls, uint64_t& t0, uint6
 // latest (next kTlEvents words). avtp_prune presets those words before its first kernel.
 // The normal build records nothing and never touches them.
 enum TimelineEvent {
-  kTlPrepBegin = 0, kTlPrepEnd, kTlScoreBegin, kTlScoreEnd, kTlSelBegin, kTlSelWaited, kTlRuleEnd, kTlSelEnd,
-  kTlCompactBegin, kTlCompactWaited, kTlCompactEnd, kTlEvents
+  kTlPrepBegin = 0, kTlPrepEnd, kTlScoreBegin, kTlScoreEnd, kTlSelBegin, kTlSelDryEnd, kTlSelWaited, kTlRuleBegin,
+  kTlRuleEnd, kTlSelEnd, kTlCompactBegin, kTlCompactWaited, kTlCompactEnd, kTlEvents
 };
 constexpr size_t kTimelineOffset = 16;  // bytes after the start of the workspace
 static_assert(kTimelineOffset + 2 * kTlEvents * sizeof(uint64_t) <= 256, "timeline must fit before the first array");
@@ -97,6 +97,22 @@ __device__ __forceinline__ void timeline_stamp(DevStatus* st, int ev) {
 #else
   (void)st;
   (void)ev;
+#endif
+}
+
+// The last of a CTA's nwarps warps to call it stamps ev, so that a CTA sends one pair of
+// atomics to the timeline words, not one per warp (thousands of same-address atomics at
+// the end of a kernel would queue behind each other and move the stamps). *count starts
+// at zero (the caller clears it and synchronises the CTA before the first call).
+__device__ __forceinline__ void timeline_stamp_cta(DevStatus* st, int ev, unsigned* count, unsigned nwarps) {
+#ifdef AVTP_TIMELINE
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0 && atomicAdd(count, 1u) == nwarps - 1) timeline_stamp(st, ev);
+#else
+  (void)st;
+  (void)ev;
+  (void)count;
+  (void)nwarps;
 #endif
 }
 
@@ -331,13 +347,12 @@ cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums,
 
 // In avtp_prune with the hidden-variation criterion on a small batch, the scoring
 // kernel leaves prune_reserve_sms(L) SMs free so that the selection kernel's CTAs (one
-// per image, alloc_select_ctas_per_sm() of them fit on an SM) start while the scores stream in
-// and warm their instruction caches (prune_warm_ctas(L) of them run the code once on
-// made-up data first); 0 otherwise. Right after the scoring stream has swept L2 a cold
-// run of the budget rule and the selection takes several times longer. On large
-// batches the scoring time would grow instead.
+// per image and one per request, one per SM) start while the scores stream in and warm
+// their instruction caches (prune_warm_ctas(L) of them run the code once on made-up data
+// first); 0 otherwise. Right after the scoring stream has swept L2 a cold run of the
+// budget rule and the selection takes several times longer. On large batches the
+// scoring time would grow instead.
 constexpr int kMaxWarmCtas = 96;
-int alloc_select_ctas_per_sm();  // from the occupancy calculator (about 4: 256 threads, 64 registers)
 int prune_reserve_sms(const avtp_layout_t& L);
 int prune_warm_ctas(const avtp_layout_t& L);
 

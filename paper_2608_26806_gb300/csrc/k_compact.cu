@@ -8,7 +8,11 @@
 // element per plane): one thread per row. All row sets go in one launch; the block index
 // range is split between the sets on the host. A single-thread bulk-copy ring per SM
 // (global -> shared -> global) was slower: the gather moves its bytes at about the HBM
-// rate already, and one issuing thread per SM kept fewer of them in flight.
+// rate already, and one issuing thread per SM kept fewer of them in flight. So was a
+// ring of bulk copies per warp with 192 KiB of slots per SM (the whole kept set in flight
+// at once): 14.9 us against 11.7 us for this kernel on the Qwen3-VL-8B-shaped gather (28 MB
+// of kept rows, h_cur read once beforehand, event-timed). Writing the 28 MB is the bound:
+// a plain 28-MB fill takes about 12 us on this part.
 #include "avtp_internal.cuh"
 
 namespace avtp {
@@ -111,12 +115,21 @@ __device__ __forceinline__ void compact_block(const CompactParams& P, int b, con
 __global__ void __launch_bounds__(kThreads)
 k_compact(CompactParams P, int n_blocks, const int32_t* __restrict__ kept_idx, int64_t n_kept, int64_t n_tokens,
           DevStatus* st) {
-  if (threadIdx.x == 0) timeline_stamp(st, kTlCompactBegin);
+#ifdef AVTP_TIMELINE
+  __shared__ unsigned s_tl_done;
+  if (threadIdx.x == 0) {
+    s_tl_done = 0;
+    timeline_stamp(st, kTlCompactBegin);
+  }
+  __syncthreads();
+#endif
   pdl_wait();  // kept_idx comes from the selection kernel
   pdl_trigger();
   if (threadIdx.x == 0) timeline_stamp(st, kTlCompactWaited);
   for (int b = blockIdx.x; b < n_blocks; b += gridDim.x) compact_block(P, b, kept_idx, n_kept, n_tokens, st);
-  if ((threadIdx.x & 31) == 0) timeline_stamp(st, kTlCompactEnd);
+#ifdef AVTP_TIMELINE
+  timeline_stamp_cta(st, kTlCompactEnd, &s_tl_done, kWarps);
+#endif
 }
 
 int compact_ctas_per_sm() {

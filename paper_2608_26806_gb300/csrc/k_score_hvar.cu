@@ -35,9 +35,8 @@ constexpr int kChunkElems = 1024;         // bf16 per tensor per slot (2 KiB)
 constexpr int kChunkBytes = kChunkElems * 2;
 constexpr int kSlotBytes = 2 * kChunkBytes;
 constexpr size_t kSmemBytes = static_cast<size_t>(kWarps) * kSlots * kSlotBytes;  // 192 KiB
-// Layouts up to this many images / requests are staged in shared memory. Kept small
-// (about 11 KiB with the barriers) so that a CTA of the selection kernel, launched
-// while this kernel still runs, fits on the same SM next to the 192-KiB pipeline.
+// Layouts up to this many images / requests are staged in shared memory (about 11 KiB
+// with the barriers, next to the 192-KiB pipeline).
 constexpr int kStageImages = 1024;
 constexpr int kStageRequests = 256;
 
@@ -142,7 +141,10 @@ __device__ void block_scan_inplace(int32_t* a, int n, int32_t* s_warp) {
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+// 64 registers a thread: on large batches (no SMs left free) a CTA of the selection
+// kernel (256 threads, up to 128 registers) can then start on the same SM as this one
+// and wait there for the scores.
+__global__ void __maxnreg__(64)
 k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const __nv_bfloat16* __restrict__ h_prior,
              int64_t prior_stride, int D, const int32_t* __restrict__ cu, int R, const int32_t* __restrict__ icu,
              const int32_t* __restrict__ ist, const int32_t* __restrict__ iln, int NI, int64_t T,
@@ -155,8 +157,16 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   __shared__ int32_t s_icu[kStageRequests + 1];
   __shared__ int32_t s_cu[kStageRequests + 1];
   __shared__ int32_t s_warp[kWarps];
+  __shared__ float s_part[kWarps][2][3];  // a warp's sums over the first / last token it shares
   pdl_trigger();
-  if (threadIdx.x == 0) timeline_stamp(st, kTlScoreBegin);
+#ifdef AVTP_TIMELINE
+  __shared__ unsigned s_tl_done;
+  if (threadIdx.x == 0) {
+    s_tl_done = 0;
+    timeline_stamp(st, kTlScoreBegin);
+  }
+  __syncthreads();
+#endif
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   unsigned char* wbuf = smem + static_cast<size_t>(warp) * kSlots * kSlotBytes;
   uint64_t* wbar = bars[warp];
@@ -203,22 +213,36 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   const uint64_t pol_last = policy_evict_last();
   const int n_chunks = (D + kChunkElems - 1) / kChunkElems;
   const int64_t n_items = min(max(map.n_vis, int64_t(0)), T);  // visual ordinals (never more than T)
-  const int64_t n_warps = static_cast<int64_t>(gridDim.x) * kWarps;
-  const int64_t per_warp = (n_items + n_warps - 1) / n_warps;
-  const int64_t w0 = (static_cast<int64_t>(blockIdx.x) * kWarps + warp) * per_warp;  // this warp's range
-  const int64_t w1 = min(n_items, w0 + per_warp);
+  // ---- work split. CTA c takes a contiguous run of visual tokens (n_items / C each, the
+  // first n_items % C one more). Inside the CTA the pieces (token, chunk) are split evenly
+  // and contiguously between the warps, so that no warp has more than one piece more than
+  // another. A token whose pieces fall to several warps is finished after the main loop
+  // from the warps' partial sums, added in warp order (the same order on every run).
+  const int64_t C = gridDim.x, cta = blockIdx.x;
+  const int64_t tok_q = n_items / C, tok_r = n_items % C;
+  const int64_t v_lo = cta * tok_q + min(cta, tok_r);
+  // pieces of this CTA: below 2^31 for every grid the launcher picks (at most 16 tokens
+  // per CTA when the grid is smaller than the SM count, otherwise n_tokens / 100 or fewer)
+  const int32_t n_pc = static_cast<int32_t>((tok_q + (cta < tok_r ? 1 : 0)) * n_chunks);
+  const int32_t pc_q = n_pc / kWarps, pc_r = n_pc % kWarps;
+  const int32_t p_lo = warp * pc_q + min(warp, pc_r);
+  const int32_t p_hi = p_lo + pc_q + (warp < pc_r ? 1 : 0);
+  const int32_t first_u = p_lo / n_chunks;  // local token of the warp's first piece
+  const int first_c = p_lo % n_chunks;
 
-  int64_t issue_v = w0;
-  int issue_chunk = 0;
+  int32_t p_issue = p_lo;
+  int32_t issue_u = first_u;
+  int issue_chunk = first_c;
   int issue_img = 0;
-  int64_t issue_t = issue_v < w1 ? map.position(issue_v, issue_img) : 0;
+  int64_t issue_t = p_issue < p_hi ? map.position(v_lo + issue_u, issue_img) : 0;
 
-  auto issue_valid = [&]() { return issue_v < w1; };
+  auto issue_valid = [&]() { return p_issue < p_hi; };
   auto advance_issue = [&]() {
+    ++p_issue;
     if (++issue_chunk < n_chunks) return;
     issue_chunk = 0;
-    ++issue_v;
-    if (issue_v < w1) issue_t = map.position(issue_v, issue_img);
+    ++issue_u;
+    if (p_issue < p_hi) issue_t = map.position(v_lo + issue_u, issue_img);
   };
   auto issue_one = [&](int slot) {
     const int e0 = issue_chunk * kChunkElems;
@@ -250,18 +274,19 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   // per lane: even and odd elements accumulate separately (one paired FMA each)
   float2 dot2 = make_float2(0.f, 0.f), na2 = dot2, nb2 = dot2;
   int slot_take = 0;
-  int64_t take_v = w0;
-  int take_chunk = 0;
+  int32_t take_p = p_lo;
+  int32_t take_u = first_u;
+  int take_chunk = first_c;
   int take_img = 0;
   int run_img = -1;     // image of the current run of rows (lane 0's view)
   int64_t run_sum = 0;  // its fixed-point sum so far
-  auto flush_run = [&]() {
+  auto add_to_image = [&](int img, int64_t v) {
+    if (img_sums == nullptr) return;
     if (!waited) {
       pdl_wait();
       waited = true;
     }
-    if (lane == 0 && run_img >= 0)
-      atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + run_img), static_cast<unsigned long long>(run_sum));
+    if (lane == 0) atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + img), static_cast<unsigned long long>(v));
   };
   while (in_flight > 0) {
     const uint32_t parity = (phase_bits >> slot_take) & 1u;
@@ -292,7 +317,7 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     }
     __syncwarp();
     --in_flight;
-    const bool row_done = take_chunk == n_chunks - 1;
+    const bool token_end = take_chunk == n_chunks - 1 || take_p == p_hi - 1;
     // refill the slot just consumed
     if (issue_valid()) {
       issue_one(slot_take);
@@ -300,28 +325,38 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
       ++in_flight;
     }
     slot_take = (slot_take + 1) % kSlots;
-    if (row_done) {
+    if (token_end) {
       const float d = warp_sum(dot2.x + dot2.y), x = warp_sum(na2.x + na2.y), y = warp_sum(nb2.x + nb2.y);
       dot2 = na2 = nb2 = make_float2(0.f, 0.f);
-      const int64_t t = map.position(take_v, take_img);
-      const bool inside = t >= 0 && t < T;
-      const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
-      const float I = 1.f - d / den;
-      if (lane == 0 && inside) scores[t] = I;
-      // run-length accumulation of the per-image sums (take_img is uniform over the warp)
-      if (take_img != run_img) {
-        if (run_img >= 0) flush_run();
-        run_img = take_img;
-        run_sum = 0;
+      const int64_t t = map.position(v_lo + take_u, take_img);
+      const bool whole = take_chunk == n_chunks - 1 && (take_u != first_u || first_c == 0);
+      if (whole) {
+        const bool inside = t >= 0 && t < T;
+        const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
+        const float I = 1.f - d / den;
+        if (lane == 0 && inside) scores[t] = I;
+        // run-length accumulation of the per-image sums (take_img is uniform over the warp)
+        if (take_img != run_img) {
+          if (run_img >= 0) add_to_image(run_img, run_sum);
+          run_img = take_img;
+          run_sum = 0;
+        }
+        if (inside) run_sum += fixed_point_score(I);
+      } else if (lane == 0) {
+        // a piece of a token shared with other warps: the first or the last of this warp's
+        const int k = take_u == first_u ? 0 : 1;
+        s_part[warp][k][0] = d;
+        s_part[warp][k][1] = x;
+        s_part[warp][k][2] = y;
       }
-      if (inside) run_sum += fixed_point_score(I);
+    }
+    ++take_p;
+    if (++take_chunk == n_chunks) {
       take_chunk = 0;
-      ++take_v;
-    } else {
-      ++take_chunk;
+      ++take_u;
     }
   }
-  if (!timed_out && run_img >= 0) flush_run();
+  if (!timed_out && run_img >= 0) add_to_image(run_img, run_sum);
   if (timed_out) {
     // drain: give the copies still in flight (slot_take and the in_flight - 1 slots after
     // it) a bounded chance to land before the CTA exits
@@ -335,8 +370,42 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     pdl_wait();  // the validation kernel resets the status word: record after it
     if (lane == 0) record_error(st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));
   }
+
+  // ---- tokens shared by several warps, finished by the warp that holds the last piece
+  __syncthreads();
+  if (p_lo < p_hi && first_c != 0 && p_hi >= (first_u + 1) * n_chunks && lane == 0) {
+    // the warps that hold pieces of token first_u, from the one with its first piece
+    const int32_t p0 = first_u * n_chunks;
+    const int32_t big = (pc_q + 1) * pc_r;  // pieces held by the warps with one extra piece
+    const int w0 = p0 < big ? p0 / (pc_q + 1) : pc_r + (p0 - big) / pc_q;
+    float d = 0.f, x = 0.f, y = 0.f;
+    for (int w = w0; w <= warp; ++w) {
+      const int32_t wp = w * pc_q + min(w, pc_r);  // first piece of warp w
+      const int k = (w == warp || wp / n_chunks == first_u) ? 0 : 1;
+      d += s_part[w][k][0];
+      x += s_part[w][k][1];
+      y += s_part[w][k][2];
+    }
+    int img = 0;
+    const int64_t t = map.position(v_lo + first_u, img);
+    if (t >= 0 && t < T) {
+      const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
+      const float I = 1.f - d / den;
+      scores[t] = I;
+      if (img_sums != nullptr) {
+        if (!waited) {
+          pdl_wait();
+          waited = true;
+        }
+        atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + img),
+                  static_cast<unsigned long long>(fixed_point_score(I)));
+      }
+    }
+  }
   pdl_wait();  // completion of this grid implies completion of the one before it
-  if (lane == 0) timeline_stamp(st, kTlScoreEnd);
+#ifdef AVTP_TIMELINE
+  timeline_stamp_cta(st, kTlScoreEnd, &s_tl_done, kWarps);
+#endif
 }
 
 }  // namespace
@@ -344,18 +413,32 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
 cudaError_t launch_score_hvar(const avtp_layout_t& L, const avtp_score_args_t& sa, float* scores,
                               int64_t* img_sums, void* ws, const WsPlan& p, cudaStream_t s, int reserve_sms) {
   if (L.n_images == 0 || L.n_tokens == 0) return cudaSuccess;
+  // The dynamic shared memory a CTA may take: all an SM offers a CTA, less the static part.
   static PerDevice attrs;
-  cudaError_t ae = once_per_device(attrs, [](int, int*) {
-    return cudaFuncSetAttribute(k_score_hvar, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                static_cast<int>(kSmemBytes));
-  });
+  int smem_max = 0;
+  cudaError_t ae = once_per_device(attrs, [](int dev, int* v) {
+    int optin = 0;
+    cudaFuncAttributes fa{};
+    cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, k_score_hvar);
+    if (e != cudaSuccess) return e;
+    *v = optin - static_cast<int>(fa.sharedSizeBytes);
+    if (*v < static_cast<int>(kSmemBytes)) return cudaErrorInvalidConfiguration;
+    return cudaFuncSetAttribute(k_score_hvar, cudaFuncAttributeMaxDynamicSharedMemorySize, *v);
+  }, &smem_max);
   if (ae != cudaSuccess) return ae;
+  // With SMs left to the selection kernel, each scoring CTA takes all the shared memory a
+  // CTA may have (the pipeline uses kSmemBytes of it): no CTA of the selection kernel can
+  // then start next to it, so they all land on the free SMs. Sharing an SM with 16
+  // streaming warps, a selection CTA fetched its code several times slower and its
+  // warm-up run did not end before the scores did.
+  const size_t smem = reserve_sms > 0 ? static_cast<size_t>(smem_max) : kSmemBytes;
   const int64_t want = (L.n_tokens + kWarps - 1) / kWarps;
   // one 192 KiB CTA per SM, except the SMs left to the next kernel
   int64_t cap = static_cast<int64_t>(device_sm_count()) - reserve_sms;
   if (cap < 1) cap = 1;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  cudaError_t e = launch_kernel(k_score_hvar, dim3(grid), dim3(kThreads), kSmemBytes, s, /*pdl=*/true,
+  cudaError_t e = launch_kernel(k_score_hvar, dim3(grid), dim3(kThreads), smem, s, /*pdl=*/true,
                                 static_cast<const __nv_bfloat16*>(sa.h_cur), sa.h_cur_stride,
                                 static_cast<const __nv_bfloat16*>(sa.h_prior), sa.h_prior_stride, sa.hidden,
                                 L.cu_seqlens, L.n_requests, L.img_cu, L.img_start, L.img_len, L.n_images, L.n_tokens,

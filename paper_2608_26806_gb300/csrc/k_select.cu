@@ -53,9 +53,12 @@ struct SelShared {
   int digit, above, count;
   // hand-over from the warps of the fused kernel
   uint32_t kmin, kmax;
-  int k, before, total, alloc_err, vis_before, n_vis;
+  int k, before, total, alloc_err, out_lo, out_hi, vis_before, n_vis;
   int ncand;      // candidates gathered from the chosen first-pass bucket
   uint32_t thr;   // the k-th largest key, found among them
+  // inputs of the fused kernel's warm-up run (see alloc_select_tail)
+  int32_t dry_status[4];  // a status word that reads "layout ok"
+  int32_t dry_out[2];
 };
 
 // Named barrier for warps 1..7 (224 threads) while warp 0 runs the budget rule.
@@ -219,7 +222,7 @@ constexpr int kCandCap = 256;
 // ascending order: every key above thr and the first k - #(key > thr) equal to it.
 // Returns false (having written nothing) when the bucket is too large; all threads call.
 // dry: compute everything but write nothing (warms the instruction cache).
-__device__ __noinline__ bool select_from_first_pass(int n, int k, int64_t t0, int64_t base,
+__device__ __forceinline__ bool select_from_first_pass(int n, int k, int64_t t0, int64_t base,
                                                     int32_t* __restrict__ kept_idx, SelShared& sh, uint32_t kmin,
                                                     uint32_t kmax, bool dry) {
   const int tid = threadIdx.x;
@@ -397,117 +400,95 @@ struct AllocParams {
   int warm_ctas;     // CTAs below this index warm their instruction cache before the wait
 };
 
-__global__ void __launch_bounds__(kThreads, 2)
-k_alloc_select(SelectArgs a, AllocParams ap) {
-  extern __shared__ __align__(16) unsigned char dsmem[];  // budget scratch for requests of > 32 images
-  __shared__ __align__(16) unsigned char rule32[warp_alloc_smem_bytes(32)];  // ... and of at most 32
-  __shared__ SelShared sh;
+// What a CTA of k_alloc_select knows before the scores exist (from the call's inputs).
+struct TailIn {
+  int r, i0, m, li;
+  int32_t s0, n, nxt, Tr;
+  int64_t t0;
+  // warp 0: the request's sizes and the scalars of the budget rule
+  int32_t N, n_lane, vis_before;
+  int64_t B, inv_n, inv_N;
+  float kr;
+  RatioRule rule;
+};
+
+// Keys of the CTA's image held per thread of warps 1..7 right after the wait.
+constexpr int kTailKeys = (kKeyCap + kThreads - 33) / (kThreads - 32);
+
+// Everything k_alloc_select does once the scores exist. The kernel runs it twice from one
+// copy of the code (a loop that is not unrolled): first with dry set, before the wait, on
+// whatever the buffers hold then (every index is in bounds for any contents; the sums are
+// replaced by equal made-up means, so that the budget rule takes its common path),
+// writing nothing to global memory; then for real. The dry run leaves exactly this code
+// in the SM's instruction cache: a cold fetch costs about a microsecond per miss once the
+// scoring stream has swept L2. Inlined, so that nothing of it lives on the stack (after
+// the wait, local memory would come back from DRAM too).
+// After the wait, one round of loads brings the status word, the request's sums, the
+// request's output offsets and the image's scores, so that only one memory latency
+// precedes the budget rule and the first histogram (which run side by side). The warm-up
+// run loads the same way from shared memory (generic loads serve both): while the scores
+// stream in, every global access waits behind them for microseconds.
+__device__ __forceinline__ void alloc_select_tail(const SelectArgs& a, const AllocParams& ap, SelShared& sh,
+                                                  const WarpAllocSmem& wsm, const WarpAllocSmem& wsm32,
+                                                  const TailIn& in, bool dry) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = blockIdx.x;
-  if (tid == 0) timeline_stamp(a.st, kTlSelBegin);
-  const WarpAllocSmem wsm = carve_warp_alloc(dsmem, ap.m_cap);
-  const WarpAllocSmem wsm32 = carve_warp_alloc(rule32, 32);
+  const int r = in.r, i0 = in.i0, m = in.m, li = in.li;
+  const int32_t s0 = in.s0, nxt = in.nxt, Tr = in.Tr;
+  const int32_t n = dry ? min(in.n, kKeyCap) : in.n;
+  const int64_t t0 = in.t0;
+  const bool image = b < a.NI;
+  // where the loads below read: the call's buffers, or shared stand-ins for the warm-up
+  const float* sc = dry ? reinterpret_cast<const float*>(sh.keys) : a.scores + t0;
+  const int32_t* status = dry ? sh.dry_status : &a.st->layout_ok;
+  const int64_t* sums = dry ? wsm32.S : ap.img_sums + i0;
+  const int32_t* out_cu = dry ? sh.dry_out : a.out_cu + r;
+  const bool stage = n <= kKeyCap;
 
-  // ---- set-up from the call's inputs only, overlapped with the scoring kernel.
-  // The layout is not validated yet, so every index is clamped; nothing here is
-  // used unless the validation kernel accepts the layout.
-  int r = 0, i0 = 0, m = 0, li = 0;
-  int32_t s0 = 0, n = 0, nxt = 0, Tr = 0;
-  int64_t t0 = 0;
-  if (b < a.NI) {
-    r = upper_index(a.icu, a.R, b);
-    i0 = min(max(a.icu[r], 0), a.NI);
-    const int i1 = min(max(a.icu[r + 1], i0), a.NI);
-    m = min(i1 - i0, ap.m_cap);
-    if (m > 0) {
-      li = min(max(b - i0, 0), m - 1);
-      Tr = a.cu[r + 1] - a.cu[r];
-      s0 = a.ist[i0 + li];
-      n = a.iln[i0 + li];
-      nxt = (li + 1 < m) ? a.ist[i0 + li + 1] : Tr;
-      t0 = static_cast<int64_t>(a.cu[r]) + s0;
+  // ---- one round of loads
+  const int layout_ok = *status;
+  int64_t S_lane = 0;
+  int32_t out_lo = 0, out_hi = 0;
+  uint32_t key[kTailKeys];
+  if (warp == 0) {
+    if (image && lane < m && m <= 32) S_lane = sums[lane];
+    if (image) {
+      out_lo = out_cu[0];
+      out_hi = out_cu[1];
     }
-  }
-  // warp 0: the request's sizes and the scalars of the budget rule
-  int32_t N = 0, n_lane = 0, vis_before = 0;
-  int64_t B = 0, inv_n = 0, inv_N = 0;
-  float kr = 0.f;
-  RatioRule rule{};
-  if (warp == 0 && b < a.NI) {
-    int64_t nsum = 0, nbefore = 0;
-    for (int j = lane; j < m; j += 32) {
-      const int32_t nj = a.iln[i0 + j];
-      if (m > 32) wsm.n[j] = nj;
-      else n_lane = nj;
-      nsum += nj;
-      nbefore += j < li ? nj : 0;
-    }
-    N = static_cast<int32_t>(warp_sum(nsum));
-    vis_before = static_cast<int32_t>(warp_sum(nbefore));
-    kr = ap.keep_ratio[r];
-    // B_r = floor(r_base * N_vis + 0.5), each operation rounded once
-    B = static_cast<int64_t>(floor(__dadd_rn(__dmul_rn(static_cast<double>(kr), static_cast<double>(N)), 0.5)));
-    rule = make_ratio_rule(kr, ap.alpha, ap.relative);
-    inv_N = recip62(N);
-    inv_n = recip62(n_lane);
-  }
-
-  // ---- warm the instruction cache. When the scoring kernel leaves SMs free
-  // (prune_reserve_sms), the first CTAs start while the scores stream in, so the budget
-  // rule and the selection run once on made-up data here, writing nothing to global
-  // memory; their code is then resident when the real data arrives (a cold fetch
-  // costs about 1 us per KiB, the L2 having been swept by the scoring kernel).
-  if (b < ap.warm_ctas && b < a.NI && m >= 1 && m <= 32) {
-    constexpr int kDryKeys = 1024;
-    if (warp == 0) {
-      const int64_t S = lane < m ? (static_cast<int64_t>(n_lane) << 30) : 0;
-      int32_t K = 0;
-      const int err = warp_allocate32(wsm32, m, S, n_lane, inv_n, B, N, inv_N, rule, ap.alpha, ap.r_min, ap.r_max, &K);
-      asm volatile("" ::"r"(K), "r"(err));
+  } else if (image && stage) {
+    const int wt = tid - 32;
 #pragma unroll
-      for (int q = 0; q < 8; ++q) sh.hist[0][lane * 8 + q] = 0;
-    } else {
-      const int wt = tid - 32;
-      for (int j = wt; j < kDryKeys; j += kThreads - 32) sh.keys[j] = 0x3f800000u + static_cast<uint32_t>(j);
-#pragma unroll
-      for (int q = 0; q < 8; ++q) sh.hist[warp][lane * 8 + q] = 0;
-      if (tid == 32) sh.ncand = 0;
-      bar_workers();
-      // keys 0x3f800000 .. +1023: the top differing bit is 9, digits are bits 2..9
-      hist_pass(KeySource{a.scores, sh.keys}, kDryKeys, ~0x3ffu, 0x3f800000u, 2, 0xffu, sh.hist[warp], wt, kThreads - 32);
+    for (int q = 0; q < kTailKeys; ++q) {
+      const int j = wt + q * (kThreads - 32);
+      key[q] = j < n ? rank_key(sc[j]) : 0u;
     }
-    __syncthreads();
-    select_from_first_pass(kDryKeys, kDryKeys / 2, 0, 0, a.kept_idx, sh, 0x3f800000u, 0x3f8003ffu, true);
-    __syncthreads();
   }
-
-  // ---- wait for the scores and per-image sums (and, through them, the validation)
-  pdl_wait();
-  pdl_trigger();
-  if (tid == 0) timeline_stamp(a.st, kTlSelWaited);
-  if (!a.st->layout_ok) return;
-  if (b >= a.NI) {
-    leading_text(a, b - a.NI);
+  if (dry) S_lane = lane < m ? (static_cast<int64_t>(in.n_lane) << 30) : 0;  // equal means
+  if (!layout_ok) return;
+  if (!image) {
+    if (!dry) leading_text(a, b - a.NI);
     return;
   }
   const int i = b;
-  const float* sc = a.scores + t0;
-  const bool stage = n <= kKeyCap;
   if (warp == 0) {
     // ---- the budget rule, one warp
     int err;
     int k, before, total;
     if (m <= 32) {
-      const int64_t S = lane < m ? ap.img_sums[i0 + lane] : 0;
+#ifdef AVTP_TIMELINE
+      if (!dry && __shfl_sync(kFull, S_lane, 0) != INT64_MIN && lane == 0) timeline_stamp(a.st, kTlRuleBegin);
+#endif
       int32_t K;
-      err = warp_allocate32(wsm32, m, S, n_lane, inv_n, B, N, inv_N, rule, ap.alpha, ap.r_min, ap.r_max, &K);
+      err = warp_allocate32(wsm32, m, S_lane, in.n_lane, in.inv_n, in.B, in.N, in.inv_N, in.rule, ap.alpha, ap.r_min,
+                            ap.r_max, &K);
       k = __shfl_sync(kFull, K, li);
-      before = warp_sum(lane < li ? K : 0);
-      total = warp_sum(lane < m ? K : 0);
+      before = static_cast<int>(__reduce_add_sync(kFull, static_cast<uint32_t>(lane < li ? K : 0)));
+      total = static_cast<int>(__reduce_add_sync(kFull, static_cast<uint32_t>(lane < m ? K : 0)));
     } else {
-      for (int j = lane; j < m; j += 32) wsm.S[j] = ap.img_sums[i0 + j];
+      for (int j = lane; j < m; j += 32) wsm.S[j] = dry ? (static_cast<int64_t>(wsm.n[j]) << 30) : ap.img_sums[i0 + j];
       __syncwarp();
-      err = warp_allocate(wsm, m, B, N, kr, ap.alpha, ap.r_min, ap.r_max, ap.relative);
+      err = warp_allocate(wsm, m, in.B, in.N, in.kr, ap.alpha, ap.r_min, ap.r_max, ap.relative);
       int bs = 0, ts = 0;
       for (int j = lane; j < m; j += 32) {
         ts += wsm.K[j];
@@ -520,23 +501,36 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
 #pragma unroll
     for (int q = 0; q < 8; ++q) sh.hist[0][lane * 8 + q] = 0;  // warp 0 takes no part in the first pass
     if (lane == 0) {
-      timeline_stamp(a.st, kTlRuleEnd);
+      if (!dry) timeline_stamp(a.st, kTlRuleEnd);
       sh.k = k;
       sh.before = before;
       sh.total = total;
       sh.alloc_err = err;
-      sh.vis_before = vis_before;
-      sh.n_vis = N;
+      sh.out_lo = out_lo;
+      sh.out_hi = out_hi;
+      sh.vis_before = in.vis_before;
+      sh.n_vis = in.N;
     }
   } else {
     // ---- warps 1..7: stage the keys, find their range, build the first histogram
     const int wt = tid - 32;
     uint32_t lo = 0xffffffffu, hi = 0u;
-    for (int j = wt; j < n; j += kThreads - 32) {
-      const uint32_t key = rank_key(sc[j]);
-      if (stage) sh.keys[j] = key;
-      lo = min(lo, key);
-      hi = max(hi, key);
+    if (stage) {
+#pragma unroll
+      for (int q = 0; q < kTailKeys; ++q) {
+        const int j = wt + q * (kThreads - 32);
+        if (j < n) {
+          sh.keys[j] = key[q];
+          lo = min(lo, key[q]);
+          hi = max(hi, key[q]);
+        }
+      }
+    } else {
+      for (int j = wt; j < n; j += kThreads - 32) {
+        const uint32_t kk = rank_key(sc[j]);
+        lo = min(lo, kk);
+        hi = max(hi, kk);
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -573,24 +567,109 @@ k_alloc_select(SelectArgs a, AllocParams ap) {
   }
   __syncthreads();
   const uint32_t kmin = sh.kmin, kmax = sh.kmax;
-  const int k = sh.k, before = sh.before, total = sh.total, vis_b = sh.vis_before, Nv = sh.n_vis;
-  if (sh.alloc_err != AVTP_OK) {
-    if (tid == 0) record_error(a.st, sh.alloc_err, r);
-    return;
+  const int k = sh.k, before = sh.before, total = sh.total;
+  const int32_t olo = sh.out_lo, ohi = sh.out_hi, vis_b = sh.vis_before, Nv = sh.n_vis;
+  if (!dry) {
+    if (sh.alloc_err != AVTP_OK) {
+      if (tid == 0) record_error(a.st, sh.alloc_err, r);
+      return;
+    }
+    if (tid == 0) ap.budgets[i] = k;
+    if (olo < 0 || ohi - olo != total + (Tr - Nv) || static_cast<int64_t>(ohi) > a.n_kept) {
+      if (tid == 0) record_error(a.st, AVTP_ERR_DEVICE_INPUT, i);
+      return;
+    }
   }
-  if (tid == 0) ap.budgets[i] = k;
-  const int32_t out_lo = a.out_cu[r], out_hi = a.out_cu[r + 1];
-  if (out_lo < 0 || out_hi - out_lo != total + (Tr - Nv) || static_cast<int64_t>(out_hi) > a.n_kept) {
-    if (tid == 0) record_error(a.st, AVTP_ERR_DEVICE_INPUT, i);
-    return;
-  }
-  const int64_t base = static_cast<int64_t>(out_lo) + (s0 - vis_b) + before;
+  const int64_t base = static_cast<int64_t>(olo) + (s0 - vis_b) + before;
   const bool fast = stage && kmin != kmax && k > 0 && k < n &&
-                    select_from_first_pass(n, k, t0, base, a.kept_idx, sh, kmin, kmax, false);
+                    select_from_first_pass(n, k, t0, base, a.kept_idx, sh, kmin, kmax, dry);
+  if (dry) {
+    __syncthreads();  // the shared state is reused by the real run
+    return;
+  }
   if (!fast) block_select(sc, n, k, t0, base, a.kept_idx, sh, stage, kmin, kmax, kmin != kmax);
   const int e = s0 + n;
   for (int p = e + tid; p < nxt; p += kThreads) a.kept_idx[base + k + (p - e)] = a.cu[r] + p;
   if (tid == 0) timeline_stamp(a.st, kTlSelEnd);
+}
+
+// 184 registers: the tail runs without spilling (at 128 it spilled about 100 bytes a
+// thread, and local memory is slow to come back right after the scoring stream). One CTA
+// per SM, which is how the free SMs are used anyway.
+__global__ void __maxnreg__(184)
+k_alloc_select(SelectArgs a, AllocParams ap) {
+  extern __shared__ __align__(16) unsigned char dsmem[];  // budget scratch for requests of > 32 images
+  __shared__ __align__(16) unsigned char rule32[warp_alloc_smem_bytes(32)];  // ... and of at most 32
+  __shared__ SelShared sh;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int b = blockIdx.x;
+  if (tid == 0) timeline_stamp(a.st, kTlSelBegin);
+  const WarpAllocSmem wsm = carve_warp_alloc(dsmem, ap.m_cap);
+  const WarpAllocSmem wsm32 = carve_warp_alloc(rule32, 32);
+
+  // ---- set-up from the call's inputs only, overlapped with the scoring kernel.
+  // The layout is not validated yet, so every index is clamped; nothing here is
+  // used unless the validation kernel accepts the layout.
+  TailIn in{};
+  if (b < a.NI) {
+    in.r = upper_index(a.icu, a.R, b);
+    in.i0 = min(max(a.icu[in.r], 0), a.NI);
+    const int i1 = min(max(a.icu[in.r + 1], in.i0), a.NI);
+    in.m = min(i1 - in.i0, ap.m_cap);
+    if (in.m > 0) {
+      in.li = min(max(b - in.i0, 0), in.m - 1);
+      in.Tr = a.cu[in.r + 1] - a.cu[in.r];
+      in.s0 = a.ist[in.i0 + in.li];
+      in.n = a.iln[in.i0 + in.li];
+      in.nxt = (in.li + 1 < in.m) ? a.ist[in.i0 + in.li + 1] : in.Tr;
+      in.t0 = static_cast<int64_t>(a.cu[in.r]) + in.s0;
+    }
+    // a span outside the scores (a malformed layout, reported by the validation kernel)
+    // is never read, not even by the dry run
+    if (in.t0 < 0 || in.n < 0 || in.t0 + in.n > a.T) {
+      in.t0 = 0;
+      in.n = 0;
+    }
+  }
+  if (warp == 0 && b < a.NI) {
+    int64_t nsum = 0, nbefore = 0;
+    for (int j = lane; j < in.m; j += 32) {
+      const int32_t nj = a.iln[in.i0 + j];
+      if (in.m > 32) wsm.n[j] = nj;
+      else in.n_lane = nj;
+      nsum += nj;
+      nbefore += j < in.li ? nj : 0;
+    }
+    in.N = static_cast<int32_t>(warp_sum(nsum));
+    in.vis_before = static_cast<int32_t>(warp_sum(nbefore));
+    in.kr = ap.keep_ratio[in.r];
+    // B_r = floor(r_base * N_vis + 0.5), each operation rounded once
+    in.B = static_cast<int64_t>(
+        floor(__dadd_rn(__dmul_rn(static_cast<double>(in.kr), static_cast<double>(in.N)), 0.5)));
+    in.rule = make_ratio_rule(in.kr, ap.alpha, ap.relative);
+    in.inv_N = recip62(in.N);
+    in.inv_n = recip62(in.n_lane);
+  }
+
+  if (tid == 0) {
+    sh.dry_status[0] = sh.dry_status[1] = sh.dry_status[2] = sh.dry_status[3] = 1;
+    sh.dry_out[0] = 0;
+    sh.dry_out[1] = 0;
+  }
+  __syncthreads();
+  // ---- the dry run (see alloc_select_tail) on the CTAs that start while the scores
+  // stream in (prune_reserve_sms), then the wait for the scores and per-image sums (and,
+  // through them, the validation), then the real run: one copy of the code for both
+#pragma unroll 1
+  for (int pass = b < ap.warm_ctas ? 0 : 1; pass < 2; ++pass) {
+    if (pass == 1) {
+      if (tid == 0 && b < ap.warm_ctas) timeline_stamp(a.st, kTlSelDryEnd);
+      pdl_wait();
+      pdl_trigger();
+      if (tid == 0) timeline_stamp(a.st, kTlSelWaited);
+    }
+    alloc_select_tail(a, ap, sh, wsm, wsm32, in, pass == 0);
+  }
 }
 
 SelectArgs make_args(const avtp_layout_t& L, const float* scores, const int32_t* out_cu_seqlens, int32_t* kept_idx,
@@ -620,15 +699,6 @@ cudaError_t launch_select(const avtp_layout_t& L, const float* scores, const int
                           const WsPlan& p, cudaStream_t s) {
   const SelectArgs a = make_args(L, scores, out_cu_seqlens, kept_idx, n_kept, ws, p);
   return launch_kernel(k_select, dim3(L.n_images + L.n_requests), dim3(kThreads), 0, s, /*pdl=*/true, a, budgets);
-}
-
-int alloc_select_ctas_per_sm() {
-  static PerDevice occ;
-  int n = 0;
-  const cudaError_t e = once_per_device(occ, [](int, int* v) {
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(v, k_alloc_select, kThreads, 0);
-  }, &n);
-  return (e == cudaSuccess && n >= 1) ? n : 1;
 }
 
 cudaError_t launch_alloc_select(const avtp_layout_t& L, const int64_t* img_sums, const avtp_alloc_args_t& aa,
