@@ -41,7 +41,7 @@ struct DevStatus {
   int32_t code;
   int32_t layout_ok;
   int32_t detail;  // index of the first offending item, for debugging
-  int32_t pad;
+  uint32_t pool;   // tokens the criterion-A scoring kernel's warps have drawn from its pool
 };
 
 __device__ __forceinline__ void record_error(DevStatus* st, int32_t code, int32_t detail) {

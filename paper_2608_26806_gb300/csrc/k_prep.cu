@@ -263,6 +263,7 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
   if (tid == 0) {
     st->code = s_err;
     st->detail = s_detail;
+    st->pool = 0;
     st->layout_ok = (s_err == 0) ? 1 : 0;
     timeline_stamp(st, kTlPrepEnd);
   }

@@ -7,19 +7,25 @@
 // 192 KiB per SM are in flight, independent of the register file. The warp then
 // accumulates dot, |a|^2 and |b|^2 in fp32 from shared memory.
 //
-// Work is split by visual ordinal: warp w of W takes a contiguous range of
-// visual tokens. Each CTA derives the ordinal -> (image, packed position) map
-// itself from the layout, staged in shared memory, so it needs nothing from the
-// validation kernel and runs alongside it (programmatic dependent launch). Every
-// position is checked to lie in [0, T) before a copy is issued, so a malformed
-// layout cannot make it read out of bounds; the validation kernel reports it.
-// Layouts too large to stage fall back to the validation kernel's prefix arrays.
+// Work is split by visual ordinal, whole tokens per warp: each warp first takes a
+// fixed contiguous run of about 80 % of its even share, then draws the remaining
+// tokens one at a time from a pool (a counter in the status word that the validation
+// kernel resets; the first draw waits for that kernel). Without the pool the CTAs
+// finished up to 6 us apart on the Qwen3-VL-8B-shaped request: SMs do not all get the
+// same share of the memory bandwidth. A token is scored by one warp either way, so the
+// scores do not depend on which warp takes it. Each CTA derives the ordinal -> (image,
+// packed position) map itself from the layout, staged in shared memory, so it needs
+// nothing from the validation kernel before its pool draws and runs alongside it
+// (programmatic dependent launch). Every position is checked to lie in [0, T) before a
+// copy is issued, so a malformed layout cannot make it read out of bounds; the
+// validation kernel reports it. Layouts too large to stage fall back to the validation
+// kernel's prefix arrays.
 //
 // Per-image sums S_i = sum rint(fx(I) * 2^32) (integers, so any order gives the
 // same value) are accumulated per warp over runs of rows of the same image and
 // added to img_sums with one atomic per run. The validation kernel zeroes
-// img_sums, so the first atomic of a warp waits for it; with contiguous ranges
-// that is normally at the end of the warp's work, when it has long finished.
+// img_sums, so the first atomic of a warp waits for it; that is normally well after
+// it has finished.
 //
 // L2 policy: h_prior evict-first, h_cur evict-last, because the compaction step
 // reads the kept h_cur rows again right after.
@@ -157,7 +163,6 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   __shared__ int32_t s_icu[kStageRequests + 1];
   __shared__ int32_t s_cu[kStageRequests + 1];
   __shared__ int32_t s_warp[kWarps];
-  __shared__ float s_part[kWarps][2][3];  // a warp's sums over the first / last token it shares
   pdl_trigger();
 #ifdef AVTP_TIMELINE
   __shared__ unsigned s_tl_done;
@@ -213,36 +218,78 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
   const uint64_t pol_last = policy_evict_last();
   const int n_chunks = (D + kChunkElems - 1) / kChunkElems;
   const int64_t n_items = min(max(map.n_vis, int64_t(0)), T);  // visual ordinals (never more than T)
-  // ---- work split. CTA c takes a contiguous run of visual tokens (n_items / C each, the
-  // first n_items % C one more). Inside the CTA the pieces (token, chunk) are split evenly
-  // and contiguously between the warps, so that no warp has more than one piece more than
-  // another. A token whose pieces fall to several warps is finished after the main loop
-  // from the warps' partial sums, added in warp order (the same order on every run).
-  const int64_t C = gridDim.x, cta = blockIdx.x;
-  const int64_t tok_q = n_items / C, tok_r = n_items % C;
-  const int64_t v_lo = cta * tok_q + min(cta, tok_r);
-  // pieces of this CTA: below 2^31 for every grid the launcher picks (at most 16 tokens
-  // per CTA when the grid is smaller than the SM count, otherwise n_tokens / 100 or fewer)
-  const int32_t n_pc = static_cast<int32_t>((tok_q + (cta < tok_r ? 1 : 0)) * n_chunks);
-  const int32_t pc_q = n_pc / kWarps, pc_r = n_pc % kWarps;
-  const int32_t p_lo = warp * pc_q + min(warp, pc_r);
-  const int32_t p_hi = p_lo + pc_q + (warp < pc_r ? 1 : 0);
-  const int32_t first_u = p_lo / n_chunks;  // local token of the warp's first piece
-  const int first_c = p_lo % n_chunks;
+  // ---- work split. Each warp first takes a fixed contiguous run of whole tokens, about
+  // 80 % of its even share; the rest of the tokens form a pool that the warps draw from
+  // one token at a time (a counter the validation kernel resets), so that SMs with more
+  // memory bandwidth take more of it and the CTAs finish together. Batches of fewer than
+  // four tokens a warp are split evenly with no pool.
+  // (visual ordinals are below 2^31: cu_seqlens are int32)
+  const int32_t n_vis32 = static_cast<int32_t>(n_items);
+  const int32_t n_warps = static_cast<int32_t>(gridDim.x) * kWarps;
+  const int32_t gw = static_cast<int32_t>(blockIdx.x) * kWarps + warp;
+  const bool pooled = n_items >= 4 * static_cast<int64_t>(n_warps);
+  int32_t v_lo, v_hi, pool_lo;
+  if (pooled) {
+    const int32_t per = (n_vis32 - n_vis32 / 5) / n_warps;
+    v_lo = gw * per;
+    v_hi = v_lo + per;
+    pool_lo = n_warps * per;
+  } else {
+    const int32_t per = n_vis32 / n_warps, extra = n_vis32 % n_warps;
+    v_lo = gw * per + min(gw, extra);
+    v_hi = v_lo + per + (gw < extra ? 1 : 0);
+    pool_lo = n_vis32;
+  }
+  unsigned int* pool = &st->pool;
+  bool waited = false;  // the validation kernel (which resets the pool and img_sums) is done
+  auto wait_prep = [&]() {
+    if (!waited) {
+      pdl_wait();
+      waited = true;
+    }
+  };
+  // The next pool token is requested one token ahead (lane 0's atomic; its value is read
+  // only when that token is due, so the request's latency hides behind the current one).
+  bool pref = false;  // a request is outstanding (its value is in lane 0's pref_raw)
+  unsigned int pref_raw = 0;
+  auto request_pool = [&]() {
+    wait_prep();
+    if (lane == 0) pref_raw = atomicAdd(pool, 1u);
+    pref = true;
+  };
+  // the token after `v` in this warp's sequence (n_items when there is none)
+  auto next_token = [&](int32_t v) -> int32_t {
+    if (v + 1 < v_hi) return v + 1;
+    if (pool_lo >= n_vis32) return n_vis32;
+    if (!pref) request_pool();
+    const uint32_t k = __shfl_sync(0xffffffffu, pref_raw, 0);
+    pref = false;
+    return k < static_cast<uint32_t>(n_vis32 - pool_lo) ? pool_lo + static_cast<int32_t>(k) : n_vis32;
+  };
 
-  int32_t p_issue = p_lo;
-  int32_t issue_u = first_u;
-  int issue_chunk = first_c;
+  // issue side: token issue_v, chunk issue_chunk
+  int32_t issue_v = v_lo < v_hi ? v_lo : next_token(v_hi - 1);
+  int issue_chunk = 0;
   int issue_img = 0;
-  int64_t issue_t = p_issue < p_hi ? map.position(v_lo + issue_u, issue_img) : 0;
+  int64_t issue_t = issue_v < n_vis32 ? map.position(issue_v, issue_img) : 0;
+  // tokens issued (and the one prepared next) not yet consumed, oldest first: at most
+  // kSlots + 1, when every token is one chunk
+  int32_t q0 = issue_v, q1 = -1, q2 = -1, q3 = -1;
+  if (issue_v < n_vis32 && issue_v + 1 >= v_hi && pool_lo < n_vis32) request_pool();
 
-  auto issue_valid = [&]() { return p_issue < p_hi; };
+  auto issue_valid = [&]() { return issue_v < n_vis32; };
   auto advance_issue = [&]() {
-    ++p_issue;
     if (++issue_chunk < n_chunks) return;
     issue_chunk = 0;
-    ++issue_u;
-    if (p_issue < p_hi) issue_t = map.position(v_lo + issue_u, issue_img);
+    issue_v = next_token(issue_v);
+    if (issue_v < n_vis32) {
+      issue_t = map.position(issue_v, issue_img);
+      if (q1 < 0) q1 = issue_v;
+      else if (q2 < 0) q2 = issue_v;
+      else q3 = issue_v;
+      // starting the last fixed token, or a pool token: request the one after it
+      if (issue_v + 1 >= v_hi && pool_lo < n_vis32 && !pref) request_pool();
+    }
   };
   auto issue_one = [&](int slot) {
     const int e0 = issue_chunk * kChunkElems;
@@ -270,22 +317,16 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     advance_issue();
   }
   bool timed_out = false;
-  bool waited = false;  // the validation kernel (which zeroes img_sums) is known to be done
   // per lane: even and odd elements accumulate separately (one paired FMA each)
   float2 dot2 = make_float2(0.f, 0.f), na2 = dot2, nb2 = dot2;
   int slot_take = 0;
-  int32_t take_p = p_lo;
-  int32_t take_u = first_u;
-  int take_chunk = first_c;
+  int take_chunk = 0;
   int take_img = 0;
   int run_img = -1;     // image of the current run of rows (lane 0's view)
   int64_t run_sum = 0;  // its fixed-point sum so far
   auto add_to_image = [&](int img, int64_t v) {
     if (img_sums == nullptr) return;
-    if (!waited) {
-      pdl_wait();
-      waited = true;
-    }
+    wait_prep();
     if (lane == 0) atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + img), static_cast<unsigned long long>(v));
   };
   while (in_flight > 0) {
@@ -317,7 +358,14 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     }
     __syncwarp();
     --in_flight;
-    const bool token_end = take_chunk == n_chunks - 1 || take_p == p_hi - 1;
+    const bool row_done = take_chunk == n_chunks - 1;
+    const int32_t take_v = q0;
+    if (row_done) {  // the token leaves the queue before the refill may add one
+      q0 = q1;
+      q1 = q2;
+      q2 = q3;
+      q3 = -1;
+    }
     // refill the slot just consumed
     if (issue_valid()) {
       issue_one(slot_take);
@@ -325,35 +373,24 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
       ++in_flight;
     }
     slot_take = (slot_take + 1) % kSlots;
-    if (token_end) {
+    if (row_done) {
       const float d = warp_sum(dot2.x + dot2.y), x = warp_sum(na2.x + na2.y), y = warp_sum(nb2.x + nb2.y);
       dot2 = na2 = nb2 = make_float2(0.f, 0.f);
-      const int64_t t = map.position(v_lo + take_u, take_img);
-      const bool whole = take_chunk == n_chunks - 1 && (take_u != first_u || first_c == 0);
-      if (whole) {
-        const bool inside = t >= 0 && t < T;
-        const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
-        const float I = 1.f - d / den;
-        if (lane == 0 && inside) scores[t] = I;
-        // run-length accumulation of the per-image sums (take_img is uniform over the warp)
-        if (take_img != run_img) {
-          if (run_img >= 0) add_to_image(run_img, run_sum);
-          run_img = take_img;
-          run_sum = 0;
-        }
-        if (inside) run_sum += fixed_point_score(I);
-      } else if (lane == 0) {
-        // a piece of a token shared with other warps: the first or the last of this warp's
-        const int k = take_u == first_u ? 0 : 1;
-        s_part[warp][k][0] = d;
-        s_part[warp][k][1] = x;
-        s_part[warp][k][2] = y;
+      const int64_t t = map.position(take_v, take_img);
+      const bool inside = t >= 0 && t < T;
+      const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
+      const float I = 1.f - d / den;
+      if (lane == 0 && inside) scores[t] = I;
+      // run-length accumulation of the per-image sums (take_img is uniform over the warp)
+      if (take_img != run_img) {
+        if (run_img >= 0) add_to_image(run_img, run_sum);
+        run_img = take_img;
+        run_sum = 0;
       }
-    }
-    ++take_p;
-    if (++take_chunk == n_chunks) {
+      if (inside) run_sum += fixed_point_score(I);
       take_chunk = 0;
-      ++take_u;
+    } else {
+      ++take_chunk;
     }
   }
   if (!timed_out && run_img >= 0) add_to_image(run_img, run_sum);
@@ -369,38 +406,6 @@ k_score_hvar(const __nv_bfloat16* __restrict__ h_cur, int64_t cur_stride, const 
     }
     pdl_wait();  // the validation kernel resets the status word: record after it
     if (lane == 0) record_error(st, AVTP_ERR_TIMEOUT, static_cast<int32_t>(blockIdx.x));
-  }
-
-  // ---- tokens shared by several warps, finished by the warp that holds the last piece
-  __syncthreads();
-  if (p_lo < p_hi && first_c != 0 && p_hi >= (first_u + 1) * n_chunks && lane == 0) {
-    // the warps that hold pieces of token first_u, from the one with its first piece
-    const int32_t p0 = first_u * n_chunks;
-    const int32_t big = (pc_q + 1) * pc_r;  // pieces held by the warps with one extra piece
-    const int w0 = p0 < big ? p0 / (pc_q + 1) : pc_r + (p0 - big) / pc_q;
-    float d = 0.f, x = 0.f, y = 0.f;
-    for (int w = w0; w <= warp; ++w) {
-      const int32_t wp = w * pc_q + min(w, pc_r);  // first piece of warp w
-      const int k = (w == warp || wp / n_chunks == first_u) ? 0 : 1;
-      d += s_part[w][k][0];
-      x += s_part[w][k][1];
-      y += s_part[w][k][2];
-    }
-    int img = 0;
-    const int64_t t = map.position(v_lo + first_u, img);
-    if (t >= 0 && t < T) {
-      const float den = fmaxf(sqrtf(x), 1e-8f) * fmaxf(sqrtf(y), 1e-8f);
-      const float I = 1.f - d / den;
-      scores[t] = I;
-      if (img_sums != nullptr) {
-        if (!waited) {
-          pdl_wait();
-          waited = true;
-        }
-        atomicAdd(reinterpret_cast<unsigned long long*>(img_sums + img),
-                  static_cast<unsigned long long>(fixed_point_score(I)));
-      }
-    }
   }
   pdl_wait();  // completion of this grid implies completion of the one before it
 #ifdef AVTP_TIMELINE
