@@ -55,6 +55,9 @@ avtp_status_t check_score_args(const avtp_layout_t* L, const avtp_score_args_t* 
     if (a->path != AVTP_PATH_AUTO && a->path != AVTP_PATH_TENSOR && a->path != AVTP_PATH_CUDA)
       return AVTP_ERR_INVALID_ARG;
     if (a->path == AVTP_PATH_TENSOR && a->query_set == AVTP_QUERIES_LAST) return AVTP_ERR_UNSUPPORTED;
+    if (attn_uses_cuda_cores(*L, *a) &&
+        narrow_plan(*L, *a, attn_plan(*L, *a).max_text).z_elems > kNarrowMaxLogitBytes / 4)
+      return AVTP_ERR_RANGE;
     return AVTP_OK;
   }
   return AVTP_ERR_INVALID_ARG;
@@ -148,8 +151,8 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
     if (attn_uses_cuda_cores(L, *sa)) {
       const NarrowPlan np = narrow_plan(L, *sa, a.max_text);
       const size_t nrows = static_cast<size_t>(np.rows);
-      p.lse_rows = take(Hkv * nrows * 4 + 4);
-      p.p1_part = (sa->lse == nullptr) ? take(Hkv * static_cast<size_t>(np.NS) * nrows * 8 + 8) : 0;
+      p.p1_part = (sa->lse == nullptr) ? take(static_cast<size_t>(np.NS) * nrows * 8 + 8) : 0;
+      p.zbuf = take(static_cast<size_t>(np.z_elems) * 4 + 4);
     } else {
       p.qt = take(Hkv * rows * static_cast<size_t>(sa->head_dim) * 2 + 16);
       p.lse_rows = (sa->lse != nullptr) ? take(Hkv * rows * 4 + 4) : 0;

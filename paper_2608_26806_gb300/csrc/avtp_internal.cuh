@@ -138,6 +138,7 @@ struct WsPlan {
   size_t lse_rows;    // float [Hkv, rows]: log2-domain LSE of every row (supplied LSE only)
   size_t p1_part;     // float2 [Hkv * n_blocks_max][256][kAttnMaxChunks]: per-CTA (max, sum) of every row
   size_t mass;        // uint64 [n_ktiles_max][128]: fixed-point probability mass of every visual key, by key tile
+  size_t zbuf;        // float: the CUDA-core path's logits, request by request [its rows][its tokens]
   size_t total;
 };
 
@@ -153,20 +154,23 @@ struct AttnPlan {
 };
 AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa);
 
-// The CUDA-core path of criterion B (k_score_narrow.cu): rows per KV group are the
-// batch's queries (at most) times G; pass 1 splits every (request, KV group) into NS key
-// ranges.
+// The CUDA-core path of criterion B (k_score_narrow.cu): rows are the batch's queries (at
+// most) times Hq; the logits pass splits every (request, KV group) into NS key ranges and
+// keeps every logit, Hq x queries x tokens of each request, at most kNarrowMaxLogitBytes.
 constexpr int kNarrowMaxSplits = 64;
+constexpr int64_t kNarrowMaxLogitBytes = int64_t(1) << 30;
 // AVTP_PATH_AUTO takes the CUDA cores for AVTP_QUERIES_LAST, and for AVTP_QUERIES_TEXT
 // only when the batch has at most this many rows per KV group (judged from its text-token
-// bound). Measured on Qwen3-shaped heads the tensor-core path was faster from 4 rows per
-// group up (flat near 33 us to 512 rows, the CUDA cores growing with the rows), so the
-// text query set keeps to the tensor cores.
-constexpr int64_t kNarrowAutoRows = 0;
+// bound). Measured on a request of four 640-token images and Qwen3-shaped heads (8 KV
+// groups of 4 heads, d = 128), score call event-timed: 33.0 us on the CUDA cores against
+// 33.4 us on tcgen05 at 4 rows per group (one text token), 35.4 against 33.4 at 8, and
+// the CUDA cores growing with the rows beyond (tcgen05 stays near 33 us up to 256 rows).
+constexpr int64_t kNarrowAutoRows = 4;
 struct NarrowPlan {
   int G;
-  int64_t rows;
+  int64_t rows;     // global rows (query ordinal x Hq + head), at most
   int NS;
+  int64_t z_elems;  // logits, at most
 };
 NarrowPlan narrow_plan(const avtp_layout_t& L, const avtp_score_args_t& sa, int64_t max_text);
 bool attn_uses_cuda_cores(const avtp_layout_t& L, const avtp_score_args_t& sa);

@@ -5,30 +5,40 @@
 //   s_t = 1/(Hq*|Q_r|) * sum_h sum_{q in Q_r, pos q >= pos t} exp2(z2(h,q,t) - lse2(h,q)),
 //   z2 = softmax_scale * log2(e) * q_h . k_{g(h)},  lse2 = log2 sum_{visible keys} exp2(z2).
 //
-// Rows: for KV group g, row o*G + j is query ordinal o with head g*G + j; the ordinal
-// is the request index for the last-token set and the text ordinal for the text set.
+// Rows: the global row of query ordinal o and head h is o*Hq + h; the ordinal is the
+// request index for the last-token set and the text ordinal for the text set.
 //
-// k_narrow_lse (pass 1): one CTA per (request, KV group, key split); a thread owns one
-// key at a time (its d elements read as 16-byte vectors; the request's rows, in blocks
-// of kRB, sit in shared memory as fp32) and keeps an online (max, sum) per row of the
-// block; the CTA leaves one partial per (row, split).
-// k_narrow_merge: merges the splits into lse2 per row (a warp per row), or converts a
-// supplied natural-log LSE, and clears the per-key mass accumulator.
-// k_narrow_mass (pass 2): one CTA per (key tile of an image, KV group), a thread per key:
-// the key's probability under every row whose query follows it, summed and added to the
-// 64-bit fixed-point accumulator that k_attn_finalize turns into scores.
-// The work per key is d FMAs per row: memory-bound for a few rows, compute-bound beyond
-// a few dozen, where the tensor-core path takes over (avtp_api.cu picks the path).
+// The keys are read once. k_narrow_logits: one CTA per (request, KV group, key split);
+// each warp takes 16-key tiles and multiplies them by the group's rows, 8 at a time, with
+// warp-level mma.sync (m16n8k16, bf16 in, fp32 accumulate): a tile too narrow for a
+// tcgen05 MMA still gets the tensor cores, and all of a tile's key loads are in flight
+// before its first MMA. (Holding the rows in shared memory and a key per thread with
+// fp32 FMAs spent 29 % of its issue slots on shared-memory loads and ran 24 us for the
+// 20 MB of keys of a 9856-token request.) It
+// writes every logit z2 of the request's rows to a buffer (rows x keys of the request,
+// fp32: 1.3 MB for one query token over 9856 keys and 32 heads) and, unless the LSE is
+// supplied, one online (max, sum) partial per (row, split). k_narrow_mass: each CTA
+// merges the partials of its request's rows into lse2 (one round of loads), then a thread
+// per visual key sums exp2(z2 - lse2) over the rows whose query follows it, reading the
+// logits back (coalesced: consecutive keys of a row are consecutive), and stores the
+// key's fixed-point mass for k_attn_finalize. No key is read twice and no mass needs
+// atomics.
+// The work per key is d multiply-adds per row; the logits buffer grows with the rows, and
+// for wide query sets the tcgen05 path takes over (avtp_api.cu picks the path).
 #include "avtp_internal.cuh"
 
 namespace avtp {
 namespace {
 
-constexpr int kNT = 128;      // threads per CTA; pass 2 handles a 128-key tile
-constexpr int kRB = 8;        // rows held in registers at a time
+constexpr int kNT = 128;      // threads per CTA; k_narrow_mass handles a 128-key tile
+constexpr int kRB = 8;        // rows per MMA tile (the N of m16n8k16)
+constexpr int kMassRows = 256;  // rows whose lse2 and query position k_narrow_mass stages at a time
+constexpr int kMassBatch = 32;  // logits a thread of k_narrow_mass loads at once
+constexpr int kSplitLanes = 4;  // lanes that merge one row's split partials in k_narrow_mass
+static_assert(kNarrowMaxSplits % kSplitLanes == 0 && 32 % kSplitLanes == 0, "split lanes");
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr unsigned long long kMassNotFinite = 1ull << 63;
-static_assert(kNT == kAttnTileM, "pass 2 works on the key tiles of the tensor-core path");
+static_assert(kNT == kAttnTileM, "k_narrow_mass works on the key tiles of the tensor-core path");
 
 struct NarrowArgs {
   const __nv_bfloat16* q;
@@ -48,12 +58,10 @@ struct NarrowArgs {
   int Hq, Hkv, G, d;
   float c2;         // softmax_scale * log2(e)
   int last;         // 1: the request's last token is the only query
-  int NS;           // key splits per (request, KV group) in pass 1
-  int64_t rows;     // rows per KV group: queries of the batch (at most) times G
-  float2* part;     // [Hkv][NS][rows]: pass-1 (max2, sum) per split
-  float* lse2;      // [Hkv][rows]
+  int NS;           // key splits per (request, KV group) in k_narrow_logits
+  float* z;         // logits, request by request: [rows of r][T_r]
+  float2* part;     // [global rows][NS]: (max2, sum) per split
   unsigned long long* mass;  // [key tiles][128], 2^-kAttnMassFracBits
-  int64_t n_mass;
   const float* lse;          // supplied natural-log LSE [Hq][lse_stride], or null
   int64_t lse_stride;
   DevStatus* st;
@@ -74,6 +82,15 @@ __device__ __forceinline__ int64_t query_pos(const NarrowArgs& a, int r, int64_t
   return a.last ? static_cast<int64_t>(a.cu[r + 1]) - 1 : static_cast<int64_t>(a.text_idx[o]);
 }
 
+// Offset of request r's logits: Hq * sum over earlier requests of queries x tokens.
+__device__ __forceinline__ int64_t logits_base(const NarrowArgs& a, int r) {
+  if (a.last) return static_cast<int64_t>(a.Hq) * a.cu[r];
+  int64_t s = 0;
+  for (int u = 0; u < r; ++u)
+    s += static_cast<int64_t>(a.text_cu[u + 1] - a.text_cu[u]) * (a.cu[u + 1] - a.cu[u]);
+  return s * a.Hq;
+}
+
 // (m, s) <- the online merge of (m, s) and (m2, s2), with -inf for "no key yet".
 __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2) {
   const float M = fmaxf(m, m2);
@@ -82,102 +99,31 @@ __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2)
   m = M;
 }
 
-// A block of up to kRB rows of request r, group g, starting at row rb: the queries as
-// fp32 in shared memory, their positions, and (pass 2) their lse2.
-struct RowBlock {
-  float* qs;       // [kRB][d]
-  int64_t* qpos;   // [kRB]; -1 for rows past the request's
-  float* l2;       // [kRB]
-};
-
-__device__ void load_rows(const NarrowArgs& a, int r, int g, int64_t o0, int n_rows, int rb, const RowBlock& B,
-                          bool want_lse) {
-  const int d = a.d;
-  for (int e = threadIdx.x; e < kRB * d / 8; e += kNT) {
-    const int rr = e / (d / 8), c = e % (d / 8);
-    const int row = rb + rr;
-    float* dst = B.qs + rr * d + c * 8;
-    if (row < n_rows) {
-      const int64_t o = o0 + row / a.G;
-      const int h = g * a.G + row % a.G;
-      const int64_t pos = query_pos(a, r, o);
-      const uint4 v = *reinterpret_cast<const uint4*>(a.q + pos * a.q_stride + static_cast<int64_t>(h) * d + c * 8);
-      const uint32_t* w = reinterpret_cast<const uint32_t*>(&v);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        dst[2 * u] = __uint_as_float(w[u] << 16);
-        dst[2 * u + 1] = __uint_as_float(w[u] & 0xffff0000u);
-      }
-    } else {
-#pragma unroll
-      for (int u = 0; u < 8; ++u) dst[u] = 0.f;
-    }
-  }
-  for (int rr = threadIdx.x; rr < kRB; rr += kNT) {
-    const int row = rb + rr;
-    if (row < n_rows) {
-      const int64_t o = o0 + row / a.G;
-      B.qpos[rr] = query_pos(a, r, o);
-      if (want_lse) B.l2[rr] = a.lse2[static_cast<int64_t>(g) * a.rows + o * a.G + row % a.G];
-    } else {
-      B.qpos[rr] = -1;
-      if (want_lse) B.l2[rr] = 0.f;
-    }
-  }
+// ---------------------------------------------------------------- the logits (and lse2)
+// D = q . k for a 16-key x 8-row tile on the tensor cores (mma.sync m16n8k16, bf16 in,
+// fp32 accumulate): the keys are the 16-row A operand, the 8 rows of a block the B
+// operand. Lane l holds keys l/4 and l/4 + 8 of the tile and rows 2(l%4), 2(l%4) + 1.
+__device__ __forceinline__ void mma_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                          uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// z[rr] = c2 * q_rr . k for the kRB rows of the block and key t of group g. All of the
-// key's D/8 16-byte loads are issued before the first FMA: a key costs one memory round
-// trip, not D/8 of them.
-template <int D>
-__device__ __forceinline__ void block_logits(const NarrowArgs& a, int64_t t, int g, const float* qs, float* z) {
-  const uint4* kp = reinterpret_cast<const uint4*>(a.k + t * a.k_stride + static_cast<int64_t>(g) * D);
-  uint4 kv[D / 8];
-#pragma unroll
-  for (int c = 0; c < D / 8; ++c) kv[c] = __ldg(kp + c);
-  float acc[kRB];
-#pragma unroll
-  for (int rr = 0; rr < kRB; ++rr) acc[rr] = 0.f;
-#pragma unroll
-  for (int c = 0; c < D / 8; ++c) {
-    const uint32_t* w = reinterpret_cast<const uint32_t*>(&kv[c]);
-    float kf[8];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      kf[2 * u] = __uint_as_float(w[u] << 16);
-      kf[2 * u + 1] = __uint_as_float(w[u] & 0xffff0000u);
-    }
-#pragma unroll
-    for (int rr = 0; rr < kRB; ++rr) {
-      const float4 q0 = *reinterpret_cast<const float4*>(qs + rr * D + c * 8);
-      const float4 q1 = *reinterpret_cast<const float4*>(qs + rr * D + c * 8 + 4);
-      float s = acc[rr];
-      s = fmaf(kf[0], q0.x, s);
-      s = fmaf(kf[1], q0.y, s);
-      s = fmaf(kf[2], q0.z, s);
-      s = fmaf(kf[3], q0.w, s);
-      s = fmaf(kf[4], q1.x, s);
-      s = fmaf(kf[5], q1.y, s);
-      s = fmaf(kf[6], q1.z, s);
-      s = fmaf(kf[7], q1.w, s);
-      acc[rr] = s;
-    }
-  }
-#pragma unroll
-  for (int rr = 0; rr < kRB; ++rr) z[rr] = acc[rr] * a.c2;
-}
-
-// ---------------------------------------------------------------- pass 1
 template <int D>
 __global__ void __launch_bounds__(kNT)
-k_narrow_lse(NarrowArgs a) {
-  extern __shared__ __align__(16) float nsm[];
-  __shared__ int64_t s_qpos[kRB];
+k_narrow_logits(NarrowArgs a) {
+  constexpr int KS = D / 16;  // k-steps
   __shared__ float s_m[kNT / 32][kRB], s_s[kNT / 32][kRB];
   pdl_wait();
   pdl_trigger();
   if (!a.st->layout_ok) return;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int kq = 2 * (lane & 3);  // this lane's column pair in a k-step
+  const int km = lane >> 2;       // this lane's keys in a tile: km and km + 8
+  const bool want_lse = a.lse == nullptr;
   const int64_t units = static_cast<int64_t>(a.R) * a.Hkv * a.NS;
   for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
     const int sp = static_cast<int>(u % a.NS);
@@ -187,43 +133,98 @@ k_narrow_lse(NarrowArgs a) {
     int nq;
     request_queries(a, r, &o0, &nq);
     const int n_rows = nq * a.G;
-    if (n_rows == 0) continue;
     const int64_t t_lo = a.cu[r], T_r = a.cu[r + 1] - a.cu[r];
     const int64_t ks = t_lo + T_r * sp / a.NS, ke = t_lo + T_r * (sp + 1) / a.NS;
+    const int64_t zb = logits_base(a, r);
     for (int rb = 0; rb < n_rows; rb += kRB) {
-      __syncthreads();  // the previous block's rows and reductions are no longer read
-      const RowBlock B{nsm, s_qpos, nullptr};
-      load_rows(a, r, g, o0, n_rows, rb, B, false);
-      __syncthreads();
-      float m[kRB], s[kRB];
+      // B operand: row rb + km of the block (the lane's row for the loads), as bf16 pairs
+      uint32_t bq[KS][2];
+      {
+        const int row = rb + km;
+        if (row < n_rows) {
+          const int64_t o = o0 + row / a.G;
+          const int h = g * a.G + row % a.G;
+          const __nv_bfloat16* qp = a.q + query_pos(a, r, o) * a.q_stride + static_cast<int64_t>(h) * D;
 #pragma unroll
-      for (int rr = 0; rr < kRB; ++rr) { m[rr] = -INFINITY; s[rr] = 0.f; }
-      for (int64_t t = ks + threadIdx.x; t < ke; t += kNT) {
-        float z[kRB];
-        block_logits<D>(a, t, g, nsm, z);
+          for (int kk = 0; kk < KS; ++kk) {
+            bq[kk][0] = *reinterpret_cast<const uint32_t*>(qp + kk * 16 + kq);
+            bq[kk][1] = *reinterpret_cast<const uint32_t*>(qp + kk * 16 + 8 + kq);
+          }
+        } else {
 #pragma unroll
-        for (int rr = 0; rr < kRB; ++rr) {
-          if (t > s_qpos[rr]) continue;  // after the query (or a row past the request's)
-          if (z[rr] > m[rr]) {
-            s[rr] = (m[rr] == -INFINITY ? 0.f : s[rr] * exp2f(m[rr] - z[rr])) + 1.f;
-            m[rr] = z[rr];
-          } else {
-            s[rr] += exp2f(z[rr] - m[rr]);
+          for (int kk = 0; kk < KS; ++kk) bq[kk][0] = bq[kk][1] = 0u;
+        }
+      }
+      // the lane's two rows of the C tile: where their logits go, their query positions
+      int64_t zrow[2], qp[2];
+      bool live[2];
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int row = rb + kq + j;
+        live[j] = row < n_rows;
+        const int64_t o_loc = row / a.G, h = g * a.G + row % a.G;
+        zrow[j] = zb + (o_loc * a.Hq + h) * T_r - t_lo;
+        qp[j] = live[j] ? query_pos(a, r, o0 + o_loc) : -1;
+      }
+      float m[2] = {-INFINITY, -INFINITY}, sm[2] = {0.f, 0.f};
+      // two tiles per step: every A load of both in flight before the first MMA
+      for (int64_t t0 = ks + warp * 32; t0 < ke; t0 += (kNT / 32) * 32) {
+        uint32_t ak[2][KS][4];
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const int64_t tA = t0 + 16 * h2 + km, tB = tA + 8;
+          const __nv_bfloat16* kA = a.k + tA * a.k_stride + static_cast<int64_t>(g) * D;
+          const __nv_bfloat16* kB = a.k + tB * a.k_stride + static_cast<int64_t>(g) * D;
+#pragma unroll
+          for (int kk = 0; kk < KS; ++kk) {
+            ak[h2][kk][0] = tA < ke ? __ldg(reinterpret_cast<const unsigned int*>(kA + kk * 16 + kq)) : 0u;
+            ak[h2][kk][1] = tB < ke ? __ldg(reinterpret_cast<const unsigned int*>(kB + kk * 16 + kq)) : 0u;
+            ak[h2][kk][2] = tA < ke ? __ldg(reinterpret_cast<const unsigned int*>(kA + kk * 16 + 8 + kq)) : 0u;
+            ak[h2][kk][3] = tB < ke ? __ldg(reinterpret_cast<const unsigned int*>(kB + kk * 16 + 8 + kq)) : 0u;
+          }
+        }
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const int64_t tA = t0 + 16 * h2 + km, tB = tA + 8;
+          float c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int kk = 0; kk < KS; ++kk)
+            mma_16816(c, ak[h2][kk][0], ak[h2][kk][1], ak[h2][kk][2], ak[h2][kk][3], bq[kk][0], bq[kk][1]);
+          // c[0], c[1]: key tA, rows kq, kq + 1; c[2], c[3]: key tB, the same rows
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int j = e & 1;
+            const int64_t t = e < 2 ? tA : tB;
+            if (!live[j] || t >= ke) continue;
+            const float z = c[e] * a.c2;
+            a.z[zrow[j] + t] = z;
+            if (!want_lse || t > qp[j]) continue;  // the key follows the query
+            if (z > m[j]) {
+              sm[j] = (m[j] == -INFINITY ? 0.f : sm[j] * exp2f(m[j] - z)) + 1.f;
+              m[j] = z;
+            } else {
+              sm[j] += exp2f(z - m[j]);
+            }
           }
         }
       }
-      // reduce over the CTA: warps by shuffles, then across the warps
+      if (!want_lse) continue;
+      // reduce over the lanes that hold the same rows (same l % 4), then over the warps
 #pragma unroll
-      for (int rr = 0; rr < kRB; ++rr) {
+      for (int j = 0; j < 2; ++j) {
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-          const float m2 = __shfl_xor_sync(0xffffffffu, m[rr], off);
-          const float s2 = __shfl_xor_sync(0xffffffffu, s[rr], off);
-          merge_ms(m[rr], s[rr], m2, s2);
+        for (int off = 4; off < 32; off <<= 1) {
+          const float m2 = __shfl_xor_sync(0xffffffffu, m[j], off);
+          const float s2 = __shfl_xor_sync(0xffffffffu, sm[j], off);
+          merge_ms(m[j], sm[j], m2, s2);
         }
-        if (lane == 0) {
-          s_m[warp][rr] = m[rr];
-          s_s[warp][rr] = s[rr];
+      }
+      __syncthreads();  // s_m / s_s of the previous block are no longer read
+      if (lane < 4) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          s_m[warp][kq + j] = m[j];
+          s_s[warp][kq + j] = sm[j];
         }
       }
       __syncthreads();
@@ -232,108 +233,110 @@ k_narrow_lse(NarrowArgs a) {
         float M = s_m[0][rr], Sm = s_s[0][rr];
         for (int w = 1; w < kNT / 32; ++w) merge_ms(M, Sm, s_m[w][rr], s_s[w][rr]);
         const int row = rb + rr;
-        const int64_t ro = (o0 + row / a.G) * a.G + row % a.G;
-        a.part[(static_cast<int64_t>(g) * a.NS + sp) * a.rows + ro] = make_float2(M, Sm);
+        const int64_t gr = (o0 + row / a.G) * a.Hq + g * a.G + row % a.G;
+        a.part[gr * a.NS + sp] = make_float2(M, Sm);
       }
     }
   }
 }
 
-// ---------------------------------------------------------------- merge
-__global__ void __launch_bounds__(256)
-k_narrow_merge(NarrowArgs a, int64_t n_rows_used) {
-  pdl_wait();
-  pdl_trigger();
-  if (!a.st->layout_ok) return;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  const int64_t tid0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  for (int64_t u = tid0; u < a.n_mass; u += stride) a.mass[u] = 0ull;
-  // rows in use: R * G (last-token set) or (text tokens of the batch) * G
-  const int64_t n_text = a.last ? 0 : a.text_cu[a.R];
-  // a warp per row: the lanes merge the splits, then a shuffle tree
-  const int lane = threadIdx.x & 31;
-  const int64_t wstride = stride >> 5;
-  for (int64_t u = tid0 >> 5; u < static_cast<int64_t>(a.Hkv) * n_rows_used; u += wstride) {
-    const int g = static_cast<int>(u / n_rows_used);
-    const int64_t ro = u % n_rows_used;
-    const int64_t o = ro / a.G;
-    if (!a.last && o >= n_text) continue;                        // no such text token in this batch
-    if (a.last && a.cu[o + 1] == a.cu[o]) continue;              // a request without tokens has no query
-    float l2;
-    if (a.lse != nullptr) {
-      const int h = g * a.G + static_cast<int>(ro % a.G);
-      const int r = a.last ? static_cast<int>(o) : upper_index(a.text_cu, a.R, o);
-      l2 = a.lse[static_cast<int64_t>(h) * a.lse_stride + query_pos(a, r, o)] * kLog2e;
-    } else {
-      float M = -INFINITY, Sm = 0.f;
-      for (int sp = lane; sp < a.NS; sp += 32) {
-        const float2 p = a.part[(static_cast<int64_t>(g) * a.NS + sp) * a.rows + ro];
-        merge_ms(M, Sm, p.x, p.y);
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float m2 = __shfl_xor_sync(0xffffffffu, M, off);
-        const float s2 = __shfl_xor_sync(0xffffffffu, Sm, off);
-        merge_ms(M, Sm, m2, s2);
-      }
-      l2 = M + log2f(Sm);
-    }
-    if (lane == 0) a.lse2[static_cast<int64_t>(g) * a.rows + ro] = l2;
-  }
-}
-
-// ---------------------------------------------------------------- pass 2
-template <int D>
+// ---------------------------------------------------------------- the mass of every visual key
 __global__ void __launch_bounds__(kNT)
 k_narrow_mass(NarrowArgs a) {
-  extern __shared__ __align__(16) float nsm[];
-  __shared__ int64_t s_qpos[kRB];
-  __shared__ float s_l2[kRB];
+  __shared__ float s_l2[kMassRows];
+  __shared__ int64_t s_qpos[kMassRows];
   pdl_wait();
   pdl_trigger();
   if (!a.st->layout_ok) return;
   const int n_tiles = a.ktile_cu[a.NI];
-  const int64_t units = static_cast<int64_t>(n_tiles) * a.Hkv;
-  for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
-    const int g = static_cast<int>(u % a.Hkv);
-    const int tile = static_cast<int>(u / a.Hkv);
+  for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
     const int i = a.ktile_img[tile];
     const int r = a.img_req[i];
     int64_t o0;
     int nq;
     request_queries(a, r, &o0, &nq);
-    const int n_rows = nq * a.G;
+    const int64_t n_rows = static_cast<int64_t>(nq) * a.Hq;
     const int ok = (tile - a.ktile_cu[i]) * kNT + static_cast<int>(threadIdx.x);  // key within the image
     const bool has = ok < a.iln[i];
-    const int64_t t = static_cast<int64_t>(a.cu[r]) + a.ist[i] + ok;
+    const int64_t t_lo = a.cu[r], T_r = a.cu[r + 1] - a.cu[r];
+    const int64_t t = t_lo + a.ist[i] + ok;
+    const float* zr = a.z + logits_base(a, r) + (t - t_lo);
     float mass = 0.f;
-    for (int rb = 0; rb < n_rows; rb += kRB) {
+    for (int64_t rb = 0; rb < n_rows; rb += kMassRows) {
+      const int nr = static_cast<int>(n_rows - rb < kMassRows ? n_rows - rb : kMassRows);
+      // the first kMassBatch logits of the key, loaded while the rows are staged
+      float zz0[kMassBatch];
+#pragma unroll
+      for (int j = 0; j < kMassBatch; ++j) zz0[j] = has && j < nr ? __ldcg(zr + (rb + j) * T_r) : 0.f;
       __syncthreads();
-      const RowBlock B{nsm, s_qpos, s_l2};
-      load_rows(a, r, g, o0, n_rows, rb, B, true);
+      for (int rr = threadIdx.x; rr < kMassRows; rr += kNT) {
+        const int64_t row = rb + rr;
+        if (row < n_rows) {
+          const int64_t o = o0 + row / a.Hq;
+          const int h = static_cast<int>(row % a.Hq);
+          const int64_t pos = query_pos(a, r, o);
+          s_qpos[rr] = pos;
+          if (a.lse != nullptr) s_l2[rr] = a.lse[static_cast<int64_t>(h) * a.lse_stride + pos] * kLog2e;
+        } else {
+          s_qpos[rr] = -1;
+          s_l2[rr] = 0.f;
+        }
+      }
+      if (a.lse == nullptr) {
+        // lse2 of the staged rows from the logits pass's (max, sum) partials: kSplitLanes
+        // lanes per row, every partial load of a lane issued before it merges
+        const int sub = threadIdx.x % kSplitLanes;
+        for (int rr0 = static_cast<int>(threadIdx.x) / kSplitLanes; rr0 < kMassRows; rr0 += kNT / kSplitLanes) {
+          float M = -INFINITY, Sm = 0.f;
+          if (rr0 < nr) {
+            const float2* pp = a.part + ((o0 * a.Hq) + rb + rr0) * a.NS;
+            float2 pv[kNarrowMaxSplits / kSplitLanes];
+#pragma unroll
+            for (int q = 0; q < kNarrowMaxSplits / kSplitLanes; ++q) {
+              const int sp = sub + q * kSplitLanes;
+              pv[q] = sp < a.NS ? __ldcg(pp + sp) : make_float2(-INFINITY, 0.f);
+            }
+#pragma unroll
+            for (int q = 0; q < kNarrowMaxSplits / kSplitLanes; ++q) merge_ms(M, Sm, pv[q].x, pv[q].y);
+          }
+#pragma unroll
+          for (int off = kSplitLanes / 2; off > 0; off >>= 1) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, M, off);
+            const float s2 = __shfl_xor_sync(0xffffffffu, Sm, off);
+            merge_ms(M, Sm, m2, s2);
+          }
+          if (sub == 0 && rr0 < nr) s_l2[rr0] = M + log2f(Sm);
+        }
+      }
       __syncthreads();
       if (!has) continue;
-      float z[kRB];
-      block_logits<D>(a, t, g, nsm, z);
 #pragma unroll
-      for (int rr = 0; rr < kRB; ++rr)
-        if (t <= s_qpos[rr]) mass += exp2f(z[rr] - s_l2[rr]);
-    }
-    if (has && n_rows > 0) {
-      unsigned long long* dst = a.mass + static_cast<int64_t>(tile) * kNT + threadIdx.x;
-      if (mass <= 512.f) {  // at most one per row
-        atomicAdd(dst, static_cast<unsigned long long>(__float2ll_rn(mass * static_cast<float>(1ull << kAttnMassFracBits))));
-      } else {
-        atomicOr(dst, kMassNotFinite);  // NaN or inf inputs: the key scores NaN
+      for (int j = 0; j < kMassBatch; ++j)
+        if (j < nr && t <= s_qpos[j]) mass += exp2f(zz0[j] - s_l2[j]);
+      // the rest, kMassBatch logits in flight before the first exp2
+      for (int r0 = kMassBatch; r0 < nr; r0 += kMassBatch) {
+        float zz[kMassBatch];
+#pragma unroll
+        for (int j = 0; j < kMassBatch; ++j) zz[j] = r0 + j < nr ? __ldcg(zr + (rb + r0 + j) * T_r) : 0.f;
+#pragma unroll
+        for (int j = 0; j < kMassBatch; ++j)
+          if (r0 + j < nr && t <= s_qpos[r0 + j]) mass += exp2f(zz[j] - s_l2[r0 + j]);
       }
     }
+    unsigned long long m = 0;
+    if (has && n_rows > 0)
+      m = mass <= 4194304.f ? static_cast<unsigned long long>(__float2ll_rn(mass * static_cast<float>(1ull << kAttnMassFracBits)))
+                            : kMassNotFinite;  // NaN or inf inputs: the key scores NaN
+    a.mass[static_cast<int64_t>(tile) * kNT + threadIdx.x] = m;
   }
 }
 
+// Key splits per (request, KV group): about two keys per thread of a unit, on average
+// over the requests.
 int narrow_splits(const avtp_layout_t& L, int Hkv) {
-  const int64_t want = 4ll * device_sm_count();
-  const int64_t per = static_cast<int64_t>(L.n_requests) * Hkv;
-  int64_t ns = (want + per - 1) / per;
+  (void)Hkv;
+  const int64_t per_request = L.n_tokens / (L.n_requests > 0 ? L.n_requests : 1);
+  const int64_t ns = (per_request + 2 * kNT - 1) / (2 * kNT);
   return static_cast<int>(ns < 1 ? 1 : (ns > kNarrowMaxSplits ? kNarrowMaxSplits : ns));
 }
 
@@ -342,8 +345,15 @@ int narrow_splits(const avtp_layout_t& L, int Hkv) {
 NarrowPlan narrow_plan(const avtp_layout_t& L, const avtp_score_args_t& sa, int64_t max_text) {
   NarrowPlan p;
   p.G = sa.n_q_heads / sa.n_kv_heads;
-  p.rows = (sa.query_set == AVTP_QUERIES_LAST ? static_cast<int64_t>(L.n_requests) : max_text) * p.G;
+  const int64_t n_q = sa.query_set == AVTP_QUERIES_LAST ? static_cast<int64_t>(L.n_requests) : max_text;
+  p.rows = n_q * sa.n_q_heads;
   p.NS = narrow_splits(L, sa.n_kv_heads);
+  // logits: Hq x queries x tokens of each request, at most Hq x n_q x T (the last-token set:
+  // Hq x T exactly)
+  p.z_elems = sa.query_set == AVTP_QUERIES_LAST ? static_cast<int64_t>(sa.n_q_heads) * L.n_tokens
+                                                : (n_q > 0 && L.n_tokens > INT64_MAX / 4 / n_q / sa.n_q_heads
+                                                       ? INT64_MAX / 4
+                                                       : p.rows * L.n_tokens);
   return p;
 }
 
@@ -373,34 +383,21 @@ cudaError_t launch_score_narrow(const avtp_layout_t& L, const avtp_score_args_t&
   a.c2 = sa.softmax_scale * kLog2e;
   a.last = sa.query_set == AVTP_QUERIES_LAST ? 1 : 0;
   a.NS = np.NS;
-  a.rows = np.rows;
+  a.z = ws_at<float>(ws, p.zbuf);
   a.part = ws_at<float2>(ws, p.p1_part);
-  a.lse2 = ws_at<float>(ws, p.lse_rows);
+  a.st = ws_at<DevStatus>(ws, p.status);
   a.mass = ws_at<unsigned long long>(ws, p.mass);
-  a.n_mass = plan.n_ktiles_max * kAttnTileM;
   a.lse = sa.lse;
   a.lse_stride = sa.lse_stride;
-  a.st = ws_at<DevStatus>(ws, p.status);
-  const size_t qsm = static_cast<size_t>(kRB) * sa.head_dim * sizeof(float);
   const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
-  if (sa.lse == nullptr) {
-    const int64_t units = static_cast<int64_t>(L.n_requests) * a.Hkv * a.NS;
-    const int grid = static_cast<int>(units < cap ? units : cap);
-    cudaError_t e = sa.head_dim == 64 ? launch_kernel(k_narrow_lse<64>, dim3(grid), dim3(kNT), qsm, s, true, a)
-                                      : launch_kernel(k_narrow_lse<128>, dim3(grid), dim3(kNT), qsm, s, true, a);
-    if (e != cudaSuccess) return e;
-  }
-  {
-    const int64_t work = (a.n_mass > 32 * a.Hkv * a.rows ? a.n_mass : 32 * a.Hkv * a.rows);
-    const int64_t want = (work + 255) / 256;
-    const int grid = static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
-    cudaError_t e = launch_kernel(k_narrow_merge, dim3(grid), dim3(256), 0, s, /*pdl=*/true, a, a.rows);
-    if (e != cudaSuccess) return e;
-  }
-  const int64_t units2 = plan.n_ktiles_max * a.Hkv;
+  const int64_t units = static_cast<int64_t>(L.n_requests) * a.Hkv * a.NS;
+  const int grid = static_cast<int>(units < cap ? units : cap);
+  cudaError_t e = sa.head_dim == 64 ? launch_kernel(k_narrow_logits<64>, dim3(grid), dim3(kNT), 0, s, true, a)
+                                    : launch_kernel(k_narrow_logits<128>, dim3(grid), dim3(kNT), 0, s, true, a);
+  if (e != cudaSuccess) return e;
+  const int64_t units2 = plan.n_ktiles_max;
   const int grid2 = static_cast<int>(units2 < 1 ? 1 : (units2 < cap ? units2 : cap));
-  cudaError_t e = sa.head_dim == 64 ? launch_kernel(k_narrow_mass<64>, dim3(grid2), dim3(kNT), qsm, s, true, a)
-                                    : launch_kernel(k_narrow_mass<128>, dim3(grid2), dim3(kNT), qsm, s, true, a);
+  e = launch_kernel(k_narrow_mass, dim3(grid2), dim3(kNT), 0, s, true, a);
   if (e != cudaSuccess) return e;
   return launch_attn_finalize(L, sa, scores, img_sums, ws, p, plan, s);
 }
