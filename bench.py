@@ -416,7 +416,7 @@ def run_ours(args, world, rank, local):
             "ms_per_step": round(ms3, 5), "steps": sec_last["steps"], "latency_us": sec_last["latency_us"],
             "steps_us": sec_last["steps_us"],
             "stage_roofline": stage_roofline(a3, ms3, hbm_s, bf16_s, peak_kind),
-            "score_roofline": {"bound": "hbm", "kernel": "score (lse + merge + mass + finalize)",
+            "score_roofline": {"bound": "hbm", "kernel": "score (logits + mass + finalize)",
                                "achieved": round(a3["score_bytes"] / (score_us * 1e-6) / 1e9, 1), "peak": hbm_s,
                                "unit": "GB/s",
                                "frac": round(a3["score_bytes"] / (score_us * 1e-6) / 1e9 / hbm_s, 4),
@@ -969,6 +969,109 @@ def run_reference(args, world, rank):
             "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+# ---------------------------------------------------------------- phase timeline (diagnostic)
+def run_timeline(args):
+    """The headline stage in the timeline build (-DAVTP_TIMELINE): per phase, the earliest
+    and latest global-timer stamp over the CTAs that reached it, in microseconds after the
+    validation kernel starts (median over the steps after a few warm-up calls), with L2
+    flushed before each call (the host enqueues the call while the flush runs) and, for
+    comparison, back to back. Not a bench line: the stamps add atomics to the kernels."""
+    os.environ["AVTP_TIMELINE"] = "1"
+    import torch
+
+    from paper_2608_26806_gb300 import avtp, build, synth
+
+    build.build(timeline=True)
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = synth.make_workload(args.config, parts=("A", "B", "pos") if args.criterion == "text_attention" else ("A", "pos"))
+    lay = wl.layout
+
+    def bf16(x):
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    L = avtp.Layout.from_host(lay.cu_seqlens, lay.img_cu, lay.img_start, lay.img_len, device=dev)
+    h_cur = bf16(wl.h_cur)
+    kr = torch.from_numpy(wl.keep_ratio).to(dev)
+    if args.criterion == "hidden_variation":
+        score = dict(h_cur=h_cur, h_prior=bf16(wl.h_prior))
+    else:
+        score = dict(q=bf16(wl.q), k=bf16(wl.k), softmax_scale=wl.softmax_scale)
+    call = avtp.PruneCall(L, args.criterion, keep_ratio=kr, keep_ratio_host=wl.keep_ratio, rows={"hidden": h_cur},
+                          planes={"pos": torch.from_numpy(wl.pos).to(dev)}, **score)
+    flush = L2Flush(dev)
+    out = {"config": args.config, "criterion": args.criterion, "unit": "us after the validation kernel starts"}
+    for mode in ("flushed", "back_to_back"):
+        runs = []
+        for i in range(max(args.steps, 8)):
+            torch.cuda.synchronize()
+            if mode == "flushed":
+                flush()
+            else:
+                call.run()
+            call.run()
+            torch.cuda.synchronize()
+            tl = avtp.timeline(call.buffers.workspace)
+            t0 = tl["prep_begin"][0]
+            runs.append({k: ((v[0] - t0) / 1e3, (v[1] - t0) / 1e3) for k, v in tl.items()})
+        keep = runs[3:]
+        out[mode] = {k: [round(float(np.median([r[k][j] for r in keep])), 2) for j in (0, 1)] for k in keep[-1]}
+    return out
+
+
+# ---------------------------------------------------------------- path crossover (diagnostic)
+def run_crossover(args):
+    """Criterion-B scoring on both paths as the query set widens: one request of four
+    640-token images followed by n text tokens, Qwen3-shaped heads (32 query heads, 8 KV
+    groups, d = 128), rows per KV group = 4n. Each avtp_score call is event-timed with L2
+    flushed before it (the host enqueues the call while the flush runs); the median of 30
+    calls per point. Not a bench line."""
+    import torch
+
+    from paper_2608_26806_gb300 import avtp, synth
+
+    import __graft_entry__
+
+    __graft_entry__.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    flush = L2Flush(dev)
+
+    def bf16(x):
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    out = []
+    texts = [args.crossover_text] if args.crossover_text else [1, 2, 4, 8, 16, 32, 64, 128]
+    paths = [args.crossover_path] if args.crossover_path else ["tensor", "cuda"]
+    for n_text in texts:
+        wl = synth.make_custom([[("i", 640)] * 4 + [("t", n_text)]], hidden=128, n_q_heads=32, n_kv_heads=8,
+                               head_dim=128, seed=3, parts=("B",))
+        lay = wl.layout
+        L = avtp.Layout.from_host(lay.cu_seqlens, lay.img_cu, lay.img_start, lay.img_len, device=dev)
+        st = dict(q=bf16(wl.q), k=bf16(wl.k), softmax_scale=wl.softmax_scale)
+        row = {"text_tokens": n_text, "rows_per_kv_group": 4 * n_text}
+        for path in paths:
+            ws = avtp.new_workspace(avtp.workspace_size(L, "text_attention", path=path, **st))
+            sc = torch.zeros(lay.n_tokens, device=dev)
+            sums = torch.zeros(lay.n_images, dtype=torch.int64, device=dev)
+            for _ in range(5):
+                avtp.score(L, "text_attention", path=path, scores=sc, img_sums=sums, workspace=ws, **st)
+            torch.cuda.synchronize()
+            ts = []
+            for _ in range(30):
+                flush()
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record()
+                avtp.score(L, "text_attention", path=path, scores=sc, img_sums=sums, workspace=ws, **st)
+                b.record()
+                torch.cuda.synchronize()
+                ts.append(a.elapsed_time(b) * 1e3)
+            row[path + "_us"] = round(float(np.median(ts)), 2)
+        out.append(row)
+    return {"crossover": out, "unit": "us per avtp_score call (event-timed, L2 flushed)"}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -985,9 +1088,21 @@ def main():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-secondary", action="store_true",
                     help="skip the attention-criterion object (timed after the headline criterion)")
+    ap.add_argument("--timeline", action="store_true",
+                    help="print the phase timeline of the headline stage (timeline build) instead of the bench line")
+    ap.add_argument("--crossover", action="store_true",
+                    help="print criterion-B scoring times of both paths as the query set widens, not the bench line")
+    ap.add_argument("--crossover-text", type=int, default=0, help="--crossover: only this many text tokens")
+    ap.add_argument("--crossover-path", default="", choices=["", "tensor", "cuda"], help="--crossover: only this path")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.timeline:
+        print(json.dumps(run_timeline(args)), flush=True)
+        return
+    if args.crossover:
+        print(json.dumps(run_crossover(args)), flush=True)
+        return
     world, rank, local = dist_env()
     if args.impl == "reference":
         line = run_reference(args, world, rank)
