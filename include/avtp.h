@@ -83,10 +83,14 @@ typedef enum {
 
 /* Where AVTP_CRIT_TEXT_ATTENTION computes its logits. */
 typedef enum {
-  AVTP_PATH_AUTO = 0,    /* tensor cores when the rows of a request and KV group (queries x
-                          * heads of the group) fill their 128-row tiles, CUDA cores otherwise */
-  AVTP_PATH_TENSOR = 1,  /* tcgen05 tensor cores (AVTP_QUERIES_TEXT only)                   */
-  AVTP_PATH_CUDA = 2     /* CUDA-core FMA, a thread per key                                  */
+  AVTP_PATH_AUTO = 0,    /* the narrow path for AVTP_QUERIES_LAST and for text query sets of
+                          * at most 4 rows per KV group (queries x heads of the group),
+                          * tcgen05 otherwise                                                  */
+  AVTP_PATH_TENSOR = 1,  /* tcgen05 tensor cores, 256-row blocks (AVTP_QUERIES_TEXT only)     */
+  AVTP_PATH_CUDA = 2     /* the narrow path: keys on the M side of warp-level mma.sync, every
+                          * key read once, every logit of the request's rows kept in the
+                          * workspace (Hq x queries x tokens x 4 bytes per request; more than
+                          * 1 GiB in all returns AVTP_ERR_RANGE)                               */
 } avtp_attn_path_t;
 
 typedef struct {
