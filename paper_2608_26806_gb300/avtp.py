@@ -133,7 +133,7 @@ def load() -> ctypes.CDLL:
 
 TIMELINE_EVENTS = ("prep_begin", "prep_end", "score_begin", "score_end", "select_begin", "select_dry_end",
                    "select_waited", "rule_begin", "rule_end", "select_end", "compact_begin", "compact_waited",
-                   "compact_end")
+                   "compact_end", "hist_done")
 
 
 def timeline(workspace: torch.Tensor) -> Dict[str, Tuple[int, int]]:

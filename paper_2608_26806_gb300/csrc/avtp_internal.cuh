@@ -82,7 +82,7 @@ __device__ __forceinline__ bool wait_expired(uint32_t polls, uint64_t& t0, uint6
 // The normal build records nothing and never touches them.
 enum TimelineEvent {
   kTlPrepBegin = 0, kTlPrepEnd, kTlScoreBegin, kTlScoreEnd, kTlSelBegin, kTlSelDryEnd, kTlSelWaited, kTlRuleBegin,
-  kTlRuleEnd, kTlSelEnd, kTlCompactBegin, kTlCompactWaited, kTlCompactEnd, kTlEvents
+  kTlRuleEnd, kTlSelEnd, kTlCompactBegin, kTlCompactWaited, kTlCompactEnd, kTlHistDone, kTlEvents
 };
 constexpr size_t kTimelineOffset = 16;  // bytes after the start of the workspace
 static_assert(kTimelineOffset + 2 * kTlEvents * sizeof(uint64_t) <= 256, "timeline must fit before the first array");

@@ -559,6 +559,10 @@ __device__ __forceinline__ void alloc_select_tail(const SelectArgs& a, const All
       hist_pass(KeySource{sc, stage ? sh.keys : nullptr}, n, mask, lo & mask, shift, dmask, sh.hist[warp], wt,
                 kThreads - 32);
     }
+#ifdef AVTP_TIMELINE
+    bar_workers();  // every worker's first pass is done
+    if (!dry && tid == 32) timeline_stamp(a.st, kTlHistDone);
+#endif
     if (tid == 32) {
       sh.kmin = lo;
       sh.kmax = hi;
