@@ -20,9 +20,10 @@
 // supplied, one online (max, sum) partial per (row, split). k_narrow_mass: each CTA
 // merges the partials of its request's rows into lse2 (one round of loads), then a thread
 // per visual key sums exp2(z2 - lse2) over the rows whose query follows it, reading the
-// logits back (coalesced: consecutive keys of a row are consecutive), and stores the
-// key's fixed-point mass for k_attn_finalize. No key is read twice and no mass needs
-// atomics.
+// logits back (coalesced: consecutive keys of a row are consecutive), and writes the key's
+// score, formed from the fixed-point mass as k_attn_finalize forms it, and the tile's share
+// of its image's fixed-point sum (one atomic per tile). No key is read twice, and no
+// finalising kernel follows.
 // The work per key is d multiply-adds per row; the logits buffer grows with the rows, and
 // for wide query sets the tcgen05 path takes over (avtp_api.cu picks the path).
 #include "avtp_internal.cuh"
@@ -37,7 +38,6 @@ constexpr int kMassBatch = 32;  // logits a thread of k_narrow_mass loads at onc
 constexpr int kSplitLanes = 4;  // lanes that merge one row's split partials in k_narrow_mass
 static_assert(kNarrowMaxSplits % kSplitLanes == 0 && 32 % kSplitLanes == 0, "split lanes");
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr unsigned long long kMassNotFinite = 1ull << 63;
 static_assert(kNT == kAttnTileM, "k_narrow_mass works on the key tiles of the tensor-core path");
 
 struct NarrowArgs {
@@ -61,7 +61,8 @@ struct NarrowArgs {
   int NS;           // key splits per (request, KV group) in k_narrow_logits
   float* z;         // logits, request by request: [rows of r][T_r]
   float2* part;     // [global rows][NS]: (max2, sum) per split
-  unsigned long long* mass;  // [key tiles][128], 2^-kAttnMassFracBits
+  float* scores;             // [T]: the visual keys' scores
+  int64_t* img_sums;         // [n_img]: fixed-point image sums (zeroed by the validation kernel)
   const float* lse;          // supplied natural-log LSE [Hq][lse_stride], or null
   int64_t lse_stride;
   DevStatus* st;
@@ -245,6 +246,7 @@ __global__ void __launch_bounds__(kNT)
 k_narrow_mass(NarrowArgs a) {
   __shared__ float s_l2[kMassRows];
   __shared__ int64_t s_qpos[kMassRows];
+  __shared__ long long s_fx[kNT / 32];
   pdl_wait();
   pdl_trigger();
   if (!a.st->layout_ok) return;
@@ -323,11 +325,34 @@ k_narrow_mass(NarrowArgs a) {
           if (r0 + j < nr && t <= s_qpos[r0 + j]) mass += exp2f(zz[j] - s_l2[r0 + j]);
       }
     }
-    unsigned long long m = 0;
-    if (has && n_rows > 0)
-      m = mass <= 4194304.f ? static_cast<unsigned long long>(__float2ll_rn(mass * static_cast<float>(1ull << kAttnMassFracBits)))
-                            : kMassNotFinite;  // NaN or inf inputs: the key scores NaN
-    a.mass[static_cast<int64_t>(tile) * kNT + threadIdx.x] = m;
+    // the score, as k_attn_finalize forms it from the fixed-point mass: s = mass * 2^-40 /
+    // (Hq * |Q_r|), NaN for a mass that is not a finite number (non-finite inputs)
+    long long fx = 0;
+    if (has) {
+      float sc = 0.f;
+      if (n_rows > 0) {
+        if (mass <= 4194304.f) {
+          const long long m = __float2ll_rn(mass * static_cast<float>(1ull << kAttnMassFracBits));
+          sc = __ll2float_rn(m) * (1.0f / static_cast<float>(1ull << kAttnMassFracBits));
+          sc = sc / static_cast<float>(n_rows);
+        } else {
+          sc = __int_as_float(0x7fc00000);
+        }
+      }
+      a.scores[t] = sc;
+      fx = fixed_point_score(sc);
+    }
+    // the tile's share of its image's fixed-point sum, one atomic
+    fx = warp_sum(fx);
+    if ((threadIdx.x & 31) == 0) s_fx[threadIdx.x >> 5] = fx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      long long sum = 0;
+#pragma unroll
+      for (int w = 0; w < kNT / 32; ++w) sum += s_fx[w];
+      atomicAdd(reinterpret_cast<unsigned long long*>(a.img_sums + i), static_cast<unsigned long long>(sum));
+    }
+    __syncthreads();  // s_fx is read before the next tile writes it
   }
 }
 
@@ -386,7 +411,8 @@ cudaError_t launch_score_narrow(const avtp_layout_t& L, const avtp_score_args_t&
   a.z = ws_at<float>(ws, p.zbuf);
   a.part = ws_at<float2>(ws, p.p1_part);
   a.st = ws_at<DevStatus>(ws, p.status);
-  a.mass = ws_at<unsigned long long>(ws, p.mass);
+  a.scores = scores;
+  a.img_sums = img_sums;
   a.lse = sa.lse;
   a.lse_stride = sa.lse_stride;
   const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
@@ -397,9 +423,7 @@ cudaError_t launch_score_narrow(const avtp_layout_t& L, const avtp_score_args_t&
   if (e != cudaSuccess) return e;
   const int64_t units2 = plan.n_ktiles_max;
   const int grid2 = static_cast<int>(units2 < 1 ? 1 : (units2 < cap ? units2 : cap));
-  e = launch_kernel(k_narrow_mass, dim3(grid2), dim3(kNT), 0, s, true, a);
-  if (e != cudaSuccess) return e;
-  return launch_attn_finalize(L, sa, scores, img_sums, ws, p, plan, s);
+  return launch_kernel(k_narrow_mass, dim3(grid2), dim3(kNT), 0, s, true, a);
 }
 
 }  // namespace avtp
