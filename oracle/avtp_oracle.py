@@ -31,6 +31,10 @@ Language Models", AVTP):
     visual tokens, the per-sample ranking of the layers, the mean rank, the top-k layers.
     The attention of step 1B may also take the request's last token as its only query
     (§4.1, the output token's attention that FAST-V ranks by).
+7.  The pruning layer's attention forward (the FlashAttention-style pass whose
+    normaliser and probabilities criterion 1B reuses, §3.2): for every token of a
+    request and every head, ``O = softmax(scale * q K^T) V`` over the causally visible
+    keys of the request, and its natural-log normaliser.
 
 Readings of points the paper leaves open (each is also listed with its reason in
 the design notes of the repository):
@@ -122,7 +126,7 @@ def score_hidden_variation(layout, h_cur: np.ndarray, h_prior: np.ndarray) -> np
 # ----------------------------------------------------------------------------
 # Step 1B: text-to-visual attention (attention quantity of paper §3.3.2)
 # ----------------------------------------------------------------------------
-QUERY_SETS = ("text", "last")
+QUERY_SETS = ("text", "last", "all")
 
 
 def query_positions(layout, r: int, query_set: str = "text") -> np.ndarray:
@@ -131,12 +135,15 @@ def query_positions(layout, r: int, query_set: str = "text") -> np.ndarray:
     ``"text"``: every text token of the request (the attention of §3.3.2 kept per token).
     ``"last"``: the request's last token alone, the token whose output predicts the first
     generated token (the attention FAST-V ranks visual tokens by, §4.1).
+    ``"all"``: every token of the request (the attention forward of the layer, §3.2).
     """
     T_r = int(layout.cu_seqlens[r + 1]) - int(layout.cu_seqlens[r])
     if query_set == "text":
         return np.nonzero(~_request_visual_local(layout, r))[0]
     if query_set == "last":
         return np.arange(T_r - 1, T_r) if T_r > 0 else np.zeros(0, dtype=np.int64)
+    if query_set == "all":
+        return np.arange(T_r)
     raise ValueError(query_set)
 
 
@@ -241,6 +248,59 @@ def fixed_point(scores_f32: np.ndarray) -> np.ndarray:
     s = np.clip(s, -FX_SCORE_LIMIT, FX_SCORE_LIMIT)
     return np.rint(s * float(2 ** FX_FRAC_BITS)).astype(np.int64)
 
+
+
+def attention_forward(layout, q, k, v, n_q_heads: int, n_kv_heads: int, scale: float):
+    """The layer's causal attention forward: ``O = softmax(scale * q K^T) V`` per token and
+    head over the request's causally visible keys, with the natural-log normaliser.
+    Follows paper §3.2 (the FlashAttention-style forward whose normaliser criterion 1B
+    reuses) and §3.3.2 (grouped-query heads ``g(h) = h // (Hq/Hkv)``).
+
+    ``q``: bf16 bits [T, Hq, d]; ``k``, ``v``: bf16 bits [T, Hkv, d]. Returns ``(O, lse)``:
+    fp64 [T, Hq, d] and fp64 [Hq, T].
+    """
+    T = int(layout.cu_seqlens[-1])
+    d = q.shape[2]
+    O = np.zeros((T, n_q_heads, d), dtype=np.float64)
+    lse = np.zeros((n_q_heads, T), dtype=np.float64)
+    G = n_q_heads // n_kv_heads
+    for r in range(len(layout.cu_seqlens) - 1):
+        a = int(layout.cu_seqlens[r])
+        b = int(layout.cu_seqlens[r + 1])
+        if b == a:
+            continue
+        for h in range(n_q_heads):
+            z, qpos = attention_logits(layout, q, k, r, h, n_q_heads, n_kv_heads, scale, "all")
+            norm = logsumexp_rows(z)
+            P = np.exp(z - norm[:, None])                       # [T_r, T_r], rows sum to 1
+            O[a + qpos, h, :] = P @ bf16_to_f64(v[a:b, h // G, :])
+            lse[h, a + qpos] = norm
+    return O, lse
+
+
+def attention_forward_rows(layout, q, k, v, n_q_heads: int, n_kv_heads: int, scale: float, r: int,
+                           rows: Sequence[int]):
+    """The attention forward of `attention_forward` for a few request-local query rows of
+    request r only (for workloads too large to run whole). Returns ``(O, lse)``:
+    fp64 [len(rows), Hq, d] and fp64 [Hq, len(rows)].
+    """
+    a = int(layout.cu_seqlens[r])
+    rows = np.asarray(rows, dtype=np.int64)
+    d = q.shape[2]
+    G = n_q_heads // n_kv_heads
+    O = np.zeros((len(rows), n_q_heads, d), dtype=np.float64)
+    lse = np.zeros((n_q_heads, len(rows)), dtype=np.float64)
+    for j, p in enumerate(rows):
+        for h in range(n_q_heads):
+            g = h // G
+            qv = bf16_to_f64(q[a + p, h, :])
+            Kg = bf16_to_f64(k[a:a + p + 1, g, :])                # keys 0..p of the request
+            z = float(scale) * (Kg @ qv)
+            m = np.max(z)
+            w = np.exp(z - m)
+            O[j, h, :] = (w / np.sum(w)) @ bf16_to_f64(v[a:a + p + 1, g, :])
+            lse[h, j] = m + np.log(np.sum(w))
+    return O, lse
 
 def image_sums(layout, scores_f32: np.ndarray) -> np.ndarray:
     """Fixed-point per-image sums ``S_i`` (int64 [n_img]) of the fp32 scores.

@@ -245,11 +245,14 @@ def build_tensors(wl: Workload, parts: Sequence[str] = ("A", "B", "pos")) -> Wor
     text and 0.25 + signal_i on image i (bf16 [T, D]).
     ``"B"``: ``q`` [T, Hq, d] and ``k`` [T, Hkv, d] N(0,1); keys of image i are shifted
     by signal_i times the mean query of their KV group over the request's text rows.
+    ``"V"``: ``v`` [T, Hkv, d] N(0,1), the values of the layer's attention forward.
     ``"pos"``: int32 [P, T] with pos[p, t] = t + p*T (distinct per plane).
     """
     lay = wl.layout
     T = lay.n_tokens
-    children = np.random.SeedSequence(wl.seed).spawn(5)
+    # child i of a fresh seed sequence is the same whatever the number spawned, so the
+    # values' stream (child 5) leaves the other tensors unchanged
+    children = np.random.SeedSequence(wl.seed).spawn(6)
     if "A" in parts:
         rng_p = np.random.default_rng(children[3])
         rng_z = np.random.default_rng(children[4])
@@ -288,6 +291,14 @@ def build_tensors(wl: Workload, parts: Sequence[str] = ("A", "B", "pos")) -> Wor
                 k32[s:e] = f32_to_bf16_bits(kf)
         wl.tensors["q"] = q
         wl.tensors["k"] = k32
+    if "V" in parts:
+        rng_v = np.random.default_rng(children[5])
+        Hkv, d = wl.n_kv_heads, wl.head_dim
+        v = np.empty((T, Hkv, d), dtype=np.uint16)
+        for r0 in range(0, T, _CHUNK_ROWS):
+            r1 = min(T, r0 + _CHUNK_ROWS)
+            v[r0:r1] = _normal_bf16(rng_v, r1 - r0, Hkv * d).reshape(r1 - r0, Hkv, d)
+        wl.tensors["v"] = v
     if "pos" in parts:
         P = wl.pos_planes
         pos = (np.arange(T, dtype=np.int64)[None, :] + np.arange(P, dtype=np.int64)[:, None] * T)

@@ -63,6 +63,13 @@ MUTATIONS = {
                                          "out[r] = sum(int(v) for v in img_sums[int(layout.img_cu[r]):int(layout.img_cu[r + 1]) - 1])"),
     "pruned image starts after its first kept token": ("starts.append(int(np.count_nonzero(local < s0)))",
                                                        "starts.append(int(np.count_nonzero(local <= s0)))"),
+    "forward takes values from the wrong KV head": ("O[a + qpos, h, :] = P @ bf16_to_f64(v[a:b, h // G, :])",
+                                                    "O[a + qpos, h, :] = P @ bf16_to_f64(v[a:b, h % n_kv_heads, :])"),
+    "forward normaliser in base 2": ("lse[h, a + qpos] = norm", "lse[h, a + qpos] = norm / np.log(2.0)"),
+    "forward query set skips the first token": ("        return np.arange(T_r)\n", "        return np.arange(1, T_r)\n"),
+    "forward rows see the next key": ("Kg = bf16_to_f64(k[a:a + p + 1, g, :])", "Kg = bf16_to_f64(k[a:a + p + 2, g, :])"),
+    "forward rows weight values unnormalised": ("O[j, h, :] = (w / np.sum(w)) @ bf16_to_f64(v[a:a + p + 1, g, :])",
+                                                "O[j, h, :] = w @ bf16_to_f64(v[a:a + p + 1, g, :])"),
     "pruned image span keeps its old length": ("lens.append(int(np.count_nonzero((local >= s0) & (local < s1))))",
                                                "lens.append(s1 - s0)"),
 }

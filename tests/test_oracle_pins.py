@@ -655,3 +655,83 @@ def test_pruned_layout_marks_exactly_the_kept_visual_tokens(seed):
                         img_len=got["img_len"])
     # the visual mask of the pruned batch is the gathered visual mask of the original
     assert np.array_equal(lay2.visual_mask(), lay.visual_mask()[kept])
+
+
+# ---------------------------------------------------------------- the layer's attention forward
+def _fwd_workload(Hq=4, Hkv=2, d=16, seed=11):
+    segs = [[("t", 3), ("i", 9), ("t", 2), ("i", 5), ("t", 4)], [("i", 7), ("t", 3)], [("t", 1)]]
+    return synth.make_custom(segs, hidden=32, n_q_heads=Hq, n_kv_heads=Hkv, head_dim=d, seed=seed,
+                             parts=("B", "V"))
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(4, 2), (3, 3), (6, 1)])
+def test_attention_forward_matches_torch_sdpa(Hq, Hkv):
+    """The forward against torch's scaled_dot_product_attention in fp64 (a library routine,
+    causal per request, GQA by repeating each KV head over its query heads), and the
+    normaliser against torch.logsumexp of the masked logits."""
+    torch = pytest.importorskip("torch")
+    wl = _fwd_workload(Hq, Hkv)
+    lay = wl.layout
+    out, lse = O.attention_forward(lay, wl.q, wl.k, wl.v, Hq, Hkv, wl.softmax_scale)
+    G = Hq // Hkv
+    for r in range(lay.n_requests):
+        a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+        q = torch.from_numpy(O.bf16_to_f64(wl.q[a:b])).permute(1, 0, 2)  # [Hq, T_r, d]
+        k = torch.from_numpy(O.bf16_to_f64(wl.k[a:b])).permute(1, 0, 2).repeat_interleave(G, dim=0)
+        v = torch.from_numpy(O.bf16_to_f64(wl.v[a:b])).permute(1, 0, 2).repeat_interleave(G, dim=0)
+        ref = torch.nn.functional.scaled_dot_product_attention(q, k, v, is_causal=True, scale=wl.softmax_scale)
+        np.testing.assert_allclose(out[a:b].transpose(1, 0, 2), ref.numpy(), rtol=1e-12, atol=1e-12)
+        z = wl.softmax_scale * torch.einsum("hqd,hkd->hqk", q, k)
+        mask = torch.ones(b - a, b - a, dtype=torch.bool).tril()
+        ref_lse = torch.logsumexp(z.masked_fill(~mask, float("-inf")), dim=-1)
+        np.testing.assert_allclose(lse[:, a:b], ref_lse.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_attention_forward_closed_forms():
+    """A request's first token sees only itself: O = its value, lse = its own logit. With
+    all queries zero every visible key weighs the same: O = the prefix mean of the values,
+    lse = ln(p + 1)."""
+    Ox = O
+    wl = _fwd_workload()
+    lay = wl.layout
+    Hq, Hkv, G = wl.n_q_heads, wl.n_kv_heads, wl.n_q_heads // wl.n_kv_heads
+    out, lse = Ox.attention_forward(lay, wl.q, wl.k, wl.v, Hq, Hkv, wl.softmax_scale)
+    for r in range(lay.n_requests):
+        a = int(lay.cu_seqlens[r])
+        for h in range(Hq):
+            np.testing.assert_array_equal(out[a, h], Ox.bf16_to_f64(wl.v[a, h // G]))
+            z0 = wl.softmax_scale * np.dot(Ox.bf16_to_f64(wl.q[a, h]), Ox.bf16_to_f64(wl.k[a, h // G]))
+            assert lse[h, a] == pytest.approx(z0, rel=1e-14, abs=1e-14)
+    q0 = np.zeros_like(wl.q)
+    out0, lse0 = Ox.attention_forward(lay, q0, wl.k, wl.v, Hq, Hkv, wl.softmax_scale)
+    for r in range(lay.n_requests):
+        a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+        vf = Ox.bf16_to_f64(wl.v[a:b])                               # [T_r, Hkv, d]
+        prefix_mean = np.cumsum(vf, axis=0) / np.arange(1, b - a + 1)[:, None, None]
+        for h in range(Hq):
+            np.testing.assert_allclose(out0[a:b, h], prefix_mean[:, h // G], rtol=1e-12, atol=1e-13)
+            np.testing.assert_allclose(lse0[h, a:b], np.log(np.arange(1, b - a + 1)), rtol=1e-13)
+
+
+def test_attention_forward_rows_match_the_whole_forward():
+    Ox = O
+    wl = _fwd_workload()
+    lay = wl.layout
+    out, lse = Ox.attention_forward(lay, wl.q, wl.k, wl.v, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
+    a = int(lay.cu_seqlens[0])
+    rows = [0, 4, 11, 22]
+    o_r, l_r = Ox.attention_forward_rows(lay, wl.q, wl.k, wl.v, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale, 0, rows)
+    np.testing.assert_allclose(o_r, out[[a + p for p in rows]], rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(l_r, lse[:, [a + p for p in rows]], rtol=1e-13)
+
+
+def test_forward_normaliser_is_criterion_b_normaliser():
+    """The forward's normaliser at the text rows is the one criterion B divides by: the
+    text-query scores computed with it (supplied) equal the scores computed from scratch."""
+    Ox = O
+    wl = _fwd_workload()
+    lay = wl.layout
+    _, lse = Ox.attention_forward(lay, wl.q, wl.k, wl.v, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
+    s_own = Ox.score_text_attention(lay, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale)
+    s_fwd = Ox.score_text_attention(lay, wl.q, wl.k, wl.n_q_heads, wl.n_kv_heads, wl.softmax_scale, lse=lse)
+    np.testing.assert_allclose(s_fwd, s_own, rtol=1e-12, atol=1e-15)
