@@ -264,7 +264,7 @@ def run_ours(args, world, rank, local):
     __graft_entry__.build()
     crit = args.criterion
     second = None if args.no_secondary or crit != "hidden_variation" else "text_attention"
-    parts = ("A", "pos") if (crit == "hidden_variation" and second is None) else ("A", "B", "pos")
+    parts = ("A", "pos") if (crit == "hidden_variation" and second is None) else ("A", "B", "V", "pos")
     wl = synth.make_workload(args.config, parts=parts)
     lay = wl.layout
 
@@ -320,7 +320,7 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     # the other scoring criterion (text-to-visual attention), timed the same way on the
     # same workload, for a secondary object of the line
-    sec = sec_lse = sec_last = prog = None
+    sec = sec_lse = sec_last = prog = fwd = None
     if second is not None:
         sec = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev)
         lse = fa_lse(wl, bf16(wl.q), bf16(wl.k), torch)
@@ -330,6 +330,7 @@ def run_ours(args, world, rank, local):
         sec_last = time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp, world, dev,
                                   query_set="last")
         prog = time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avtp, world, dev)
+        fwd = time_forward(args, wl, L, bf16, stream, flush, torch, avtp, world, dev)
     variants = time_variants(args, call, stream, flush, torch, avtp, 4 if crit == "hidden_variation" else 7)
     clocks = sampler.stop() if sampler else None
     barrier(world)
@@ -427,6 +428,25 @@ def run_ours(args, world, rank, local):
     if prog is not None:
         line["progressive"] = prog
         line["gpu_launches"] += prog["gpu_launches"]
+    if fwd is not None:
+        res, Kf = fwd
+        flops = forward_flops(wl)
+        plain, with_b = res["plain"]["ms"], res["with_scores"]["ms"]
+        achieved = flops / (plain * 1e-3) / 1e12
+        line["attn_forward"] = {
+            "what": "the pruning layer's causal attention forward (O fp32, natural-log LSE) through "
+                    "avtp_attn_forward, plain and with criterion B's scores from the forward's LSE",
+            "steps": Kf, "l2": "flushed before every timed call",
+            "plain_us": round(plain * 1e3, 2), "plain_p50_us": res["plain"]["p50_us"],
+            "with_scores_us": round(with_b * 1e3, 2), "with_scores_p50_us": res["with_scores"]["p50_us"],
+            "criterion_b_marginal_us": round((with_b - plain) * 1e3, 2),
+            "criterion_b_marginal_frac": round((with_b - plain) / plain, 4),
+            "roofline": {"bound": "tensor", "kernel": "forward (query tiles + value transpose + k_attn_fwd)",
+                         "achieved": round(achieved, 2), "peak": bf16_s, "unit": "TFLOP/s",
+                         "frac": round(achieved / bf16_s, 4), "peak_kind": peak_kind,
+                         "algorithmic_flops_per_launch": flops},
+            "gpu_launches": res["plain"]["launches"] + res["with_scores"]["launches"]}
+        line["gpu_launches"] += line["attn_forward"]["gpu_launches"]
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, crit, args.cpu_seconds)
         if not args.no_all_core_baseline:
@@ -555,6 +575,45 @@ def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp
                            "p90": round(step_ms[int(len(step_ms) * 0.9)] * 1e3, 2)},
             "steps_us": {k: round(v * 1e3, 2) for k, v in per_step.items()},
             "launches": K * ((7 if lse is None else 6) if query_set == "text" else 7)}
+
+
+def forward_flops(wl):
+    """Causal attention forward FLOPs: every visible (query, key) pair of every query head
+    costs d multiply-adds in Q K^T and d in P V."""
+    cu = wl.layout.cu_seqlens
+    pairs = sum(int(n) * (int(n) + 1) // 2 for n in np.diff(cu))
+    return 4 * pairs * wl.n_q_heads * wl.head_dim
+
+
+def time_forward(args, wl, L, bf16, stream, flush, torch, avtp, world, dev):
+    """The layer's attention forward (avtp_attn_forward) on the same workload, plain and
+    with criterion B's scores from its own LSE: B's marginal cost is the difference."""
+    q, k, v = bf16(wl.q), bf16(wl.k), bf16(wl.v)
+    K = max(5, min(args.steps, 100))
+    out = {}
+    for key, with_scores in (("plain", False), ("with_scores", True)):
+        call = avtp.ForwardCall(L, q=q, k=k, v=v, softmax_scale=wl.softmax_scale, scores=with_scores)
+        for _ in range(max(3, args.warmup)):
+            flush()
+            call.run(stream)
+        torch.cuda.synchronize()
+        st = avtp.read_device_status(call.workspace)
+        if st != avtp.OK:
+            raise RuntimeError(f"device status after warm-up (attention forward): {avtp.status_string(st)}")
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+        barrier(world)
+        torch.cuda.synchronize()
+        for i in range(K):
+            flush()
+            ev[i][0].record(stream)
+            call.run(stream)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        ms = sorted(a.elapsed_time(b) for a, b in ev)
+        out[key] = {"ms": reduce_max(sum(ms), world, dev) / K, "p50_us": round(ms[len(ms) // 2] * 1e3, 2),
+                    "launches": K * (7 if with_scores else 4)}  # k_prep, qtiles, transpose, forward (+ pack, mass, finalize)
+        del call
+    return out, K
 
 
 def time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avtp, world, dev, stages=3):

@@ -189,6 +189,43 @@ AVTP_API avtp_status_t avtp_workspace_size(const avtp_layout_t* layout, const av
 AVTP_API avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_args_t* args, float* scores,
                          int64_t* img_sums, void* workspace, size_t workspace_bytes, avtp_stream_t stream);
 
+/* The pruning layer's causal attention forward, with the text-attention criterion as
+ * a side output (paper §3.2: FlashAttention-style attention keeps the natural-log
+ * normaliser of every query row, which is what the criterion needs; §3.3.2 for the
+ * criterion). For every token t and query head h of the batch:
+ *   O[t, h]   = sum_u softmax_u(softmax_scale * q[t, h] . k[u, g(h)]) v[u, g(h)]
+ *   lse[h, t] = ln sum_u exp(softmax_scale * q[t, h] . k[u, g(h)])
+ * over the keys u of t's request with u <= t, g(h) = h / (n_q_heads / n_kv_heads).
+ * bf16 tensor-core products with fp32 accumulation; P is rounded to bf16 before P V,
+ * as in FlashAttention. */
+typedef struct {
+  const void* v;       /* device bf16 [T, n_kv_heads, head_dim], token stride v_stride
+                        * elements (a multiple of 8), 16-byte aligned                  */
+  int64_t v_stride;
+  float* o;            /* device fp32 [T, n_q_heads, head_dim], token stride o_stride
+                        * elements (a multiple of 4), 16-byte aligned: written          */
+  int64_t o_stride;
+  float* lse;          /* device fp32 [n_q_heads, T], row stride lse_stride >= T: written */
+  int64_t lse_stride;
+} avtp_forward_args_t;
+
+/* Workspace bytes of avtp_attn_forward for these arguments (the same checks as the call). */
+AVTP_API avtp_status_t avtp_forward_workspace_size(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
+                                                   const avtp_forward_args_t* fwd_args, size_t* bytes);
+
+/* Runs the forward above for every token of the batch: q, k, the heads, head_dim,
+ * strides and softmax_scale come from score_args (criterion AVTP_CRIT_TEXT_ATTENTION,
+ * lse NULL: the forward writes it), v, O and the LSE from fwd_args. When scores and
+ * img_sums are non-NULL it then scores the visual tokens as avtp_score does with
+ * score_args' query set and path, reading the LSE the forward just wrote: criterion B
+ * costs its mass pass (one more Q K^T over the query set and the visual keys) and no
+ * pass of its own for the normaliser. The exact per-key mass needs each query's final
+ * normaliser, so it cannot be formed inside the forward's own key loop. Both NULL: the
+ * plain forward. The layout is validated as in avtp_score; asynchronous on `stream`. */
+AVTP_API avtp_status_t avtp_attn_forward(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
+                                         const avtp_forward_args_t* fwd_args, float* scores, int64_t* img_sums,
+                                         void* workspace, size_t workspace_bytes, avtp_stream_t stream);
+
 /* Step 2 (paper §3.3.3, App. A.2). From img_sums (device int64 [n_images]) writes
  * budgets (device int32 [n_images]) and out_cu_seqlens (device int32 [R+1]),
  * the packed offsets of the pruned batch. Per request, in exact rational arithmetic:

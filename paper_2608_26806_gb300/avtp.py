@@ -75,6 +75,11 @@ class _Rows(ctypes.Structure):
                 ("out_stride", c_int64)]
 
 
+class _ForwardArgs(ctypes.Structure):
+    _fields_ = [("v", c_void_p), ("v_stride", c_int64), ("o", c_void_p), ("o_stride", c_int64), ("lse", c_void_p),
+                ("lse_stride", c_int64)]
+
+
 # ---------------------------------------------------------------- library
 _LIB = None
 
@@ -82,6 +87,10 @@ _LIB = None
 SIGNATURES = {
     "avtp_workspace_size": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(c_size_t)]),
     "avtp_score": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
+    "avtp_forward_workspace_size": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(_ForwardArgs),
+                                            POINTER(c_size_t)]),
+    "avtp_attn_forward": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(_ForwardArgs), c_void_p, c_void_p,
+                                  c_void_p, c_size_t, c_void_p]),
     "avtp_allocate": (c_int, [POINTER(_Layout), c_void_p, POINTER(_AllocArgs), c_void_p, c_void_p, c_void_p,
                               c_size_t, c_void_p]),
     "avtp_select": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
@@ -313,6 +322,62 @@ def score(layout: Layout, criterion, *, h_cur=None, h_prior=None, q=None, k=None
     _check(load().avtp_score(ctypes.byref(lay), ctypes.byref(sa), _ptr(scores), _ptr(img_sums), _ptr(workspace),
                              workspace.numel(), _stream(stream)), "avtp_score")
     return scores, img_sums[:layout.n_images]
+
+
+def _forward_args(v: torch.Tensor, o: torch.Tensor, lse: torch.Tensor) -> _ForwardArgs:
+    if v.dtype != torch.bfloat16 or v.dim() != 3 or v.stride(2) != 1 or v.stride(1) != v.shape[2]:
+        raise ValueError("v must be bf16 [T, Hkv, head_dim] with contiguous heads")
+    if o.dtype != torch.float32 or o.dim() != 3 or o.stride(2) != 1 or o.stride(1) != o.shape[2]:
+        raise ValueError("o must be fp32 [T, Hq, head_dim] with contiguous heads")
+    if lse.dtype != torch.float32 or lse.dim() != 2 or lse.stride(1) != 1:
+        raise ValueError("lse must be fp32 [Hq, T] with a contiguous last dim")
+    return _ForwardArgs(_ptr(v), v.stride(0), _ptr(o), o.stride(0), _ptr(lse), lse.stride(0))
+
+
+class ForwardCall:
+    """A prepared avtp_attn_forward call: arguments marshalled once, outputs and workspace
+    allocated once, so that ``run()`` is the C call alone (for timing and graphs)."""
+
+    def __init__(self, layout: Layout, *, q, k, v, softmax_scale=None, scores: bool = True, query_set="text",
+                 path="auto", o=None, lse=None, workspace=None):
+        dev = layout.cu_seqlens.device
+        T, Hq, d = q.shape
+        self.layout = layout
+        self.o = o if o is not None else torch.empty(T, Hq, d, dtype=torch.float32, device=dev)
+        self.lse = lse if lse is not None else torch.empty(Hq, max(T, 1), dtype=torch.float32, device=dev)
+        self.scores = torch.zeros(T, dtype=torch.float32, device=dev) if scores else None
+        self.img_sums = torch.empty(max(layout.n_images, 1), dtype=torch.int64, device=dev) if scores else None
+        self._keep = (q, k, v)
+        self._sa = _score_args(CRIT_TEXT_ATTENTION, q=q, k=k, softmax_scale=softmax_scale,
+                               max_text_tokens=layout.n_text, query_set=query_set, path=path)
+        self._fa = _forward_args(v, self.o, self.lse)
+        self._lay = layout.c()
+        lib = load()
+        if workspace is None:
+            n = c_size_t()
+            _check(lib.avtp_forward_workspace_size(ctypes.byref(self._lay), ctypes.byref(self._sa),
+                                                   ctypes.byref(self._fa), ctypes.byref(n)),
+                   "avtp_forward_workspace_size")
+            workspace = new_workspace(int(n.value), dev)
+        self.workspace = workspace
+
+    def run(self, stream=None):
+        _check(load().avtp_attn_forward(ctypes.byref(self._lay), ctypes.byref(self._sa), ctypes.byref(self._fa),
+                                        _ptr(self.scores), _ptr(self.img_sums), _ptr(self.workspace),
+                                        self.workspace.numel(), _stream(stream)), "avtp_attn_forward")
+        return self
+
+
+def attn_forward(layout: Layout, *, q, k, v, softmax_scale=None, scores: bool = True, query_set="text",
+                 path="auto", stream=None):
+    """avtp_attn_forward: the layer's causal attention forward, O (fp32 [T, Hq, d]) and the
+    natural-log LSE (fp32 [Hq, T]), and with ``scores`` the text-attention scores and
+    fixed-point image sums from that LSE. Returns (o, lse, scores, img_sums); the last
+    two are None without ``scores``."""
+    c = ForwardCall(layout, q=q, k=k, v=v, softmax_scale=softmax_scale, scores=scores, query_set=query_set,
+                    path=path).run(stream)
+    sums = c.img_sums[:layout.n_images] if c.img_sums is not None else None
+    return c.o, c.lse[:, :layout.n_tokens], c.scores, sums
 
 
 def allocate(layout: Layout, img_sums: torch.Tensor, keep_ratio: torch.Tensor, alpha=1.0, r_min=0.05, r_max=0.95,

@@ -4,6 +4,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include "avtp_fwd.cuh"
 #include "avtp_internal.cuh"
 
 namespace avtp {
@@ -166,6 +167,18 @@ WsPlan plan_workspace(const avtp_layout_t& L, const avtp_score_args_t* sa) {
   return p;
 }
 
+FwdWs plan_forward_workspace(const avtp_layout_t& L, const avtp_score_args_t& sa, size_t base_bytes) {
+  FwdWs f{};
+  size_t off = align_up(base_bytes);
+  f.Tp = (L.n_tokens + 7) & ~static_cast<int64_t>(7);
+  f.vt = off;
+  off = align_up(off + static_cast<size_t>(sa.n_kv_heads) * sa.head_dim * static_cast<size_t>(f.Tp) * 2 + 16);
+  f.qtile_cu = off;
+  off = align_up(off + (static_cast<size_t>(L.n_requests) + 1) * 4);
+  f.total = off;
+  return f;
+}
+
 bool pdl_enabled() {
   static const bool on = [] {
     const char* v = getenv("AVTP_PDL");
@@ -245,6 +258,64 @@ avtp_status_t avtp_score(const avtp_layout_t* layout, const avtp_score_args_t* a
   }
   if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
   return score_impl(layout, args, scores, img_sums, workspace, p, s);
+}
+
+// The forward's arguments, and the score arguments of its criterion-B side output (the
+// caller's, with the LSE the forward writes supplied).
+static avtp_status_t forward_args(const avtp_layout_t* L, const avtp_score_args_t* a, const avtp_forward_args_t* f,
+                                  avtp_score_args_t* sa_out) {
+  if (a == nullptr || f == nullptr) return AVTP_ERR_INVALID_ARG;
+  if (a->criterion != AVTP_CRIT_TEXT_ATTENTION || a->lse != nullptr) return AVTP_ERR_INVALID_ARG;
+  if (f->v == nullptr || f->o == nullptr || f->lse == nullptr) return AVTP_ERR_INVALID_ARG;
+  avtp_score_args_t sa = *a;
+  sa.lse = f->lse;
+  sa.lse_stride = f->lse_stride;
+  avtp_status_t st = check_score_args(L, &sa);
+  if (st != AVTP_OK) return st;
+  const int64_t Hq = sa.n_q_heads, Hkv = sa.n_kv_heads, d = sa.head_dim;
+  if (f->v_stride < Hkv * d || f->o_stride < Hq * d) return AVTP_ERR_INVALID_ARG;
+  if (f->v_stride % 8 != 0 || f->o_stride % 4 != 0) return AVTP_ERR_UNSUPPORTED;
+  if (!aligned16(f->v) || !aligned16(f->o)) return AVTP_ERR_UNSUPPORTED;
+  // query tiles x heads, the forward's grid: (T / 128 + R) * Hq CTAs
+  if ((L->n_tokens / 128 + L->n_requests) * Hq > 0x7fffffffLL) return AVTP_ERR_RANGE;
+  *sa_out = sa;
+  return AVTP_OK;
+}
+
+avtp_status_t avtp_forward_workspace_size(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
+                                          const avtp_forward_args_t* fwd_args, size_t* bytes) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  if (bytes == nullptr) return AVTP_ERR_INVALID_ARG;
+  avtp_score_args_t sa{};
+  if ((st = forward_args(layout, score_args, fwd_args, &sa)) != AVTP_OK) return st;
+  *bytes = plan_forward_workspace(*layout, sa, plan_workspace(*layout, &sa).total).total;
+  return AVTP_OK;
+}
+
+avtp_status_t avtp_attn_forward(const avtp_layout_t* layout, const avtp_score_args_t* score_args,
+                                const avtp_forward_args_t* fwd_args, float* scores, int64_t* img_sums,
+                                void* workspace, size_t workspace_bytes, avtp_stream_t stream) {
+  avtp_status_t st = check_layout(layout);
+  if (st != AVTP_OK) return st;
+  avtp_score_args_t sa{};
+  if ((st = forward_args(layout, score_args, fwd_args, &sa)) != AVTP_OK) return st;
+  if ((scores == nullptr) != (img_sums == nullptr)) return AVTP_ERR_INVALID_ARG;
+  const WsPlan p = plan_workspace(*layout, &sa);
+  const FwdWs f = plan_forward_workspace(*layout, sa, p.total);
+  WsPlan whole = p;
+  whole.total = f.total;
+  if ((st = check_ws(workspace, workspace_bytes, whole)) != AVTP_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PrepArgs pa{};
+  pa.L = *layout;
+  pa.zero_img_sums = img_sums;
+  pa.build_text_tiles = scores != nullptr;
+  if (pa.build_text_tiles) pa.attn = attn_plan(*layout, sa);
+  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
+  if ((st = from_cuda(launch_attn_forward(*layout, sa, *fwd_args, workspace, p, f, s))) != AVTP_OK) return st;
+  if (scores == nullptr) return AVTP_OK;
+  return score_impl(layout, &sa, scores, img_sums, workspace, p, s);
 }
 
 avtp_status_t avtp_allocate(const avtp_layout_t* layout, const int64_t* img_sums, const avtp_alloc_args_t* args,

@@ -216,6 +216,50 @@ def test_workspace_size_grows_with_attention_bookkeeping(lib):
     assert a.value % 256 == 0 and b.value % 256 == 0
 
 
+def _fwd_args(d=128, hq=32, hkv=8, T=100):
+    return avtp._ForwardArgs(FAKE, hkv * d, FAKE, hq * d, FAKE, T)
+
+
+def _forward(lib, lay, sa, fa, scores=FAKE, sums=FAKE, ws=FAKE, ws_bytes=1 << 34):
+    return lib.avtp_attn_forward(ctypes.byref(lay), ctypes.byref(sa) if sa is not None else None,
+                                 ctypes.byref(fa) if fa is not None else None, scores, sums, ws, ws_bytes, None)
+
+
+def test_host_validation_of_forward_arguments(lib):
+    lay = _layout(T=100)
+    assert _forward(lib, lay, None, _fwd_args()) == avtp.ERR_INVALID_ARG
+    assert _forward(lib, lay, _attn_args(), None) == avtp.ERR_INVALID_ARG
+    assert _forward(lib, lay, _hv_args(), _fwd_args()) == avtp.ERR_INVALID_ARG  # the criterion of the forward is B
+    supplied = _attn_args()
+    supplied.lse, supplied.lse_stride = FAKE, 100  # the forward writes the LSE itself
+    assert _forward(lib, lay, supplied, _fwd_args()) == avtp.ERR_INVALID_ARG
+    assert _forward(lib, lay, _attn_args(d=96), _fwd_args(d=96)) == avtp.ERR_UNSUPPORTED
+    for field, value, code in [("v", None, avtp.ERR_INVALID_ARG), ("o", None, avtp.ERR_INVALID_ARG),
+                               ("lse", None, avtp.ERR_INVALID_ARG), ("v", FAKE + 8, avtp.ERR_UNSUPPORTED),
+                               ("o", FAKE + 4, avtp.ERR_UNSUPPORTED), ("v_stride", 8 * 128 - 8, avtp.ERR_INVALID_ARG),
+                               ("v_stride", 8 * 128 + 4, avtp.ERR_UNSUPPORTED),
+                               ("o_stride", 32 * 128 + 2, avtp.ERR_UNSUPPORTED),
+                               ("o_stride", 32 * 128 - 4, avtp.ERR_INVALID_ARG),
+                               ("lse_stride", 99, avtp.ERR_INVALID_ARG)]:
+        fa = _fwd_args()
+        setattr(fa, field, value)
+        assert _forward(lib, lay, _attn_args(), fa) == code, (field, value)
+    assert _forward(lib, lay, _attn_args(), _fwd_args(), sums=None) == avtp.ERR_INVALID_ARG  # both or neither
+    assert _forward(lib, lay, _attn_args(), _fwd_args(), ws_bytes=1024) == avtp.ERR_WORKSPACE
+    assert _forward(lib, lay, _attn_args(), _fwd_args(), ws=FAKE + 16) == avtp.ERR_WORKSPACE
+
+
+def test_forward_workspace_holds_the_transposed_values(lib):
+    lay = _layout(n_req=2, n_img=5, T=10000)
+    a, b = ctypes.c_size_t(), ctypes.c_size_t()
+    sa = _attn_args()
+    assert lib.avtp_workspace_size(ctypes.byref(lay), ctypes.byref(sa), ctypes.byref(a)) == avtp.OK
+    fa = _fwd_args(T=10000)
+    assert lib.avtp_forward_workspace_size(ctypes.byref(lay), ctypes.byref(sa), ctypes.byref(fa),
+                                           ctypes.byref(b)) == avtp.OK
+    assert b.value >= 8 * 128 * 10000 * 2 and b.value % 256 == 0
+
+
 def test_host_validation_of_wait_selftest_arguments(lib):
     for bad in (-1, 0, 999, 10_000_000_001):
         assert lib.avtp_wait_selftest(bad, 0, FAKE, 256, None) == avtp.ERR_INVALID_ARG
@@ -230,7 +274,8 @@ def test_binding_structs_match_the_c_layout(tmp_path):
     # sizeof and every field offset of the ABI structs, from the header compiled by the
     # host C compiler, against the ctypes mirrors of the binding
     structs = {"avtp_layout_t": avtp._Layout, "avtp_score_args_t": avtp._ScoreArgs,
-               "avtp_alloc_args_t": avtp._AllocArgs, "avtp_rows_t": avtp._Rows}
+               "avtp_alloc_args_t": avtp._AllocArgs, "avtp_rows_t": avtp._Rows,
+               "avtp_forward_args_t": avtp._ForwardArgs}
     renamed = {"in_": "in"}  # a Python keyword in the mirror
     lines = ["#include <stdio.h>", "#include <stddef.h>", '#include "avtp.h"', "int main(void) {"]
     for c_name, py in structs.items():
