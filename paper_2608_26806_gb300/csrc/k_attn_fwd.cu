@@ -15,15 +15,20 @@
 //   S_j = Q K_j^T        tcgen05, M = 128 queries, N = 128 keys, K = d; fp32 in TMEM
 //   P_j = exp2(c2 S_j - m)  softmax warps, bf16 into shared memory (128-byte swizzle)
 //   O  += P_j V_j        tcgen05, M = 128, N = d, K = 128 keys; fp32 in TMEM
-// with c2 = scale * log2(e). A row's reference max m moves only when a block's max
-// exceeds it by more than 8 (log2 units), so the accumulator in TMEM is rescaled rarely
-// and every P entry stays below 2^8. P V needs V with keys contiguous (the MMA's K-major
-// operand), so a first kernel writes the values transposed, Vt[g][c][t].
+// with c2 = scale * log2(e). The two 64-key halves of every block are softmaxed by
+// different warps, each half of a row with its own reference max, sum and accumulator
+// (O_0 += P[:, 0:64] V[0:64], O_1 += P[:, 64:128] V[64:128]); the two halves of a row
+// are merged once, in the epilogue, the way split-key partial softmaxes combine. A
+// half's reference max moves only when a block's max exceeds it by more than 8 (log2
+// units), so its accumulator in TMEM is rescaled rarely and every P entry stays below
+// 2^8. P V needs V with keys contiguous (the MMA's K-major operand), so a first kernel
+// writes the values transposed, Vt[g][c][t].
 //
-// Warps 0-3: softmax and epilogue (thread i owns query row i = TMEM lane i). Warp 4
-// issues the TMA loads (Q once, K and Vt double-buffered). Warp 5 owns TMEM and issues
-// the MMAs: S_j before P_{j-1} V_{j-1}, so the softmax of block j overlaps the P V of
-// block j - 1. TMEM: S double buffer in columns 0-255, O in columns 256 .. 256 + d.
+// Warps 0-7: softmax and epilogue; warp w owns query rows 32 (w % 4) .. + 31 (TMEM lanes)
+// and key half w / 4, so two warps share every SM sub-partition. Warp 8 issues the TMA
+// loads (Q once, K and Vt double-buffered). Warp 9 owns TMEM and issues the MMAs: S_j
+// before P_{j-1} V_{j-1}, so the softmax of block j overlaps the P V of block j - 1.
+// TMEM: S double buffer in columns 0-255, O_0 from column 256, O_1 from column 384.
 // Every wait is bounded; a CTA whose wait gives up records AVTP_ERR_TIMEOUT and returns.
 #include <cudaTypedefs.h>
 
@@ -35,11 +40,14 @@ namespace {
 
 constexpr int kQT = 128;  // query rows per tile (MMA M, TMEM lanes)
 constexpr int kKB = 128;  // keys per block (MMA N of Q K^T, K of P V)
-constexpr int kThreads = 192;
-constexpr int kTmaWarp = 4;
-constexpr int kMmaWarp = 5;
+constexpr int kHalf = kKB / 2;  // keys of a block per softmax warp
+constexpr int kThreads = 320;
+constexpr int kSoftWarps = 8;
+constexpr int kTmaWarp = 8;
+constexpr int kMmaWarp = 9;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kOCol = 256;
+constexpr uint32_t kOCol = 256;   // O_0; O_1 at kOCol + kOHalf
+constexpr uint32_t kOHalf = 128;
 constexpr float kRescaleTau = 8.f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -97,6 +105,8 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+__device__ __forceinline__ void bar_softmax() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&b);
@@ -110,6 +120,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
            const __grid_constant__ CUtensorMap mapV, FwdArgs a) {
   extern __shared__ unsigned char smem_raw[];
   __shared__ FwdSync sy;
+  __shared__ float2 s_ml[2][kQT];  // (reference max, sum) of each key half of each row
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int d = a.d;
@@ -144,9 +155,9 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       tc::mbar_init(&sy.v_full[s], 1);
       tc::mbar_init(&sy.v_empty[s], 1);
       tc::mbar_init(&sy.s_full[s], 1);
-      tc::mbar_init(&sy.s_empty[s], 4);
+      tc::mbar_init(&sy.s_empty[s], kSoftWarps);
     }
-    tc::mbar_init(&sy.p_full, 4);
+    tc::mbar_init(&sy.p_full, kSoftWarps);
     tc::mbar_init(&sy.pv_done, 1);
     tc::mbar_init(&sy.drain, 1);
     sy.abort = 0;
@@ -195,7 +206,8 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
     if (lane == 0) {
       const uint32_t idS = tc::idesc_bf16(kQT, kKB), idO = tc::idesc_bf16(kQT, d);
       const uint32_t aQ = tc::smem_u32(sQ), aP = tc::smem_u32(sP);
-      // O += P_i V_i: A = P (128 rows x 128 keys), B = Vt block (d rows x 128 keys)
+      // O_h += P_i[:, 64h .. 64h + 63] V_i[64h .. 64h + 63]: A = panel h of P (128 rows x 64
+      // keys), B = panel h of the Vt block (d rows x 64 keys)
       auto issue_pv = [&](int i) -> bool {
         const int sb = i & 1;
         if (!tc::mbar_wait(&sy.p_full, i & 1)) return false;
@@ -203,11 +215,14 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         tc::fence_after_sync();
         const uint32_t bV = tc::smem_u32(sV + sb * v_bytes(d));
 #pragma unroll
-        for (int ks = 0; ks < kKB / 16; ++ks) {
-          const uint32_t off = static_cast<uint32_t>(ks & 3) * 32u;
-          const uint32_t ap = aP + static_cast<uint32_t>(ks >> 2) * (kQT * 128) + off;
-          const uint32_t bp = bV + static_cast<uint32_t>(ks >> 2) * static_cast<uint32_t>(d * 128) + off;
-          tc::mma_bf16(tmem + kOCol, tc::desc_k_sw128(ap), tc::desc_k_sw128(bp), idO, (i > 0 || ks > 0) ? 1u : 0u);
+        for (int hh = 0; hh < 2; ++hh) {
+#pragma unroll
+          for (int ks = 0; ks < kHalf / 16; ++ks) {
+            const uint32_t ap = aP + static_cast<uint32_t>(hh * (kQT * 128) + ks * 32);
+            const uint32_t bp = bV + static_cast<uint32_t>(hh * (d * 128) + ks * 32);
+            tc::mma_bf16(tmem + kOCol + hh * kOHalf, tc::desc_k_sw128(ap), tc::desc_k_sw128(bp), idO,
+                         (i > 0 || ks > 0) ? 1u : 0u);
+          }
         }
         tc::mma_commit(&sy.pv_done);
         tc::mma_commit(&sy.v_empty[sb]);
@@ -231,17 +246,20 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       tc::mbar_wait(&sy.drain, 0);
     }
   } else {
-    // ------------------------------------------------------------ softmax and epilogue (warps 0-3)
-    const int row = warp * 32 + lane;
+    // ------------------------------------------------------------ softmax and epilogue (warps 0-7)
+    const int quad = warp & 3, half = warp >> 2;
+    const int row = quad * 32 + lane;
     const int qpos = q0 + row;
-    const uint32_t tl = tmem + (static_cast<uint32_t>(warp * 32) << 16);  // this warp's TMEM lanes
+    const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16);  // this warp's TMEM lanes
+    const uint32_t ocol = kOCol + half * kOHalf;                           // this half's accumulator
     const float c2 = a.c2;
-    float m = -INFINITY, l = 0.f;  // reference max (log2 units) and sum of exp2(c2 s - m)
+    const float2 cc = make_float2(c2, c2);
+    float m = -INFINITY, l = 0.f;  // reference max (log2 units) and sum of exp2(c2 s - m), this half
     bool ok = true;
-    unsigned char* prow = sP + row * 128;
+    unsigned char* prow = sP + half * (kQT * 128) + row * 128;  // this row of P panel `half`
     for (int j = 0; j < nblk; ++j) {
       const int sb = j & 1;
-      const int key0 = (kb0 + j) * kKB;
+      const int key0 = (kb0 + j) * kKB + half * kHalf;
       if (__any_sync(0xffffffffu, *abort_flag != 0)) { ok = false; break; }
       if (!tc::mbar_wait_warp(&sy.s_full[sb], (j >> 1) & 1)) {
         if (lane == 0) *abort_flag = 1;
@@ -249,31 +267,29 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         break;
       }
       tc::fence_after_sync();
-      float s[kKB];
-#pragma unroll
-      for (int c4 = 0; c4 < kKB / 32; ++c4)
-        tc::tmem_ld32(tl + sb * kKB + c4 * 32, *reinterpret_cast<float(*)[32]>(s + c4 * 32));
+      float s[kHalf];
+      tc::tmem_ld64(tl + sb * kKB + half * kHalf, s);
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&sy.s_empty[sb]);
       // key key0 + c is visible to this row when cu_r <= key0 + c <= qpos
       const int lo = cu_r - key0, hi = qpos - key0;
-      if (__any_sync(0xffffffffu, lo > 0 || hi < kKB - 1)) {
+      if (__any_sync(0xffffffffu, lo > 0 || hi < kHalf - 1)) {
 #pragma unroll
-        for (int c = 0; c < kKB; ++c) s[c] = (c >= lo && c <= hi) ? s[c] : -INFINITY;
+        for (int c = 0; c < kHalf; ++c) s[c] = (c >= lo && c <= hi) ? s[c] : -INFINITY;
       }
-      // row max: eight running maxima (columns c mod 8), then their tree; exact in any order
+      // max: eight running maxima (columns c mod 8), then their tree; exact in any order
       float t[8];
 #pragma unroll
       for (int c = 0; c < 8; ++c) t[c] = s[c];
 #pragma unroll
-      for (int c = 8; c < kKB; ++c) t[c & 7] = fmaxf(t[c & 7], s[c]);
+      for (int c = 8; c < kHalf; ++c) t[c & 7] = fmaxf(t[c & 7], s[c]);
 #pragma unroll
       for (int w = 4; w >= 1; w >>= 1) {
 #pragma unroll
         for (int c = 0; c < w; ++c) t[c] = fmaxf(t[c], t[c + w]);
       }
-      const float mb = t[0] * c2;  // -inf when nothing in the block is visible
+      const float mb = t[0] * c2;  // -inf when nothing in the half is visible
       float factor = 1.f;
       bool resc = false;
       if (mb > m + kRescaleTau) {
@@ -285,18 +301,21 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         m = mb;
       }
       const float nm = (m == -INFINITY) ? 0.f : -m;
-      uint32_t pk[kKB / 2];
-      float l0 = 0.f, l1 = 0.f;
+      const float2 nn = make_float2(nm, nm);
+      uint32_t pk[kHalf / 2];
+      float2 acc0 = make_float2(0.f, 0.f), acc1 = acc0;
 #pragma unroll
-      for (int c = 0; c < kKB; c += 2) {
-        const float p0 = tc::ex2(fmaf(s[c], c2, nm));
-        const float p1 = tc::ex2(fmaf(s[c + 1], c2, nm));
-        l0 += p0;
-        l1 += p1;
+      for (int c = 0; c < kHalf; c += 4) {
+        const float2 z01 = tc::ffma2(make_float2(s[c], s[c + 1]), cc, nn);
+        const float2 z23 = tc::ffma2(make_float2(s[c + 2], s[c + 3]), cc, nn);
+        const float p0 = tc::ex2(z01.x), p1 = tc::ex2(z01.y), p2 = tc::ex2(z23.x), p3 = tc::ex2(z23.y);
+        acc0 = tc::add2(acc0, make_float2(p0, p1));
+        acc1 = tc::add2(acc1, make_float2(p2, p3));
         pk[c / 2] = pack_bf16x2(p0, p1);
+        pk[c / 2 + 1] = pack_bf16x2(p2, p3);
       }
-      l += l0 + l1;
-      // the P buffer is free and O is final up to block j - 1 once P_{j-1} V_{j-1} is done
+      l += (acc0.x + acc0.y) + (acc1.x + acc1.y);
+      // the P buffer is free and O_h is final up to block j - 1 once P_{j-1} V_{j-1} is done
       if (j >= 1) {
         if (!tc::mbar_wait_warp(&sy.pv_done, (j - 1) & 1)) {
           if (lane == 0) *abort_flag = 1;
@@ -307,21 +326,21 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         if (__any_sync(0xffffffffu, resc)) {
           for (int oc = 0; oc < d / 32; ++oc) {
             uint32_t ov[32];
-            tc::tmem_ld32_async(tl + kOCol + oc * 32, ov);
+            tc::tmem_ld32_async(tl + ocol + oc * 32, ov);
             tc::tmem_wait(ov);
 #pragma unroll
             for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * factor);
-            tmem_st32(tl + kOCol + oc * 32, ov);
+            tmem_st32(tl + ocol + oc * 32, ov);
           }
           tmem_wait_st();
         }
       }
-      // P row: two panels of 64 keys, 128 bytes per row, 16-byte chunk c of row i at
-      // chunk position c ^ (i % 8) (the layout a 128-byte-swizzled TMA load writes)
+      // this row of P panel `half`: 128 bytes, 16-byte chunk c at chunk position c ^ (row % 8)
+      // (the layout a 128-byte-swizzled TMA load writes)
 #pragma unroll
-      for (int c16 = 0; c16 < kKB / 8; ++c16) {
-        const int panel = c16 >> 3, ch = (c16 & 7) ^ (row & 7);
-        *reinterpret_cast<uint4*>(prow + panel * (kQT * 128) + ch * 16) =
+      for (int c16 = 0; c16 < kHalf / 8; ++c16) {
+        const int ch = c16 ^ (row & 7);
+        *reinterpret_cast<uint4*>(prow + ch * 16) =
             make_uint4(pk[4 * c16], pk[4 * c16 + 1], pk[4 * c16 + 2], pk[4 * c16 + 3]);
       }
       fence_proxy_async_smem();
@@ -329,26 +348,39 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&sy.p_full);
     }
-    if (ok && !__any_sync(0xffffffffu, *abort_flag != 0)) {
-      if (!tc::mbar_wait_warp(&sy.pv_done, (nblk - 1) & 1)) {
-        if (lane == 0) *abort_flag = 1;
-      } else {
-        tc::fence_after_sync();
-        const bool live = qpos <= q_last;
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        float* orow = a.o + static_cast<int64_t>(qpos) * a.o_stride + static_cast<int64_t>(h) * d;
-        for (int oc = 0; oc < d / 32; ++oc) {
-          float v[32];
-          tc::tmem_ld32(tl + kOCol + oc * 32, v);
-          if (live) {
+    bool fin = ok && !__any_sync(0xffffffffu, *abort_flag != 0);
+    if (fin && !tc::mbar_wait_warp(&sy.pv_done, (nblk - 1) & 1)) {
+      if (lane == 0) *abort_flag = 1;
+      fin = false;
+    }
+    // merge the two key halves of every row; every softmax warp passes this barrier once
+    s_ml[half][row] = make_float2(m, l);
+    bar_softmax();
+    if (fin) {
+      tc::fence_after_sync();
+      const float2 h0 = s_ml[0][row], h1 = s_ml[1][row];
+      const float M = fmaxf(h0.x, h1.x);
+      const float s0 = h0.x == -INFINITY ? 0.f : tc::ex2(h0.x - M);
+      const float s1 = h1.x == -INFINITY ? 0.f : tc::ex2(h1.x - M);
+      const float L = h0.y * s0 + h1.y * s1;
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      const float w0 = s0 * inv, w1 = s1 * inv;
+      const bool live = qpos <= q_last;
+      const int c0 = half * (d / 2);  // this warp writes output columns c0 .. c0 + d/2 - 1
+      float* orow = a.o + static_cast<int64_t>(qpos) * a.o_stride + static_cast<int64_t>(h) * d + c0;
+      for (int oc = 0; oc < d / 64; ++oc) {
+        float v0[32], v1[32];
+        tc::tmem_ld32(tl + kOCol + c0 + oc * 32, v0);
+        tc::tmem_ld32(tl + kOCol + kOHalf + c0 + oc * 32, v1);
+        if (live) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-              *reinterpret_cast<float4*>(orow + oc * 32 + 4 * i) =
-                  make_float4(v[4 * i] * inv, v[4 * i + 1] * inv, v[4 * i + 2] * inv, v[4 * i + 3] * inv);
-          }
+          for (int i = 0; i < 8; ++i)
+            *reinterpret_cast<float4*>(orow + oc * 32 + 4 * i) =
+                make_float4(v0[4 * i] * w0 + v1[4 * i] * w1, v0[4 * i + 1] * w0 + v1[4 * i + 1] * w1,
+                            v0[4 * i + 2] * w0 + v1[4 * i + 2] * w1, v0[4 * i + 3] * w0 + v1[4 * i + 3] * w1);
         }
-        if (live) a.lse[static_cast<int64_t>(h) * a.lse_stride + qpos] = (m + log2f(l)) * kLn2;
       }
+      if (live && half == 0) a.lse[static_cast<int64_t>(h) * a.lse_stride + qpos] = (M + log2f(L)) * kLn2;
     }
   }
   tc::fence_before_sync();
