@@ -13,8 +13,8 @@
 //
 // Per key block j:
 //   S_j = Q K_j^T        tcgen05, M = 128 queries, N = 128 keys, K = d; fp32 in TMEM
-//   P_j = exp2(c2 S_j - m)  softmax warps, bf16 into shared memory (128-byte swizzle)
-//   O  += P_j V_j        tcgen05, M = 128, N = d, K = 128 keys; fp32 in TMEM
+//   P_j = exp2(c2 S_j - m)  softmax warps, bf16, written back into S_j's own TMEM columns
+//   O  += P_j V_j        tcgen05 with A (P) read from TMEM, M = 128, N = d, K = 128 keys
 // with c2 = scale * log2(e). The two 64-key halves of every block are softmaxed by
 // different warps, each half of a row with its own reference max, sum and accumulator
 // (O_0 += P[:, 0:64] V[0:64], O_1 += P[:, 64:128] V[64:128]); the two halves of a row
@@ -28,7 +28,9 @@
 // and key half w / 4, so two warps share every SM sub-partition. Warp 8 issues the TMA
 // loads (Q once, K and Vt double-buffered). Warp 9 owns TMEM and issues the MMAs: S_j
 // before P_{j-1} V_{j-1}, so the softmax of block j overlaps the P V of block j - 1.
-// TMEM: S double buffer in columns 0-255, O_0 from column 256, O_1 from column 384.
+// TMEM: S double buffer in columns 0-255, O_0 from column 256, O_1 from column 384. P_j
+// lives in the first 32 columns of each key half of S_j (two bf16 per column), so S
+// buffer j % 2 is free again once P_j V_j has completed; P never touches shared memory.
 // Every wait is bounded; a CTA whose wait gives up records AVTP_ERR_TIMEOUT and returns.
 #include <cudaTypedefs.h>
 
@@ -55,20 +57,17 @@ constexpr float kLog2e = 1.4426950408889634f;
 __host__ __device__ constexpr size_t q_bytes(int d) { return static_cast<size_t>(kQT) * d * 2; }
 __host__ __device__ constexpr size_t k_bytes(int d) { return static_cast<size_t>(kKB) * d * 2; }
 __host__ __device__ constexpr size_t v_bytes(int d) { return static_cast<size_t>(d) * kKB * 2; }
-constexpr size_t kPBytes = static_cast<size_t>(kQT) * kKB * 2;
-__host__ __device__ constexpr size_t fwd_smem_bytes(int d) {
-  return 1024 + q_bytes(d) + 2 * k_bytes(d) + 2 * v_bytes(d) + kPBytes;
-}
-// Every head_dim requests the d = 128 size, so that no second CTA (and its 512 TMEM
-// columns) shares an SM.
-constexpr size_t kFwdSmem = fwd_smem_bytes(128);
+__host__ __device__ constexpr size_t fwd_smem_bytes(int d) { return 1024 + q_bytes(d) + 2 * k_bytes(d) + 2 * v_bytes(d); }
+// Every head_dim requests more than half the SM's shared memory, so that no second CTA
+// (and its 512 TMEM columns) shares an SM.
+constexpr size_t kFwdSmem = fwd_smem_bytes(128) > 116 * 1024 ? fwd_smem_bytes(128) : 116 * 1024;
 static_assert(kFwdSmem <= 227 * 1024, "shared memory of one CTA");
 
 struct FwdSync {
   uint64_t q_full;
   uint64_t k_full[2], k_empty[2];
   uint64_t v_full[2], v_empty[2];
-  uint64_t s_full[2], s_empty[2];
+  uint64_t s_full[2];
   uint64_t p_full, pv_done, drain;
   uint32_t tmem;
   int abort;
@@ -100,9 +99,15 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
       : "memory");
 }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-// Orders this thread's shared-memory stores before later tensor-core reads of them.
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+// D[tmem] (+)= A[tmem] * B^T for one K = 16 step, A (M x 16, two bf16 per column) read
+// from tensor memory; issued by a single thread.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
 }
 
 __device__ __forceinline__ void bar_softmax() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
@@ -128,7 +133,6 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
   // key stage b at sK + b * k_bytes(d), value stage b at sV + b * v_bytes(d)
   unsigned char* sK = sQ + q_bytes(d);
   unsigned char* sV = sK + 2 * k_bytes(d);
-  unsigned char* sP = sV + 2 * v_bytes(d);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   pdl_wait();
@@ -155,7 +159,6 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       tc::mbar_init(&sy.v_full[s], 1);
       tc::mbar_init(&sy.v_empty[s], 1);
       tc::mbar_init(&sy.s_full[s], 1);
-      tc::mbar_init(&sy.s_empty[s], kSoftWarps);
     }
     tc::mbar_init(&sy.p_full, kSoftWarps);
     tc::mbar_init(&sy.pv_done, 1);
@@ -205,9 +208,9 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idS = tc::idesc_bf16(kQT, kKB), idO = tc::idesc_bf16(kQT, d);
-      const uint32_t aQ = tc::smem_u32(sQ), aP = tc::smem_u32(sP);
-      // O_h += P_i[:, 64h .. 64h + 63] V_i[64h .. 64h + 63]: A = panel h of P (128 rows x 64
-      // keys), B = panel h of the Vt block (d rows x 64 keys)
+      const uint32_t aQ = tc::smem_u32(sQ);
+      // O_h += P_i[:, 64h .. 64h + 63] V_i[64h .. 64h + 63]: A = P's half h in TMEM (128 lanes
+      // x 32 columns), B = panel h of the Vt block (d rows x 64 keys)
       auto issue_pv = [&](int i) -> bool {
         const int sb = i & 1;
         if (!tc::mbar_wait(&sy.p_full, i & 1)) return false;
@@ -218,10 +221,9 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         for (int hh = 0; hh < 2; ++hh) {
 #pragma unroll
           for (int ks = 0; ks < kHalf / 16; ++ks) {
-            const uint32_t ap = aP + static_cast<uint32_t>(hh * (kQT * 128) + ks * 32);
+            const uint32_t ap = tmem + static_cast<uint32_t>(sb * kKB + hh * kHalf + ks * 8);
             const uint32_t bp = bV + static_cast<uint32_t>(hh * (d * 128) + ks * 32);
-            tc::mma_bf16(tmem + kOCol + hh * kOHalf, tc::desc_k_sw128(ap), tc::desc_k_sw128(bp), idO,
-                         (i > 0 || ks > 0) ? 1u : 0u);
+            mma_bf16_ts(tmem + kOCol + hh * kOHalf, ap, tc::desc_k_sw128(bp), idO, (i > 0 || ks > 0) ? 1u : 0u);
           }
         }
         tc::mma_commit(&sy.pv_done);
@@ -232,7 +234,8 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       for (int j = 0; ok && j < nblk && !*abort_flag; ++j) {
         const int sb = j & 1;
         if (!tc::mbar_wait(&sy.k_full[sb], (j >> 1) & 1)) { ok = false; break; }
-        if (j >= 2 && !tc::mbar_wait(&sy.s_empty[sb], ((j >> 1) - 1) & 1)) { ok = false; break; }
+        // S buffer sb holds P_{j-2} until P_{j-2} V_{j-2} has completed
+        if (j >= 2 && !tc::mbar_wait(&sy.pv_done, (j - 2) & 1)) { ok = false; break; }
         tc::fence_after_sync();
         tc::mma_rows(tmem + sb * kKB, aQ, kQT * 128, tc::smem_u32(sK + sb * k_bytes(d)), kKB * 128, d, idS);
         tc::mma_commit(&sy.s_full[sb]);
@@ -256,7 +259,6 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
     const float2 cc = make_float2(c2, c2);
     float m = -INFINITY, l = 0.f;  // reference max (log2 units) and sum of exp2(c2 s - m), this half
     bool ok = true;
-    unsigned char* prow = sP + half * (kQT * 128) + row * 128;  // this row of P panel `half`
     for (int j = 0; j < nblk; ++j) {
       const int sb = j & 1;
       const int key0 = (kb0 + j) * kKB + half * kHalf;
@@ -269,9 +271,6 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       tc::fence_after_sync();
       float s[kHalf];
       tc::tmem_ld64(tl + sb * kKB + half * kHalf, s);
-      tc::fence_before_sync();
-      __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&sy.s_empty[sb]);
       // key key0 + c is visible to this row when cu_r <= key0 + c <= qpos
       const int lo = cu_r - key0, hi = qpos - key0;
       if (__any_sync(0xffffffffu, lo > 0 || hi < kHalf - 1)) {
@@ -315,15 +314,15 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         pk[c / 2 + 1] = pack_bf16x2(p2, p3);
       }
       l += (acc0.x + acc0.y) + (acc1.x + acc1.y);
-      // the P buffer is free and O_h is final up to block j - 1 once P_{j-1} V_{j-1} is done
-      if (j >= 1) {
+      // O_h is final up to block j - 1 once P_{j-1} V_{j-1} is done: rescaling waits for it
+      if (j >= 1 && __any_sync(0xffffffffu, resc)) {
         if (!tc::mbar_wait_warp(&sy.pv_done, (j - 1) & 1)) {
           if (lane == 0) *abort_flag = 1;
           ok = false;
           break;
         }
         tc::fence_after_sync();
-        if (__any_sync(0xffffffffu, resc)) {
+        {
           for (int oc = 0; oc < d / 32; ++oc) {
             uint32_t ov[32];
             tc::tmem_ld32_async(tl + ocol + oc * 32, ov);
@@ -335,15 +334,9 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
           tmem_wait_st();
         }
       }
-      // this row of P panel `half`: 128 bytes, 16-byte chunk c at chunk position c ^ (row % 8)
-      // (the layout a 128-byte-swizzled TMA load writes)
-#pragma unroll
-      for (int c16 = 0; c16 < kHalf / 8; ++c16) {
-        const int ch = c16 ^ (row & 7);
-        *reinterpret_cast<uint4*>(prow + ch * 16) =
-            make_uint4(pk[4 * c16], pk[4 * c16 + 1], pk[4 * c16 + 2], pk[4 * c16 + 3]);
-      }
-      fence_proxy_async_smem();
+      // P_j's half: the first 32 columns of this half of S_j, already read into registers
+      tmem_st32(tl + sb * kKB + half * kHalf, pk);
+      tmem_wait_st();
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&sy.p_full);
