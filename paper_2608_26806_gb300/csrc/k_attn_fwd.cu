@@ -12,25 +12,26 @@
 // request or after the query are masked.
 //
 // Per key block j:
-//   S_j = Q K_j^T        tcgen05, M = 128 queries, N = 128 keys, K = d; fp32 in TMEM
-//   P_j = exp2(c2 S_j - m)  softmax warps, bf16, written back into S_j's own TMEM columns
-//   O  += P_j V_j        tcgen05 with A (P) read from TMEM, M = 128, N = d, K = 128 keys
-// with c2 = scale * log2(e). The two 64-key halves of every block are softmaxed by
-// different warps, each half of a row with its own reference max, sum and accumulator
-// (O_0 += P[:, 0:64] V[0:64], O_1 += P[:, 64:128] V[64:128]); the two halves of a row
-// are merged once, in the epilogue, the way split-key partial softmaxes combine. A
-// half's reference max moves only when a block's max exceeds it by more than 8 (log2
-// units), so its accumulator in TMEM is rescaled rarely and every P entry stays below
-// 2^8. P V needs V with keys contiguous (the MMA's K-major operand), so a first kernel
-// writes the values transposed, Vt[g][c][t].
+//   S_j = Q K_j^T           tcgen05 with A (Q) read from TMEM, M = 128 queries, N = 128 keys
+//   P_j = exp2(c2 S_j - m)  softmax warps; bf16, two per column, into a TMEM P buffer
+//   O  += P_j V_j           tcgen05 with A (P) read from TMEM, M = 128, N = d, K = 128 keys
+// with c2 = scale * log2(e). A row's reference max m moves only when a block's max
+// exceeds it by more than 8 (log2 units), so the accumulator in TMEM is rescaled rarely
+// and every P entry stays below 2^8. P V needs V with keys contiguous (the MMA's K-major
+// operand), so a first kernel writes the values transposed, Vt[g][c][t].
 //
-// Warps 0-7: softmax and epilogue; warp w owns query rows 32 (w % 4) .. + 31 (TMEM lanes)
-// and key half w / 4, so two warps share every SM sub-partition. Warp 8 issues the TMA
-// loads (Q once, K and Vt double-buffered). Warp 9 owns TMEM and issues the MMAs: S_j
-// before P_{j-1} V_{j-1}, so the softmax of block j overlaps the P V of block j - 1.
-// TMEM: S double buffer in columns 0-255, O_0 from column 256, O_1 from column 384. P_j
-// lives in the first 32 columns of each key half of S_j (two bf16 per column), so S
-// buffer j % 2 is free again once P_j V_j has completed; P never touches shared memory.
+// Warps 0-7: softmax and epilogue. Warp w owns query rows 32 (w % 4) .. + 31 (TMEM lanes)
+// and key half w / 4 of every block, so two warps share every SM sub-partition; the two
+// warps of a row range exchange their half maxima through shared memory once per block
+// (a 64-thread named barrier), so a row has one reference max and one accumulator. Warp
+// 8 issues the TMA loads (Q once, K and Vt double-buffered). Warp 9 owns TMEM and issues
+// the MMAs in the order S_{j+1}, P_j V_j: S_{j+1} as soon as the softmax has read S_j
+// out of TMEM, P_j V_j once P_j is written, so the tensor core has the next block's work
+// queued while the softmax runs. One thread issues every MMA, and an MMA is issued no
+// faster than the tensor core takes its operands, so the operands come from TMEM where
+// they can: Q (copied there once by the softmax warps) and P are the A operands, and
+// only K and V are read from shared memory. TMEM: S in columns 0-127, P buffers in
+// 128-255 (64 columns each), Q in 256-319, O in 384 .. 384 + d.
 // Every wait is bounded; a CTA whose wait gives up records AVTP_ERR_TIMEOUT and returns.
 #include <cudaTypedefs.h>
 
@@ -48,8 +49,10 @@ constexpr int kSoftWarps = 8;
 constexpr int kTmaWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kOCol = 256;   // O_0; O_1 at kOCol + kOHalf
-constexpr uint32_t kOHalf = 128;
+constexpr uint32_t kSCol = 0;
+constexpr uint32_t kPCol = 128;  // P buffer b at kPCol + 64 b (two bf16 per column)
+constexpr uint32_t kQCol = 256;  // Q, two bf16 per column (d / 2 columns)
+constexpr uint32_t kOCol = 384;
 constexpr float kRescaleTau = 8.f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -67,8 +70,10 @@ struct FwdSync {
   uint64_t q_full;
   uint64_t k_full[2], k_empty[2];
   uint64_t v_full[2], v_empty[2];
-  uint64_t s_full[2];
-  uint64_t p_full, pv_done, drain;
+  uint64_t q_tmem;                 // Q copied into TMEM by the softmax warps
+  uint64_t s_full, s_empty;        // S: written by the MMA / read out by the softmax
+  uint64_t p_full[2], pv_done[2];  // P buffer b: written by the softmax / read by P V
+  uint64_t drain;
   uint32_t tmem;
   int abort;
 };
@@ -110,7 +115,19 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       : "memory");
 }
 
-__device__ __forceinline__ void bar_softmax() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+__device__ __forceinline__ void bar_softmax() { asm volatile("bar.sync 5, 256;" ::: "memory"); }
+// Barrier of the two softmax warps of TMEM lane quadrant `quad` (ids 1-4, 64 threads); true
+// when `bad` holds for any of their threads.
+__device__ __forceinline__ bool bar_pair_any(int quad, bool bad) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %2, 0;\n\t"
+      "barrier.red.or.pred q, %1, 64, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(1 + quad), "r"(bad ? 1u : 0u)
+      : "memory");
+  return r != 0;
+}
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
@@ -125,7 +142,8 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
            const __grid_constant__ CUtensorMap mapV, FwdArgs a) {
   extern __shared__ unsigned char smem_raw[];
   __shared__ FwdSync sy;
-  __shared__ float2 s_ml[2][kQT];  // (reference max, sum) of each key half of each row
+  __shared__ float2 s_ml[2][kQT];    // (reference max, sum over the half) of each row, at the end
+  __shared__ float s_mx[2][2][kQT];   // [S buffer][key half][row]: block max of the half
   unsigned char* smem =
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int d = a.d;
@@ -158,10 +176,12 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       tc::mbar_init(&sy.k_empty[s], 1);
       tc::mbar_init(&sy.v_full[s], 1);
       tc::mbar_init(&sy.v_empty[s], 1);
-      tc::mbar_init(&sy.s_full[s], 1);
+      tc::mbar_init(&sy.p_full[s], kSoftWarps);
+      tc::mbar_init(&sy.pv_done[s], 1);
     }
-    tc::mbar_init(&sy.p_full, kSoftWarps);
-    tc::mbar_init(&sy.pv_done, 1);
+    tc::mbar_init(&sy.q_tmem, kSoftWarps);
+    tc::mbar_init(&sy.s_full, 1);
+    tc::mbar_init(&sy.s_empty, kSoftWarps);
     tc::mbar_init(&sy.drain, 1);
     sy.abort = 0;
     tc::fence_mbar_init();
@@ -208,41 +228,46 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idS = tc::idesc_bf16(kQT, kKB), idO = tc::idesc_bf16(kQT, d);
-      const uint32_t aQ = tc::smem_u32(sQ);
-      // O_h += P_i[:, 64h .. 64h + 63] V_i[64h .. 64h + 63]: A = P's half h in TMEM (128 lanes
-      // x 32 columns), B = panel h of the Vt block (d rows x 64 keys)
+      // S_j = Q K_j^T into S, once the softmax has read S_{j-1} out of it: A = Q in TMEM
+      // (128 lanes x d / 2 columns), B = key stage j % 2 (128 keys x d, K-major)
+      auto issue_s = [&](int j) -> bool {
+        const int sb = j & 1;
+        if (!tc::mbar_wait(&sy.k_full[sb], (j >> 1) & 1)) return false;
+        if (j >= 1 && !tc::mbar_wait(&sy.s_empty, (j - 1) & 1)) return false;
+        tc::fence_after_sync();
+        const uint32_t bK = tc::smem_u32(sK + sb * k_bytes(d));
+        for (int ks = 0; ks < d / 16; ++ks) {
+          const uint32_t bp = bK + static_cast<uint32_t>((ks >> 2) * (kKB * 128) + (ks & 3) * 32);
+          mma_bf16_ts(tmem + kSCol, tmem + kQCol + static_cast<uint32_t>(ks * 8), tc::desc_k_sw128(bp), idS,
+                      ks > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(&sy.s_full);
+        tc::mma_commit(&sy.k_empty[sb]);
+        return true;
+      };
+      // O += P_i V_i: A = P buffer i % 2 in TMEM (128 lanes x 64 columns), B = the Vt block
+      // (d rows x 128 keys, two 64-key panels)
       auto issue_pv = [&](int i) -> bool {
         const int sb = i & 1;
-        if (!tc::mbar_wait(&sy.p_full, i & 1)) return false;
+        if (!tc::mbar_wait(&sy.p_full[sb], (i >> 1) & 1)) return false;
         if (!tc::mbar_wait(&sy.v_full[sb], (i >> 1) & 1)) return false;
         tc::fence_after_sync();
         const uint32_t bV = tc::smem_u32(sV + sb * v_bytes(d));
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-#pragma unroll
-          for (int ks = 0; ks < kHalf / 16; ++ks) {
-            const uint32_t ap = tmem + static_cast<uint32_t>(sb * kKB + hh * kHalf + ks * 8);
-            const uint32_t bp = bV + static_cast<uint32_t>(hh * (d * 128) + ks * 32);
-            mma_bf16_ts(tmem + kOCol + hh * kOHalf, ap, tc::desc_k_sw128(bp), idO, (i > 0 || ks > 0) ? 1u : 0u);
-          }
+        for (int ks = 0; ks < kKB / 16; ++ks) {
+          const uint32_t ap = tmem + kPCol + static_cast<uint32_t>(sb * 64 + ks * 8);
+          const uint32_t bp = bV + static_cast<uint32_t>((ks >> 2) * (d * 128) + (ks & 3) * 32);
+          mma_bf16_ts(tmem + kOCol, ap, tc::desc_k_sw128(bp), idO, (i > 0 || ks > 0) ? 1u : 0u);
         }
-        tc::mma_commit(&sy.pv_done);
+        tc::mma_commit(&sy.pv_done[sb]);
         tc::mma_commit(&sy.v_empty[sb]);
         return true;
       };
-      bool ok = tc::mbar_wait(&sy.q_full, 0);
+      bool ok = tc::mbar_wait(&sy.q_tmem, 0) && issue_s(0);
       for (int j = 0; ok && j < nblk && !*abort_flag; ++j) {
-        const int sb = j & 1;
-        if (!tc::mbar_wait(&sy.k_full[sb], (j >> 1) & 1)) { ok = false; break; }
-        // S buffer sb holds P_{j-2} until P_{j-2} V_{j-2} has completed
-        if (j >= 2 && !tc::mbar_wait(&sy.pv_done, (j - 2) & 1)) { ok = false; break; }
-        tc::fence_after_sync();
-        tc::mma_rows(tmem + sb * kKB, aQ, kQT * 128, tc::smem_u32(sK + sb * k_bytes(d)), kKB * 128, d, idS);
-        tc::mma_commit(&sy.s_full[sb]);
-        tc::mma_commit(&sy.k_empty[sb]);
-        if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
+        if (j + 1 < nblk && !issue_s(j + 1)) { ok = false; break; }
+        if (!issue_pv(j)) { ok = false; break; }
       }
-      if (ok && !*abort_flag && !issue_pv(nblk - 1)) ok = false;
       if (!ok) *abort_flag = 1;
       // every MMA issued has completed once this arrives
       tc::mma_commit(&sy.drain);
@@ -254,41 +279,71 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
     const int row = quad * 32 + lane;
     const int qpos = q0 + row;
     const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16);  // this warp's TMEM lanes
-    const uint32_t ocol = kOCol + half * kOHalf;                           // this half's accumulator
+    const int oc0 = half * (d / 2);  // O columns this warp rescales and writes out
     const float c2 = a.c2;
     const float2 cc = make_float2(c2, c2);
-    float m = -INFINITY, l = 0.f;  // reference max (log2 units) and sum of exp2(c2 s - m), this half
-    bool ok = true;
+    float m = -INFINITY, l = 0.f;  // row reference max (log2 units); sum of exp2(c2 s - m) over this half
+    bool bad = false;               // a wait gave up (here or, through the pair barrier, in the partner)
+    // Q into TMEM: warp (quad, half) copies 64-element panel `half` of its 32 rows (d = 64:
+    // half 0 alone), unswizzling the 128-byte TMA layout (16-byte chunk c of row r at
+    // chunk position c ^ (r % 8))
+    if (!tc::mbar_wait_warp(&sy.q_full, 0)) bad = true;
+    if (!bad && half < d / 64) {
+      const unsigned char* qrow = sQ + half * (kQT * 128) + row * 128;
+      uint32_t qv[32];
+#pragma unroll
+      for (int c16 = 0; c16 < 8; ++c16) {
+        const uint4 u = *reinterpret_cast<const uint4*>(qrow + ((c16 ^ (row & 7)) << 4));
+        qv[4 * c16] = u.x;
+        qv[4 * c16 + 1] = u.y;
+        qv[4 * c16 + 2] = u.z;
+        qv[4 * c16 + 3] = u.w;
+      }
+      tmem_st32(tl + kQCol + half * 32, qv);
+      tmem_wait_st();
+    }
+    tc::fence_before_sync();
+    __syncwarp();
+    if (!bad && lane == 0) tc::mbar_arrive(&sy.q_tmem);
     for (int j = 0; j < nblk; ++j) {
       const int sb = j & 1;
       const int key0 = (kb0 + j) * kKB + half * kHalf;
-      if (__any_sync(0xffffffffu, *abort_flag != 0)) { ok = false; break; }
-      if (!tc::mbar_wait_warp(&sy.s_full[sb], (j >> 1) & 1)) {
+      bad = bad || __any_sync(0xffffffffu, *abort_flag != 0);
+      if (!bad && !tc::mbar_wait_warp(&sy.s_full, j & 1)) bad = true;
+      float s[kHalf];
+      float mh = -INFINITY;
+      if (!bad) {
+        tc::fence_after_sync();
+        tc::tmem_ld64(tl + kSCol + half * kHalf, s);
+        tc::fence_before_sync();
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&sy.s_empty);
+        // key key0 + c is visible to this row when cu_r <= key0 + c <= qpos
+        const int lo = cu_r - key0, hi = qpos - key0;
+        if (__any_sync(0xffffffffu, lo > 0 || hi < kHalf - 1)) {
+#pragma unroll
+          for (int c = 0; c < kHalf; ++c) s[c] = (c >= lo && c <= hi) ? s[c] : -INFINITY;
+        }
+        // max: eight running maxima (columns c mod 8), then their tree; exact in any order
+        float t[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) t[c] = s[c];
+#pragma unroll
+        for (int c = 8; c < kHalf; ++c) t[c & 7] = fmaxf(t[c & 7], s[c]);
+#pragma unroll
+        for (int w = 4; w >= 1; w >>= 1) {
+#pragma unroll
+          for (int c = 0; c < w; ++c) t[c] = fmaxf(t[c], t[c + w]);
+        }
+        mh = t[0];
+      }
+      // the row's block max from both halves; both warps of the pair leave together
+      s_mx[sb][half][row] = mh;
+      if (bar_pair_any(quad, bad)) {
         if (lane == 0) *abort_flag = 1;
-        ok = false;
         break;
       }
-      tc::fence_after_sync();
-      float s[kHalf];
-      tc::tmem_ld64(tl + sb * kKB + half * kHalf, s);
-      // key key0 + c is visible to this row when cu_r <= key0 + c <= qpos
-      const int lo = cu_r - key0, hi = qpos - key0;
-      if (__any_sync(0xffffffffu, lo > 0 || hi < kHalf - 1)) {
-#pragma unroll
-        for (int c = 0; c < kHalf; ++c) s[c] = (c >= lo && c <= hi) ? s[c] : -INFINITY;
-      }
-      // max: eight running maxima (columns c mod 8), then their tree; exact in any order
-      float t[8];
-#pragma unroll
-      for (int c = 0; c < 8; ++c) t[c] = s[c];
-#pragma unroll
-      for (int c = 8; c < kHalf; ++c) t[c & 7] = fmaxf(t[c & 7], s[c]);
-#pragma unroll
-      for (int w = 4; w >= 1; w >>= 1) {
-#pragma unroll
-        for (int c = 0; c < w; ++c) t[c] = fmaxf(t[c], t[c + w]);
-      }
-      const float mb = t[0] * c2;  // -inf when nothing in the half is visible
+      const float mb = fmaxf(mh, s_mx[sb][half ^ 1][row]) * c2;  // -inf when nothing is visible
       float factor = 1.f;
       bool resc = false;
       if (mb > m + kRescaleTau) {
@@ -314,66 +369,61 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         pk[c / 2 + 1] = pack_bf16x2(p2, p3);
       }
       l += (acc0.x + acc0.y) + (acc1.x + acc1.y);
-      // O_h is final up to block j - 1 once P_{j-1} V_{j-1} is done: rescaling waits for it
+      // O is final up to block j - 1 once P_{j-1} V_{j-1} is done: a rescale waits for it and
+      // scales this warp's half of the columns (both warps of the pair took the same factor)
       if (j >= 1 && __any_sync(0xffffffffu, resc)) {
-        if (!tc::mbar_wait_warp(&sy.pv_done, (j - 1) & 1)) {
-          if (lane == 0) *abort_flag = 1;
-          ok = false;
-          break;
+        if (!tc::mbar_wait_warp(&sy.pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1)) {
+          bad = true;
+          continue;  // to the next pair barrier, where both warps stop
         }
         tc::fence_after_sync();
-        {
-          for (int oc = 0; oc < d / 32; ++oc) {
-            uint32_t ov[32];
-            tc::tmem_ld32_async(tl + ocol + oc * 32, ov);
-            tc::tmem_wait(ov);
+        for (int oc = 0; oc < d / 64; ++oc) {
+          uint32_t ov[32];
+          tc::tmem_ld32_async(tl + kOCol + oc0 + oc * 32, ov);
+          tc::tmem_wait(ov);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * factor);
-            tmem_st32(tl + ocol + oc * 32, ov);
-          }
-          tmem_wait_st();
+          for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * factor);
+          tmem_st32(tl + kOCol + oc0 + oc * 32, ov);
         }
+        tmem_wait_st();
       }
-      // P_j's half: the first 32 columns of this half of S_j, already read into registers
-      tmem_st32(tl + sb * kKB + half * kHalf, pk);
+      // P buffer sb is free once P_{j-2} V_{j-2} has completed
+      if (j >= 2 && !tc::mbar_wait_warp(&sy.pv_done[sb], ((j >> 1) - 1) & 1)) {
+        bad = true;
+        continue;
+      }
+      tc::fence_after_sync();
+      tmem_st32(tl + kPCol + sb * 64 + half * 32, pk);
       tmem_wait_st();
       tc::fence_before_sync();
       __syncwarp();
-      if (lane == 0) tc::mbar_arrive(&sy.p_full);
+      if (lane == 0) tc::mbar_arrive(&sy.p_full[sb]);
     }
-    bool fin = ok && !__any_sync(0xffffffffu, *abort_flag != 0);
-    if (fin && !tc::mbar_wait_warp(&sy.pv_done, (nblk - 1) & 1)) {
+    bool fin = !bad && !__any_sync(0xffffffffu, *abort_flag != 0);
+    if (fin && !tc::mbar_wait_warp(&sy.pv_done[(nblk - 1) & 1], ((nblk - 1) >> 1) & 1)) {
       if (lane == 0) *abort_flag = 1;
       fin = false;
     }
-    // merge the two key halves of every row; every softmax warp passes this barrier once
+    // the row's sum over both halves; every softmax warp passes this barrier once
     s_ml[half][row] = make_float2(m, l);
     bar_softmax();
     if (fin) {
       tc::fence_after_sync();
-      const float2 h0 = s_ml[0][row], h1 = s_ml[1][row];
-      const float M = fmaxf(h0.x, h1.x);
-      const float s0 = h0.x == -INFINITY ? 0.f : tc::ex2(h0.x - M);
-      const float s1 = h1.x == -INFINITY ? 0.f : tc::ex2(h1.x - M);
-      const float L = h0.y * s0 + h1.y * s1;
+      const float L = s_ml[0][row].y + s_ml[1][row].y;
       const float inv = L > 0.f ? 1.f / L : 0.f;
-      const float w0 = s0 * inv, w1 = s1 * inv;
       const bool live = qpos <= q_last;
-      const int c0 = half * (d / 2);  // this warp writes output columns c0 .. c0 + d/2 - 1
-      float* orow = a.o + static_cast<int64_t>(qpos) * a.o_stride + static_cast<int64_t>(h) * d + c0;
+      float* orow = a.o + static_cast<int64_t>(qpos) * a.o_stride + static_cast<int64_t>(h) * d + oc0;
       for (int oc = 0; oc < d / 64; ++oc) {
-        float v0[32], v1[32];
-        tc::tmem_ld32(tl + kOCol + c0 + oc * 32, v0);
-        tc::tmem_ld32(tl + kOCol + kOHalf + c0 + oc * 32, v1);
+        float v[32];
+        tc::tmem_ld32(tl + kOCol + oc0 + oc * 32, v);
         if (live) {
 #pragma unroll
           for (int i = 0; i < 8; ++i)
             *reinterpret_cast<float4*>(orow + oc * 32 + 4 * i) =
-                make_float4(v0[4 * i] * w0 + v1[4 * i] * w1, v0[4 * i + 1] * w0 + v1[4 * i + 1] * w1,
-                            v0[4 * i + 2] * w0 + v1[4 * i + 2] * w1, v0[4 * i + 3] * w0 + v1[4 * i + 3] * w1);
+                make_float4(v[4 * i] * inv, v[4 * i + 1] * inv, v[4 * i + 2] * inv, v[4 * i + 3] * inv);
         }
       }
-      if (live && half == 0) a.lse[static_cast<int64_t>(h) * a.lse_stride + qpos] = (M + log2f(L)) * kLn2;
+      if (live && half == 0) a.lse[static_cast<int64_t>(h) * a.lse_stride + qpos] = (m + log2f(L)) * kLn2;
     }
   }
   tc::fence_before_sync();
