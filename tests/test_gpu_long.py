@@ -95,3 +95,38 @@ def test_prune_long_workload(long_workload, criterion):
         b = exp["budgets"].reshape(lay.n_requests, -1)
         strong = wl.signal.reshape(lay.n_requests, -1) > 1.0
         assert np.all(b[strong].min() > b[~strong].max())
+
+
+def test_attention_forward_long_workload(long_workload):
+    """The layer's attention forward over all 264,192 tokens: sampled rows (tile edges, the
+    middle, the last token) of requests 0 and 3 against the oracle's per-row forward, at
+    the bound of the bf16 probabilities (2^-8 of the forward of |v|). Request 3's rows of O
+    start 3.2 GB into the output, past 2^31 bytes, where a 32-bit offset would show. Criterion B's scores from the
+    forward's LSE on every visual key of request 3."""
+    wl, dw = long_workload
+    lay = wl.layout
+    synth.build_tensors(wl, parts=("V",))  # the values only; the other tensors stay as drawn
+    v = torch.from_numpy(np.ascontiguousarray(wl.v).view(np.int16)).cuda().view(torch.bfloat16)
+    Hq, Hkv = wl.n_q_heads, wl.n_kv_heads
+    o, lse, scores, _ = avtp.attn_forward(dw.L, q=dw.t["q"], k=dw.t["k"], v=v, softmax_scale=wl.softmax_scale)
+    torch.cuda.synchronize()
+    v_abs = (wl.v & np.uint16(0x7FFF)).astype(np.uint16)
+    for r in (0, lay.n_requests - 1):
+        a, b = int(lay.cu_seqlens[r]), int(lay.cu_seqlens[r + 1])
+        n = b - a
+        if r == lay.n_requests - 1:
+            assert a * Hq * wl.head_dim * 4 > 2 ** 31  # O rows of the last request start past 2^31 bytes
+        rows = sorted({0, 127, 128, n // 2, n - 129, n - 1})
+        ref_o, ref_lse = O.attention_forward_rows(lay, wl.q, wl.k, wl.v, Hq, Hkv, wl.softmax_scale, r, rows)
+        ref_abs, _ = O.attention_forward_rows(lay, wl.q, wl.k, v_abs, Hq, Hkv, wl.softmax_scale, r, rows)
+        g = [a + p for p in rows]
+        got_o = o[g].cpu().numpy()
+        assert np.all(np.abs(got_o - ref_o) <= 2.0 ** -8 * ref_abs + 1e-5), f"request {r}"
+        np.testing.assert_allclose(lse[:, g].cpu().numpy(), ref_lse, rtol=RTOL, atol=ATOL, err_msg=f"request {r}")
+    sub, a, b = _request(wl, lay.n_requests - 1)
+    ref = O.score_text_attention(sub, wl.q[a:b], wl.k[a:b], Hq, Hkv, wl.softmax_scale)
+    vis = sub.visual_mask()
+    np.testing.assert_allclose(scores.cpu().numpy()[a:b][vis], ref[vis], rtol=RTOL, atol=ATOL)
+    del o, lse, scores, v
+    wl.tensors.pop("v")
+    torch.cuda.empty_cache()
