@@ -84,3 +84,21 @@ def test_stage_roofline_takes_the_slower_bound():
     r = bench.stage_roofline(acct, 0.004, 6794.1, 1910.0, "measured")
     assert r["bound"] == "tensor"
     assert abs(r["frac"] - 0.25) < 1e-4
+
+
+def test_forward_flops_equal_brute_force_mask_counts():
+    # the forward's FLOPs: Q K^T and P V, 2 d each per query head and visible (query, key)
+    # pair, pairs counted from an explicit causal mask per request
+    rng = np.random.default_rng(5)
+    for _ in range(20):
+        reqs = [[("t", int(rng.integers(1, 9))), ("i", int(rng.integers(1, 9)))] for _ in range(int(rng.integers(1, 4)))]
+        wl = _wl(reqs, Hq=int(rng.integers(1, 5)), d=int(rng.choice([4, 8])))
+        cu = wl.layout.cu_seqlens
+        pairs = 0
+        for r in range(len(cu) - 1):
+            n = int(cu[r + 1] - cu[r])
+            pairs += int(np.tril(np.ones((n, n), dtype=np.int64)).sum())
+        assert bench.forward_flops(wl) == 4 * wl.head_dim * wl.n_q_heads * pairs
+    # the Qwen3-VL-8B-shaped request: 796 GFLOP
+    q3 = synth.make_workload("qwen3_vl_8b", parts=())
+    assert bench.forward_flops(q3) == 795_857_649_664
