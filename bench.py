@@ -417,7 +417,7 @@ def run_ours(args, world, rank, local):
             "ms_per_step": round(ms3, 5), "steps": sec_last["steps"], "latency_us": sec_last["latency_us"],
             "steps_us": sec_last["steps_us"],
             "stage_roofline": stage_roofline(a3, ms3, hbm_s, bf16_s, peak_kind),
-            "score_roofline": {"bound": "hbm", "kernel": "score (logits + mass + finalize)",
+            "score_roofline": {"bound": "hbm", "kernel": "score (logits + mass)",
                                "achieved": round(a3["score_bytes"] / (score_us * 1e-6) / 1e9, 1), "peak": hbm_s,
                                "unit": "GB/s",
                                "frac": round(a3["score_bytes"] / (score_us * 1e-6) / 1e9 / hbm_s, 4),
@@ -574,7 +574,10 @@ def time_secondary(args, wl, L, kr, h_cur, pos, bf16, stream, flush, torch, avtp
             "latency_us": {"p50": round(step_ms[len(step_ms) // 2] * 1e3, 2),
                            "p90": round(step_ms[int(len(step_ms) * 0.9)] * 1e3, 2)},
             "steps_us": {k: round(v * 1e3, 2) for k, v in per_step.items()},
-            "launches": K * ((7 if lse is None else 6) if query_set == "text" else 7)}
+            # k_prep, k_attn_pack, k_attn_lse (computed LSE only), k_attn_mass, k_attn_finalize,
+            # k_alloc_select, k_compact; the last-token set: k_prep, k_narrow_logits,
+            # k_narrow_mass, k_alloc_select, k_compact
+            "launches": K * ((7 if lse is None else 6) if query_set == "text" else 5)}
 
 
 def forward_flops(wl):
