@@ -452,8 +452,10 @@ avtp_status_t avtp_pruned_layout(const avtp_layout_t* layout, const int32_t* bud
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   PrepArgs pa{};
   pa.L = *layout;
-  if ((st = from_cuda(launch_prep(pa, workspace, p, s))) != AVTP_OK) return st;
-  return from_cuda(launch_pruned_layout(*layout, budgets, out_img_start, out_img_len, workspace, p, s));
+  pa.pl_budgets = budgets;
+  pa.pl_out_start = out_img_start;
+  pa.pl_out_len = out_img_len;
+  return from_cuda(launch_prep(pa, workspace, p, s));
 }
 
 int64_t avtp_kept_count_vis_host(const int32_t* cu_seqlens, const int32_t* n_vis, const float* keep_ratio,

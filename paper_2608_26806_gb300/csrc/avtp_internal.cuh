@@ -320,6 +320,10 @@ struct PrepArgs {
   int64_t* zero_img_sums;    // NULL: not zeroed
   int build_text_tiles;      // criterion B bookkeeping, sized by `attn`
   AttnPlan attn;
+  // The image spans of the pruned batch (avtp_pruned_layout), from these budgets; NULL: none.
+  const int32_t* pl_budgets;
+  int32_t* pl_out_start;
+  int32_t* pl_out_len;
 };
 cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s);
 
@@ -360,8 +364,6 @@ constexpr int kMaxWarmCtas = 96;
 int prune_reserve_sms(const avtp_layout_t& L);
 int prune_warm_ctas(const avtp_layout_t& L);
 
-cudaError_t launch_pruned_layout(const avtp_layout_t& L, const int32_t* budgets, int32_t* out_start, int32_t* out_len,
-                                 void* ws, const WsPlan& p, cudaStream_t s);
 
 cudaError_t launch_compact(const int32_t* kept_idx, int64_t n_kept, int64_t n_tokens, const avtp_rows_t* sets,
                            int n_sets, void* ws, const WsPlan& p, cudaStream_t s);

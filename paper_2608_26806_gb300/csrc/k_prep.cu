@@ -5,7 +5,8 @@
 // Writes into the workspace: the status word, vis_cu (visual-token prefix over
 // all images), img_req (request of each image), and optionally the global
 // budgets B_r = floor(r_base * N_vis + 0.5) (paper §3.3.3 base keep ratio),
-// out_cu_seqlens, and the text-query bookkeeping of the attention criterion.
+// out_cu_seqlens, the text-query bookkeeping of the attention criterion, and the
+// image spans of the pruned batch (progressive pruning, paper §3.3.2).
 #include "avtp_internal.cuh"
 
 namespace avtp {
@@ -58,7 +59,7 @@ constexpr int kStageInts = 2560;
 __global__ void __launch_bounds__(kPrepThreads)
 k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t* req_budget, int32_t* text_idx,
        int32_t* text_cu, int32_t* blk_cu, int32_t* p1s_cu, int32_t* p2t_cu, int32_t* ktile_cu, int32_t* ktile_img,
-       int32_t* meta) {
+       int32_t* meta, int32_t* g_scratch) {
   __shared__ int s_err, s_detail, s_max_steps;
   __shared__ int32_t s_warp[32];
   __shared__ int32_t s_stage[kStageInts];
@@ -267,47 +268,39 @@ k_prep(PrepArgs a, DevStatus* st, int32_t* g_vis_cu, int32_t* g_img_req, int32_t
     st->layout_ok = (s_err == 0) ? 1 : 0;
     timeline_stamp(st, kTlPrepEnd);
   }
-}
-
-// The image spans of the pruned batch: image i of request r moves left by the tokens
-// pruned from the request's earlier images and keeps budgets[i] tokens. One CTA: an
-// exclusive scan of the pruned counts over all images, less the request's first entry.
-__global__ void __launch_bounds__(kPrepThreads)
-k_pruned_layout(avtp_layout_t L, const int32_t* __restrict__ budgets, const int32_t* __restrict__ img_req,
-                int32_t* __restrict__ out_start, int32_t* __restrict__ out_len, int32_t* __restrict__ scratch,
-                DevStatus* st) {
-  __shared__ int32_t s_warp[32];
-  if (!st->layout_ok) return;
-  const int NI = L.n_images;
-  // dropped[i] = img_len - budget (0 for a budget outside [0, img_len], which is recorded)
-  auto dropped = [&](int i) {
-    const int32_t k = budgets[i], n = L.img_len[i];
-    return (k >= 0 && k <= n) ? n - k : 0;
-  };
-  block_exclusive_scan<int32_t>(NI, dropped, scratch, s_warp);
-  for (int i = threadIdx.x; i < NI; i += blockDim.x) {
-    const int32_t k = budgets[i], n = L.img_len[i];
-    if (k < 0 || k > n) {
-      record_error(st, AVTP_ERR_DEVICE_INPUT, i);
-      out_start[i] = 0;
-      out_len[i] = 0;
-      continue;
+  if (a.pl_budgets != nullptr) {
+    // The image spans of the pruned batch: image i of request r moves left by the tokens
+    // pruned from the request's earlier images and keeps budgets[i] tokens (an exclusive
+    // scan of the pruned counts over all images, less the request's first entry). A budget
+    // outside [0, img_len] is recorded (after the status word above is written) and its
+    // image gets an empty span.
+    __syncthreads();
+    if (s_err == 0) {
+      const int32_t* budgets = a.pl_budgets;
+      block_exclusive_scan<int32_t>(
+          NI,
+          [&](int i) {
+            const int32_t k = budgets[i], n = iln[i];
+            return (k >= 0 && k <= n) ? n - k : 0;
+          },
+          g_scratch, s_warp);
+      for (int i = tid; i < NI; i += blockDim.x) {
+        const int32_t k = budgets[i], n = iln[i];
+        if (k < 0 || k > n) {
+          record_error(st, AVTP_ERR_DEVICE_INPUT, i);
+          a.pl_out_start[i] = 0;
+          a.pl_out_len[i] = 0;
+          continue;
+        }
+        const int first = icu[img_req[i]];  // the request's first image
+        a.pl_out_start[i] = ist[i] - (g_scratch[i] - g_scratch[first]);
+        a.pl_out_len[i] = k;
+      }
     }
-    const int first = L.img_cu[img_req[i]];  // the request's first image
-    out_start[i] = L.img_start[i] - (scratch[i] - scratch[first]);
-    out_len[i] = k;
   }
 }
 
 }  // namespace
-
-cudaError_t launch_pruned_layout(const avtp_layout_t& L, const int32_t* budgets, int32_t* out_start, int32_t* out_len,
-                                 void* ws, const WsPlan& p, cudaStream_t s) {
-  if (L.n_images == 0) return cudaSuccess;
-  k_pruned_layout<<<1, kPrepThreads, 0, s>>>(L, budgets, ws_at<int32_t>(ws, p.img_req), out_start, out_len,
-                                             ws_at<int32_t>(ws, p.scratch), ws_at<DevStatus>(ws, p.status));
-  return cudaGetLastError();
-}
 
 cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream_t s) {
   const bool b = a.build_text_tiles != 0;
@@ -320,7 +313,8 @@ cudaError_t launch_prep(const PrepArgs& a, void* ws, const WsPlan& p, cudaStream
                                     b ? ws_at<int32_t>(ws, p.p2t_cu) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.ktile_cu) : nullptr,
                                     b ? ws_at<int32_t>(ws, p.ktile_img) : nullptr,
-                                    b ? ws_at<int32_t>(ws, p.meta) : nullptr);
+                                    b ? ws_at<int32_t>(ws, p.meta) : nullptr,
+                                    a.pl_budgets != nullptr ? ws_at<int32_t>(ws, p.scratch) : nullptr);
   return cudaGetLastError();
 }
 
