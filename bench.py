@@ -688,7 +688,7 @@ def time_progressive(args, wl, L, h_cur, h_prior, pos, stream, flush, torch, avt
             "latency_us": {"p50": round(p50 * 1e3, 2), "p90": round(ms[int(len(ms) * 0.9)] * 1e3, 2)},
             "stage_roofline": {"bound": "hbm", "algorithmic_bytes": int(bytes_total), "bound_us": round(bound_us, 2),
                                "frac": round(bound_us / (p50 * 1e3), 4), "peak_gbs": hbm, "peak_kind": peak_kind},
-            "gpu_launches": K * (4 * stages + 2 * (stages - 1))}
+            "gpu_launches": K * (4 * stages + (stages - 1))}  # each boundary: one k_prep (it builds the spans)
 
 
 def run_e2e(args, wl, crit, L, call, dev, stream, torch, avtp):
