@@ -437,12 +437,14 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
 
 // ---------------------------------------------------------------- transposed values
 // Vt[g][c][t] = v[t][g][c] for t < T and 0 for T <= t < Tp. A CTA moves a tile of 64
-// tokens x 64 channels of one KV head through shared memory, 16 bytes per access on both
-// sides.
+// tokens x 64 channels of one KV head through shared memory, 16 bytes per global access on
+// both sides. The tile is read down its columns, so its 16-byte chunks are swizzled: chunk
+// c of token row t sits at chunk position c ^ (t / 8 % 8), and the eight token rows a warp
+// reads at once fall on different banks.
 __global__ void __launch_bounds__(256)
 k_attn_vt(const __nv_bfloat16* __restrict__ v, int64_t v_stride, int d, int64_t T, int64_t Tp,
           __nv_bfloat16* __restrict__ vt, const DevStatus* st) {
-  __shared__ __align__(16) uint16_t tile[64][64 + 8];  // [token][channel]; rows of 144 bytes
+  __shared__ __align__(16) uint16_t tile[64][64];  // [token][channel], swizzled 16-byte chunks
   pdl_wait();
   pdl_trigger();
   if (!st->layout_ok) return;
@@ -454,18 +456,20 @@ k_attn_vt(const __nv_bfloat16* __restrict__ v, int64_t v_stride, int d, int64_t 
     const int64_t t = t0 + tt;
     uint4 val = make_uint4(0u, 0u, 0u, 0u);
     if (t < T) val = *reinterpret_cast<const uint4*>(v + t * v_stride + static_cast<int64_t>(g) * d + c0 + ch * 8);
-    *reinterpret_cast<uint4*>(&tile[tt][ch * 8]) = val;
+    *reinterpret_cast<uint4*>(&tile[tt][(ch ^ ((tt >> 3) & 7)) * 8]) = val;
   }
   __syncthreads();
   for (int e = threadIdx.x; e < 64 * 8; e += blockDim.x) {
     const int cc = e >> 3, tch = e & 7;
     const int64_t t = t0 + tch * 8;
     if (t >= Tp) continue;
+    // token rows tch * 8 .. + 7 all lie in row group tch
+    const int col = (((cc >> 3) ^ tch) << 3) | (cc & 7);
     uint32_t w[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k)
-      w[k] = static_cast<uint32_t>(tile[tch * 8 + 2 * k][cc]) |
-             (static_cast<uint32_t>(tile[tch * 8 + 2 * k + 1][cc]) << 16);
+      w[k] = static_cast<uint32_t>(tile[tch * 8 + 2 * k][col]) |
+             (static_cast<uint32_t>(tile[tch * 8 + 2 * k + 1][col]) << 16);
     *reinterpret_cast<uint4*>(vt + (static_cast<int64_t>(g) * d + c0 + cc) * Tp + t) =
         make_uint4(w[0], w[1], w[2], w[3]);
   }
