@@ -1081,6 +1081,64 @@ def run_timeline(args):
     return out
 
 
+# ---------------------------------------------------------------- forward timeline (diagnostic)
+def run_timeline_forward(args):
+    """The attention forward in the timeline build (-DAVTP_TIMELINE): clock stamps per key
+    block of the CTA with the most key blocks (head 0), medians over its steady blocks and
+    over calls, in SM cycles: the block period, the softmax's phases and the MMA-issuing
+    thread's. Not a bench line: the stamps add stores to the kernel."""
+    os.environ["AVTP_TIMELINE"] = "1"
+    import torch
+
+    from paper_2608_26806_gb300 import avtp, build, synth
+
+    build.build(timeline=True)
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = synth.make_workload(args.config, parts=("B", "V"))
+    lay = wl.layout
+
+    def bf16(x):
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    L = avtp.Layout.from_host(lay.cu_seqlens, lay.img_cu, lay.img_start, lay.img_len, device=dev)
+    call = avtp.ForwardCall(L, q=bf16(wl.q), k=bf16(wl.k), v=bf16(wl.v), softmax_scale=wl.softmax_scale,
+                            scores=False)
+    # the first CTA runs the last query tile of the last request: its key blocks
+    cu = lay.cu_seqlens
+    a, b = int(cu[-2]), int(cu[-1])
+    nblk = (b - 1) // 128 - a // 128 + 1
+    n = min(nblk, 256)  # the timeline build keeps the first 256 blocks
+    flush = L2Flush(dev)
+    per_call = []
+    for i in range(max(args.steps, 8)):
+        flush()
+        call.run()
+        torch.cuda.synchronize()
+        if i >= 3:
+            per_call.append(avtp.forward_timeline(n))
+    st = avtp.read_device_status(call.workspace)
+    if st != avtp.OK:
+        raise RuntimeError(f"device status (forward timeline): {avtp.status_string(st)}")
+    S = {n: i for i, n in enumerate(avtp.FORWARD_TIMELINE_SLOTS)}
+
+    def med(f):
+        vals = []
+        for t in per_call:
+            vals += [f(t, j) for j in range(2, n - 1)]
+        return round(float(np.median(vals)), 1)
+
+    return {"config": args.config, "blocks": nblk, "blocks_stamped": n, "unit": "SM cycles per 128-key block (median)",
+            "period": med(lambda t, j: t[j, S["p_handed"]] - t[j - 1, S["p_handed"]]),
+            "softmax": {"wait_for_S": med(lambda t, j: t[j, S["s_ready"]] - t[j, S["top"]]),
+                        "load_mask_max_exchange": med(lambda t, j: t[j, S["exchanged"]] - t[j, S["s_ready"]]),
+                        "exponentials": med(lambda t, j: t[j, S["exp_done"]] - t[j, S["exchanged"]]),
+                        "p_handover": med(lambda t, j: t[j, S["p_handed"]] - t[j, S["exp_done"]])},
+            "mma_thread": {"S_waits_and_issue": med(lambda t, j: t[j, S["mma_s_issued"]] - t[j, S["mma_s_entry"]]),
+                           "PV_waits": med(lambda t, j: t[j, S["mma_pv_ready"]] - t[j, S["mma_pv_entry"]]),
+                           "PV_issue": med(lambda t, j: t[j, S["mma_pv_issued"]] - t[j, S["mma_pv_ready"]])}}
+
+
 # ---------------------------------------------------------------- path crossover (diagnostic)
 def run_crossover(args):
     """Criterion-B scoring on both paths as the query set widens: one request of four
@@ -1152,6 +1210,8 @@ def main():
                     help="skip the attention-criterion object (timed after the headline criterion)")
     ap.add_argument("--timeline", action="store_true",
                     help="print the phase timeline of the headline stage (timeline build) instead of the bench line")
+    ap.add_argument("--timeline-forward", action="store_true",
+                    help="per-block phase timings of the attention forward (timeline build), not a bench line")
     ap.add_argument("--crossover", action="store_true",
                     help="print criterion-B scoring times of both paths as the query set widens, not the bench line")
     ap.add_argument("--crossover-text", type=int, default=0, help="--crossover: only this many text tokens")
@@ -1161,6 +1221,9 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.timeline:
         print(json.dumps(run_timeline(args)), flush=True)
+        return
+    if args.timeline_forward:
+        print(json.dumps(run_timeline_forward(args)), flush=True)
         return
     if args.crossover:
         print(json.dumps(run_crossover(args)), flush=True)

@@ -226,6 +226,15 @@ AVTP_API avtp_status_t avtp_attn_forward(const avtp_layout_t* layout, const avtp
                                          const avtp_forward_args_t* fwd_args, float* scores, int64_t* img_sums,
                                          void* workspace, size_t workspace_bytes, avtp_stream_t stream);
 
+/* Diagnostic: per-key-block clock stamps (SM cycles) of the last avtp_attn_forward call's
+ * first CTA, the query tile with the most key blocks, head 0. Available in the library's
+ * timeline build (compiled with AVTP_TIMELINE); the default build returns
+ * AVTP_ERR_UNSUPPORTED. out: host int64 [max_blocks][10]: per block j, from softmax warp 0
+ * the loop top, S ready, the half maxima exchanged, the exponentials done and P handed
+ * over, then from the MMA-issuing thread S_j's entry and issue and P_j V_j's entry,
+ * operands ready and issue. Synchronises the device. */
+AVTP_API avtp_status_t avtp_forward_timeline(int64_t* out, int32_t max_blocks);
+
 /* Step 2 (paper §3.3.3, App. A.2). From img_sums (device int64 [n_images]) writes
  * budgets (device int32 [n_images]) and out_cu_seqlens (device int32 [R+1]),
  * the packed offsets of the pruned batch. Per request, in exact rational arithmetic:

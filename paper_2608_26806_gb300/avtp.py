@@ -91,6 +91,7 @@ SIGNATURES = {
                                             POINTER(c_size_t)]),
     "avtp_attn_forward": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(_ForwardArgs), c_void_p, c_void_p,
                                   c_void_p, c_size_t, c_void_p]),
+    "avtp_forward_timeline": (c_int, [c_void_p, c_int32]),
     "avtp_allocate": (c_int, [POINTER(_Layout), c_void_p, POINTER(_AllocArgs), c_void_p, c_void_p, c_void_p,
                               c_size_t, c_void_p]),
     "avtp_select": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
@@ -366,6 +367,18 @@ class ForwardCall:
                                         _ptr(self.scores), _ptr(self.img_sums), _ptr(self.workspace),
                                         self.workspace.numel(), _stream(stream)), "avtp_attn_forward")
         return self
+
+
+FORWARD_TIMELINE_SLOTS = ("top", "s_ready", "exchanged", "exp_done", "p_handed", "mma_s_entry", "mma_s_issued",
+                          "mma_pv_entry", "mma_pv_ready", "mma_pv_issued")
+
+
+def forward_timeline(n_blocks: int) -> np.ndarray:
+    """avtp_forward_timeline: clock stamps int64 [n_blocks, 10] (FORWARD_TIMELINE_SLOTS) of the
+    last forward call's first CTA; needs the timeline build (AVTP_TIMELINE=1)."""
+    out = np.zeros((n_blocks, len(FORWARD_TIMELINE_SLOTS)), dtype=np.int64)
+    _check(load().avtp_forward_timeline(out.ctypes.data, n_blocks), "avtp_forward_timeline")
+    return out
 
 
 def attn_forward(layout: Layout, *, q, k, v, softmax_scale=None, scores: bool = True, query_set="text",

@@ -115,6 +115,25 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       : "memory");
 }
 
+// Diagnostic timeline build (-DAVTP_TIMELINE): clock stamps of the grid's first CTA (the
+// tile with the most key blocks, head 0), per key block j. Slots: 0-4 from softmax warp 0
+// (loop top, S ready, half maxima exchanged, exponentials done, P handed over); 5-9 from
+// the MMA thread (S_j: entry, issued; P_j V_j: entry, operands ready, issued). Read with
+// avtp_forward_timeline().
+constexpr int kFwdTlBlocks = 256;
+constexpr int kFwdTlSlots = 10;
+#ifdef AVTP_TIMELINE
+__device__ long long g_fwd_tl[kFwdTlBlocks][kFwdTlSlots];
+#endif
+__device__ __forceinline__ void fwd_stamp(int j, int slot) {
+#ifdef AVTP_TIMELINE
+  if (blockIdx.x == 0 && j < kFwdTlBlocks) g_fwd_tl[j][slot] = clock64();
+#else
+  (void)j;
+  (void)slot;
+#endif
+}
+
 __device__ __forceinline__ void bar_softmax() { asm volatile("bar.sync 5, 256;" ::: "memory"); }
 // Barrier of the two softmax warps of TMEM lane quadrant `quad` (ids 1-4, 64 threads); true
 // when `bad` holds for any of their threads.
@@ -232,6 +251,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       // (128 lanes x d / 2 columns), B = key stage j % 2 (128 keys x d, K-major)
       auto issue_s = [&](int j) -> bool {
         const int sb = j & 1;
+        fwd_stamp(j, 5);
         if (!tc::mbar_wait(&sy.k_full[sb], (j >> 1) & 1)) return false;
         if (j >= 1 && !tc::mbar_wait(&sy.s_empty, (j - 1) & 1)) return false;
         tc::fence_after_sync();
@@ -243,14 +263,17 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         }
         tc::mma_commit(&sy.s_full);
         tc::mma_commit(&sy.k_empty[sb]);
+        fwd_stamp(j, 6);
         return true;
       };
       // O += P_i V_i: A = P buffer i % 2 in TMEM (128 lanes x 64 columns), B = the Vt block
       // (d rows x 128 keys, two 64-key panels)
       auto issue_pv = [&](int i) -> bool {
         const int sb = i & 1;
+        fwd_stamp(i, 7);
         if (!tc::mbar_wait(&sy.p_full[sb], (i >> 1) & 1)) return false;
         if (!tc::mbar_wait(&sy.v_full[sb], (i >> 1) & 1)) return false;
+        fwd_stamp(i, 8);
         tc::fence_after_sync();
         const uint32_t bV = tc::smem_u32(sV + sb * v_bytes(d));
 #pragma unroll
@@ -261,6 +284,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         }
         tc::mma_commit(&sy.pv_done[sb]);
         tc::mma_commit(&sy.v_empty[sb]);
+        fwd_stamp(i, 9);
         return true;
       };
       bool ok = tc::mbar_wait(&sy.q_tmem, 0) && issue_s(0);
@@ -308,8 +332,11 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
     for (int j = 0; j < nblk; ++j) {
       const int sb = j & 1;
       const int key0 = (kb0 + j) * kKB + half * kHalf;
+      const bool stamp = warp == 0 && lane == 0;
+      if (stamp) fwd_stamp(j, 0);
       bad = bad || __any_sync(0xffffffffu, *abort_flag != 0);
       if (!bad && !tc::mbar_wait_warp(&sy.s_full, j & 1)) bad = true;
+      if (stamp) fwd_stamp(j, 1);
       float s[kHalf];
       float mh = -INFINITY;
       if (!bad) {
@@ -343,6 +370,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         if (lane == 0) *abort_flag = 1;
         break;
       }
+      if (stamp) fwd_stamp(j, 2);
       const float mb = fmaxf(mh, s_mx[sb][half ^ 1][row]) * c2;  // -inf when nothing is visible
       float factor = 1.f;
       bool resc = false;
@@ -369,6 +397,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         pk[c / 2 + 1] = pack_bf16x2(p2, p3);
       }
       l += (acc0.x + acc0.y) + (acc1.x + acc1.y);
+      if (stamp) fwd_stamp(j, 3);
       // O is final up to block j - 1 once P_{j-1} V_{j-1} is done: a rescale waits for it and
       // scales this warp's half of the columns (both warps of the pair took the same factor)
       if (j >= 1 && __any_sync(0xffffffffu, resc)) {
@@ -398,6 +427,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&sy.p_full[sb]);
+      if (stamp) fwd_stamp(j, 4);
     }
     bool fin = !bad && !__any_sync(0xffffffffu, *abort_flag != 0);
     if (fin && !tc::mbar_wait_warp(&sy.pv_done[(nblk - 1) & 1], ((nblk - 1) >> 1) & 1)) {
@@ -595,3 +625,18 @@ cudaError_t launch_attn_forward(const avtp_layout_t& L, const avtp_score_args_t&
 }
 
 }  // namespace avtp
+
+extern "C" avtp_status_t avtp_forward_timeline(int64_t* out, int32_t max_blocks) {
+#ifdef AVTP_TIMELINE
+  if (out == nullptr || max_blocks < 1) return AVTP_ERR_INVALID_ARG;
+  const int n = max_blocks < avtp::kFwdTlBlocks ? max_blocks : avtp::kFwdTlBlocks;
+  return cudaMemcpyFromSymbol(out, avtp::g_fwd_tl, static_cast<size_t>(n) * avtp::kFwdTlSlots * sizeof(long long)) ==
+                 cudaSuccess
+             ? AVTP_OK
+             : AVTP_ERR_CUDA;
+#else
+  (void)out;
+  (void)max_blocks;
+  return AVTP_ERR_UNSUPPORTED;
+#endif
+}

@@ -260,6 +260,11 @@ def test_forward_workspace_holds_the_transposed_values(lib):
     assert b.value >= 8 * 128 * 10000 * 2 and b.value % 256 == 0
 
 
+def test_forward_timeline_needs_the_timeline_build(lib):
+    out = np.zeros((4, 10), dtype=np.int64)
+    assert lib.avtp_forward_timeline(out.ctypes.data, 4) == avtp.ERR_UNSUPPORTED
+
+
 def test_host_validation_of_wait_selftest_arguments(lib):
     for bad in (-1, 0, 999, 10_000_000_001):
         assert lib.avtp_wait_selftest(bad, 0, FAKE, 256, None) == avtp.ERR_INVALID_ARG
