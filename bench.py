@@ -1139,6 +1139,61 @@ def run_timeline_forward(args):
                            "PV_issue": med(lambda t, j: t[j, S["mma_pv_issued"]] - t[j, S["mma_pv_ready"]])}}
 
 
+# ---------------------------------------------------------------- criterion-B pass timelines (diagnostic)
+def run_timeline_attn(args):
+    """Criterion B's tensor-core passes in the timeline build (-DAVTP_TIMELINE): clock stamps
+    per step of each pass's first CTA, medians over its steps after the first and over calls,
+    in SM cycles: the step period, the MMA thread's wait for its operands and accumulators,
+    its issue, the epilogue's hold of the accumulators, and the time from a key tile's load
+    to the MMA thread finding it ready. Not a bench line: the stamps add stores."""
+    os.environ["AVTP_TIMELINE"] = "1"
+    import torch
+
+    from paper_2608_26806_gb300 import avtp, build, synth
+
+    build.build(timeline=True)
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = synth.make_workload(args.config, parts=("B",))
+    lay = wl.layout
+
+    def bf16(x):
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    L = avtp.Layout.from_host(lay.cu_seqlens, lay.img_cu, lay.img_start, lay.img_len, device=dev)
+    q, k = bf16(wl.q), bf16(wl.k)
+    ws = avtp.new_workspace(avtp.workspace_size(L, "text_attention", q=q, k=k, path="tensor"), dev)
+    flush = L2Flush(dev)
+    S = {n: i for i, n in enumerate(avtp.SCORE_TIMELINE_SLOTS)}
+    stamps = {1: [], 2: []}
+    for i in range(max(args.steps, 8)):
+        flush()
+        avtp.score(L, "text_attention", q=q, k=k, softmax_scale=wl.softmax_scale, path="tensor", workspace=ws)
+        torch.cuda.synchronize()
+        if i >= 3:
+            for p in (1, 2):
+                stamps[p].append(avtp.score_timeline(p, 64))
+    st = avtp.read_device_status(ws)
+    if st != avtp.OK:
+        raise RuntimeError(f"device status (criterion-B timeline): {avtp.status_string(st)}")
+    out = {"config": args.config, "unit": "SM cycles per step (median)"}
+    for p in (1, 2):
+        def med(f):
+            vals = []
+            for t in stamps[p]:
+                n = int(np.count_nonzero(t[:, S["mma_issued"]]))  # steps the first CTA ran
+                vals += [f(t, j) for j in range(1, n)]
+            return round(float(np.median(vals)), 1) if vals else None
+        out[f"pass{p}"] = {
+            "steps_stamped": int(np.count_nonzero(stamps[p][-1][:, S["mma_issued"]])),
+            "period": med(lambda t, j: t[j, S["mma_issued"]] - t[j - 1, S["mma_issued"]]),
+            "mma_wait_for_operands": med(lambda t, j: t[j, S["mma_ready"]] - t[j, S["mma_step"]]),
+            "mma_issue": med(lambda t, j: t[j, S["mma_issued"]] - t[j, S["mma_ready"]]),
+            "epilogue_hold": med(lambda t, j: t[j, S["acc_released"]] - t[j, S["acc_ready"]]),
+            "load_to_ready": med(lambda t, j: t[j, S["mma_ready"]] - t[j, S["load_issued"]])}
+    return out
+
+
 # ---------------------------------------------------------------- path crossover (diagnostic)
 def run_crossover(args):
     """Criterion-B scoring on both paths as the query set widens: one request of four
@@ -1212,6 +1267,8 @@ def main():
                     help="print the phase timeline of the headline stage (timeline build) instead of the bench line")
     ap.add_argument("--timeline-forward", action="store_true",
                     help="per-block phase timings of the attention forward (timeline build), not a bench line")
+    ap.add_argument("--timeline-attn", action="store_true",
+                    help="per-step phase timings of criterion B's tensor-core passes (timeline build), not a bench line")
     ap.add_argument("--crossover", action="store_true",
                     help="print criterion-B scoring times of both paths as the query set widens, not the bench line")
     ap.add_argument("--crossover-text", type=int, default=0, help="--crossover: only this many text tokens")
@@ -1224,6 +1281,9 @@ def main():
         return
     if args.timeline_forward:
         print(json.dumps(run_timeline_forward(args)), flush=True)
+        return
+    if args.timeline_attn:
+        print(json.dumps(run_timeline_attn(args)), flush=True)
         return
     if args.crossover:
         print(json.dumps(run_crossover(args)), flush=True)

@@ -235,6 +235,15 @@ AVTP_API avtp_status_t avtp_attn_forward(const avtp_layout_t* layout, const avtp
  * operands ready and issue. Synchronises the device. */
 AVTP_API avtp_status_t avtp_forward_timeline(int64_t* out, int32_t max_blocks);
 
+/* Diagnostic: per-step clock stamps (SM cycles) of the first CTA of criterion B's tensor-core
+ * pass `pass` (1: the log-sum-exp pass, 2: the mass pass) in the last avtp_score call that
+ * ran it, for the first max_steps (at most 64) steps of that CTA's run. Timeline build only
+ * (AVTP_TIMELINE); the default build returns AVTP_ERR_UNSUPPORTED. out: host int64
+ * [max_steps][6]: the key tile's load issued, the MMA thread at the step, its operands and
+ * accumulators ready, its MMAs issued, the step's first accumulator ready for epilogue
+ * warp 0, the step's last accumulator released by it. Synchronises the device. */
+AVTP_API avtp_status_t avtp_score_timeline(int32_t pass, int64_t* out, int32_t max_steps);
+
 /* Step 2 (paper §3.3.3, App. A.2). From img_sums (device int64 [n_images]) writes
  * budgets (device int32 [n_images]) and out_cu_seqlens (device int32 [R+1]),
  * the packed offsets of the pruned batch. Per request, in exact rational arithmetic:

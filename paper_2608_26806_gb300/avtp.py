@@ -92,6 +92,7 @@ SIGNATURES = {
     "avtp_attn_forward": (c_int, [POINTER(_Layout), POINTER(_ScoreArgs), POINTER(_ForwardArgs), c_void_p, c_void_p,
                                   c_void_p, c_size_t, c_void_p]),
     "avtp_forward_timeline": (c_int, [c_void_p, c_int32]),
+    "avtp_score_timeline": (c_int, [c_int32, c_void_p, c_int32]),
     "avtp_allocate": (c_int, [POINTER(_Layout), c_void_p, POINTER(_AllocArgs), c_void_p, c_void_p, c_void_p,
                               c_size_t, c_void_p]),
     "avtp_select": (c_int, [POINTER(_Layout), c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_void_p, c_size_t,
@@ -378,6 +379,17 @@ def forward_timeline(n_blocks: int) -> np.ndarray:
     last forward call's first CTA; needs the timeline build (AVTP_TIMELINE=1)."""
     out = np.zeros((n_blocks, len(FORWARD_TIMELINE_SLOTS)), dtype=np.int64)
     _check(load().avtp_forward_timeline(out.ctypes.data, n_blocks), "avtp_forward_timeline")
+    return out
+
+
+SCORE_TIMELINE_SLOTS = ("load_issued", "mma_step", "mma_ready", "mma_issued", "acc_ready", "acc_released")
+
+
+def score_timeline(pass_: int, n_steps: int) -> np.ndarray:
+    """avtp_score_timeline: clock stamps int64 [n_steps, 6] (SCORE_TIMELINE_SLOTS) of the first
+    CTA of criterion B's tensor-core pass 1 or 2; needs the timeline build (AVTP_TIMELINE=1)."""
+    out = np.zeros((n_steps, len(SCORE_TIMELINE_SLOTS)), dtype=np.int64)
+    _check(load().avtp_score_timeline(int(pass_), out.ctypes.data, n_steps), "avtp_score_timeline")
     return out
 
 

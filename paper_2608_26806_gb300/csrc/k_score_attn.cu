@@ -97,6 +97,26 @@ struct AttnArgs {
 
 __device__ __forceinline__ void bar_epi() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
+// Diagnostic timeline build (-DAVTP_TIMELINE): clock stamps of each pass's first CTA, per
+// step s of its run. Slots: 0 the key tile's load issued (TMA thread); 1 the MMA thread at
+// the step, 2 its operands and accumulators ready, 3 its MMAs issued and committed; 4 the
+// step's (first) accumulator ready for epilogue warp 0, 5 the step's (last) accumulator
+// released by it. Read with avtp_score_timeline().
+constexpr int kAttnTlSteps = 64;
+constexpr int kAttnTlSlots = 6;
+#ifdef AVTP_TIMELINE
+__device__ long long g_attn_tl[2][kAttnTlSteps][kAttnTlSlots];
+#endif
+__device__ __forceinline__ void attn_stamp(int pass, int st, int slot) {
+#ifdef AVTP_TIMELINE
+  if (blockIdx.x == 0 && st < kAttnTlSteps) g_attn_tl[pass][st][slot] = clock64();
+#else
+  (void)pass;
+  (void)st;
+  (void)slot;
+#endif
+}
+
 // A (KV group, row block) pair: rows [R0, R1) of group g belong to request r.
 struct Seg {
   int g, b, r;
@@ -385,6 +405,7 @@ k_attn_lse(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         tc::mbar_arrive_expect_tx(&sy.b_full[sb], static_cast<uint32_t>(b_bytes(d)));
         for (int ac = 0; ac < d / 64; ++ac)
           tc::tma_load_3d(sB[sb] + ac * atomB, &mapK, ac * 64, cur.g, key_base + cur.j * kN, &sy.b_full[sb]);
+        attn_stamp(0, st, 0);
         ++nb;
         new_seg = st + 1 < n_steps && cur.next(a.p1s_cu, NB);
       }
@@ -399,6 +420,7 @@ k_attn_lse(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
       uint32_t na = 0, nb = 0;
       bool new_seg = true, stop = false;
       for (int st = 0; st < n_steps && !stop && !*abort_flag; ++st) {
+        attn_stamp(0, st, 1);
         if (new_seg) {
           if (!tc::mbar_wait(&sy.a_full[0], na & 1)) { *abort_flag = 1; break; }
           ++na;
@@ -408,12 +430,14 @@ k_attn_lse(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         for (int t = 0; t < 2; ++t) {
           // accumulator t: its previous use (step nb - 1) must have been read out
           if (nb >= 1 && !tc::mbar_wait(&sy.acc_empty[t], (nb - 1) & 1)) { *abort_flag = 1; stop = true; break; }
+          if (t == 0) attn_stamp(0, st, 2);
           tc::fence_after_sync();
           tc::mma_rows(tmem + t * kN, tc::smem_u32(sA + t * a_bytes(d)), atomA, tc::smem_u32(sB[sb]), atomB, d, idesc);
           tc::mma_commit(&sy.acc_full[t]);
         }
         if (stop) break;
         tc::mma_commit(&sy.b_empty[sb]);
+        attn_stamp(0, st, 3);
         ++nb;
         const bool more = st + 1 < n_steps;
         if (!more || cur.last_of_block()) tc::mma_commit(&sy.a_empty[0]);
@@ -461,6 +485,7 @@ k_attn_lse(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
           if (lane == 0) *abort_flag = 1;
           ok = false;
         }
+        if (t == 0 && warp == 0 && lane == 0) attn_stamp(0, st, 4);
         tc::fence_after_sync();
         // columns 0..lim of this warp's half are visible to the row
         const int lim = (t ? qpos1 : qpos0) - (key_base + cur.j * kN + half * (kN / 2));
@@ -479,6 +504,7 @@ k_attn_lse(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUt
         tc::fence_before_sync();
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(&sy.acc_empty[t]);
+        if (t == 1 && warp == 0 && lane == 0) attn_stamp(0, st, 5);
       }
       const bool more = st + 1 < n_steps;
       if (!more || cur.last_of_block()) {
@@ -567,6 +593,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CU
         tc::mbar_arrive_expect_tx(&sy.a_full[sa], static_cast<uint32_t>(a_bytes(d)));
         for (int ac = 0; ac < d / 64; ++ac)
           tc::tma_load_3d(sA0 + sa * a_bytes(d) + ac * atomA, &mapK, ac * 64, cur.g, tile.kp0, &sy.a_full[sa]);
+        attn_stamp(1, st, 0);
         ++na;
         new_seg = st + 1 < n_steps && cur.next(a.p2t_cu, NB);
       }
@@ -581,6 +608,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CU
       uint32_t na = 0, nbl = 0;
       bool new_seg = true;
       for (int st = 0; st < n_steps && !*abort_flag; ++st) {
+        attn_stamp(1, st, 1);
         if (new_seg) {
           if (!tc::mbar_wait(&sy.b_full[0], nbl & 1)) { *abort_flag = 1; break; }
           ++nbl;
@@ -589,10 +617,12 @@ k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CU
         if (!tc::mbar_wait(&sy.a_full[sa], (na / kP2Stages) & 1)) { *abort_flag = 1; break; }
         const int t = na & 1;  // accumulator of this step
         if (na >= 2 && !tc::mbar_wait(&sy.acc_empty[t], ((na >> 1) - 1) & 1)) { *abort_flag = 1; break; }
+        attn_stamp(1, st, 2);
         tc::fence_after_sync();
         tc::mma_rows(tmem + t * kN, tc::smem_u32(sA0 + sa * a_bytes(d)), atomA, tc::smem_u32(sB), atomB, d, idesc);
         tc::mma_commit(&sy.a_empty[sa]);
         tc::mma_commit(&sy.acc_full[t]);
+        attn_stamp(1, st, 3);
         ++na;
         const bool more = st + 1 < n_steps;
         if (!more || cur.last_of_block()) tc::mma_commit(&sy.b_empty[0]);
@@ -669,6 +699,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CU
         if (lane == 0) *abort_flag = 1;
         ok = false;
       }
+      if (warp == 0 && lane == 0) attn_stamp(1, st, 4);
       tc::fence_after_sync();
       // does this warp's column half hold a visible row? (CTA-uniform)
       const bool any = tile.c0 < (half + 1) * kHalf && c1 > half * kHalf;
@@ -677,6 +708,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CU
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive(&sy.acc_empty[t]);
+      if (warp == 0 && lane == 0) attn_stamp(1, st, 5);
       const int w = st % kMassWindow;
       s_mass[w][half][klane] = mass;
       if (etid == 0) {
@@ -904,3 +936,20 @@ cudaError_t launch_attn_finalize(const avtp_layout_t& L, const avtp_score_args_t
 }
 
 }  // namespace avtp
+
+extern "C" avtp_status_t avtp_score_timeline(int32_t pass, int64_t* out, int32_t max_steps) {
+#ifdef AVTP_TIMELINE
+  if (out == nullptr || max_steps < 1 || (pass != 1 && pass != 2)) return AVTP_ERR_INVALID_ARG;
+  const int n = max_steps < avtp::kAttnTlSteps ? max_steps : avtp::kAttnTlSteps;
+  const size_t row = static_cast<size_t>(avtp::kAttnTlSteps) * avtp::kAttnTlSlots * sizeof(long long);
+  return cudaMemcpyFromSymbol(out, avtp::g_attn_tl, static_cast<size_t>(n) * avtp::kAttnTlSlots * sizeof(long long),
+                              (pass - 1) * row) == cudaSuccess
+             ? AVTP_OK
+             : AVTP_ERR_CUDA;
+#else
+  (void)pass;
+  (void)out;
+  (void)max_steps;
+  return AVTP_ERR_UNSUPPORTED;
+#endif
+}

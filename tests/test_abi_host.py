@@ -263,6 +263,7 @@ def test_forward_workspace_holds_the_transposed_values(lib):
 def test_forward_timeline_needs_the_timeline_build(lib):
     out = np.zeros((4, 10), dtype=np.int64)
     assert lib.avtp_forward_timeline(out.ctypes.data, 4) == avtp.ERR_UNSUPPORTED
+    assert lib.avtp_score_timeline(1, out.ctypes.data, 4) == avtp.ERR_UNSUPPORTED
 
 
 def test_host_validation_of_wait_selftest_arguments(lib):
