@@ -227,7 +227,8 @@ AVTP_API avtp_status_t avtp_attn_forward(const avtp_layout_t* layout, const avtp
                                          void* workspace, size_t workspace_bytes, avtp_stream_t stream);
 
 /* Diagnostic: per-key-block clock stamps (SM cycles) of the last avtp_attn_forward call's
- * first CTA, the query tile with the most key blocks, head 0. Available in the library's
+ * first CTA, the query tile with the most key blocks, head 0, for its first max_blocks (at
+ * most 256; the rest of out is left untouched) key blocks. Available in the library's
  * timeline build (compiled with AVTP_TIMELINE); the default build returns
  * AVTP_ERR_UNSUPPORTED. out: host int64 [max_blocks][10]: per block j, from softmax warp 0
  * the loop top, S ready, the half maxima exchanged, the exponentials done and P handed
@@ -237,7 +238,8 @@ AVTP_API avtp_status_t avtp_forward_timeline(int64_t* out, int32_t max_blocks);
 
 /* Diagnostic: per-step clock stamps (SM cycles) of the first CTA of criterion B's tensor-core
  * pass `pass` (1: the log-sum-exp pass, 2: the mass pass) in the last avtp_score call that
- * ran it, for the first max_steps (at most 64) steps of that CTA's run. Timeline build only
+ * ran it, for the first max_steps (at most 64; the rest of out is left untouched) steps of
+ * that CTA's run. Timeline build only
  * (AVTP_TIMELINE); the default build returns AVTP_ERR_UNSUPPORTED. out: host int64
  * [max_steps][6]: the key tile's load issued, the MMA thread at the step, its operands and
  * accumulators ready, its MMAs issued, the step's first accumulator ready for epilogue
