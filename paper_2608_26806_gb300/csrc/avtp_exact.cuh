@@ -394,7 +394,7 @@ __device__ __noinline__ void exact_search(const WarpAllocSmem& sm, int m, const 
 #pragma unroll 1
   for (int round = 0; round < 2 * kMaxImagesPerRequest + 2; ++round) {
     // ---- pivot: an alive breakpoint chosen by a 64-bit key, largest key wins
-    // key bits: 63 alive, 62 preferred this round, 61..14 order value, 13..0 breakpoint index
+    // key bits: 63 alive, 62 preferred in this iteration, 61..14 order value, 13..0 breakpoint index
     uint64_t best = 0;
     for (int j = lane; j < m; j += 32) {
       const int al = sm.alive[j];

@@ -160,10 +160,10 @@ AttnPlan attn_plan(const avtp_layout_t& L, const avtp_score_args_t& sa);
 constexpr int kNarrowMaxSplits = 64;
 constexpr int64_t kNarrowMaxLogitBytes = int64_t(1) << 30;
 // AVTP_PATH_AUTO takes the CUDA cores for AVTP_QUERIES_LAST, and for AVTP_QUERIES_TEXT
-// only when the batch has at most this many rows per KV group (judged from its text-token
+// only when the batch has at most this many rows per KV group (decided from its text-token
 // bound). Measured on a request of four 640-token images and Qwen3-shaped heads (8 KV
-// groups of 4 heads, d = 128), score call event-timed: 31.4 us on the narrow path against
-// 34.5 us on tcgen05 at 4 rows per group (one text token), 34.5 against 34.5 at 8, and
+// groups of 4 heads, d = 128), score call event-timed: 29.3 us on the narrow path against
+// 34.4 us on tcgen05 at 4 rows per group (one text token), 33.4 against 34.4 at 8, and
 // the narrow path growing with the rows beyond (tcgen05 stays near 33 us up to 256 rows).
 constexpr int64_t kNarrowAutoRows = 4;
 struct NarrowPlan {
