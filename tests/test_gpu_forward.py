@@ -169,3 +169,55 @@ def test_forward_serving_batch_sampled_rows():
         g = [int(cu[r]) + p for p in rows]
         _check_o(o_h[g], ref_o, ref_abs)
         np.testing.assert_allclose(lse_h[:, g], ref_lse, rtol=RTOL, atol=ATOL)
+
+
+def test_forward_many_small_requests():
+    """Forty requests of 1 to 300 tokens: many query tiles per call, tiles and key blocks
+    that straddle request boundaries at every offset, requests shorter than a tile."""
+    rng = np.random.default_rng(17)
+    reqs = []
+    for _ in range(40):
+        segs = []
+        for _ in range(int(rng.integers(1, 4))):
+            segs.append(("t" if rng.random() < 0.5 else "i", int(rng.integers(1, 101))))
+        reqs.append(segs)
+    wl = synth.make_custom(reqs, n_q_heads=4, n_kv_heads=1, head_dim=64, hidden=64, seed=23, parts=("B", "V"))
+    L, q, k, v = _dev(wl)
+    o, lse, scores, sums = avtp.attn_forward(L, q=q, k=k, v=v, softmax_scale=wl.softmax_scale)
+    torch.cuda.synchronize()
+    ref_o, ref_lse = O.attention_forward(wl.layout, wl.q, wl.k, wl.v, 4, 1, wl.softmax_scale)
+    ref_abs, _ = O.attention_forward(wl.layout, wl.q, wl.k, _abs_v(wl.v), 4, 1, wl.softmax_scale)
+    _check_o(o.cpu().numpy(), ref_o, ref_abs)
+    np.testing.assert_allclose(lse.cpu().numpy(), ref_lse, rtol=RTOL, atol=ATOL)
+    vis = wl.layout.visual_mask()
+    ref = O.score_text_attention(wl.layout, wl.q, wl.k, 4, 1, wl.softmax_scale)
+    assert_scores_close(scores.cpu().numpy(), ref, vis)
+
+
+def test_forward_strided_tensors():
+    """q, k and v rows with padded token strides, O and the LSE written into wider buffers:
+    the strides of the ABI are honoured and nothing outside the views is written."""
+    Hq, Hkv, d = 6, 2, 128
+    wl = synth.make_custom(_FWD_LAYOUTS[2], n_q_heads=Hq, n_kv_heads=Hkv, head_dim=d, hidden=64, seed=41,
+                           parts=("B", "V"))
+    T = wl.layout.n_tokens
+    L = dev_layout(wl.layout)
+
+    def padded(bits, heads):
+        big = torch.zeros(T, heads + 1, d, dtype=torch.bfloat16, device="cuda")
+        big[:, :heads] = bf16_dev(bits)
+        return big[:, :heads]
+
+    q, k, v = padded(wl.q, Hq), padded(wl.k, Hkv), padded(wl.v, Hkv)
+    o_big = torch.full((T, Hq + 2, d), 7.0, dtype=torch.float32, device="cuda")
+    lse_big = torch.full((Hq, T + 24), 7.0, dtype=torch.float32, device="cuda")
+    c = avtp.ForwardCall(L, q=q, k=k, v=v, softmax_scale=wl.softmax_scale, o=o_big[:, :Hq], lse=lse_big[:, :T])
+    c.run()
+    torch.cuda.synchronize()
+    ref_o, ref_lse = O.attention_forward(wl.layout, wl.q, wl.k, wl.v, Hq, Hkv, wl.softmax_scale)
+    ref_abs, _ = O.attention_forward(wl.layout, wl.q, wl.k, _abs_v(wl.v), Hq, Hkv, wl.softmax_scale)
+    _check_o(o_big[:, :Hq].cpu().numpy(), ref_o, ref_abs)
+    np.testing.assert_allclose(lse_big[:, :T].cpu().numpy(), ref_lse, rtol=RTOL, atol=ATOL)
+    assert torch.all(o_big[:, Hq:] == 7.0) and torch.all(lse_big[:, T:] == 7.0)
+    ref = O.score_text_attention(wl.layout, wl.q, wl.k, Hq, Hkv, wl.softmax_scale)
+    assert_scores_close(c.scores.cpu().numpy(), ref, wl.layout.visual_mask())
