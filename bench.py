@@ -1139,6 +1139,82 @@ def run_timeline_forward(args):
                            "PV_issue": med(lambda t, j: t[j, S["mma_pv_issued"]] - t[j, S["mma_pv_ready"]])}}
 
 
+# ---------------------------------------------------------------- single-step entry points (diagnostic)
+def run_standalone(args):
+    """The steps as separate calls (avtp_score, avtp_allocate, avtp_select, avtp_compact) on
+    the workload, and the pruning-layer statistic (avtp_layer_attention for every layer of a
+    36-layer model, then avtp_layer_select over 256 samples): event-timed calls, L2 flushed
+    before each, medians in microseconds. Not a bench line: each call also runs the
+    validation kernel, and nothing is chained."""
+    import torch
+
+    from paper_2608_26806_gb300 import avtp, synth
+
+    import __graft_entry__
+
+    __graft_entry__.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = synth.make_workload(args.config, parts=("A", "pos"))
+    lay = wl.layout
+
+    def bf16(x):
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    L = avtp.Layout.from_host(lay.cu_seqlens, lay.img_cu, lay.img_start, lay.img_len, device=dev)
+    h_cur, h_prior = bf16(wl.h_cur), bf16(wl.h_prior)
+    pos = torch.from_numpy(wl.pos).to(dev)
+    kr = torch.from_numpy(wl.keep_ratio).to(dev)
+    n_kept = avtp.kept_count_host({"cu_seqlens": lay.cu_seqlens, "img_cu": lay.img_cu, "img_len": lay.img_len},
+                                  wl.keep_ratio)
+    ws = avtp.new_workspace(avtp.workspace_size(L, "hidden_variation", h_cur=h_cur, h_prior=h_prior), dev)
+    scores = torch.zeros(lay.n_tokens, dtype=torch.float32, device=dev)
+    sums = torch.empty(max(lay.n_images, 1), dtype=torch.int64, device=dev)
+    budgets = torch.empty(max(lay.n_images, 1), dtype=torch.int32, device=dev)
+    ocu = torch.empty(lay.n_requests + 1, dtype=torch.int32, device=dev)
+    kept = torch.empty(max(n_kept, 1), dtype=torch.int32, device=dev)
+    hid_out = torch.empty(max(n_kept, 1), h_cur.shape[1], dtype=torch.bfloat16, device=dev)
+    pos_out = torch.empty(pos.shape[0], max(n_kept, 1), dtype=pos.dtype, device=dev)
+    rows = [(h_cur, hid_out)] + [(pos[p_], pos_out[p_]) for p_ in range(pos.shape[0])]
+    n_layers, n_samples = 36, 256
+    A = torch.zeros(n_samples, n_layers, dtype=torch.int64, device=dev)
+    A.copy_(torch.randint(0, 1 << 40, (n_samples, n_layers), generator=torch.Generator().manual_seed(3)).to(dev))
+    A1 = torch.zeros(lay.n_requests, n_layers, dtype=torch.int64, device=dev)
+    steps = {
+        "score": lambda: avtp.score(L, "hidden_variation", h_cur=h_cur, h_prior=h_prior, scores=scores,
+                                    img_sums=sums, workspace=ws),
+        "allocate": lambda: avtp.allocate(L, sums, kr, budgets=budgets, out_cu_seqlens=ocu, workspace=ws),
+        "select": lambda: avtp.select(L, scores, budgets, ocu, n_kept, kept_idx=kept, workspace=ws),
+        "compact": lambda: avtp.compact(kept[:n_kept], lay.n_tokens, [(a_, b_[:n_kept]) for a_, b_ in rows],
+                                        workspace=ws),
+        "layer_attention_36_layers": lambda: [avtp.layer_attention(L, sums, A1, l_, workspace=ws)
+                                              for l_ in range(n_layers)],
+        "layer_select_256_samples": lambda: avtp.layer_select(A, 3),
+    }
+    flush = L2Flush(dev)
+    K = max(10, min(args.steps, 100))
+    out = {"config": args.config, "unit": "us per call (median, L2 flushed before each)", "calls": K}
+    for name, fn in steps.items():
+        for _ in range(3):
+            flush()
+            fn()
+        torch.cuda.synchronize()
+        ms = []
+        for _ in range(K):
+            flush()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            fn()
+            e1.record()
+            torch.cuda.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        out[name] = round(float(np.median(ms)) * 1e3, 2)
+    st = avtp.read_device_status(ws)
+    if st != avtp.OK:
+        raise RuntimeError(f"device status (standalone steps): {avtp.status_string(st)}")
+    return out
+
+
 # ---------------------------------------------------------------- criterion-B pass timelines (diagnostic)
 def run_timeline_attn(args):
     """Criterion B's tensor-core passes in the timeline build (-DAVTP_TIMELINE): clock stamps
@@ -1267,6 +1343,8 @@ def main():
                     help="print the phase timeline of the headline stage (timeline build) instead of the bench line")
     ap.add_argument("--timeline-forward", action="store_true",
                     help="per-block phase timings of the attention forward (timeline build), not a bench line")
+    ap.add_argument("--standalone", action="store_true",
+                    help="time the single-step entry points and the layer statistic, not the bench line")
     ap.add_argument("--timeline-attn", action="store_true",
                     help="per-step phase timings of criterion B's tensor-core passes (timeline build), not a bench line")
     ap.add_argument("--crossover", action="store_true",
@@ -1284,6 +1362,9 @@ def main():
         return
     if args.timeline_attn:
         print(json.dumps(run_timeline_attn(args)), flush=True)
+        return
+    if args.standalone:
+        print(json.dumps(run_standalone(args)), flush=True)
         return
     if args.crossover:
         print(json.dumps(run_crossover(args)), flush=True)
