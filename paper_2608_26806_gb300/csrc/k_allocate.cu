@@ -1,7 +1,8 @@
 // Step 2 as its own kernel (avtp_allocate): one warp per request runs the budget
 // rule of avtp_alloc.cuh (paper §3.3.3 adaptive keep ratio, App. A.2 clamps) and
-// writes the request's budgets. The fused stage (avtp_prune) runs the same rule
-// inside the selection kernel instead.
+// writes the request's budgets: the register form (a lane per image) for requests of up
+// to 32 images, the shared-memory form beyond, as in the fused stage (avtp_prune), which
+// runs the same rule inside the selection kernel.
 #include "avtp_alloc.cuh"
 
 namespace avtp {
@@ -10,7 +11,7 @@ namespace {
 constexpr int kMaxWarpsPerCta = 4;
 constexpr size_t kSmemBudget = 200 * 1024;
 
-__global__ void __launch_bounds__(kMaxWarpsPerCta * 32)
+__global__ void __launch_bounds__(kMaxWarpsPerCta * 32, 1)
 k_allocate(const int32_t* __restrict__ img_cu, const int32_t* __restrict__ img_len,
            const int64_t* __restrict__ img_sums, const float* __restrict__ keep_ratio, float alpha, float r_min,
            float r_max, int relative, const int32_t* __restrict__ vis_cu, const int32_t* __restrict__ req_budget,
@@ -25,6 +26,22 @@ k_allocate(const int32_t* __restrict__ img_cu, const int32_t* __restrict__ img_l
   const int m = img_cu[r + 1] - i0;
   if (m == 0) return;
   const WarpAllocSmem sm = carve_warp_alloc(smem + static_cast<size_t>(warp) * warp_alloc_smem_bytes(m_cap), m_cap);
+  if (m <= 32) {
+    const bool has = lane < m;
+    const int64_t S = has ? img_sums[i0 + lane] : 0;
+    const int32_t n = has ? img_len[i0 + lane] : 0;
+    const int32_t N = vis_cu[i0 + m] - vis_cu[i0];
+    const RatioRule rule = make_ratio_rule(keep_ratio[r], alpha, relative);
+    int32_t K = 0;
+    const int err = warp_allocate32(sm, m, S, n, recip62(n), req_budget[r], N, recip62(N), rule, alpha, r_min, r_max,
+                                    &K);
+    if (err != AVTP_OK) {
+      if (lane == 0) record_error(st, err, r);
+      return;
+    }
+    if (has) budgets[i0 + lane] = K;
+    return;
+  }
   for (int j = lane; j < m; j += 32) {
     sm.S[j] = img_sums[i0 + j];
     sm.n[j] = img_len[i0 + j];
